@@ -1,0 +1,210 @@
+/*
+ * kvq — packed low-bit KV-cache attention step with LoRA-adapted Q/K/V
+ * projections, for NVIDIA GB300 (sm_103a).  C ABI.
+ *
+ * The step follows "Quality Recovery for Quantized KV Caches via Low-Rank
+ * Attention Adaptation" (arXiv 2609.04263):
+ *   kvq_project_lora    Section 3, Eq. (1) and Eq. (lora): Q/K/V = H W'^T with
+ *                       W' = W + (alpha/r) B A, kept as an explicit rank-r
+ *                       branch (Section 3.4), then rotary positions on Q, K.
+ *   kvq_append_pack     Section 3.1, Eq. (affine) and the symmetric control;
+ *                       KIVI and KVarN formats: new keys/values are coded and
+ *                       appended; no unquantized copy is kept beyond the
+ *                       format's own full-precision window.
+ *   kvq_attend_prefill  Sections 3.1-3.3: causal attention of the newly
+ *   kvq_attend_decode   appended tokens over the stored reconstruction
+ *                       R_phi(K, V) of every cached token.
+ *
+ * Conventions for every call:
+ *   - Tensor arguments are DEVICE pointers owned by the caller, row-major and
+ *     contiguous.  The library never allocates device memory: a cache lives
+ *     in a caller-provided buffer of kvq_cache_bytes() bytes.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *     asynchronous on that stream; the caller orders calls on one cache.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     failed validation returns a status, launches nothing and leaves the
+ *     cache unchanged.  kvq_last_error() describes the last failure of the
+ *     calling thread.
+ *   - Inputs must be finite.
+ *   - The dtype (KVQ_F32 or KVQ_BF16) is the activation dtype: it applies to
+ *     hidden states, weights, LoRA factors, q/k/v, outputs and the
+ *     full-precision cache windows.  Accumulation is fp32; cache metadata is
+ *     fp16.
+ */
+#ifndef KVQ_H
+#define KVQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define KVQ_ABI_VERSION 1
+
+typedef enum {
+  KVQ_OK = 0,
+  KVQ_ERR_ARG = 1,          /* null pointer, bad enum, negative size         */
+  KVQ_ERR_SHAPE = 2,        /* inconsistent or unsupported dimensions        */
+  KVQ_ERR_CAPACITY = 3,     /* append beyond max_tokens, buffer too small    */
+  KVQ_ERR_UNSUPPORTED = 4,  /* format/bit-width/dtype combination not built  */
+  KVQ_ERR_CUDA = 5,         /* a CUDA launch or query failed                 */
+  KVQ_ERR_TIMEOUT = 6       /* a bounded device-side wait gave up            */
+} kvq_status;
+
+/* Cache formats (Section 3.1). */
+typedef enum {
+  KVQ_FMT_FLOAT = 0,      /* control: K/V stored in the activation dtype        */
+  KVQ_FMT_AFFINE = 1,     /* Eq. (affine): groups of `group_size` along D, codes
+                             round((x - min)/s), fp16 scale and fp16 offset     */
+  KVQ_FMT_SYMMETRIC = 2,  /* maximum-magnitude fp16 scale, no offset; signed
+                             code q in [-(2^(b-1)-1), 2^(b-1)-1] stored as
+                             q + 2^(b-1)                                        */
+  KVQ_FMT_KIVI = 3,       /* keys per channel (group = 32-token block x one
+                             channel), values per token (groups along D), the
+                             newest R..R+G-1 tokens kept at full precision      */
+  KVQ_FMT_KVARN = 4       /* first `sink_tokens` kept at full precision; then
+                             blocks of `group_size` tokens: normalised Hadamard
+                             on D, `norm_iters` rounds of dual-axis variance
+                             normalisation, grouped affine codes                */
+} kvq_format;
+
+typedef enum { KVQ_F32 = 0, KVQ_BF16 = 1 } kvq_dtype;
+
+/* Geometry and format of one layer's cache. */
+typedef struct {
+  int32_t fmt;              /* kvq_format                                       */
+  int32_t key_bits;         /* 2, 4 or 8 (ignored for FLOAT)                     */
+  int32_t value_bits;       /* 2, 4 or 8 (ignored for FLOAT)                     */
+  int32_t group_size;       /* G: divides head_dim; KIVI/KVarN: also the token
+                               block length (power of two for KVarN)            */
+  int32_t residual_tokens;  /* KIVI: R (>= 0)                                    */
+  int32_t sink_tokens;      /* KVarN: S (>= 0)                                   */
+  int32_t norm_iters;       /* KVarN: normalisation iterations (paper: 8)        */
+  int32_t batch;            /* B sequences, all holding the same token count    */
+  int32_t kv_heads;         /* Hkv                                               */
+  int32_t q_heads;          /* Hq (multiple of Hkv); sizes the decode workspace */
+  int32_t head_dim;         /* D: 64, 128 or 256                                 */
+  int32_t max_tokens;       /* capacity per sequence                             */
+  int32_t dtype;            /* kvq_dtype of the full-precision windows           */
+} kvq_cache_desc;
+
+typedef struct kvq_cache kvq_cache;   /* opaque, host-side bookkeeping only */
+
+/* Planes of a cache, for inspection and tests (kvq_cache_view). */
+enum {
+  KVQ_PLANE_K_CODES = 0,  /* uint8 [B][Hkv][rows][D*kb/8], LSB-first bit order   */
+  KVQ_PLANE_K_SCALE,      /* fp16: per token [rows][D/G]; KIVI [blocks][D]       */
+  KVQ_PLANE_K_ZERO,       /* fp16, same shape as K_SCALE (affine formats)        */
+  KVQ_PLANE_V_CODES,
+  KVQ_PLANE_V_SCALE,
+  KVQ_PLANE_V_ZERO,
+  KVQ_PLANE_K_FULL,       /* act dtype: FLOAT all tokens; KIVI residual ring of
+                             R+G slots (token t in slot t mod (R+G)); KVarN sinks */
+  KVQ_PLANE_V_FULL,
+  KVQ_PLANE_K_PEND,       /* act dtype, KVarN staging ring [G][D], slot (t-S) mod G */
+  KVQ_PLANE_V_PEND,
+  KVQ_PLANE_K_ROW,        /* fp16 KVarN row scales, one per quantized token      */
+  KVQ_PLANE_K_COL,        /* fp16 KVarN column scales [blocks][D]                */
+  KVQ_PLANE_V_ROW,
+  KVQ_PLANE_V_COL,
+  KVQ_PLANE_WORKSPACE,    /* fp32 decode split-K partials (not cache state)      */
+  KVQ_NUM_PLANES
+};
+
+typedef struct {
+  void* ptr[KVQ_NUM_PLANES];          /* device pointer, NULL if absent        */
+  int64_t dims[KVQ_NUM_PLANES][4];    /* [B][Hkv][rows][cols], row-major       */
+  int32_t elem_bytes[KVQ_NUM_PLANES]; /* 1 codes, 2 fp16/bf16, 4 fp32           */
+  int32_t tokens;                     /* T: tokens stored per sequence          */
+  int32_t quantized_tokens;           /* tokens held as codes (KIVI/KVarN: the
+                                         quantized prefix; AFFINE/SYM: T)      */
+} kvq_cache_planes;
+
+/* Device bytes a cache with this descriptor needs (0 if the descriptor is
+ * invalid; see kvq_last_error). */
+size_t kvq_cache_bytes(const kvq_cache_desc* desc);
+
+/* Bind a cache to `dev_buf` (caller-owned, >= kvq_cache_bytes, 256-byte
+ * aligned).  Allocates only the host-side handle; the buffer contents need no
+ * initialisation.  The cache starts empty (T = 0). */
+kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t bytes,
+                            kvq_cache** out);
+
+/* Free the host handle.  The device buffer stays the caller's. */
+kvq_status kvq_destroy_cache(kvq_cache* cache);
+
+/* Forget every stored token (host bookkeeping only; nothing is launched). */
+kvq_status kvq_reset_cache(kvq_cache* cache);
+
+/* Tokens stored per sequence, or -1 for a NULL cache. */
+int kvq_cache_tokens(const kvq_cache* cache);
+
+/* Device pointers and shapes of every plane (for tests and export). */
+kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out);
+
+/*
+ * Q/K/V projection with explicit LoRA branches and rotary positions
+ * (Section 3, Eq. 1 and Eq. lora; cost per token per Section 3.4).
+ *
+ *   x       [B][L][d_in]                     hidden states
+ *   w_qkv   [(Hq + 2 Hkv) * D][d_in]          frozen W_Q, W_K, W_V stacked by rows
+ *   a_p     [r_p][d_in], b_p [d_out_p][r_p]   LoRA factors of p in {q,k,v};
+ *                                             r_p = 0 (pointers ignored) means no
+ *                                             adapter on p (placements Q/K/QK/QKV)
+ *   out     q [B][Hq][L][D], k and v [B][Hkv][L][D]   (head-major)
+ *
+ *   y_p = x W_p^T + alpha_over_r * (x A_p^T) B_p^T, then rotate-half RoPE on
+ *   q and k at positions pos0 + l with frequencies rope_base^(-2i/D)
+ *   (rope_base = 0 disables RoPE).  r_p <= 64, multiple of 8 for KVQ_BF16.
+ */
+kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w_qkv,
+                            const void* a_q, const void* b_q, int r_q,
+                            const void* a_k, const void* b_k, int r_k,
+                            const void* a_v, const void* b_v, int r_v,
+                            float alpha_over_r, int n_q_heads, int n_kv_heads,
+                            int head_dim, int pos0, float rope_base, int dtype,
+                            void* q, void* k, void* v, void* stream);
+
+/*
+ * Append L new tokens per sequence: k, v [B][Hkv][L][D] (activation dtype).
+ * Codes them per the cache format (Section 3.1) into the packed planes.  The
+ * cache after T tokens is the same whether they arrive in one call or in
+ * chunks.  KVQ_ERR_CAPACITY if T + L > max_tokens.
+ */
+kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L,
+                           void* stream);
+
+/*
+ * Causal attention of the L most recently appended tokens' queries over the
+ * reconstruction of all T cached tokens (Sections 3.2-3.3).  Query l sits at
+ * position T - L + l and sees tokens 0 .. T - L + l.  q, out [B][Hq][L][D];
+ * query head h reads kv head h / (Hq / Hkv).  softmax_scale is usually
+ * 1/sqrt(D).  Must follow kvq_append_pack of the same L tokens.
+ */
+kvq_status kvq_attend_prefill(kvq_cache* cache, const void* q, int L, int n_q_heads,
+                              float softmax_scale, void* out, void* stream);
+
+/*
+ * Decode step: kvq_attend_prefill with L = 1, split over the tokens across
+ * thread blocks with a log-sum-exp merge (partials in the cache's workspace
+ * plane, so calls on one cache must not overlap).  q, out [B][Hq][1][D].
+ */
+kvq_status kvq_attend_decode(kvq_cache* cache, const void* q, int n_q_heads,
+                             float softmax_scale, void* out, void* stream);
+
+/* Read and clear the device-side error word of the library (synchronises
+ * `stream`).  *out = 0 when no bounded wait has timed out. */
+kvq_status kvq_device_status(void* stream, int* out);
+
+/* Description of the last failure on this thread ("" if none). */
+const char* kvq_last_error(void);
+
+/* KVQ_ABI_VERSION of the loaded library. */
+int kvq_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVQ_H */

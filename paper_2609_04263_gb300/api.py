@@ -1,0 +1,123 @@
+"""PyTorch-facing wrappers over the C ABI: device memory and streams come from
+torch, every computation runs in libkvq.so."""
+from __future__ import annotations
+
+import math
+
+import torch
+
+from . import kvq
+
+_DT = {torch.float32: kvq.KVQ_F32, torch.bfloat16: kvq.KVQ_BF16}
+_TORCH = {kvq.KVQ_F32: torch.float32, kvq.KVQ_BF16: torch.bfloat16}
+_PLANE_DTYPE = {1: torch.uint8, 2: torch.float16, 4: torch.float32}
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("tensor arguments must be contiguous CUDA tensors")
+    return t.data_ptr()
+
+
+def make_desc(fmt, key_bits, value_bits, group_size, batch, kv_heads, q_heads, head_dim,
+              max_tokens, dtype, residual_tokens=0, sink_tokens=0, norm_iters=8):
+    return kvq.kvq_cache_desc(fmt=fmt, key_bits=key_bits, value_bits=value_bits,
+                              group_size=group_size, residual_tokens=residual_tokens,
+                              sink_tokens=sink_tokens, norm_iters=norm_iters, batch=batch,
+                              kv_heads=kv_heads, q_heads=q_heads, head_dim=head_dim,
+                              max_tokens=max_tokens, dtype=_DT.get(dtype, dtype))
+
+
+class Cache:
+    """One layer's packed cache in a torch-owned device buffer."""
+
+    def __init__(self, desc: kvq.kvq_cache_desc, device="cuda", buffer=None):
+        self.desc = desc
+        self.nbytes = kvq.kvq_cache_bytes(desc)
+        if buffer is None:
+            buffer = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        self.buffer = buffer
+        self.handle = kvq.kvq_create_cache(desc, buffer.data_ptr(), self.nbytes)
+        self.act = _TORCH[desc.dtype]
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h:
+            kvq.kvq_destroy_cache(h)
+            self.handle = None
+
+    @property
+    def tokens(self) -> int:
+        return kvq.kvq_cache_tokens(self.handle)
+
+    def reset(self) -> None:
+        kvq.kvq_reset_cache(self.handle)
+
+    def append(self, k: torch.Tensor, v: torch.Tensor) -> None:
+        kvq.kvq_append_pack(self.handle, _ptr(k), _ptr(v), k.shape[2], _stream())
+
+    def attend_prefill(self, q: torch.Tensor, out=None, scale=None) -> torch.Tensor:
+        out = torch.empty_like(q) if out is None else out
+        scale = 1.0 / math.sqrt(self.desc.head_dim) if scale is None else scale
+        kvq.kvq_attend_prefill(self.handle, _ptr(q), q.shape[2], q.shape[1], scale, _ptr(out),
+                               _stream())
+        return out
+
+    def attend_decode(self, q: torch.Tensor, out=None, scale=None) -> torch.Tensor:
+        out = torch.empty_like(q) if out is None else out
+        scale = 1.0 / math.sqrt(self.desc.head_dim) if scale is None else scale
+        kvq.kvq_attend_decode(self.handle, _ptr(q), q.shape[1], scale, _ptr(out), _stream())
+        return out
+
+    def planes(self) -> dict:
+        """name -> tensor view [B, H, rows, cols] of each present plane."""
+        v = kvq.kvq_cache_view(self.handle)
+        base = self.buffer.data_ptr()
+        out = {}
+        for i, name in enumerate(kvq.PLANES):
+            p = v.ptr[i]
+            if not p:
+                continue
+            dims = [int(d) for d in v.dims[i]]
+            eb = int(v.elem_bytes[i])
+            n = dims[0] * dims[1] * dims[2] * dims[3] * eb
+            off = p - base
+            raw = self.buffer[off:off + n]
+            dt = _PLANE_DTYPE[eb]
+            if name.endswith(("_full", "_pend")):
+                dt = self.act
+            out[name] = raw.view(dt).view(*dims)
+        out["_tokens"] = int(v.tokens)
+        out["_quantized_tokens"] = int(v.quantized_tokens)
+        return out
+
+
+def project_lora(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0=0,
+                 rope_base=0.0, out=None):
+    """q [B,Hq,L,D], k, v [B,Hkv,L,D] = RoPE(x W'^T) with W' = W + (alpha/r) B A.
+
+    lora: dict p -> (A [r, d_in], B [d_out, r]) or None for p in 'qkv'.
+    """
+    B, L, d_in = x.shape
+    D = head_dim
+    if out is None:
+        out = (torch.empty(B, n_q_heads, L, D, dtype=x.dtype, device=x.device),
+               torch.empty(B, n_kv_heads, L, D, dtype=x.dtype, device=x.device),
+               torch.empty(B, n_kv_heads, L, D, dtype=x.dtype, device=x.device))
+    args = []
+    for p in "qkv":
+        ab = lora.get(p)
+        if ab is None:
+            args += [None, None, 0]
+        else:
+            args += [_ptr(ab[0]), _ptr(ab[1]), ab[0].shape[0]]
+    kvq.kvq_project_lora(_ptr(x), B, L, d_in, _ptr(w_qkv), *args, alpha_over_r, n_q_heads,
+                         n_kv_heads, head_dim, pos0, rope_base, _DT[x.dtype], _ptr(out[0]),
+                         _ptr(out[1]), _ptr(out[2]), _stream())
+    return out

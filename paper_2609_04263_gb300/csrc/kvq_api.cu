@@ -1,0 +1,392 @@
+// C-ABI entry points: argument validation, cache geometry and bookkeeping.
+// Kernels live in pack.cu, attend.cu and project.cu.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "kvq_internal.cuh"
+
+using namespace kvq;
+
+struct kvq_cache {
+  kvq_cache_desc desc;
+  Geom g;
+  char* base;
+  size_t bytes;
+  int T;
+};
+
+namespace {
+
+thread_local std::string g_last_error;
+
+kvq_status fail(kvq_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+kvq_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(KVQ_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool misaligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) != 0; }
+
+bool valid_bits(int b) { return b == 2 || b == 4 || b == 8; }
+bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Validate a descriptor and lay out its planes.  Offsets are relative to the
+// buffer start; returns the total size, or 0 with g_last_error set.
+size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
+              kvq_status* st) {
+  *st = KVQ_ERR_ARG;
+  if (!d) { fail(KVQ_ERR_ARG, "descriptor is NULL"); return 0; }
+  if (d->fmt < KVQ_FMT_FLOAT || d->fmt > KVQ_FMT_KVARN) {
+    fail(KVQ_ERR_ARG, "unknown format %d", d->fmt); return 0;
+  }
+  if (d->dtype != KVQ_F32 && d->dtype != KVQ_BF16) {
+    fail(KVQ_ERR_ARG, "unknown dtype %d", d->dtype); return 0;
+  }
+  *st = KVQ_ERR_SHAPE;
+  if (d->batch <= 0 || d->kv_heads <= 0 || d->q_heads <= 0 || d->max_tokens <= 0) {
+    fail(KVQ_ERR_SHAPE, "batch, kv_heads, q_heads and max_tokens must be positive"); return 0;
+  }
+  if (d->q_heads % d->kv_heads != 0) {
+    fail(KVQ_ERR_SHAPE, "q_heads %d is not a multiple of kv_heads %d", d->q_heads, d->kv_heads);
+    return 0;
+  }
+  if (d->q_heads / d->kv_heads > 16) {
+    fail(KVQ_ERR_UNSUPPORTED, "GQA group %d > 16", d->q_heads / d->kv_heads);
+    *st = KVQ_ERR_UNSUPPORTED; return 0;
+  }
+  if (d->head_dim != 64 && d->head_dim != 128 && d->head_dim != 256) {
+    fail(KVQ_ERR_UNSUPPORTED, "head_dim %d (supported: 64, 128, 256)", d->head_dim);
+    *st = KVQ_ERR_UNSUPPORTED; return 0;
+  }
+  const int D = d->head_dim, G = d->group_size;
+  if (d->fmt != KVQ_FMT_FLOAT) {
+    if (!valid_bits(d->key_bits) || !valid_bits(d->value_bits)) {
+      fail(KVQ_ERR_UNSUPPORTED, "bit widths %d/%d (supported: 2, 4, 8)", d->key_bits,
+           d->value_bits);
+      *st = KVQ_ERR_UNSUPPORTED; return 0;
+    }
+    if (G < 8 || !pow2(G) || D % G != 0 || G > D) {
+      fail(KVQ_ERR_SHAPE, "group_size %d must be a power of two in [8, head_dim] dividing %d",
+           G, D);
+      return 0;
+    }
+  }
+  if (d->fmt == KVQ_FMT_KIVI && d->residual_tokens < 0) {
+    fail(KVQ_ERR_SHAPE, "residual_tokens must be >= 0"); return 0;
+  }
+  if (d->fmt == KVQ_FMT_KVARN) {
+    if (d->sink_tokens < 0 || d->norm_iters < 0 || d->norm_iters > 64) {
+      fail(KVQ_ERR_SHAPE, "sink_tokens >= 0 and 0 <= norm_iters <= 64 required"); return 0;
+    }
+    if (G > 128 || G * D > 16384) {
+      fail(KVQ_ERR_UNSUPPORTED, "KVarN block of %d tokens x %d channels (max 128 tokens, "
+           "16384 elements)", G, D);
+      *st = KVQ_ERR_UNSUPPORTED; return 0;
+    }
+  }
+  const int B = d->batch, H = d->kv_heads, Tm = d->max_tokens;
+  const int act = d->dtype == KVQ_BF16 ? 2 : 4;
+  memset(g, 0, sizeof *g);
+  g->fmt = d->fmt; g->kb = d->key_bits; g->vb = d->value_bits; g->G = G;
+  g->R = d->residual_tokens; g->S = d->sink_tokens; g->iters = d->norm_iters;
+  g->B = B; g->H = H; g->Hq = d->q_heads; g->D = D; g->Tmax = Tm; g->act = d->dtype;
+  g->ring = d->residual_tokens + G;
+  auto set = [&](int which, int64_t rows, int64_t cols, int elem) {
+    g->pl[which].rows = rows; g->pl[which].cols = cols; g->pl[which].elem = elem;
+  };
+  switch (d->fmt) {
+    case KVQ_FMT_FLOAT:
+      set(KVQ_PLANE_K_FULL, Tm, D, act);
+      set(KVQ_PLANE_V_FULL, Tm, D, act);
+      break;
+    case KVQ_FMT_AFFINE:
+    case KVQ_FMT_SYMMETRIC:
+      set(KVQ_PLANE_K_CODES, Tm, D * d->key_bits / 8, 1);
+      set(KVQ_PLANE_K_SCALE, Tm, D / G, 2);
+      set(KVQ_PLANE_V_CODES, Tm, D * d->value_bits / 8, 1);
+      set(KVQ_PLANE_V_SCALE, Tm, D / G, 2);
+      if (d->fmt == KVQ_FMT_AFFINE) {
+        set(KVQ_PLANE_K_ZERO, Tm, D / G, 2);
+        set(KVQ_PLANE_V_ZERO, Tm, D / G, 2);
+      }
+      break;
+    case KVQ_FMT_KIVI: {
+      const int64_t nblk = (Tm + G - 1) / G;
+      set(KVQ_PLANE_K_CODES, nblk * G, D * d->key_bits / 8, 1);
+      set(KVQ_PLANE_K_SCALE, nblk, D, 2);
+      set(KVQ_PLANE_K_ZERO, nblk, D, 2);
+      set(KVQ_PLANE_V_CODES, nblk * G, D * d->value_bits / 8, 1);
+      set(KVQ_PLANE_V_SCALE, nblk * G, D / G, 2);
+      set(KVQ_PLANE_V_ZERO, nblk * G, D / G, 2);
+      set(KVQ_PLANE_K_FULL, g->ring, D, act);
+      set(KVQ_PLANE_V_FULL, g->ring, D, act);
+      break;
+    }
+    case KVQ_FMT_KVARN: {
+      const int64_t nblk = Tm > d->sink_tokens ? (Tm - d->sink_tokens) / G : 0;
+      const int64_t Q = nblk * G;
+      if (d->sink_tokens > 0) {
+        set(KVQ_PLANE_K_FULL, d->sink_tokens, D, act);
+        set(KVQ_PLANE_V_FULL, d->sink_tokens, D, act);
+      }
+      set(KVQ_PLANE_K_PEND, G, D, act);
+      set(KVQ_PLANE_V_PEND, G, D, act);
+      if (nblk > 0) {
+        set(KVQ_PLANE_K_CODES, Q, D * d->key_bits / 8, 1);
+        set(KVQ_PLANE_K_SCALE, Q, D / G, 2);
+        set(KVQ_PLANE_K_ZERO, Q, D / G, 2);
+        set(KVQ_PLANE_K_ROW, 1, Q, 2);
+        set(KVQ_PLANE_K_COL, nblk, D, 2);
+        set(KVQ_PLANE_V_CODES, Q, D * d->value_bits / 8, 1);
+        set(KVQ_PLANE_V_SCALE, Q, D / G, 2);
+        set(KVQ_PLANE_V_ZERO, Q, D / G, 2);
+        set(KVQ_PLANE_V_ROW, 1, Q, 2);
+        set(KVQ_PLANE_V_COL, nblk, D, 2);
+      }
+      break;
+    }
+  }
+  size_t total = 0;
+  for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
+    off[i] = 0;
+    if (i == KVQ_PLANE_WORKSPACE) continue;
+    Plane& p = g->pl[i];
+    if (p.rows == 0) continue;
+    off[i] = total;
+    total = align256(total + (size_t)B * H * p.rows * p.cols * p.elem);
+  }
+  // decode workspace: [B][Hq][kMaxSplits][D + 2] fp32, indexed by q head
+  off[KVQ_PLANE_WORKSPACE] = total;
+  g->pl[KVQ_PLANE_WORKSPACE].rows = kMaxSplits;
+  g->pl[KVQ_PLANE_WORKSPACE].cols = D + kWsStride;
+  g->pl[KVQ_PLANE_WORKSPACE].elem = 4;
+  total = align256(total + (size_t)B * d->q_heads * kMaxSplits * (D + kWsStride) * 4);
+  *st = KVQ_OK;
+  return total;
+}
+
+int g_num_sms = 0;
+std::mutex g_mu;
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// device error word: one int in static device memory, address looked up per
+// device on first use
+// ---------------------------------------------------------------------------
+static __device__ int g_kvq_device_error;
+
+namespace kvq {
+int* device_error_word() {
+  static int* addr[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_kvq_device_error) != cudaSuccess) return nullptr;
+    addr[dev] = static_cast<int*>(p);
+  }
+  return addr[dev];
+}
+
+int num_sms() {
+  if (g_num_sms == 0) {
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    g_num_sms = n > 0 ? n : 148;
+  }
+  return g_num_sms;
+}
+}  // namespace kvq
+
+extern "C" {
+
+int kvq_abi_version(void) { return KVQ_ABI_VERSION; }
+
+const char* kvq_last_error(void) { return g_last_error.c_str(); }
+
+size_t kvq_cache_bytes(const kvq_cache_desc* desc) {
+  Geom g;
+  size_t off[KVQ_NUM_PLANES];
+  kvq_status st;
+  return layout(desc, &g, off, &st);
+}
+
+kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t bytes,
+                            kvq_cache** out) {
+  if (!out) return fail(KVQ_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  if (!dev_buf) return fail(KVQ_ERR_ARG, "dev_buf is NULL");
+  if (reinterpret_cast<uintptr_t>(dev_buf) % 256 != 0)
+    return fail(KVQ_ERR_ARG, "dev_buf must be 256-byte aligned");
+  Geom g;
+  size_t off[KVQ_NUM_PLANES];
+  kvq_status st;
+  size_t need = layout(desc, &g, off, &st);
+  if (need == 0) return st;
+  if (bytes < need)
+    return fail(KVQ_ERR_CAPACITY, "buffer of %zu bytes < %zu needed", bytes, need);
+  kvq_cache* c = new kvq_cache;
+  c->desc = *desc;
+  c->g = g;
+  c->base = static_cast<char*>(dev_buf);
+  c->bytes = bytes;
+  c->T = 0;
+  for (int i = 0; i < KVQ_NUM_PLANES; ++i)
+    c->g.pl[i].p = c->g.pl[i].rows ? c->base + off[i] : nullptr;
+  *out = c;
+  g_last_error.clear();
+  return KVQ_OK;
+}
+
+kvq_status kvq_destroy_cache(kvq_cache* cache) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  delete cache;
+  return KVQ_OK;
+}
+
+kvq_status kvq_reset_cache(kvq_cache* cache) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  cache->T = 0;
+  return KVQ_OK;
+}
+
+int kvq_cache_tokens(const kvq_cache* cache) { return cache ? cache->T : -1; }
+
+kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out) {
+  if (!cache || !out) return fail(KVQ_ERR_ARG, "cache or out is NULL");
+  const Geom& g = cache->g;
+  for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
+    out->ptr[i] = g.pl[i].p;
+    out->dims[i][0] = g.pl[i].rows ? g.B : 0;
+    out->dims[i][1] = g.pl[i].rows ? (i == KVQ_PLANE_WORKSPACE ? g.Hq : g.H) : 0;
+    out->dims[i][2] = g.pl[i].rows;
+    out->dims[i][3] = g.pl[i].cols;
+    out->elem_bytes[i] = g.pl[i].elem;
+  }
+  out->tokens = cache->T;
+  switch (g.fmt) {
+    case KVQ_FMT_FLOAT: out->quantized_tokens = 0; break;
+    case KVQ_FMT_KIVI: out->quantized_tokens = kivi_tq(cache->T, g.R, g.G); break;
+    case KVQ_FMT_KVARN: out->quantized_tokens = kvarn_nblocks(cache->T, g.S, g.G) * g.G; break;
+    default: out->quantized_tokens = cache->T;
+  }
+  return KVQ_OK;
+}
+
+kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L,
+                           void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (L < 0) return fail(KVQ_ERR_ARG, "L = %d < 0", L);
+  if (L == 0) return KVQ_OK;
+  if (!k || !v) return fail(KVQ_ERR_ARG, "k or v is NULL");
+  if (misaligned(k) || misaligned(v)) return fail(KVQ_ERR_ARG, "k and v must be 16-byte aligned");
+  if ((int64_t)cache->T + L > cache->g.Tmax)
+    return fail(KVQ_ERR_CAPACITY, "append of %d tokens to %d exceeds max_tokens %d", L,
+                cache->T, cache->g.Tmax);
+  cudaError_t e = launch_append(cache->g, cache->T, L, k, v, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_append_pack launch");
+  cache->T += L;
+  return KVQ_OK;
+}
+
+static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_heads,
+                                float scale, void* out, void* stream, bool decode) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (!q || !out) return fail(KVQ_ERR_ARG, "q or out is NULL");
+  if (misaligned(q) || misaligned(out)) return fail(KVQ_ERR_ARG, "q and out must be 16-byte aligned");
+  if (L <= 0) return fail(KVQ_ERR_ARG, "L = %d must be positive", L);
+  if (n_q_heads != cache->g.Hq)
+    return fail(KVQ_ERR_SHAPE, "n_q_heads %d != cache q_heads %d", n_q_heads, cache->g.Hq);
+  if (L > cache->T)
+    return fail(KVQ_ERR_SHAPE, "%d queries but only %d cached tokens (append first)", L,
+                cache->T);
+  if (!(scale > 0.f) || scale != scale) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
+  cudaError_t e = launch_attend(cache->g, cache->T, q, L, scale, out, decode,
+                                (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_attend launch");
+  return KVQ_OK;
+}
+
+kvq_status kvq_attend_prefill(kvq_cache* cache, const void* q, int L, int n_q_heads,
+                              float softmax_scale, void* out, void* stream) {
+  return attend_common(cache, q, L, n_q_heads, softmax_scale, out, stream, false);
+}
+
+kvq_status kvq_attend_decode(kvq_cache* cache, const void* q, int n_q_heads,
+                             float softmax_scale, void* out, void* stream) {
+  return attend_common(cache, q, 1, n_q_heads, softmax_scale, out, stream, true);
+}
+
+kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w_qkv,
+                            const void* a_q, const void* b_q, int r_q,
+                            const void* a_k, const void* b_k, int r_k,
+                            const void* a_v, const void* b_v, int r_v,
+                            float alpha_over_r, int n_q_heads, int n_kv_heads,
+                            int head_dim, int pos0, float rope_base, int dtype,
+                            void* q, void* k, void* v, void* stream) {
+  if (dtype != KVQ_F32 && dtype != KVQ_BF16) return fail(KVQ_ERR_ARG, "unknown dtype %d", dtype);
+  if (B < 0 || L < 0 || d_in <= 0) return fail(KVQ_ERR_SHAPE, "bad B/L/d_in");
+  if (n_q_heads <= 0 || n_kv_heads <= 0 || n_q_heads % n_kv_heads)
+    return fail(KVQ_ERR_SHAPE, "heads %d/%d", n_q_heads, n_kv_heads);
+  if (head_dim != 64 && head_dim != 128 && head_dim != 256)
+    return fail(KVQ_ERR_UNSUPPORTED, "head_dim %d (supported: 64, 128, 256)", head_dim);
+  if (pos0 < 0) return fail(KVQ_ERR_ARG, "pos0 < 0");
+  if (!(rope_base >= 0.f)) return fail(KVQ_ERR_ARG, "rope_base < 0");
+  if (dtype == KVQ_BF16 && d_in % 64 != 0)
+    return fail(KVQ_ERR_SHAPE, "d_in %d must be a multiple of 64 for bf16", d_in);
+  if (B == 0 || L == 0) return KVQ_OK;
+  if (!x || !w_qkv || !q || !k || !v) return fail(KVQ_ERR_ARG, "NULL tensor pointer");
+  if (misaligned(x) || misaligned(w_qkv) || misaligned(q) || misaligned(k) || misaligned(v))
+    return fail(KVQ_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  const void* a[3] = {a_q, a_k, a_v};
+  const void* bm[3] = {b_q, b_k, b_v};
+  int r[3] = {r_q, r_k, r_v};
+  for (int p = 0; p < 3; ++p) {
+    if (r[p] < 0 || r[p] > 64) return fail(KVQ_ERR_SHAPE, "rank %d outside [0, 64]", r[p]);
+    if (r[p] > 0 && (!a[p] || !bm[p])) return fail(KVQ_ERR_ARG, "rank %d but NULL factor", r[p]);
+    if (dtype == KVQ_BF16 && r[p] % 8) return fail(KVQ_ERR_SHAPE, "bf16 rank %d not a multiple of 8", r[p]);
+    if (r[p] == 0) { a[p] = nullptr; bm[p] = nullptr; }
+    if (misaligned(a[p]) || misaligned(bm[p]))
+      return fail(KVQ_ERR_ARG, "LoRA factors must be 16-byte aligned");
+  }
+  void* out[3] = {q, k, v};
+  int* err = device_error_word();
+  if (!err) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
+  cudaError_t e = launch_project(x, B, L, d_in, w_qkv, a, bm, r, alpha_over_r, n_q_heads,
+                                 n_kv_heads, head_dim, pos0, rope_base, dtype, out, err,
+                                 (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora launch");
+  return KVQ_OK;
+}
+
+kvq_status kvq_device_status(void* stream, int* out) {
+  if (!out) return fail(KVQ_ERR_ARG, "out is NULL");
+  int* p = device_error_word();
+  if (!p) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
+  cudaStream_t s = (cudaStream_t)stream;
+  int h = 0;
+  cudaError_t e = cudaMemcpyAsync(&h, p, sizeof(int), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(p, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_device_status");
+  *out = h;
+  return h ? KVQ_ERR_TIMEOUT : KVQ_OK;
+}
+
+}  // extern "C"

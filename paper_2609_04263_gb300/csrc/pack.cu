@@ -1,0 +1,427 @@
+// Quantize-and-pack of new keys/values into the physical incremental cache
+// (Section 3.1).  Every value that decides a code is computed in IEEE fp32
+// with explicitly rounded operations (no contraction), in the order the cache
+// format fixes, so codes and fp16 metadata are reproducible bit for bit.
+#include <math.h>
+
+#include "kvq_internal.cuh"
+
+namespace kvq {
+namespace {
+
+// Where token t of a (b, h) row comes from: the new input for t >= T0,
+// otherwise a full-precision ring plane (KIVI residual or KVarN staging).
+struct TokSrc {
+  const void* x;      // [B][H][L][D] new tokens
+  int T0, L;
+  int ring_plane;     // plane index of the ring, -1 if none
+  int ring_off, ring_rows;
+};
+
+__device__ __forceinline__ int64_t tok_elem(const Geom& g, const TokSrc& s, int b, int h,
+                                            int t, const void** base) {
+  if (t >= s.T0) {
+    *base = s.x;
+    return (((int64_t)b * g.H + h) * s.L + (t - s.T0)) * g.D;
+  }
+  const Plane& pl = g.pl[s.ring_plane];
+  *base = pl.p;
+  int slot = (t - s.ring_off) % s.ring_rows;
+  return plane_index(pl, b, h, g.H, slot, 0);
+}
+
+// Load 8 consecutive activation elements (16-byte aligned) as fp32.
+__device__ __forceinline__ void load8(const void* base, int64_t e, int act, float v[8]) {
+  if (act == KVQ_BF16) {
+    uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(base) + e);
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 f = __bfloat1622float2(p[i]);
+      v[2 * i] = f.x;
+      v[2 * i + 1] = f.y;
+    }
+  } else {
+    const float4* p = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + e);
+    float4 a = p[0], b = p[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+}
+
+// Eq. (affine) scale for one group: max((mx - mn) / (2^b - 1), 1e-8).
+__device__ __forceinline__ float affine_scale(float mn, float mx, int bits) {
+  return fmaxf(__fdiv_rn(__fsub_rn(mx, mn), (float)((1 << bits) - 1)), 1e-8f);
+}
+__device__ __forceinline__ int affine_code(float x, float mn, float s, int bits) {
+  float c = rintf(__fdiv_rn(__fsub_rn(x, mn), s));
+  c = fminf(fmaxf(c, 0.f), (float)((1 << bits) - 1));
+  return (int)c;
+}
+// Symmetric control: s = max(absmax / qmax, 1e-8), q = round(x / s) in
+// [-qmax, qmax], stored as q + 2^(b-1).
+__device__ __forceinline__ float sym_scale(float amax, int bits) {
+  return fmaxf(__fdiv_rn(amax, (float)((1 << (bits - 1)) - 1)), 1e-8f);
+}
+__device__ __forceinline__ int sym_code(float x, float s, int bits) {
+  const float qmax = (float)((1 << (bits - 1)) - 1);
+  float q = rintf(__fdiv_rn(x, s));
+  q = fminf(fmaxf(q, -qmax), qmax);
+  return (int)q + (1 << (bits - 1));
+}
+
+// ---------------------------------------------------------------------------
+// Per-token grouped coding: AFFINE / SYMMETRIC keys and values, KIVI values.
+// A group of G elements is held by G/8 consecutive lanes, 8 elements each;
+// min/max (or absmax) is a butterfly over those lanes; each lane packs its 8
+// codes LSB-first into one 16/32/64-bit store.
+// ---------------------------------------------------------------------------
+__global__ void pack_pertoken_kernel(Geom g, int which, int bits, int sym, TokSrc src,
+                                     int t_begin, int t_end) {
+  const int lpg = g.G / 8;                 // lanes per group
+  const int gpw = 32 / lpg;                // groups per warp pass
+  const int lane = threadIdx.x & 31;
+  const int sub = lane / lpg, li = lane % lpg;
+  const int groups_per_tok = g.D / g.G;
+  const int64_t ntok = (int64_t)(t_end - t_begin);
+  const int64_t units = (int64_t)g.B * g.H * ntok * groups_per_tok;
+  const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t base = warp * gpw; base < units; base += nwarps * gpw) {
+    const int64_t u = base + sub;
+    const bool live = u < units;
+    const int64_t uu = live ? u : units - 1;
+    const int grp = (int)(uu % groups_per_tok);
+    int64_t rest = uu / groups_per_tok;
+    const int t = t_begin + (int)(rest % ntok);
+    rest /= ntok;
+    const int h = (int)(rest % g.H);
+    const int b = (int)(rest / g.H);
+    const void* sb;
+    const int64_t e = tok_elem(g, src, b, h, t, &sb) + grp * g.G + li * 8;
+    float v[8];
+    load8(sb, e, g.act, v);
+    float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) {
+      if (sym) hi = fmaxf(hi, fabsf(v[i]));
+      else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
+    }
+    for (int off = lpg / 2; off > 0; off >>= 1) {
+      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
+      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
+    }
+    float s;
+    uint64_t word = 0;
+    if (sym) {
+      s = sym_scale(hi, bits);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) word |= (uint64_t)sym_code(v[i], s, bits) << (i * bits);
+    } else {
+      s = affine_scale(lo, hi, bits);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) word |= (uint64_t)affine_code(v[i], lo, s, bits) << (i * bits);
+    }
+    if (!live) continue;
+    uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
+    const int byte0 = (grp * g.G + li * 8) * bits / 8;
+    if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
+    else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
+    else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
+    if (li == 0) {
+      *plane_ptr<__half>(g, scale_plane, b, h, t, grp) = __float2half_rn(s);
+      if (!sym) *plane_ptr<__half>(g, zero_plane, b, h, t, grp) = __float2half_rn(lo + 0.0f);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Copy new tokens into a full-precision plane at slot (t - off) mod rows:
+// FLOAT cache, KIVI residual ring, KVarN sinks and staging ring.
+// ---------------------------------------------------------------------------
+__global__ void store_full_kernel(Geom g, int plane, const void* x, int T0, int L,
+                                  int t_begin, int t_end, int off, int rows) {
+  const int es = g.act == KVQ_BF16 ? 2 : 4;
+  const int vec_per_tok = g.D * es / 16;
+  const int64_t ntok = t_end - t_begin;
+  const int64_t total = (int64_t)g.B * g.H * ntok * vec_per_tok;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int vi = (int)(i % vec_per_tok);
+    int64_t rest = i / vec_per_tok;
+    const int t = t_begin + (int)(rest % ntok);
+    rest /= ntok;
+    const int h = (int)(rest % g.H), b = (int)(rest / g.H);
+    const uint4* src = reinterpret_cast<const uint4*>(
+        reinterpret_cast<const char*>(x) + ((((int64_t)b * g.H + h) * L + (t - T0)) * g.D) * es);
+    const Plane& pl = g.pl[plane];
+    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<char*>(pl.p) +
+                                          plane_index(pl, b, h, g.H, (t - off) % rows, 0) * es);
+    dst[vi] = src[vi];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// KIVI keys: one group per (32-token block, channel).  One CTA per block.
+// ---------------------------------------------------------------------------
+__global__ void kivi_key_flush_kernel(Geom g, TokSrc src, int blk_begin) {
+  extern __shared__ float smem[];
+  const int G = g.G, D = g.D, bits = g.kb;
+  float* xs = smem;                                   // [G][D]
+  uint8_t* cs = reinterpret_cast<uint8_t*>(xs + G * D); // [G][D]
+  const int blk = blk_begin + blockIdx.x;
+  const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
+  const int t0 = blk * G;
+  for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
+    const int r = i / D, d = i % D;
+    const void* sb;
+    int64_t e = tok_elem(g, src, b, h, t0 + r, &sb);
+    xs[i] = ld_act(sb, e + d, g.act);
+  }
+  __syncthreads();
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    float mn = xs[d], mx = xs[d];
+    for (int r = 1; r < G; ++r) {
+      mn = fminf(mn, xs[r * D + d]);
+      mx = fmaxf(mx, xs[r * D + d]);
+    }
+    const float s = affine_scale(mn, mx, bits);
+    for (int r = 0; r < G; ++r) cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, bits);
+    *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
+    *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+  }
+  __syncthreads();
+  const int per = 8 / bits, row_bytes = D * bits / 8;
+  for (int i = threadIdx.x; i < G * row_bytes; i += blockDim.x) {
+    const int r = i / row_bytes, j = i % row_bytes;
+    unsigned byte = 0;
+    for (int e = 0; e < per; ++e) byte |= (unsigned)cs[r * D + j * per + e] << (e * bits);
+    plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r)[j] = (uint8_t)byte;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// KVarN block: normalised Hadamard on D, dual-axis variance normalisation,
+// grouped affine along D.  One CTA per (block, b*h); keys and values are
+// separate launches (the value launch gets the value planes in the key
+// slots).  Sums follow the stride-halving pairwise tree in fp32.
+// ---------------------------------------------------------------------------
+__global__ void kvarn_block_kernel(Geom g, TokSrc src, int blk_begin, float inv_sqrt_d) {
+  extern __shared__ float smem[];
+  const int G = g.G, D = g.D;
+  const int bits = g.kb;   // the host passes value planes in the key slots
+  float* y = smem;                 // [G][D]
+  float* acc = y + G * D;          // [G][D] scratch for the sums, then codes
+  float* sig = acc + G * D;        // [max(G, D)]
+  float* rsc = sig + 256;          // [G] row scales
+  float* csc = rsc + 128;          // [D] column scales
+  const int blk = blk_begin + blockIdx.x;
+  const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
+  const int q0 = blk * G;          // first quantized row of the block
+  const int t0 = g.S + q0;
+  const int nt = blockDim.x;
+  for (int i = threadIdx.x; i < G * D; i += nt) {
+    const int r = i / D, d = i % D;
+    const void* sb;
+    int64_t e = tok_elem(g, src, b, h, t0 + r, &sb);
+    y[i] = ld_act(sb, e + d, g.act);
+  }
+  for (int i = threadIdx.x; i < G; i += nt) rsc[i] = 1.f;
+  for (int i = threadIdx.x; i < D; i += nt) csc[i] = 1.f;
+  __syncthreads();
+  // Hadamard butterflies, h = 1, 2, ..., D/2
+  for (int hs = 1; hs < D; hs <<= 1) {
+    for (int p = threadIdx.x; p < G * D / 2; p += nt) {
+      const int r = p / (D / 2), k = p % (D / 2);
+      const int j = (k / hs) * 2 * hs + (k % hs);
+      float a = y[r * D + j], c = y[r * D + j + hs];
+      y[r * D + j] = __fadd_rn(a, c);
+      y[r * D + j + hs] = __fsub_rn(a, c);
+    }
+    __syncthreads();
+  }
+  for (int i = threadIdx.x; i < G * D; i += nt) y[i] = __fmul_rn(y[i], inv_sqrt_d);
+  __syncthreads();
+  const float inv_d = 1.f / (float)D, inv_g = 1.f / (float)G;
+  for (int it = 0; it < g.iters; ++it) {
+    // rows
+    for (int i = threadIdx.x; i < G * D; i += nt) acc[i] = __fmul_rn(y[i], y[i]);
+    __syncthreads();
+    for (int n = D / 2; n >= 1; n >>= 1) {
+      for (int p = threadIdx.x; p < G * n; p += nt) {
+        const int r = p / n, j = p % n;
+        acc[r * D + j] = __fadd_rn(acc[r * D + j], acc[r * D + j + n]);
+      }
+      __syncthreads();
+    }
+    for (int r = threadIdx.x; r < G; r += nt) {
+      const float sg = fmaxf(__fsqrt_rn(__fmul_rn(acc[r * D], inv_d)), 1e-8f);
+      sig[r] = sg;
+      rsc[r] = __fmul_rn(rsc[r], sg);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < G * D; i += nt) y[i] = __fdiv_rn(y[i], sig[i / D]);
+    __syncthreads();
+    // columns
+    for (int i = threadIdx.x; i < G * D; i += nt) acc[i] = __fmul_rn(y[i], y[i]);
+    __syncthreads();
+    for (int n = G / 2; n >= 1; n >>= 1) {
+      for (int p = threadIdx.x; p < n * D; p += nt) {
+        const int r = p / D, j = p % D;
+        acc[r * D + j] = __fadd_rn(acc[r * D + j], acc[(r + n) * D + j]);
+      }
+      __syncthreads();
+    }
+    for (int j = threadIdx.x; j < D; j += nt) {
+      const float sg = fmaxf(__fsqrt_rn(__fmul_rn(acc[j], inv_g)), 1e-8f);
+      sig[j] = sg;
+      csc[j] = __fmul_rn(csc[j], sg);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < G * D; i += nt) y[i] = __fdiv_rn(y[i], sig[i % D]);
+    __syncthreads();
+  }
+  // grouped affine along D (groups of G channels)
+  const int codes_plane = KVQ_PLANE_K_CODES, scale_plane = KVQ_PLANE_K_SCALE;
+  const int zero_plane = KVQ_PLANE_K_ZERO, row_plane = KVQ_PLANE_K_ROW;
+  const int col_plane = KVQ_PLANE_K_COL;
+  uint8_t* cs = reinterpret_cast<uint8_t*>(acc);
+  const int ng = D / G;
+  for (int p = threadIdx.x; p < G * ng; p += nt) {
+    const int r = p / ng, gq = p % ng;
+    const float* row = y + r * D + gq * G;
+    float mn = row[0], mx = row[0];
+    for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
+    const float sc = affine_scale(mn, mx, bits);
+    for (int j = 0; j < G; ++j) cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, bits);
+    *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
+    *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
+  }
+  for (int r = threadIdx.x; r < G; r += nt)
+    *plane_ptr<__half>(g, row_plane, b, h, 0, q0 + r) = __float2half_rn(rsc[r]);
+  for (int j = threadIdx.x; j < D; j += nt)
+    *plane_ptr<__half>(g, col_plane, b, h, blk, j) = __float2half_rn(csc[j]);
+  __syncthreads();
+  const int per = 8 / bits, row_bytes = D * bits / 8;
+  for (int i = threadIdx.x; i < G * row_bytes; i += nt) {
+    const int r = i / row_bytes, j = i % row_bytes;
+    unsigned byte = 0;
+    for (int e = 0; e < per; ++e) byte |= (unsigned)cs[r * D + j * per + e] << (e * bits);
+    plane_ptr<uint8_t>(g, codes_plane, b, h, q0 + r)[j] = (uint8_t)byte;
+  }
+}
+
+int grid_for(int64_t threads_needed, int block) {
+  int64_t n = (threads_needed + block - 1) / block;
+  int64_t cap = (int64_t)num_sms() * 16;
+  if (n > cap) n = cap;
+  return (int)(n < 1 ? 1 : n);
+}
+
+cudaError_t store_full(const Geom& g, int plane, const void* x, int T0, int L, int ta, int tb,
+                       int off, int rows, cudaStream_t s) {
+  if (tb <= ta) return cudaSuccess;
+  const int es = g.act == KVQ_BF16 ? 2 : 4;
+  int64_t n = (int64_t)g.B * g.H * (tb - ta) * (g.D * es / 16);
+  store_full_kernel<<<grid_for(n, 256), 256, 0, s>>>(g, plane, x, T0, L, ta, tb, off, rows);
+  return cudaGetLastError();
+}
+
+cudaError_t pack_pertoken(const Geom& g, int which, int bits, int sym, const TokSrc& src,
+                          int ta, int tb, cudaStream_t s) {
+  if (tb <= ta) return cudaSuccess;
+  int64_t units = (int64_t)g.B * g.H * (tb - ta) * (g.D / g.G);
+  int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
+  pack_pertoken_kernel<<<grid_for(threads, 256), 256, 0, s>>>(g, which, bits, sym, src, ta, tb);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_append(const Geom& g, int T0, int L, const void* k, const void* v,
+                          cudaStream_t s) {
+  const int T1 = T0 + L;
+  cudaError_t e = cudaSuccess;
+  TokSrc sk{k, T0, L, -1, 0, 1}, sv{v, T0, L, -1, 0, 1};
+  switch (g.fmt) {
+    case KVQ_FMT_FLOAT:
+      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, T0, T1, 0, g.Tmax, s);
+      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, T0, T1, 0, g.Tmax, s);
+      return e;
+    case KVQ_FMT_AFFINE:
+    case KVQ_FMT_SYMMETRIC: {
+      const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
+      e = pack_pertoken(g, 0, g.kb, sym, sk, T0, T1, s);
+      if (e == cudaSuccess) e = pack_pertoken(g, 1, g.vb, sym, sv, T0, T1, s);
+      return e;
+    }
+    case KVQ_FMT_KIVI: {
+      const int q0 = kivi_tq(T0, g.R, g.G), q1 = kivi_tq(T1, g.R, g.G);
+      sk.ring_plane = KVQ_PLANE_K_FULL; sk.ring_rows = g.ring;
+      sv.ring_plane = KVQ_PLANE_V_FULL; sv.ring_rows = g.ring;
+      if (q1 > q0) {
+        dim3 grid((q1 - q0) / g.G, g.B * g.H);
+        size_t sm = (size_t)g.G * g.D * 5;
+        e = cudaFuncSetAttribute(kivi_key_flush_kernel,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        if (e != cudaSuccess) return e;
+        kivi_key_flush_kernel<<<grid, 128, sm, s>>>(g, sk, q0 / g.G);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = pack_pertoken(g, 1, g.vb, 0, sv, q0, q1, s);
+        if (e != cudaSuccess) return e;
+      }
+      const int ta = q1 > T0 ? q1 : T0;
+      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, ta, T1, 0, g.ring, s);
+      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, ta, T1, 0, g.ring, s);
+      return e;
+    }
+    case KVQ_FMT_KVARN: {
+      const int S = g.S, G = g.G;
+      const int se = T1 < S ? T1 : S;
+      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, T0, se, 0, S > 0 ? S : 1, s);
+      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, T0, se, 0, S > 0 ? S : 1, s);
+      if (e != cudaSuccess) return e;
+      const int n0 = kvarn_nblocks(T0, S, G), n1 = kvarn_nblocks(T1, S, G);
+      if (n1 > n0) {
+        const size_t sm = ((size_t)2 * G * g.D + 256 + 128 + 256) * sizeof(float);
+        const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));
+        e = cudaFuncSetAttribute(kvarn_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)sm);
+        if (e != cudaSuccess) return e;
+        TokSrc src[2] = {sk, sv};
+        for (int w = 0; w < 2; ++w) {
+          src[w].ring_plane = w ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
+          src[w].ring_off = S;
+          src[w].ring_rows = G;
+        }
+        // keys and values are separate launches (different sources)
+        for (int w = 0; w < 2; ++w) {
+          dim3 grid(n1 - n0, g.B * g.H, 1);
+          Geom gw = g;
+          if (w) {  // value launch: value planes and bit width in the key slots
+            gw.kb = g.vb;
+            gw.pl[KVQ_PLANE_K_CODES] = g.pl[KVQ_PLANE_V_CODES];
+            gw.pl[KVQ_PLANE_K_SCALE] = g.pl[KVQ_PLANE_V_SCALE];
+            gw.pl[KVQ_PLANE_K_ZERO] = g.pl[KVQ_PLANE_V_ZERO];
+            gw.pl[KVQ_PLANE_K_ROW] = g.pl[KVQ_PLANE_V_ROW];
+            gw.pl[KVQ_PLANE_K_COL] = g.pl[KVQ_PLANE_V_COL];
+          }
+          kvarn_block_kernel<<<grid, 256, sm, s>>>(gw, src[w], n0, inv_sqrt_d);
+          e = cudaGetLastError();
+          if (e != cudaSuccess) return e;
+        }
+      }
+      int ta = S + n1 * G;
+      if (ta < T0) ta = T0;
+      e = store_full(g, KVQ_PLANE_K_PEND, k, T0, L, ta, T1, S, G, s);
+      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_PEND, v, T0, L, ta, T1, S, G, s);
+      return e;
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace kvq

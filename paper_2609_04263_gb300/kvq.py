@@ -1,0 +1,162 @@
+"""ctypes binding of libkvq.so: the same entry points as include/kvq.h.
+
+Argument marshalling only.  Every step of the attention path runs in the
+library's CUDA kernels; PyTorch provides device memory and streams.  The
+library is loaded on first use and a missing build raises immediately.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libkvq.so")
+
+KVQ_OK, KVQ_ERR_ARG, KVQ_ERR_SHAPE, KVQ_ERR_CAPACITY, KVQ_ERR_UNSUPPORTED, \
+    KVQ_ERR_CUDA, KVQ_ERR_TIMEOUT = range(7)
+KVQ_FMT_FLOAT, KVQ_FMT_AFFINE, KVQ_FMT_SYMMETRIC, KVQ_FMT_KIVI, KVQ_FMT_KVARN = range(5)
+KVQ_F32, KVQ_BF16 = 0, 1
+
+PLANES = ["k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "k_full",
+          "v_full", "k_pend", "v_pend", "k_row", "k_col", "v_row", "v_col", "workspace"]
+NUM_PLANES = len(PLANES)
+
+c_int, c_float, c_void_p, c_size_t = ctypes.c_int, ctypes.c_float, ctypes.c_void_p, ctypes.c_size_t
+
+
+class KvqError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"kvq status {status}: {msg}")
+        self.status = status
+
+
+class kvq_cache_desc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "fmt", "key_bits", "value_bits", "group_size", "residual_tokens", "sink_tokens",
+        "norm_iters", "batch", "kv_heads", "q_heads", "head_dim", "max_tokens", "dtype")]
+
+
+class kvq_cache_planes(ctypes.Structure):
+    _fields_ = [("ptr", c_void_p * NUM_PLANES),
+                ("dims", (ctypes.c_int64 * 4) * NUM_PLANES),
+                ("elem_bytes", ctypes.c_int32 * NUM_PLANES),
+                ("tokens", ctypes.c_int32),
+                ("quantized_tokens", ctypes.c_int32)]
+
+
+_SIGS = {
+    "kvq_abi_version": (c_int, []),
+    "kvq_last_error": (ctypes.c_char_p, []),
+    "kvq_cache_bytes": (c_size_t, [ctypes.POINTER(kvq_cache_desc)]),
+    "kvq_create_cache": (c_int, [ctypes.POINTER(kvq_cache_desc), c_void_p, c_size_t,
+                                 ctypes.POINTER(c_void_p)]),
+    "kvq_destroy_cache": (c_int, [c_void_p]),
+    "kvq_reset_cache": (c_int, [c_void_p]),
+    "kvq_cache_tokens": (c_int, [c_void_p]),
+    "kvq_cache_view": (c_int, [c_void_p, ctypes.POINTER(kvq_cache_planes)]),
+    "kvq_project_lora": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p,
+                                 c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
+                                 c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
+                                 c_int, c_float, c_int, c_void_p, c_void_p, c_void_p,
+                                 c_void_p]),
+    "kvq_append_pack": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_void_p]),
+    "kvq_attend_prefill": (c_int, [c_void_p, c_void_p, c_int, c_int, c_float, c_void_p,
+                                   c_void_p]),
+    "kvq_attend_decode": (c_int, [c_void_p, c_void_p, c_int, c_float, c_void_p, c_void_p]),
+    "kvq_device_status": (c_int, [c_void_p, ctypes.POINTER(c_int)]),
+}
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "paper_2609_04263_gb300.build.build()")
+        so = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(so, name)
+            fn.restype, fn.argtypes = res, args
+        _lib = so
+    return _lib
+
+
+def _check(status: int) -> None:
+    if status != KVQ_OK:
+        raise KvqError(status, kvq_last_error())
+
+
+def kvq_last_error() -> str:
+    return lib().kvq_last_error().decode()
+
+
+def kvq_abi_version() -> int:
+    return lib().kvq_abi_version()
+
+
+def kvq_cache_bytes(desc: kvq_cache_desc) -> int:
+    n = lib().kvq_cache_bytes(ctypes.byref(desc))
+    if n == 0:
+        raise KvqError(KVQ_ERR_SHAPE, kvq_last_error())
+    return n
+
+
+def kvq_create_cache(desc: kvq_cache_desc, dev_buf: int, nbytes: int) -> int:
+    out = c_void_p()
+    _check(lib().kvq_create_cache(ctypes.byref(desc), c_void_p(dev_buf), nbytes,
+                                  ctypes.byref(out)))
+    return out.value
+
+
+def kvq_destroy_cache(handle: int) -> None:
+    _check(lib().kvq_destroy_cache(c_void_p(handle)))
+
+
+def kvq_reset_cache(handle: int) -> None:
+    _check(lib().kvq_reset_cache(c_void_p(handle)))
+
+
+def kvq_cache_tokens(handle: int) -> int:
+    return lib().kvq_cache_tokens(c_void_p(handle))
+
+
+def kvq_cache_view(handle: int) -> kvq_cache_planes:
+    out = kvq_cache_planes()
+    _check(lib().kvq_cache_view(c_void_p(handle), ctypes.byref(out)))
+    return out
+
+
+def kvq_project_lora(x, B, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,
+                     alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, rope_base, dtype,
+                     q, k, v, stream) -> None:
+    P = lambda t: c_void_p(t or 0)
+    _check(lib().kvq_project_lora(P(x), B, L, d_in, P(w_qkv), P(a_q), P(b_q), r_q, P(a_k),
+                                  P(b_k), r_k, P(a_v), P(b_v), r_v, alpha_over_r, n_q_heads,
+                                  n_kv_heads, head_dim, pos0, rope_base, dtype, P(q), P(k),
+                                  P(v), P(stream)))
+
+
+def kvq_append_pack(handle, k, v, L, stream) -> None:
+    _check(lib().kvq_append_pack(c_void_p(handle), c_void_p(k), c_void_p(v), L,
+                                 c_void_p(stream or 0)))
+
+
+def kvq_attend_prefill(handle, q, L, n_q_heads, softmax_scale, out, stream) -> None:
+    _check(lib().kvq_attend_prefill(c_void_p(handle), c_void_p(q), L, n_q_heads,
+                                    softmax_scale, c_void_p(out), c_void_p(stream or 0)))
+
+
+def kvq_attend_decode(handle, q, n_q_heads, softmax_scale, out, stream) -> None:
+    _check(lib().kvq_attend_decode(c_void_p(handle), c_void_p(q), n_q_heads, softmax_scale,
+                                   c_void_p(out), c_void_p(stream or 0)))
+
+
+def kvq_device_status(stream=0) -> int:
+    out = c_int(0)
+    st = lib().kvq_device_status(c_void_p(stream or 0), ctypes.byref(out))
+    if st not in (KVQ_OK, KVQ_ERR_TIMEOUT):
+        _check(st)
+    return out.value

@@ -142,17 +142,18 @@ def layer_weights(wl: Workload, layer: int, seed: int = 0, rank=None):
 
 
 def kv_states(shape, seed: int = 0, stream: int = 0,
-              channel_spread: float = 4.0) -> np.ndarray:
+              channel_spread: float = 2.0) -> np.ndarray:
     """Key/value-like tensors [B, H, L, D] for exercising the cache alone.
 
-    Each channel gets its own scale (log-uniform over `channel_spread`) and
-    offset, which gives the per-channel structure real keys have.
+    Each channel gets its own scale (log-uniform in [1/spread, spread]) and
+    offset (N(0, 0.25)), which gives the per-channel structure real keys have
+    at the unit scale of projected activations.
     """
     rng = np.random.default_rng([seed, 3, stream])
     D = shape[-1]
     crng = np.random.default_rng([seed, 4])
     scale = np.exp(crng.uniform(-math.log(channel_spread), math.log(channel_spread), D))
-    offset = crng.normal(0.0, 0.5, D)
+    offset = crng.normal(0.0, 0.25, D)
     x = rng.standard_normal(shape) * scale + offset
     return x.astype(np.float32)
 

@@ -1,0 +1,113 @@
+"""Shared helpers of the parity tests: cache construction on both sides and
+plane comparison restricted to live rows."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import kvq_oracle as O
+from paper_2609_04263_gb300 import synth
+
+ACT = {"bf16": torch.bfloat16, "f32": torch.float32}
+
+# small formats used across the parity tests
+FORMATS = {
+    "float": dict(fmt=O.FMT_FLOAT, key_bits=4, value_bits=4, group_size=32),
+    "affine4": dict(fmt=O.FMT_AFFINE, key_bits=4, value_bits=4, group_size=32),
+    "affine2": dict(fmt=O.FMT_AFFINE, key_bits=2, value_bits=2, group_size=32),
+    "affine8_g64": dict(fmt=O.FMT_AFFINE, key_bits=8, value_bits=8, group_size=64),
+    "affine4_g128": dict(fmt=O.FMT_AFFINE, key_bits=4, value_bits=2, group_size=128),
+    "sym2": dict(fmt=O.FMT_SYMMETRIC, key_bits=2, value_bits=2, group_size=32),
+    "sym4": dict(fmt=O.FMT_SYMMETRIC, key_bits=4, value_bits=4, group_size=32),
+    "kivi2": dict(fmt=O.FMT_KIVI, key_bits=2, value_bits=2, group_size=32,
+                  residual_tokens=128),
+    "kivi_r0": dict(fmt=O.FMT_KIVI, key_bits=2, value_bits=4, group_size=32,
+                    residual_tokens=0),
+    "kvarn": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=64,
+                  sink_tokens=128, norm_iters=8),
+    "kvarn_small": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=32,
+                        sink_tokens=40, norm_iters=8),
+}
+
+
+def oracle_cache(spec, B, H, D, Tmax, act):
+    kw = dict(spec)
+    fmt = kw.pop("fmt")
+    return O.OracleCache(fmt, batch=B, kv_heads=H, head_dim=D, max_tokens=Tmax, act=act, **kw)
+
+
+def gpu_cache(spec, B, H, Hq, D, Tmax, act):
+    from paper_2609_04263_gb300 import api
+    kw = dict(spec)
+    fmt = kw.pop("fmt")
+    desc = api.make_desc(fmt, kw.get("key_bits", 4), kw.get("value_bits", 4),
+                         kw.get("group_size", 32), B, H, Hq, D, Tmax, ACT[act],
+                         residual_tokens=kw.get("residual_tokens", 0),
+                         sink_tokens=kw.get("sink_tokens", 0),
+                         norm_iters=kw.get("norm_iters", 8))
+    return api.Cache(desc)
+
+
+def kv_pair(B, H, L, D, act, seed=0, stream=0, device="cuda"):
+    """Seeded k, v: torch tensors on the device and the same values as fp32
+    numpy arrays for the oracle."""
+    k = synth.kv_states((B, H, L, D), seed=seed, stream=2 * stream)
+    v = synth.kv_states((B, H, L, D), seed=seed + 1000, stream=2 * stream + 1)
+    kt = torch.from_numpy(k).to(ACT[act])
+    vt = torch.from_numpy(v).to(ACT[act])
+    return (kt.to(device), vt.to(device), kt.float().numpy(), vt.float().numpy())
+
+
+def live(name, arr, oc):
+    """Rows of a plane that hold live tokens (oc: the oracle cache state)."""
+    T, G = oc.T, oc.G
+    if name in ("k_row", "v_row"):
+        arr = arr.reshape(arr.shape[0], arr.shape[1], -1)
+    if oc.fmt == O.FMT_KIVI:
+        tq = O.kivi_quantized_prefix(T, oc.R, G)
+        if name.endswith("_full"):
+            ring = oc.R + G
+            return np.stack([arr[:, :, t % ring] for t in range(tq, T)], 2) if T > tq else arr[:, :, :0]
+        if name in ("k_scale", "k_zero"):
+            return arr[:, :, :tq // G]
+        return arr[:, :, :tq]
+    if oc.fmt == O.FMT_KVARN:
+        nb = O.kvarn_blocks(T, oc.S, G)
+        if name.endswith("_pend"):
+            ts = range(oc.S + nb * G, T)
+            return np.stack([arr[:, :, (t - oc.S) % G] for t in ts], 2) if len(ts) else arr[:, :, :0]
+        if name.endswith("_col"):
+            return arr[:, :, :nb]
+        if name.endswith("_full"):
+            return arr[:, :, :min(T, oc.S)]
+        return arr[:, :, :nb * G]
+    return arr[:, :, :T]
+
+
+def to_numpy_plane(t: torch.Tensor) -> np.ndarray:
+    if t.dtype == torch.bfloat16:
+        return t.float().cpu().numpy()
+    return t.cpu().numpy()
+
+
+def compare_planes(gc, oc):
+    """Bit-exact comparison of every oracle plane with the GPU plane."""
+    gp = gc.planes()
+    assert gp["_tokens"] == oc.T
+    for name, ref in oc.planes.items():
+        if ref.size == 0:
+            continue
+        assert name in gp, f"plane {name} missing on the GPU side"
+        got = to_numpy_plane(gp[name])
+        a, b = live(name, got, oc), live(name, ref, oc)
+        assert a.shape == b.shape, (name, a.shape, b.shape)
+        if a.dtype == np.float16:
+            same = np.array_equal(a.view(np.uint16), b.view(np.uint16))
+        elif a.dtype == np.float32:
+            same = np.array_equal(a.view(np.uint32), b.astype(np.float32).view(np.uint32))
+        else:
+            same = np.array_equal(a, b)
+        if not same:
+            diff = np.argwhere(a.view(np.uint8) != b.view(np.uint8)) if a.dtype != np.float32 \
+                else np.argwhere(a != b)
+            raise AssertionError(f"plane {name}: {len(diff)} mismatches, first at {diff[:3].tolist()}")

@@ -1,0 +1,126 @@
+"""The C-ABI library loads, exports every entry point include/kvq.h declares,
+and validates arguments on the host (no GPU needed: nothing here launches)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def kvq():
+    from paper_2609_04263_gb300 import build, kvq as K
+    build.build()
+    K.lib()
+    return K
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "kvq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvq_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(kvq):
+    names = _declared()
+    assert len(names) >= 12
+    so = ctypes.CDLL(kvq.LIB_PATH)
+    for n in names:
+        assert hasattr(so, n), f"{n} declared in kvq.h but not exported"
+
+
+def test_binding_names_match_header(kvq):
+    for n in _declared():
+        assert hasattr(kvq, n), f"binding lacks {n}"
+
+
+def test_abi_version(kvq):
+    assert kvq.kvq_abi_version() == 1
+
+
+def _desc(kvq, **kw):
+    base = dict(fmt=kvq.KVQ_FMT_AFFINE, key_bits=4, value_bits=4, group_size=32,
+                residual_tokens=0, sink_tokens=0, norm_iters=8, batch=4, kv_heads=4,
+                q_heads=32, head_dim=64, max_tokens=2304, dtype=kvq.KVQ_BF16)
+    base.update(kw)
+    return kvq.kvq_cache_desc(**base)
+
+
+def test_cache_bytes_accounts_for_every_plane(kvq):
+    d = _desc(kvq)
+    n = kvq.kvq_cache_bytes(d)
+    B, H, T, D = 4, 4, 2304, 64
+    codes = B * H * T * D * 4 // 8
+    meta = B * H * T * (D // 32) * 2
+    ws = B * 32 * 32 * (D + 2) * 4
+    assert n >= 2 * codes + 4 * meta + ws
+    assert n <= 2 * codes + 4 * meta + ws + 16 * 256
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(fmt=9), 1), (dict(dtype=7), 1), (dict(batch=0), 2),
+    (dict(q_heads=30), 2), (dict(head_dim=96), 4), (dict(key_bits=3), 4),
+    (dict(group_size=48), 2), (dict(group_size=128), 2),
+    (dict(fmt=4, group_size=128, head_dim=256), 4),
+])
+def test_descriptor_validation(kvq, kw, status):
+    d = _desc(kvq, **kw)
+    assert kvq.lib().kvq_cache_bytes(ctypes.byref(d)) == 0
+    assert kvq.kvq_last_error() != ""
+    with pytest.raises(kvq.KvqError) as ei:
+        kvq.kvq_create_cache(d, 1 << 20, 1 << 40)
+    assert ei.value.status == status
+
+
+def test_create_view_and_host_validation(kvq):
+    d = _desc(kvq, max_tokens=100)
+    n = kvq.kvq_cache_bytes(d)
+    fake = 1 << 32                         # never dereferenced on the host
+    with pytest.raises(kvq.KvqError) as ei:
+        kvq.kvq_create_cache(d, fake, n - 1)
+    assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+    with pytest.raises(kvq.KvqError):
+        kvq.kvq_create_cache(d, fake + 16, n)          # misaligned
+    h = kvq.kvq_create_cache(d, fake, n)
+    try:
+        assert kvq.kvq_cache_tokens(h) == 0
+        v = kvq.kvq_cache_view(h)
+        ptrs = [v.ptr[i] for i in range(kvq.NUM_PLANES) if v.ptr[i]]
+        assert all(fake <= p < fake + n and p % 256 == 0 for p in ptrs)
+        assert v.dims[0][2] == 100 and v.dims[0][3] == 32 and v.elem_bytes[0] == 1
+        # capacity and argument errors are caught before any launch
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_append_pack(h, 1 << 33, 1 << 33, 101, 0)
+        assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+        with pytest.raises(kvq.KvqError):
+            kvq.kvq_append_pack(h, 0, 0, 4, 0)
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_attend_decode(h, 1 << 33, 32, 0.125, 1 << 33, 0)
+        assert ei.value.status == kvq.KVQ_ERR_SHAPE        # nothing cached yet
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_attend_prefill(h, 1 << 33, 1, 16, 0.125, 1 << 33, 0)
+        assert ei.value.status == kvq.KVQ_ERR_SHAPE        # wrong head count
+        assert kvq.kvq_cache_tokens(h) == 0
+    finally:
+        kvq.kvq_destroy_cache(h)
+    assert kvq.kvq_cache_tokens(None) == -1
+
+
+def test_project_validation(kvq):
+    P = 1 << 33
+    cases = [
+        dict(d_in=100),            # bf16 needs d_in % 64 == 0
+        dict(head_dim=80),
+        dict(r_q=12),              # bf16 rank must be a multiple of 8
+        dict(r_q=80),
+        dict(heads=(30, 4)),
+        dict(dtype=5),
+    ]
+    for c in cases:
+        hq, hkv = c.get("heads", (32, 4))
+        with pytest.raises(kvq.KvqError):
+            kvq.kvq_project_lora(P, 1, 4, c.get("d_in", 2048), P, P, P, c.get("r_q", 16), P, P,
+                                 16, P, P, 16, 2.0, hq, hkv, c.get("head_dim", 64), 0, 1e4,
+                                 c.get("dtype", kvq.KVQ_BF16), P, P, P, 0)
