@@ -1,0 +1,555 @@
+"""Benchmark of the packed-cache attention step on GB300.
+
+One step is one pass of the whole path over one batch of the TinyLlama-shaped
+workload (22 layers, batch 4, hidden 2048, 32 query / 4 KV heads, head_dim 64,
+4-bit affine cache with groups of 32, rank-16 LoRA on Q, K and V): reset the
+caches, prefill 2048 tokens per sequence (LoRA Q/K/V projection with RoPE,
+quantize-and-pack append, causal prefill attention, per layer), then 256 decode
+steps (projection, append, split-K decode attention, per layer; one captured
+CUDA graph per decode step).  `value` is tokens processed per second
+(batch x (prefill + decode) tokens per step); the decode phase alone, pack
+bandwidth and projection TFLOP/s are reported beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl kvq|reference]
+
+--impl reference times the CPU oracle on the host cores over a bounded sample
+of the same workload.  Under torchrun each rank runs an independent replica
+(the path has no exchange step); rank 0 prints the JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2609_04263_gb300 import synth  # noqa: E402
+
+METRIC = ("packed-KV decode attention tokens/s and % HBM roofline; pack GB/s; "
+          "QKV TFLOP/s")
+WORKLOAD = "tinyllama_affine4"
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_PATH) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work per launch (numerators of the roofline)
+# ---------------------------------------------------------------------------
+def code_bytes_per_token(wl):
+    """Packed bytes one token adds per KV head (codes + fp16 metadata)."""
+    D, G = wl.head_dim, wl.group_size
+    meta = 2 if wl.fmt == synth.FMT_SYMMETRIC else 4
+    return D * (wl.key_bits + wl.value_bits) // 8 + 2 * (D // G) * meta
+
+
+def proj_flops(wl, M):
+    D = wl.head_dim
+    N = wl.n_out
+    douts = (wl.n_q_heads * D, wl.n_kv_heads * D, wl.n_kv_heads * D)
+    r = wl.rank
+    return 2 * M * wl.d_in * N + 2 * M * wl.d_in * 3 * r + 2 * M * r * sum(douts)
+
+
+def proj_bytes(wl, M):
+    """HBM bytes of a projection launch: weights, LoRA factors, x, outputs."""
+    D, r = wl.head_dim, wl.rank
+    w = wl.n_out * wl.d_in
+    lora = 3 * r * wl.d_in + r * wl.n_out
+    return 2 * (w + lora + M * wl.d_in + M * wl.n_out)
+
+
+def pack_bytes(wl, L):
+    B, H, D = wl.batch, wl.n_kv_heads, wl.head_dim
+    return B * H * L * (2 * D * 2 + code_bytes_per_token(wl))
+
+
+def decode_attn_bytes(wl, T):
+    B, H, Hq, D = wl.batch, wl.n_kv_heads, wl.n_q_heads, wl.head_dim
+    return B * H * T * code_bytes_per_token(wl) + 2 * B * Hq * D * 2
+
+
+def prefill_attn_flops(wl, L, T):
+    """Causal: query l (position T - L + l) sees T - L + l + 1 keys; QK^T and
+    PV each 2 D flops per visible key."""
+    B, Hq, D = wl.batch, wl.n_q_heads, wl.head_dim
+    visible = L * (T - L) + L * (L + 1) // 2
+    return 4 * B * Hq * D * visible
+
+
+# ---------------------------------------------------------------------------
+# the GPU path
+# ---------------------------------------------------------------------------
+class Runner:
+    def __init__(self, wl: synth.Workload, device: str):
+        from paper_2609_04263_gb300 import api
+        self.api, self.wl, self.dev = api, wl, device
+        dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+        self.dt = dt
+        B, P, Dn, D = wl.batch, wl.prefill, wl.decode, wl.head_dim
+        self.layers = []
+        for l in range(wl.layers):
+            w, lora = synth.layer_weights(wl, l)
+            self.layers.append((
+                torch.from_numpy(w).to(dt).to(device),
+                {p: tuple(torch.from_numpy(t).to(dt).to(device) for t in lora[p]) for p in "qkv"},
+            ))
+        desc = api.make_desc(wl.fmt, wl.key_bits, wl.value_bits, wl.group_size, B,
+                             wl.n_kv_heads, wl.n_q_heads, D, wl.max_tokens, dt,
+                             residual_tokens=wl.residual_tokens, sink_tokens=wl.sink_tokens,
+                             norm_iters=wl.norm_iters)
+        self.caches = [api.Cache(desc, device=device) for _ in range(wl.layers)]
+        self.cache_bytes = self.caches[0].nbytes
+        x_pre = synth.hidden_states((B, P, wl.d_in), wl.hidden, wl.outlier_frac, seed=0)
+        x_dec = synth.hidden_states((B, Dn, wl.d_in), wl.hidden, wl.outlier_frac, seed=0,
+                                    stream=1)
+        self.x_pre_host = torch.from_numpy(x_pre).to(dt).pin_memory()
+        self.x_dec_host = torch.from_numpy(
+            np.ascontiguousarray(x_dec.transpose(1, 0, 2)[:, :, None, :])).to(dt).pin_memory()
+        self.x_pre = self.x_pre_host.to(device)
+        self.x_dec = self.x_dec_host.to(device)         # [Dn, B, 1, d_in]
+        Hq, Hkv = wl.n_q_heads, wl.n_kv_heads
+        e = lambda *s: torch.empty(*s, dtype=dt, device=device)
+        self.pre = (e(B, Hq, P, D), e(B, Hkv, P, D), e(B, Hkv, P, D))
+        self.o_pre = e(B, Hq, P, D)
+        self.xs = e(B, 1, wl.d_in)
+        self.dec = (e(B, Hq, 1, D), e(B, Hkv, 1, D), e(B, Hkv, 1, D))
+        self.o_dec = e(B, Hq, 1, D)
+        self.graph = None
+        self.events = None
+
+    # one layer's calls ----------------------------------------------------
+    def _project(self, l, x, out):
+        w, lora = self.layers[l]
+        wl = self.wl
+        return self.api.project_lora(x, w, lora, wl.alpha_over_r, wl.n_q_heads, wl.n_kv_heads,
+                                     wl.head_dim, rope_base=wl.rope_base, out=out,
+                                     pos_cache=self.caches[l])
+
+    def reset(self):
+        for c in self.caches:
+            c.reset()
+
+    def prefill(self, timer=None):
+        for l, c in enumerate(self.caches):
+            if timer:
+                timer("project", 0)
+            q, k, v = self._project(l, self.x_pre, self.pre)
+            if timer:
+                timer("project", 1)
+                timer("append", 0)
+            c.append(k, v)
+            if timer:
+                timer("append", 1)
+                timer("attend_prefill", 0)
+            c.attend_prefill(q, out=self.o_pre)
+            if timer:
+                timer("attend_prefill", 1)
+
+    def decode_step_eager(self, timer=None):
+        for l, c in enumerate(self.caches):
+            if timer:
+                timer("project_decode", 0)
+            q, k, v = self._project(l, self.xs, self.dec)
+            if timer:
+                timer("project_decode", 1)
+                timer("append_decode", 0)
+            c.append(k, v)
+            if timer:
+                timer("append_decode", 1)
+                timer("attend_decode", 0)
+            c.attend_decode(q, out=self.o_dec)
+            if timer:
+                timer("attend_decode", 1)
+
+    def capture(self):
+        """Capture one decode step (all layers) in a CUDA graph."""
+        self.reset()
+        self.prefill()                       # the caches' device state is initialised
+        torch.cuda.synchronize()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            self.decode_step_eager()
+        torch.cuda.synchronize()
+        self.graph = g
+
+    def decode(self):
+        for s in range(self.wl.decode):
+            self.xs.copy_(self.x_dec[s])
+            self.graph.replay()
+
+    def job(self, phase_events=None):
+        self.reset()
+        if phase_events:
+            phase_events[0].record()
+        self.prefill()
+        if phase_events:
+            phase_events[1].record()
+        self.decode()
+        if phase_events:
+            phase_events[2].record()
+
+    def launches_per_step(self):
+        wl = self.wl
+        append = {synth.FMT_FLOAT: 1, synth.FMT_AFFINE: 1, synth.FMT_SYMMETRIC: 1,
+                  synth.FMT_KIVI: 3, synth.FMT_KVARN: 2}[wl.fmt]
+        prefill = wl.layers * (1 + append + 1)
+        decode = wl.decode * wl.layers * (1 + append + 2)
+        return prefill + decode
+
+
+class EventTimer:
+    """Per-call-class CUDA events on the current stream."""
+
+    def __init__(self):
+        self.open = {}
+        self.pairs = {}
+
+    def __call__(self, name, edge):
+        ev = torch.cuda.Event(enable_timing=True)
+        ev.record()
+        if edge == 0:
+            self.open[name] = ev
+        else:
+            self.pairs.setdefault(name, []).append((self.open.pop(name), ev))
+
+    def mean_ms(self):
+        torch.cuda.synchronize()
+        return {k: statistics.mean(a.elapsed_time(b) for a, b in v) for k, v in self.pairs.items()}
+
+    def total_ms(self):
+        torch.cuda.synchronize()
+        return {k: sum(a.elapsed_time(b) for a, b in v) for k, v in self.pairs.items()}
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.proc, self.path = index, None, None
+
+    def start(self):
+        out_dir = os.path.join(ROOT, "gpurun_out")
+        os.makedirs(out_dir, exist_ok=True)
+        self.path = os.path.join(out_dir, f"clocks_rank{self.index}.csv")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait(timeout=10)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def l2_flush(buf):
+    buf.fill_(1)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (the reported baseline and the reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, decode_steps=8, prefill=None):
+    """Time the CPU oracle on one layer of one sequence: a full-length prefill
+    (projection, pack, attention) and `decode_steps` decode steps.  Returns
+    (seconds, job-equivalent tokens/s) where the per-layer-per-sequence cost
+    is scaled to all layers and sequences and the decode steps to the full
+    count (decode steps cost the same to within the cache growth)."""
+    from oracle import kvq_oracle as O
+    P = wl.prefill if prefill is None else prefill
+    w, lora = synth.layer_weights(wl, 0)
+    act = wl.dtype
+    w = O.round_to(w, act)
+    lora = {p: tuple(O.round_to(t, act) for t in lora[p]) for p in "qkv"}
+    x_pre = O.round_to(synth.hidden_states((1, P, wl.d_in), wl.hidden, wl.outlier_frac), act)
+    x_dec = O.round_to(synth.hidden_states((1, decode_steps, wl.d_in), wl.hidden,
+                                           wl.outlier_frac, stream=1), act)
+    cache = O.OracleCache(wl.fmt, wl.key_bits, wl.value_bits, wl.group_size, 1, wl.n_kv_heads,
+                          wl.head_dim, P + decode_steps, act=act,
+                          residual_tokens=wl.residual_tokens, sink_tokens=wl.sink_tokens,
+                          norm_iters=wl.norm_iters)
+    args = (wl.alpha_over_r, wl.n_q_heads, wl.n_kv_heads, wl.head_dim)
+    t0 = time.perf_counter()
+    q, k, v = O.project_lora(x_pre, w, lora, *args, pos0=0, rope_base=wl.rope_base)
+    cache.append(O.round_to(k, act), O.round_to(v, act))
+    O.attend(cache, O.round_to(q, act))
+    t1 = time.perf_counter()
+    for s in range(decode_steps):
+        q, k, v = O.project_lora(x_dec[:, s:s + 1], w, lora, *args, pos0=P + s,
+                                 rope_base=wl.rope_base)
+        cache.append(O.round_to(k, act), O.round_to(v, act))
+        O.attend(cache, O.round_to(q, act))
+    t2 = time.perf_counter()
+    job_s = ((t1 - t0) + (t2 - t1) * wl.decode / decode_steps) * wl.layers * wl.batch
+    tokens = wl.batch * (wl.prefill + wl.decode)
+    return t2 - t0, tokens / job_s, (f"1 of {wl.layers} layers x 1 of {wl.batch} sequences: "
+                                     f"{P}-token prefill + {decode_steps} of {wl.decode} decode "
+                                     f"steps, scaled to the full job")
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ---------------------------------------------------------------------------
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(world, x):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64,
+                     device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    wl = synth.WORKLOADS[args.workload]
+    vals, secs = [], []
+    for _ in range(args.warmup):
+        oracle_sample(wl, decode_steps=2)
+    sample = None
+    for _ in range(args.steps):
+        s, v, sample = oracle_sample(wl, decode_steps=4)
+        vals.append(v)
+        secs.append(s)
+    value = statistics.mean(vals)
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * wl.batch * (wl.prefill + wl.decode) / value,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch,
+                       "prefill": wl.prefill, "decode": wl.decode},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="kvq", choices=["kvq", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py --impl kvq needs a CUDA GPU")
+    from paper_2609_04263_gb300 import build
+    if rank == 0 or world == 1:
+        build.build()
+    barrier(world)
+    device = f"cuda:{local}"
+    torch.cuda.set_device(device)
+    wl = synth.WORKLOADS[args.workload]
+    peaks, peak_kind = load_peaks()
+    run = Runner(wl, device)
+    run.capture()
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=device)
+
+    for _ in range(max(args.warmup, 3)):
+        run.job()
+    torch.cuda.synchronize()
+
+    # ---- timed region: K whole-job steps, L2 flushed between steps --------
+    clocks = ClockSampler(local)
+    clocks.start()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    for s in range(args.steps):
+        l2_flush(flush)
+        run.job(ev[s])
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    barrier(world)
+    clk = clocks.stop()
+    step_ms = [e[0].elapsed_time(e[2]) for e in ev]
+    pre_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    total_s = max_over_ranks(world, sum(step_ms) / 1000.0)
+    tokens_per_step = wl.batch * (wl.prefill + wl.decode)
+    value = world * tokens_per_step * args.steps / total_s
+    decode_tps = wl.batch * wl.decode / (statistics.mean(dec_ms) / 1000.0)
+
+    # ---- per-kernel durations: eager prefill and decode with events -------
+    timer = EventTimer()
+    run.reset()
+    run.prefill(timer)
+    for s in range(32):
+        run.xs.copy_(run.x_dec[s])
+        run.decode_step_eager(timer)
+    mean_ms = timer.mean_ms()
+    T_dec = wl.prefill + wl.decode // 2
+    work = {
+        "project": ("tensor", proj_flops(wl, wl.batch * wl.prefill), wl.layers),
+        "attend_prefill": ("tensor", prefill_attn_flops(wl, wl.prefill, wl.prefill), wl.layers),
+        "append": ("hbm", pack_bytes(wl, wl.prefill), wl.layers),
+        "project_decode": ("hbm", proj_bytes(wl, wl.batch), wl.layers * wl.decode),
+        "append_decode": ("hbm", pack_bytes(wl, 1), wl.layers * wl.decode),
+        "attend_decode": ("hbm", decode_attn_bytes(wl, T_dec), wl.layers * wl.decode),
+    }
+    share = {k: mean_ms[k] * work[k][2] for k in work}
+    dominant = max(share, key=share.get)
+    bound, amount, _ = work[dominant]
+    dur_s = mean_ms[dominant] / 1000.0
+    if bound == "tensor":
+        achieved = amount / dur_s / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        unit = "TFLOP/s"
+    else:
+        achieved = amount / dur_s / 1e9
+        peak = peaks["hbm_gbs"]
+        unit = "GB/s"
+    kernels = {}
+    for k, (b, amt, n) in work.items():
+        d = mean_ms[k] / 1000.0
+        rate = amt / d / (1e12 if b == "tensor" else 1e9)
+        pk = peaks["bf16_tflops_sustained"] if b == "tensor" else peaks["hbm_gbs"]
+        kernels[k] = {"mean_ms": round(mean_ms[k], 5), "launches_per_step": n,
+                      "ms_per_step": round(mean_ms[k] * n, 3),
+                      "achieved": round(rate, 3), "unit": "TFLOP/s" if b == "tensor" else "GB/s",
+                      "frac": round(rate / pk, 4)}
+
+    # ---- end to end through the public API with host buffers --------------
+    e2e_vals = []
+    o_host = torch.empty(run.o_pre.shape, dtype=run.dt, pin_memory=True)
+    od_host = torch.empty(run.o_dec.shape, dtype=run.dt, pin_memory=True)
+    h2d = run.x_pre_host.numel() * run.x_pre_host.element_size() + \
+        run.x_dec_host.numel() * run.x_dec_host.element_size()
+    d2h = o_host.numel() * o_host.element_size() + od_host.numel() * od_host.element_size()
+    for s in range(args.steps):
+        l2_flush(flush)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        run.x_pre.copy_(run.x_pre_host, non_blocking=True)
+        run.x_dec.copy_(run.x_dec_host, non_blocking=True)
+        run.job()
+        o_host.copy_(run.o_pre, non_blocking=True)
+        od_host.copy_(run.o_dec, non_blocking=True)
+        torch.cuda.synchronize()
+        e2e_vals.append(time.perf_counter() - t0)
+    e2e_s = max_over_ranks(world, statistics.mean(e2e_vals))
+    e2e_value = world * tokens_per_step / e2e_s
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        secs, cval, sample = oracle_sample(wl, decode_steps=8)
+        cpu = {"value": cval, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": sample + f" ({secs:.1f} s of CPU time)"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(args.warmup, 3),
+            "ms_per_step": statistics.mean(step_ms), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+            "config": {
+                "workload": wl.name, "layers": wl.layers, "batch": wl.batch,
+                "prefill": wl.prefill, "decode": wl.decode, "d_in": wl.d_in,
+                "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+                "cache": f"{synth.FMT_NAMES[wl.fmt]} K{wl.key_bits}V{wl.value_bits} G{wl.group_size}",
+                "lora_rank": wl.rank, "tokens_per_step": tokens_per_step,
+                "l2": "flushed (256 MiB write) between timed steps; job working set > L2",
+                "parallelism": f"replicas x{world}",
+            },
+            "phases": {"prefill_ms": statistics.mean(pre_ms), "decode_ms": statistics.mean(dec_ms),
+                       "decode_tokens_per_s": decode_tps,
+                       "pack_gbs": kernels["append"]["achieved"],
+                       "qkv_tflops": kernels["project"]["achieved"]},
+            "roofline": {"bound": bound, "kernel": dominant, "achieved": round(achieved, 3),
+                         "peak": peak, "unit": unit, "frac": round(achieved / peak, 4),
+                         "peak_source": f"{peak_kind} "
+                                        f"({'bf16_tflops_sustained' if bound == 'tensor' else 'hbm_gbs'})",
+                         "traffic": None},
+            "kernels": kernels,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": run.launches_per_step() * args.steps,
+            "clocks": clk,
+            "wall_s_timed": t_wall,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -128,18 +128,31 @@ size_t kvq_cache_bytes(const kvq_cache_desc* desc);
 
 /* Bind a cache to `dev_buf` (caller-owned, >= kvq_cache_bytes, 256-byte
  * aligned).  Allocates only the host-side handle; the buffer contents need no
- * initialisation.  The cache starts empty (T = 0). */
+ * initialisation (the first launching call zeroes the cache's 256-byte device
+ * state block on its stream).  The cache starts empty (T = 0).
+ *
+ * The token count T lives in device memory and kernels read it there, so a
+ * sequence of calls can be captured into a CUDA graph and replayed: every
+ * replayed append advances T on the device.  The host keeps a mirror for
+ * argument checks; after replays, kvq_cache_sync() refreshes it. */
 kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t bytes,
                             kvq_cache** out);
 
 /* Free the host handle.  The device buffer stays the caller's. */
 kvq_status kvq_destroy_cache(kvq_cache* cache);
 
-/* Forget every stored token (host bookkeeping only; nothing is launched). */
+/* Forget every stored token.  Nothing is launched here: the device state is
+ * zeroed, on the caller's stream, by the next launching call. */
 kvq_status kvq_reset_cache(kvq_cache* cache);
 
-/* Tokens stored per sequence, or -1 for a NULL cache. */
+/* Tokens stored per sequence according to the host mirror, -1 for NULL. */
 int kvq_cache_tokens(const kvq_cache* cache);
+
+/* Read the device token count into the host mirror (synchronises `stream`).
+ * Returns KVQ_ERR_CAPACITY (and clears the flag) if a replayed append was
+ * refused on the device because it would exceed max_tokens; a refused
+ * append writes nothing and leaves T unchanged. */
+kvq_status kvq_cache_sync(kvq_cache* cache, void* stream);
 
 /* Device pointers and shapes of every plane (for tests and export). */
 kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out);
@@ -156,22 +169,27 @@ kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out);
  *   out     q [B][Hq][L][D], k and v [B][Hkv][L][D]   (head-major)
  *
  *   y_p = x W_p^T + alpha_over_r * (x A_p^T) B_p^T, then rotate-half RoPE on
- *   q and k at positions pos0 + l with frequencies rope_base^(-2i/D)
- *   (rope_base = 0 disables RoPE).  r_p <= 64, multiple of 8 for KVQ_BF16.
+ *   q and k at positions P + pos0 + l with frequencies rope_base^(-2i/D)
+ *   (rope_base = 0 disables RoPE), where P = 0 if pos_cache is NULL, else the
+ *   token count of pos_cache read on the device when the kernel runs (the
+ *   usual choice: new tokens continue the cached sequence, and a captured
+ *   decode step stays correct on replay).  r_p <= 64, multiple of 8 for
+ *   KVQ_BF16.  d_in must be a multiple of 64 for KVQ_BF16.
  */
 kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w_qkv,
                             const void* a_q, const void* b_q, int r_q,
                             const void* a_k, const void* b_k, int r_k,
                             const void* a_v, const void* b_v, int r_v,
                             float alpha_over_r, int n_q_heads, int n_kv_heads,
-                            int head_dim, int pos0, float rope_base, int dtype,
-                            void* q, void* k, void* v, void* stream);
+                            int head_dim, int pos0, kvq_cache* pos_cache, float rope_base,
+                            int dtype, void* q, void* k, void* v, void* stream);
 
 /*
  * Append L new tokens per sequence: k, v [B][Hkv][L][D] (activation dtype).
  * Codes them per the cache format (Section 3.1) into the packed planes.  The
  * cache after T tokens is the same whether they arrive in one call or in
- * chunks.  KVQ_ERR_CAPACITY if T + L > max_tokens.
+ * chunks.  KVQ_ERR_CAPACITY if T + L > max_tokens (host mirror); the kernels
+ * check the device count again and refuse an overflowing replayed append.
  */
 kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L,
                            void* stream);

@@ -59,6 +59,11 @@ class Cache:
     def reset(self) -> None:
         kvq.kvq_reset_cache(self.handle)
 
+    def sync(self) -> int:
+        """Refresh the host token count from the device (after graph replays)."""
+        kvq.kvq_cache_sync(self.handle, _stream())
+        return self.tokens
+
     def append(self, k: torch.Tensor, v: torch.Tensor) -> None:
         kvq.kvq_append_pack(self.handle, _ptr(k), _ptr(v), k.shape[2], _stream())
 
@@ -99,10 +104,11 @@ class Cache:
 
 
 def project_lora(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0=0,
-                 rope_base=0.0, out=None):
+                 rope_base=0.0, out=None, pos_cache: "Cache | None" = None):
     """q [B,Hq,L,D], k, v [B,Hkv,L,D] = RoPE(x W'^T) with W' = W + (alpha/r) B A.
 
     lora: dict p -> (A [r, d_in], B [d_out, r]) or None for p in 'qkv'.
+    Positions are pos0 + l, plus pos_cache's device token count if given.
     """
     B, L, d_in = x.shape
     D = head_dim
@@ -118,6 +124,8 @@ def project_lora(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, 
         else:
             args += [_ptr(ab[0]), _ptr(ab[1]), ab[0].shape[0]]
     kvq.kvq_project_lora(_ptr(x), B, L, d_in, _ptr(w_qkv), *args, alpha_over_r, n_q_heads,
-                         n_kv_heads, head_dim, pos0, rope_base, _DT[x.dtype], _ptr(out[0]),
+                         n_kv_heads, head_dim, pos0,
+                         pos_cache.handle if pos_cache is not None else None, rope_base,
+                         _DT[x.dtype], _ptr(out[0]),
                          _ptr(out[1]), _ptr(out[2]), _stream())
     return out

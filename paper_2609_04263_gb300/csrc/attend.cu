@@ -120,9 +120,10 @@ __device__ void dequant_tile(const Geom& g, int which, int b, int h, int t0, int
 // [ts, te).  Shared memory holds the K/V tiles, q, scores and accumulators.
 // decode: writes (m, l, o) partials to the workspace, else the output.
 __global__ void __launch_bounds__(kThreads)
-attend_generic_kernel(Geom g, int T, const void* q, int L, float scale, void* out,
+attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
                       int nq, int splits, int decode, float inv_sqrt_d) {
   extern __shared__ float sm[];
+  const int T = cache_tokens(g);
   const int D = g.D, grp = g.Hq / g.H;
   const int rows = grp * nq;
   const int ldk = D + 1;
@@ -143,11 +144,7 @@ attend_generic_kernel(Geom g, int T, const void* q, int L, float scale, void* ou
   const int pos_last = pos_first + nql - 1;
   // tokens of this split
   int ts = 0, te = pos_last + 1;
-  if (decode) {
-    const int per = (T + splits - 1) / splits;
-    ts = split * per;
-    te = min(T, ts + per);
-  }
+  if (decode) split_range(T, splits, split, kTile, &ts, &te);
   for (int i = threadIdx.x; i < rows * D; i += blockDim.x) {
     const int r = i / D, d = i % D;
     const int hl = r / nq, qi = r % nq;
@@ -256,23 +253,21 @@ __global__ void combine_kernel(Geom g, int splits, void* out) {
 
 }  // namespace
 
-int decode_splits(const Geom& g, int T) {
+int decode_splits(const Geom& g) {
   const int bh = g.B * g.H;
   int s = (2 * num_sms() + bh - 1) / bh;
-  const int by_len = (T + kTile - 1) / kTile;
-  if (s > by_len) s = by_len;
   if (s > kMaxSplits) s = kMaxSplits;
   return s < 1 ? 1 : s;
 }
 
-cudaError_t launch_attend(const Geom& g, int T, const void* q, int L, float scale, void* out,
+cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
                           bool decode, cudaStream_t s) {
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));
   int nq, splits;
   if (decode) {
     nq = 1;
-    splits = decode_splits(g, T);
+    splits = g.splits;
   } else {
     int rows = 8192 / g.D;
     if (rows > 128) rows = 128;
@@ -288,7 +283,7 @@ cudaError_t launch_attend(const Geom& g, int T, const void* q, int L, float scal
   if (e != cudaSuccess) return e;
   const int nqt = (L + nq - 1) / nq;
   dim3 grid(nqt * splits, g.H, g.B);
-  attend_generic_kernel<<<grid, kThreads, sm, s>>>(g, T, q, L, scale, out, nq, splits,
+  attend_generic_kernel<<<grid, kThreads, sm, s>>>(g, q, L, scale, out, nq, splits,
                                                    decode ? 1 : 0, inv_sqrt_d);
   e = cudaGetLastError();
   if (e != cudaSuccess || !decode) return e;

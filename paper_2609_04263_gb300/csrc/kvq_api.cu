@@ -15,7 +15,8 @@ struct kvq_cache {
   Geom g;
   char* base;
   size_t bytes;
-  int T;
+  int T;            // host mirror of the device token count
+  bool need_init;   // device state not yet zeroed since create/reset
 };
 
 namespace {
@@ -159,7 +160,9 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
       break;
     }
   }
-  size_t total = 0;
+  g->splits = decode_splits(*g);
+  size_t total = sizeof(CacheState);   // device state block at offset 0
+  static_assert(sizeof(CacheState) == 256, "state block is 256 bytes");
   for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
     off[i] = 0;
     if (i == KVQ_PLANE_WORKSPACE) continue;
@@ -247,6 +250,8 @@ kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t by
   c->base = static_cast<char*>(dev_buf);
   c->bytes = bytes;
   c->T = 0;
+  c->need_init = true;
+  c->g.state = reinterpret_cast<CacheState*>(c->base);
   for (int i = 0; i < KVQ_NUM_PLANES; ++i)
     c->g.pl[i].p = c->g.pl[i].rows ? c->base + off[i] : nullptr;
   *out = c;
@@ -263,6 +268,33 @@ kvq_status kvq_destroy_cache(kvq_cache* cache) {
 kvq_status kvq_reset_cache(kvq_cache* cache) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
   cache->T = 0;
+  cache->need_init = true;
+  return KVQ_OK;
+}
+
+// Zero the device state before the first launch after create/reset
+// (stream-ordered, so it can be captured with the calls that follow).
+static cudaError_t ensure_init(kvq_cache* c, cudaStream_t s) {
+  if (!c->need_init) return cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(c->g.state, 0, sizeof(CacheState), s);
+  if (e == cudaSuccess) c->need_init = false;
+  return e;
+}
+
+kvq_status kvq_cache_sync(kvq_cache* cache, void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = ensure_init(cache, s);
+  CacheState st;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&st, cache->g.state, 3 * sizeof(int32_t),
+                                            cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && st.error)
+    e = cudaMemsetAsync(&cache->g.state->error, 0, sizeof(int32_t), s);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_cache_sync");
+  cache->T = st.tokens;
+  if (st.error & kErrCapacity)
+    return fail(KVQ_ERR_CAPACITY, "a device-side append was refused: capacity exceeded");
   return KVQ_OK;
 }
 
@@ -299,7 +331,8 @@ kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L
   if ((int64_t)cache->T + L > cache->g.Tmax)
     return fail(KVQ_ERR_CAPACITY, "append of %d tokens to %d exceeds max_tokens %d", L,
                 cache->T, cache->g.Tmax);
-  cudaError_t e = launch_append(cache->g, cache->T, L, k, v, (cudaStream_t)stream);
+  cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
+  if (e == cudaSuccess) e = launch_append(cache->g, L, k, v, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_append_pack launch");
   cache->T += L;
   return KVQ_OK;
@@ -317,8 +350,8 @@ static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_
     return fail(KVQ_ERR_SHAPE, "%d queries but only %d cached tokens (append first)", L,
                 cache->T);
   if (!(scale > 0.f) || scale != scale) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
-  cudaError_t e = launch_attend(cache->g, cache->T, q, L, scale, out, decode,
-                                (cudaStream_t)stream);
+  cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
+  if (e == cudaSuccess) e = launch_attend(cache->g, q, L, scale, out, decode, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_attend launch");
   return KVQ_OK;
 }
@@ -338,8 +371,8 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
                             const void* a_k, const void* b_k, int r_k,
                             const void* a_v, const void* b_v, int r_v,
                             float alpha_over_r, int n_q_heads, int n_kv_heads,
-                            int head_dim, int pos0, float rope_base, int dtype,
-                            void* q, void* k, void* v, void* stream) {
+                            int head_dim, int pos0, kvq_cache* pos_cache, float rope_base,
+                            int dtype, void* q, void* k, void* v, void* stream) {
   if (dtype != KVQ_F32 && dtype != KVQ_BF16) return fail(KVQ_ERR_ARG, "unknown dtype %d", dtype);
   if (B < 0 || L < 0 || d_in <= 0) return fail(KVQ_ERR_SHAPE, "bad B/L/d_in");
   if (n_q_heads <= 0 || n_kv_heads <= 0 || n_q_heads % n_kv_heads)
@@ -368,9 +401,15 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
   void* out[3] = {q, k, v};
   int* err = device_error_word();
   if (!err) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
+  const int* pos_dev = nullptr;
+  if (pos_cache) {
+    cudaError_t e0 = ensure_init(pos_cache, (cudaStream_t)stream);
+    if (e0 != cudaSuccess) return cuda_fail(e0, "kvq_project_lora");
+    pos_dev = &pos_cache->g.state->tokens;
+  }
   cudaError_t e = launch_project(x, B, L, d_in, w_qkv, a, bm, r, alpha_over_r, n_q_heads,
-                                 n_kv_heads, head_dim, pos0, rope_base, dtype, out, err,
-                                 (cudaStream_t)stream);
+                                 n_kv_heads, head_dim, pos0, pos_dev, rope_base, dtype, out,
+                                 err, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora launch");
   return KVQ_OK;
 }

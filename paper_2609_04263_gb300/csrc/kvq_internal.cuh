@@ -22,11 +22,27 @@ struct Plane {
   int32_t elem;
 };
 
+// Device-resident state of a cache (first 256 bytes of its buffer).
+// tokens: T, the number of stored tokens per sequence; kernels read it, so
+// launches do not bake it in and a captured decode step can be replayed.
+// done: arrival counter of the last kernel of an append (the last CTA to
+// arrive advances `tokens`).  error: bit flags set by kernels that refuse
+// work (see kErr*).
+struct CacheState {
+  int32_t tokens;
+  uint32_t done;
+  int32_t error;
+  int32_t pad[61];
+};
+constexpr int kErrCapacity = 1;   // an append would exceed max_tokens
+
 // Everything a kernel needs to address a cache.  Passed by value.
 struct Geom {
   int32_t fmt, kb, vb, G, R, S, iters;
   int32_t B, H, Hq, D, Tmax, act;
   int32_t ring;          // KIVI: R + G residual slots
+  int32_t splits;        // decode split-K width (fixed per cache)
+  CacheState* state;
   Plane pl[KVQ_NUM_PLANES];
 };
 
@@ -66,18 +82,61 @@ __device__ __forceinline__ void st_act(void* p, int64_t i, float v, int act) {
 
 // Host-side launchers (each defined in the translation unit of its kernels).
 // They return cudaGetLastError() of their launches.
-cudaError_t launch_append(const Geom& g, int T0, int L, const void* k, const void* v,
-                          cudaStream_t s);
-cudaError_t launch_attend(const Geom& g, int T, const void* q, int L, float scale,
-                          void* out, bool decode, cudaStream_t s);
+// All launchers read the token count from g.state on the device.
+cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cudaStream_t s);
+cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
+                          bool decode, cudaStream_t s);
+// pos_dev: if non-NULL, positions start at *pos_dev + pos0 (a cache's token
+// count read on the device), else at pos0.
 cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const void* const a[3], const void* const bm[3], const int r[3],
                            float alpha_over_r, int Hq, int Hkv, int D, int pos0,
-                           float rope_base, int act, void* const out[3], int* err,
-                           cudaStream_t s);
+                           const int* pos_dev, float rope_base, int act,
+                           void* const out[3], int* err, cudaStream_t s);
 
-// Number of decode splits the attention launcher uses for a cache state.
-int decode_splits(const Geom& g, int T);
+// Decode split-K width for a cache geometry (fixed, independent of T).
+int decode_splits(const Geom& g);
+
+// Token range of split `s` of `splits` over T tokens (tiles of `tile`).
+__host__ __device__ inline void split_range(int T, int splits, int s, int tile, int* ts,
+                                            int* te) {
+  int per = (T + splits - 1) / splits;
+  per = (per + tile - 1) / tile * tile;
+  *ts = s * per;
+  *te = min(T, *ts + per);
+}
+
+// Token count at the start of an append of L tokens; sets the capacity
+// error bit (and the kernels skip all work) if the append would overflow.
+__device__ __forceinline__ int append_begin(const Geom& g, int L, bool* ok) {
+  const int T0 = *reinterpret_cast<volatile int32_t*>(&g.state->tokens);
+  *ok = T0 >= 0 && (int64_t)T0 + L <= g.Tmax;
+  if (!*ok && threadIdx.x == 0 && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0)
+    atomicOr(&g.state->error, kErrCapacity);
+  return T0;
+}
+
+// Called by every CTA of the final kernel of an append after it has read the
+// token count: the last CTA to arrive advances it by L (unless the append
+// was refused).
+__device__ __forceinline__ void append_arrive(CacheState* st, int T0, int L, bool ok) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned total = gridDim.x * gridDim.y * gridDim.z;
+    const unsigned prev = atomicAdd(&st->done, 1u);
+    if (prev == total - 1) {
+      if (ok) st->tokens = T0 + L;
+      st->done = 0;
+      __threadfence();
+    }
+  }
+}
+
+// Tokens stored, as read by attention kernels.
+__device__ __forceinline__ int cache_tokens(const Geom& g) {
+  return *reinterpret_cast<volatile int32_t*>(&g.state->tokens);
+}
 
 // Device address of the library's error word (set up once per device).
 int* device_error_word();

@@ -74,105 +74,159 @@ __device__ __forceinline__ int sym_code(float x, float s, int bits) {
 // Per-token grouped coding: AFFINE / SYMMETRIC keys and values, KIVI values.
 // A group of G elements is held by G/8 consecutive lanes, 8 elements each;
 // min/max (or absmax) is a butterfly over those lanes; each lane packs its 8
-// codes LSB-first into one 16/32/64-bit store.
+// codes LSB-first into one 16/32/64-bit store.  blockIdx.y selects keys (0)
+// or values (1).  kivi = 1: code the values of the KIVI blocks that this
+// append completes (tokens [q0, q1), read from the residual ring or the
+// input); else code the new tokens [T0, T0 + L).  max_tok bounds the token
+// count for the grid-stride loop.
 // ---------------------------------------------------------------------------
-__global__ void pack_pertoken_kernel(Geom g, int which, int bits, int sym, TokSrc src,
-                                     int t_begin, int t_end) {
-  const int lpg = g.G / 8;                 // lanes per group
-  const int gpw = 32 / lpg;                // groups per warp pass
-  const int lane = threadIdx.x & 31;
-  const int sub = lane / lpg, li = lane % lpg;
-  const int groups_per_tok = g.D / g.G;
-  const int64_t ntok = (int64_t)(t_end - t_begin);
-  const int64_t units = (int64_t)g.B * g.H * ntok * groups_per_tok;
-  const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
-  const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
-  const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t base = warp * gpw; base < units; base += nwarps * gpw) {
-    const int64_t u = base + sub;
-    const bool live = u < units;
-    const int64_t uu = live ? u : units - 1;
-    const int grp = (int)(uu % groups_per_tok);
-    int64_t rest = uu / groups_per_tok;
-    const int t = t_begin + (int)(rest % ntok);
-    rest /= ntok;
-    const int h = (int)(rest % g.H);
-    const int b = (int)(rest / g.H);
-    const void* sb;
-    const int64_t e = tok_elem(g, src, b, h, t, &sb) + grp * g.G + li * 8;
-    float v[8];
-    load8(sb, e, g.act, v);
-    float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
+__global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
+                                     int final_kernel) {
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
+  const int which = kivi ? 1 : blockIdx.y;
+  int t_begin = T0, t_end = T0 + L;
+  if (kivi) {
+    t_begin = kivi_tq(T0, g.R, g.G);
+    t_end = kivi_tq(T0 + L, g.R, g.G);
+  }
+  if (ok && t_end > t_begin) {
+    TokSrc src = which ? sv : sk;
+    src.T0 = T0;
+    const int bits = which ? g.vb : g.kb;
+    const int lpg = g.G / 8;                 // lanes per group
+    const int gpw = 32 / lpg;                // groups per warp pass
+    const int lane = threadIdx.x & 31;
+    const int sub = lane / lpg, li = lane % lpg;
+    const int groups_per_tok = g.D / g.G;
+    const int64_t ntok = (int64_t)(t_end - t_begin);
+    const int64_t units = (int64_t)g.B * g.H * ntok * groups_per_tok;
+    const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+    const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+    const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t base = warp * gpw; base < units; base += nwarps * gpw) {
+      const int64_t u = base + sub;
+      const bool live = u < units;
+      const int64_t uu = live ? u : units - 1;
+      const int grp = (int)(uu % groups_per_tok);
+      int64_t rest = uu / groups_per_tok;
+      const int t = t_begin + (int)(rest % ntok);
+      rest /= ntok;
+      const int h = (int)(rest % g.H);
+      const int b = (int)(rest / g.H);
+      const void* sb;
+      const int64_t e = tok_elem(g, src, b, h, t, &sb) + grp * g.G + li * 8;
+      float v[8];
+      load8(sb, e, g.act, v);
+      float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
 #pragma unroll
-    for (int i = 1; i < 8; ++i) {
-      if (sym) hi = fmaxf(hi, fabsf(v[i]));
-      else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
-    }
-    for (int off = lpg / 2; off > 0; off >>= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
-    }
-    float s;
-    uint64_t word = 0;
-    if (sym) {
-      s = sym_scale(hi, bits);
+      for (int i = 1; i < 8; ++i) {
+        if (sym) hi = fmaxf(hi, fabsf(v[i]));
+        else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
+      }
+      for (int off = lpg / 2; off > 0; off >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
+      }
+      float s;
+      uint64_t word = 0;
+      if (sym) {
+        s = sym_scale(hi, bits);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) word |= (uint64_t)sym_code(v[i], s, bits) << (i * bits);
-    } else {
-      s = affine_scale(lo, hi, bits);
+        for (int i = 0; i < 8; ++i) word |= (uint64_t)sym_code(v[i], s, bits) << (i * bits);
+      } else {
+        s = affine_scale(lo, hi, bits);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) word |= (uint64_t)affine_code(v[i], lo, s, bits) << (i * bits);
-    }
-    if (!live) continue;
-    uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
-    const int byte0 = (grp * g.G + li * 8) * bits / 8;
-    if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
-    else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
-    else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
-    if (li == 0) {
-      *plane_ptr<__half>(g, scale_plane, b, h, t, grp) = __float2half_rn(s);
-      if (!sym) *plane_ptr<__half>(g, zero_plane, b, h, t, grp) = __float2half_rn(lo + 0.0f);
+        for (int i = 0; i < 8; ++i) word |= (uint64_t)affine_code(v[i], lo, s, bits) << (i * bits);
+      }
+      if (!live) continue;
+      uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
+      const int byte0 = (grp * g.G + li * 8) * bits / 8;
+      if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
+      else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
+      else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
+      if (li == 0) {
+        *plane_ptr<__half>(g, scale_plane, b, h, t, grp) = __float2half_rn(s);
+        if (!sym) *plane_ptr<__half>(g, zero_plane, b, h, t, grp) = __float2half_rn(lo + 0.0f);
+      }
     }
   }
+  if (final_kernel) append_arrive(g.state, T0, L, ok);
 }
 
 // ---------------------------------------------------------------------------
-// Copy new tokens into a full-precision plane at slot (t - off) mod rows:
-// FLOAT cache, KIVI residual ring, KVarN sinks and staging ring.
+// Copy new tokens into the full-precision planes (blockIdx.y: 0 keys, 1
+// values): FLOAT cache (slot t), KIVI residual ring (tokens t >= q1, slot
+// t mod (R + G)), KVarN sinks (t < S, slot t) and staging ring (t >= S + n1 G,
+// slot (t - S) mod G).  Always the final kernel of an append.
 // ---------------------------------------------------------------------------
-__global__ void store_full_kernel(Geom g, int plane, const void* x, int T0, int L,
-                                  int t_begin, int t_end, int off, int rows) {
-  const int es = g.act == KVQ_BF16 ? 2 : 4;
-  const int vec_per_tok = g.D * es / 16;
-  const int64_t ntok = t_end - t_begin;
-  const int64_t total = (int64_t)g.B * g.H * ntok * vec_per_tok;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int vi = (int)(i % vec_per_tok);
-    int64_t rest = i / vec_per_tok;
-    const int t = t_begin + (int)(rest % ntok);
-    rest /= ntok;
-    const int h = (int)(rest % g.H), b = (int)(rest / g.H);
-    const uint4* src = reinterpret_cast<const uint4*>(
-        reinterpret_cast<const char*>(x) + ((((int64_t)b * g.H + h) * L + (t - T0)) * g.D) * es);
-    const Plane& pl = g.pl[plane];
-    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<char*>(pl.p) +
-                                          plane_index(pl, b, h, g.H, (t - off) % rows, 0) * es);
-    dst[vi] = src[vi];
+__global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
+  const int T1 = T0 + L;
+  if (ok) {
+    const int which = blockIdx.y;
+    const void* x = which ? v : k;
+    const int es = g.act == KVQ_BF16 ? 2 : 4;
+    const int vec_per_tok = g.D * es / 16;
+    const int64_t total = (int64_t)g.B * g.H * L * vec_per_tok;
+    int lo = T0;        // first token that goes to a full-precision plane
+    if (g.fmt == KVQ_FMT_KIVI) lo = max(T0, kivi_tq(T1, g.R, g.G));
+    const int pend_lo = g.S + kvarn_nblocks(T1, g.S, g.G) * g.G;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+      const int vi = (int)(i % vec_per_tok);
+      int64_t rest = i / vec_per_tok;
+      const int t = T0 + (int)(rest % L);
+      rest /= L;
+      const int h = (int)(rest % g.H), b = (int)(rest / g.H);
+      int plane, slot;
+      if (g.fmt == KVQ_FMT_FLOAT) {
+        plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+        slot = t;
+      } else if (g.fmt == KVQ_FMT_KIVI) {
+        if (t < lo) continue;
+        plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+        slot = t % g.ring;
+      } else {  // KVARN
+        if (t < g.S) {
+          plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+          slot = t;
+        } else if (t >= pend_lo) {
+          plane = which ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
+          slot = (t - g.S) % g.G;
+        } else {
+          continue;
+        }
+      }
+      const uint4* src = reinterpret_cast<const uint4*>(
+          reinterpret_cast<const char*>(x) + ((((int64_t)b * g.H + h) * L + (t - T0)) * g.D) * es);
+      const Plane& pl = g.pl[plane];
+      uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<char*>(pl.p) +
+                                            plane_index(pl, b, h, g.H, slot, 0) * es);
+      dst[vi] = src[vi];
+    }
   }
+  append_arrive(g.state, T0, L, ok);
 }
 
 // ---------------------------------------------------------------------------
-// KIVI keys: one group per (32-token block, channel).  One CTA per block.
+// KIVI keys: one group per (G-token block, channel).  One CTA per block that
+// this append completes (grid sized for the most an append of L can flush).
 // ---------------------------------------------------------------------------
-__global__ void kivi_key_flush_kernel(Geom g, TokSrc src, int blk_begin) {
+__global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
   extern __shared__ float smem[];
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
   const int G = g.G, D = g.D, bits = g.kb;
+  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + L, g.R, G);
+  const int blk = q0 / G + blockIdx.x;
+  if (!ok || blk >= q1 / G) return;
+  src.T0 = T0;
   float* xs = smem;                                   // [G][D]
   uint8_t* cs = reinterpret_cast<uint8_t*>(xs + G * D); // [G][D]
-  const int blk = blk_begin + blockIdx.x;
   const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
   const int t0 = blk * G;
   for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
@@ -205,20 +259,26 @@ __global__ void kivi_key_flush_kernel(Geom g, TokSrc src, int blk_begin) {
 
 // ---------------------------------------------------------------------------
 // KVarN block: normalised Hadamard on D, dual-axis variance normalisation,
-// grouped affine along D.  One CTA per (block, b*h); keys and values are
-// separate launches (the value launch gets the value planes in the key
-// slots).  Sums follow the stride-halving pairwise tree in fp32.
+// grouped affine along D.  One CTA per (block this append completes, b*h,
+// k|v).  Sums follow the stride-halving pairwise tree in fp32.
 // ---------------------------------------------------------------------------
-__global__ void kvarn_block_kernel(Geom g, TokSrc src, int blk_begin, float inv_sqrt_d) {
+__global__ void kvarn_block_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
   extern __shared__ float smem[];
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
   const int G = g.G, D = g.D;
-  const int bits = g.kb;   // the host passes value planes in the key slots
+  const int n0 = kvarn_nblocks(T0, g.S, G), n1 = kvarn_nblocks(T0 + L, g.S, G);
+  const int blk = n0 + blockIdx.x;
+  if (!ok || blk >= n1) return;
+  const int which = blockIdx.z;
+  TokSrc src = which ? sv : sk;
+  src.T0 = T0;
+  const int bits = which ? g.vb : g.kb;
   float* y = smem;                 // [G][D]
   float* acc = y + G * D;          // [G][D] scratch for the sums, then codes
   float* sig = acc + G * D;        // [max(G, D)]
   float* rsc = sig + 256;          // [G] row scales
   float* csc = rsc + 128;          // [D] column scales
-  const int blk = blk_begin + blockIdx.x;
   const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
   const int q0 = blk * G;          // first quantized row of the block
   const int t0 = g.S + q0;
@@ -285,9 +345,11 @@ __global__ void kvarn_block_kernel(Geom g, TokSrc src, int blk_begin, float inv_
     __syncthreads();
   }
   // grouped affine along D (groups of G channels)
-  const int codes_plane = KVQ_PLANE_K_CODES, scale_plane = KVQ_PLANE_K_SCALE;
-  const int zero_plane = KVQ_PLANE_K_ZERO, row_plane = KVQ_PLANE_K_ROW;
-  const int col_plane = KVQ_PLANE_K_COL;
+  const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int row_plane = which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW;
+  const int col_plane = which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL;
   uint8_t* cs = reinterpret_cast<uint8_t*>(acc);
   const int ng = D / G;
   for (int p = threadIdx.x; p < G * ng; p += nt) {
@@ -316,109 +378,56 @@ __global__ void kvarn_block_kernel(Geom g, TokSrc src, int blk_begin, float inv_
 
 int grid_for(int64_t threads_needed, int block) {
   int64_t n = (threads_needed + block - 1) / block;
-  int64_t cap = (int64_t)num_sms() * 16;
+  int64_t cap = (int64_t)num_sms() * 8;
   if (n > cap) n = cap;
   return (int)(n < 1 ? 1 : n);
 }
 
-cudaError_t store_full(const Geom& g, int plane, const void* x, int T0, int L, int ta, int tb,
-                       int off, int rows, cudaStream_t s) {
-  if (tb <= ta) return cudaSuccess;
-  const int es = g.act == KVQ_BF16 ? 2 : 4;
-  int64_t n = (int64_t)g.B * g.H * (tb - ta) * (g.D * es / 16);
-  store_full_kernel<<<grid_for(n, 256), 256, 0, s>>>(g, plane, x, T0, L, ta, tb, off, rows);
-  return cudaGetLastError();
-}
-
-cudaError_t pack_pertoken(const Geom& g, int which, int bits, int sym, const TokSrc& src,
-                          int ta, int tb, cudaStream_t s) {
-  if (tb <= ta) return cudaSuccess;
-  int64_t units = (int64_t)g.B * g.H * (tb - ta) * (g.D / g.G);
-  int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
-  pack_pertoken_kernel<<<grid_for(threads, 256), 256, 0, s>>>(g, which, bits, sym, src, ta, tb);
-  return cudaGetLastError();
-}
-
 }  // namespace
 
-cudaError_t launch_append(const Geom& g, int T0, int L, const void* k, const void* v,
-                          cudaStream_t s) {
-  const int T1 = T0 + L;
-  cudaError_t e = cudaSuccess;
-  TokSrc sk{k, T0, L, -1, 0, 1}, sv{v, T0, L, -1, 0, 1};
+cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cudaStream_t s) {
+  TokSrc sk{k, 0, L, -1, 0, 1}, sv{v, 0, L, -1, 0, 1};
+  const int es = g.act == KVQ_BF16 ? 2 : 4;
+  const int64_t full_threads = (int64_t)g.B * g.H * L * (g.D * es / 16);
+  const int max_blocks = L / g.G + 1;     // most G-blocks an append of L completes
+  cudaError_t e;
   switch (g.fmt) {
     case KVQ_FMT_FLOAT:
-      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, T0, T1, 0, g.Tmax, s);
-      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, T0, T1, 0, g.Tmax, s);
-      return e;
+      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      return cudaGetLastError();
     case KVQ_FMT_AFFINE:
     case KVQ_FMT_SYMMETRIC: {
       const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
-      e = pack_pertoken(g, 0, g.kb, sym, sk, T0, T1, s);
-      if (e == cudaSuccess) e = pack_pertoken(g, 1, g.vb, sym, sv, T0, T1, s);
-      return e;
+      const int64_t units = (int64_t)g.B * g.H * L * (g.D / g.G);
+      const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
+      pack_pertoken_kernel<<<dim3(grid_for(threads, 256), 2), 256, 0, s>>>(g, L, sk, sv, sym, 0, 1);
+      return cudaGetLastError();
     }
     case KVQ_FMT_KIVI: {
-      const int q0 = kivi_tq(T0, g.R, g.G), q1 = kivi_tq(T1, g.R, g.G);
       sk.ring_plane = KVQ_PLANE_K_FULL; sk.ring_rows = g.ring;
       sv.ring_plane = KVQ_PLANE_V_FULL; sv.ring_rows = g.ring;
-      if (q1 > q0) {
-        dim3 grid((q1 - q0) / g.G, g.B * g.H);
-        size_t sm = (size_t)g.G * g.D * 5;
-        e = cudaFuncSetAttribute(kivi_key_flush_kernel,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        if (e != cudaSuccess) return e;
-        kivi_key_flush_kernel<<<grid, 128, sm, s>>>(g, sk, q0 / g.G);
-        e = cudaGetLastError();
-        if (e == cudaSuccess) e = pack_pertoken(g, 1, g.vb, 0, sv, q0, q1, s);
-        if (e != cudaSuccess) return e;
-      }
-      const int ta = q1 > T0 ? q1 : T0;
-      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, ta, T1, 0, g.ring, s);
-      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, ta, T1, 0, g.ring, s);
-      return e;
+      const size_t sm = (size_t)g.G * g.D * 5;
+      e = cudaFuncSetAttribute(kivi_key_flush_kernel,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+      if (e != cudaSuccess) return e;
+      kivi_key_flush_kernel<<<dim3(max_blocks, g.B * g.H), 128, sm, s>>>(g, L, sk);
+      const int64_t units = (int64_t)g.B * g.H * max_blocks * g.G * (g.D / g.G);
+      const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
+      pack_pertoken_kernel<<<dim3(grid_for(threads, 256), 1), 256, 0, s>>>(g, L, sk, sv, 0, 1, 0);
+      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      return cudaGetLastError();
     }
     case KVQ_FMT_KVARN: {
-      const int S = g.S, G = g.G;
-      const int se = T1 < S ? T1 : S;
-      e = store_full(g, KVQ_PLANE_K_FULL, k, T0, L, T0, se, 0, S > 0 ? S : 1, s);
-      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_FULL, v, T0, L, T0, se, 0, S > 0 ? S : 1, s);
+      const size_t sm = ((size_t)2 * g.G * g.D + 256 + 128 + 256) * sizeof(float);
+      const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));
+      e = cudaFuncSetAttribute(kvarn_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)sm);
       if (e != cudaSuccess) return e;
-      const int n0 = kvarn_nblocks(T0, S, G), n1 = kvarn_nblocks(T1, S, G);
-      if (n1 > n0) {
-        const size_t sm = ((size_t)2 * G * g.D + 256 + 128 + 256) * sizeof(float);
-        const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));
-        e = cudaFuncSetAttribute(kvarn_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)sm);
-        if (e != cudaSuccess) return e;
-        TokSrc src[2] = {sk, sv};
-        for (int w = 0; w < 2; ++w) {
-          src[w].ring_plane = w ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
-          src[w].ring_off = S;
-          src[w].ring_rows = G;
-        }
-        // keys and values are separate launches (different sources)
-        for (int w = 0; w < 2; ++w) {
-          dim3 grid(n1 - n0, g.B * g.H, 1);
-          Geom gw = g;
-          if (w) {  // value launch: value planes and bit width in the key slots
-            gw.kb = g.vb;
-            gw.pl[KVQ_PLANE_K_CODES] = g.pl[KVQ_PLANE_V_CODES];
-            gw.pl[KVQ_PLANE_K_SCALE] = g.pl[KVQ_PLANE_V_SCALE];
-            gw.pl[KVQ_PLANE_K_ZERO] = g.pl[KVQ_PLANE_V_ZERO];
-            gw.pl[KVQ_PLANE_K_ROW] = g.pl[KVQ_PLANE_V_ROW];
-            gw.pl[KVQ_PLANE_K_COL] = g.pl[KVQ_PLANE_V_COL];
-          }
-          kvarn_block_kernel<<<grid, 256, sm, s>>>(gw, src[w], n0, inv_sqrt_d);
-          e = cudaGetLastError();
-          if (e != cudaSuccess) return e;
-        }
-      }
-      int ta = S + n1 * G;
-      if (ta < T0) ta = T0;
-      e = store_full(g, KVQ_PLANE_K_PEND, k, T0, L, ta, T1, S, G, s);
-      if (e == cudaSuccess) e = store_full(g, KVQ_PLANE_V_PEND, v, T0, L, ta, T1, S, G, s);
-      return e;
+      sk.ring_plane = KVQ_PLANE_K_PEND; sk.ring_off = g.S; sk.ring_rows = g.G;
+      sv.ring_plane = KVQ_PLANE_V_PEND; sv.ring_off = g.S; sv.ring_rows = g.G;
+      kvarn_block_kernel<<<dim3(max_blocks, g.B * g.H, 2), 256, sm, s>>>(g, L, sk, sv, inv_sqrt_d);
+      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      return cudaGetLastError();
     }
   }
   return cudaErrorInvalidValue;

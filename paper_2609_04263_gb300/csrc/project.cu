@@ -20,6 +20,7 @@ struct ProjArgs {
   int r[3];
   void* out[3];
   int B, L, d_in, Hq, Hkv, D, pos0, act;
+  const int* pos_dev;   // if set, positions start at *pos_dev + pos0
   float alpha_over_r, rope_base;
 };
 
@@ -112,6 +113,7 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
   __syncthreads();
   // RoPE (rotate-half) on q and k; angle in fp64 for accuracy
   const bool rope = proj < 2 && p.rope_base > 0.f;
+  const int pos_base = p.pos0 + (p.pos_dev ? *p.pos_dev : 0);
   const int H = proj == 0 ? p.Hq : p.Hkv;
   for (int i = threadIdx.x; i < kMT * D; i += kThreads) {
     const int m = i / D, d = i % D;
@@ -122,7 +124,7 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
     if (rope) {
       const int half = D / 2, fi = d % half;
       const double theta = pow((double)p.rope_base, -2.0 * fi / D);
-      const double ang = (double)(p.pos0 + l) * theta;
+      const double ang = (double)(pos_base + l) * theta;
       const float c = (float)cos(ang), s = (float)sin(ang);
       if (d < half) v = Y[m * D + d] * c - Y[m * D + d + half] * s;
       else v = Y[m * D + d] * c + Y[m * D + d - half] * s;
@@ -131,20 +133,189 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Few rows (M = B * L <= 16, the decode step): weight streaming.  Each warp
+// owns one RoPE column pair (c, c + D/2) of one head and streams both weight
+// rows with 16-byte loads; x (all M rows) sits in shared memory.  The
+// rank-r branch: the CTA first forms (alpha/r) x A_p^T for its projection.
+// ---------------------------------------------------------------------------
+constexpr int kSkinnyWarps = 8;
+constexpr int kSkinnyMaxM = 16;
+
+template <typename T>
+__device__ __forceinline__ void load8f(const T* p, float f[8]);
+template <>
+__device__ __forceinline__ void load8f<__nv_bfloat16>(const __nv_bfloat16* p, float f[8]) {
+  uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float2 t = __bfloat1622float2(h[i]);
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+template <>
+__device__ __forceinline__ void load8f<float>(const float* p, float f[8]) {
+  float4 a = __ldg(reinterpret_cast<const float4*>(p));
+  float4 b = __ldg(reinterpret_cast<const float4*>(p) + 1);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+}
+
+template <typename T, int MM>
+__global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjArgs p) {
+  extern __shared__ float xsm[];             // [M][d_in] fp32, then U [M][64]
+  const int M = p.B * p.L, D = p.D, K = p.d_in;
+  const int half = D / 2;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int pairs_per_head = half;
+  const int pair0 = blockIdx.x * kSkinnyWarps;      // CTA's first pair (stacked heads)
+  const int hh = pair0 / pairs_per_head;           // all 8 pairs of a CTA share a head
+  const int proj = hh < p.Hq ? 0 : hh < p.Hq + p.Hkv ? 1 : 2;
+  const int head = proj == 0 ? hh : proj == 1 ? hh - p.Hq : hh - p.Hq - p.Hkv;
+  const int r = p.r[proj];
+  float* U = xsm + M * K;
+  const T* x = reinterpret_cast<const T*>(p.x);
+  for (int i = threadIdx.x * 8; i < M * K; i += blockDim.x * 8) {
+    float f[8];
+    load8f<T>(x + i, f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) xsm[i + j] = f[j];
+  }
+  __syncthreads();
+  // (alpha/r) x A_p^T: warp w takes ranks w, w + 8, ...
+  if (r > 0) {
+    const T* A = reinterpret_cast<const T*>(p.a[proj]);
+    for (int j = warp; j < r; j += kSkinnyWarps) {
+      float acc[MM];
+#pragma unroll
+      for (int m = 0; m < MM; ++m) acc[m] = 0.f;
+      for (int k = lane * 8; k < K; k += 256) {
+        float a[8];
+        load8f<T>(A + (int64_t)j * K + k, a);
+#pragma unroll
+        for (int m = 0; m < MM; ++m) {
+          if (m < M) {
+            const float* xr = xsm + m * K + k;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[m] += a[e] * xr[e];
+          }
+        }
+      }
+#pragma unroll
+      for (int m = 0; m < MM; ++m) {
+        float v = acc[m];
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0 && m < M) U[m * 64 + j] = v * p.alpha_over_r;
+      }
+    }
+  }
+  __syncthreads();
+  const int c = (pair0 + warp) % pairs_per_head;    // channel within the first half
+  const int n1 = hh * D + c, n2 = n1 + half;
+  const T* W = reinterpret_cast<const T*>(p.w);
+  const T* w1 = W + (int64_t)n1 * K;
+  const T* w2 = W + (int64_t)n2 * K;
+  float acc1[MM], acc2[MM];
+#pragma unroll
+  for (int m = 0; m < MM; ++m) { acc1[m] = 0.f; acc2[m] = 0.f; }
+  constexpr int kUnroll = 4;
+  for (int k0 = lane * 8; k0 < K; k0 += 256 * kUnroll) {
+    float a[kUnroll][8], b[kUnroll][8];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int k = k0 + u * 256;
+      if (k < K) {
+        load8f<T>(w1 + k, a[u]);
+        load8f<T>(w2 + k, b[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int k = k0 + u * 256;
+      if (k < K) {
+#pragma unroll
+        for (int m = 0; m < MM; ++m) {
+          if (m < M) {
+            const float* xr = xsm + m * K + k;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              acc1[m] += a[u][e] * xr[e];
+              acc2[m] += b[u][e] * xr[e];
+            }
+          }
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int m = 0; m < MM; ++m) {
+    for (int o = 16; o > 0; o >>= 1) {
+      acc1[m] += __shfl_xor_sync(0xffffffffu, acc1[m], o);
+      acc2[m] += __shfl_xor_sync(0xffffffffu, acc2[m], o);
+    }
+  }
+  // rank-r up projection, RoPE, head-major store: lane m handles row m
+  if (lane < M) {
+    float y1 = 0.f, y2 = 0.f;
+#pragma unroll
+    for (int m = 0; m < MM; ++m)
+      if (m == lane) { y1 = acc1[m]; y2 = acc2[m]; }
+    if (r > 0) {
+      const T* Bm = reinterpret_cast<const T*>(p.bm[proj]);
+      const int64_t b1 = ((int64_t)head * D + c) * r, b2 = ((int64_t)head * D + c + half) * r;
+      for (int j = 0; j < r; ++j) {
+        const float u = U[lane * 64 + j];
+        y1 += u * ld_act(Bm, b1 + j, p.act);
+        y2 += u * ld_act(Bm, b2 + j, p.act);
+      }
+    }
+    const int b = lane / p.L, l = lane % p.L;
+    if (proj < 2 && p.rope_base > 0.f) {
+      const int pos = p.pos0 + (p.pos_dev ? *p.pos_dev : 0) + l;
+      const double theta = pow((double)p.rope_base, -2.0 * c / D);
+      const double ang = (double)pos * theta;
+      const float cs = (float)cos(ang), sn = (float)sin(ang);
+      const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
+      y1 = o1;
+      y2 = o2;
+    }
+    const int H = proj == 0 ? p.Hq : proj == 1 ? p.Hkv : p.Hkv;
+    const int64_t base = (((int64_t)b * H + head) * p.L + l) * D;
+    st_act(p.out[proj], base + c, y1, p.act);
+    st_act(p.out[proj], base + c + half, y2, p.act);
+  }
+}
+
+template <typename T>
+cudaError_t launch_skinny(const ProjArgs& p, cudaStream_t s) {
+  const int M = p.B * p.L;
+  const int pairs = (p.Hq + 2 * p.Hkv) * p.D / 2;
+  const size_t sm = ((size_t)M * p.d_in + (size_t)M * 64) * sizeof(float);
+  auto kern = M <= 4 ? project_skinny_kernel<T, 4> : project_skinny_kernel<T, kSkinnyMaxM>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  kern<<<pairs / kSkinnyWarps, kSkinnyWarps * 32, sm, s>>>(p);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const void* const a[3], const void* const bm[3], const int r[3],
                            float alpha_over_r, int Hq, int Hkv, int D, int pos0,
-                           float rope_base, int act, void* const out[3], int* err,
-                           cudaStream_t s) {
+                           const int* pos_dev, float rope_base, int act,
+                           void* const out[3], int* err, cudaStream_t s) {
   (void)err;
   ProjArgs p;
   p.x = x; p.w = w;
   for (int i = 0; i < 3; ++i) { p.a[i] = a[i]; p.bm[i] = bm[i]; p.r[i] = r[i]; p.out[i] = out[i]; }
   p.B = B; p.L = L; p.d_in = d_in; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.pos0 = pos0; p.act = act;
+  p.pos_dev = pos_dev;
   p.alpha_over_r = alpha_over_r; p.rope_base = rope_base;
   const int M = B * L;
+  if (M <= kSkinnyMaxM && (size_t)M * d_in * 4 <= 160 * 1024 && d_in % 8 == 0)
+    return act == KVQ_BF16 ? launch_skinny<__nv_bfloat16>(p, s) : launch_skinny<float>(p, s);
   const size_t sm = (size_t)(kMT * (kKC + 1) + 256 * (kKC + 1) + kMT * 64 + kMT * D) *
                     sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(project_simt_kernel,

@@ -57,8 +57,9 @@ _SIGS = {
     "kvq_project_lora": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p,
                                  c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
                                  c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
-                                 c_int, c_float, c_int, c_void_p, c_void_p, c_void_p,
+                                 c_int, c_void_p, c_float, c_int, c_void_p, c_void_p, c_void_p,
                                  c_void_p]),
+    "kvq_cache_sync": (c_int, [c_void_p, c_void_p]),
     "kvq_append_pack": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_void_p]),
     "kvq_attend_prefill": (c_int, [c_void_p, c_void_p, c_int, c_int, c_float, c_void_p,
                                    c_void_p]),
@@ -130,13 +131,17 @@ def kvq_cache_view(handle: int) -> kvq_cache_planes:
 
 
 def kvq_project_lora(x, B, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,
-                     alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, rope_base, dtype,
-                     q, k, v, stream) -> None:
+                     alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, pos_cache,
+                     rope_base, dtype, q, k, v, stream) -> None:
     P = lambda t: c_void_p(t or 0)
     _check(lib().kvq_project_lora(P(x), B, L, d_in, P(w_qkv), P(a_q), P(b_q), r_q, P(a_k),
                                   P(b_k), r_k, P(a_v), P(b_v), r_v, alpha_over_r, n_q_heads,
-                                  n_kv_heads, head_dim, pos0, rope_base, dtype, P(q), P(k),
-                                  P(v), P(stream)))
+                                  n_kv_heads, head_dim, pos0, P(pos_cache), rope_base, dtype,
+                                  P(q), P(k), P(v), P(stream)))
+
+
+def kvq_cache_sync(handle, stream=0) -> None:
+    _check(lib().kvq_cache_sync(c_void_p(handle), c_void_p(stream or 0)))
 
 
 def kvq_append_pack(handle, k, v, L, stream) -> None:

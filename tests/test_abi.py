@@ -122,5 +122,5 @@ def test_project_validation(kvq):
         hq, hkv = c.get("heads", (32, 4))
         with pytest.raises(kvq.KvqError):
             kvq.kvq_project_lora(P, 1, 4, c.get("d_in", 2048), P, P, P, c.get("r_q", 16), P, P,
-                                 16, P, P, 16, 2.0, hq, hkv, c.get("head_dim", 64), 0, 1e4,
+                                 16, P, P, 16, 2.0, hq, hkv, c.get("head_dim", 64), 0, None, 1e4,
                                  c.get("dtype", kvq.KVQ_BF16), P, P, P, 0)
