@@ -212,6 +212,31 @@ kvq_status kvq_attend_prefill(kvq_cache* cache, const void* q, int L, int n_q_he
 kvq_status kvq_attend_decode(kvq_cache* cache, const void* q, int n_q_heads,
                              float softmax_scale, void* out, void* stream);
 
+/*
+ * kvq_attend_decode for callers that cannot allocate device memory.  (No
+ * counterpart in the paper: this is a deployment variant of the decode step.)
+ *
+ * kvq_attend_decode keeps its split-K partials in the cache buffer's
+ * workspace plane.  Callers that cannot provide extra device memory when they
+ * call (a plugin or custom-op host that passes only input and output tensors
+ * and forbids allocation, allocation-free serving loops where cudaMalloc
+ * would synchronise the device, a process whose memory pool has reserved all
+ * free HBM) use this variant instead: the partials go to one fixed array in
+ * the library's static device memory (4 MiB per GPU, held from library load
+ * until process exit), and the call allocates nothing.
+ *
+ * Same arguments, semantics and results as kvq_attend_decode.  Returns
+ * KVQ_ERR_CAPACITY, launching nothing, if batch * q_heads * 32 * (head_dim + 2)
+ * floats exceed the array (1,048,576 floats).  The first call on each device
+ * looks up the array's device address with that device current; make that
+ * first call before any stream capture.  Every call uses the same array and
+ * leaves its contents behind (the kernels write every partial they later
+ * read, so nothing needs clearing), so calls that overlap on the GPU (other
+ * streams, other threads) race: serialise them.
+ */
+kvq_status kvq_attend_decode_noalloc(kvq_cache* cache, const void* q, int n_q_heads,
+                                     float softmax_scale, void* out, void* stream);
+
 /* Read and clear the device-side error word of the library (synchronises
  * `stream`).  *out = 0 when no bounded wait has timed out. */
 kvq_status kvq_device_status(void* stream, int* out);

@@ -10,26 +10,22 @@
 
 using namespace kvq;
 
-struct kvq_cache {
-  kvq_cache_desc desc;
-  Geom g;
-  char* base;
-  size_t bytes;
-  int T;            // host mirror of the device token count
-  bool need_init;   // device state not yet zeroed since create/reset
-};
-
 namespace {
 
 thread_local std::string g_last_error;
 
-kvq_status fail(kvq_status st, const char* fmt, ...) {
+kvq_status vfail(kvq_status st, const char* fmt, va_list ap) {
   char buf[512];
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  g_last_error = buf;
+  return st;
+}
+
+kvq_status fail(kvq_status st, const char* fmt, ...) {
   va_list ap;
   va_start(ap, fmt);
-  vsnprintf(buf, sizeof buf, fmt, ap);
+  vfail(st, fmt, ap);
   va_end(ap);
-  g_last_error = buf;
   return st;
 }
 
@@ -206,6 +202,23 @@ int* device_error_word() {
   return addr[dev];
 }
 
+// Zero the device state before the first launch after create/reset
+// (stream-ordered, so it can be captured with the calls that follow).
+cudaError_t ensure_cache_init(kvq_cache* c, cudaStream_t s) {
+  if (!c->need_init) return cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(c->g.state, 0, sizeof(CacheState), s);
+  if (e == cudaSuccess) c->need_init = false;
+  return e;
+}
+
+kvq_status set_error(kvq_status st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vfail(st, fmt, ap);
+  va_end(ap);
+  return st;
+}
+
 int num_sms() {
   if (g_num_sms == 0) {
     int dev = 0, n = 0;
@@ -272,14 +285,7 @@ kvq_status kvq_reset_cache(kvq_cache* cache) {
   return KVQ_OK;
 }
 
-// Zero the device state before the first launch after create/reset
-// (stream-ordered, so it can be captured with the calls that follow).
-static cudaError_t ensure_init(kvq_cache* c, cudaStream_t s) {
-  if (!c->need_init) return cudaSuccess;
-  cudaError_t e = cudaMemsetAsync(c->g.state, 0, sizeof(CacheState), s);
-  if (e == cudaSuccess) c->need_init = false;
-  return e;
-}
+static cudaError_t ensure_init(kvq_cache* c, cudaStream_t s) { return ensure_cache_init(c, s); }
 
 kvq_status kvq_cache_sync(kvq_cache* cache, void* stream) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");

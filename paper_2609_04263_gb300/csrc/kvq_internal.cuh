@@ -141,6 +141,31 @@ __device__ __forceinline__ int cache_tokens(const Geom& g) {
 // Device address of the library's error word (set up once per device).
 int* device_error_word();
 
+// Floats of split-K partials a decode over this geometry addresses:
+// [B][Hq][kMaxSplits][D + kWsStride].
+inline size_t workspace_floats(const Geom& g) {
+  return (size_t)g.B * g.Hq * kMaxSplits * (g.D + kWsStride);
+}
+
+// Record a failure for kvq_last_error() and return `st`.
+kvq_status set_error(kvq_status st, const char* fmt, ...);
+
 int num_sms();
 
+}  // namespace kvq
+
+// Host-side handle of a cache (opaque to users of kvq.h).
+struct kvq_cache {
+  kvq_cache_desc desc;
+  kvq::Geom g;
+  char* base;
+  size_t bytes;
+  int T;            // host mirror of the device token count
+  bool need_init;   // device state not yet zeroed since create/reset
+};
+
+namespace kvq {
+// Zero the cache's device state if this is the first launch since
+// create/reset (stream-ordered memset).
+cudaError_t ensure_cache_init(kvq_cache* c, cudaStream_t s);
 }  // namespace kvq

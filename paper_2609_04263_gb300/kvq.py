@@ -65,6 +65,8 @@ _SIGS = {
                                    c_void_p]),
     "kvq_attend_decode": (c_int, [c_void_p, c_void_p, c_int, c_float, c_void_p, c_void_p]),
     "kvq_device_status": (c_int, [c_void_p, ctypes.POINTER(c_int)]),
+    "kvq_attend_decode_noalloc": (c_int, [c_void_p, c_void_p, c_int, c_float, c_void_p,
+                                          c_void_p]),
 }
 
 _lib = None
@@ -157,6 +159,13 @@ def kvq_attend_prefill(handle, q, L, n_q_heads, softmax_scale, out, stream) -> N
 def kvq_attend_decode(handle, q, n_q_heads, softmax_scale, out, stream) -> None:
     _check(lib().kvq_attend_decode(c_void_p(handle), c_void_p(q), n_q_heads, softmax_scale,
                                    c_void_p(out), c_void_p(stream or 0)))
+
+
+def kvq_attend_decode_noalloc(handle, q, n_q_heads, softmax_scale, out, stream) -> None:
+    """Decode attention whose split-K partials live in the library's static
+    device memory instead of the cache's workspace (nothing is allocated)."""
+    _check(lib().kvq_attend_decode_noalloc(c_void_p(handle), c_void_p(q), n_q_heads,
+                                           softmax_scale, c_void_p(out), c_void_p(stream or 0)))
 
 
 def kvq_device_status(stream=0) -> int:
