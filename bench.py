@@ -179,6 +179,19 @@ class Runner:
             if timer:
                 timer("attend_decode", 1)
 
+    # the three decode call classes, each over all layers (for timing)
+    def decode_project_layers(self):
+        for l in range(len(self.caches)):
+            self._project(l, self.xs, self.dec)
+
+    def decode_append_layers(self):
+        for c in self.caches:
+            c.append(self.dec[1], self.dec[2])
+
+    def decode_attend_layers(self):
+        for c in self.caches:
+            c.attend_decode(self.dec[0], out=self.o_dec)
+
     def capture(self):
         """Capture one decode step (all layers) in a CUDA graph."""
         self.reset()
@@ -287,6 +300,27 @@ class ClockSampler:
 
 def l2_flush(buf):
     buf.fill_(1)
+
+
+def graph_time_ms(fn, reps):
+    """Mean device time of one call of `fn` (a sequence of launches), from a
+    captured graph replayed `reps` times between CUDA events (two untimed
+    replays first)."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        fn()
+    torch.cuda.synchronize()
+    for _ in range(2):
+        g.replay()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
 
 
 # ---------------------------------------------------------------------------
@@ -447,15 +481,24 @@ def main():
     value = world * tokens_per_step * args.steps / total_s
     decode_tps = wl.batch * wl.decode / (statistics.mean(dec_ms) / 1000.0)
 
-    # ---- per-kernel durations: eager prefill and decode with events -------
+    # ---- per-kernel durations ---------------------------------------------
+    # Prefill kernels run for milliseconds: CUDA events around each eager
+    # call.  Decode kernels run for microseconds, so each class (projection,
+    # append, attention) is captured as a graph of its 22 per-layer calls and
+    # timed over repeated replays; the graph keeps the device busy, so the
+    # events measure kernel time, not host launch gaps.
     timer = EventTimer()
     run.reset()
     run.prefill(timer)
-    for s in range(32):
-        run.xs.copy_(run.x_dec[s])
-        run.decode_step_eager(timer)
     mean_ms = timer.mean_ms()
-    T_dec = wl.prefill + wl.decode // 2
+    run.xs.copy_(run.x_dec[0])
+    reps = 10
+    T_prof = wl.prefill + 2 + reps          # cache length during the attention replays
+    for name, fn in (("project_decode", run.decode_project_layers),
+                     ("append_decode", run.decode_append_layers),
+                     ("attend_decode", run.decode_attend_layers)):
+        mean_ms[name] = graph_time_ms(fn, reps) / wl.layers
+    T_dec = T_prof
     work = {
         "project": ("tensor", proj_flops(wl, wl.batch * wl.prefill), wl.layers),
         "attend_prefill": ("tensor", prefill_attn_flops(wl, wl.prefill, wl.prefill), wl.layers),

@@ -95,6 +95,9 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     }
   }
   const int B = d->batch, H = d->kv_heads, Tm = d->max_tokens;
+  // per-token planes hold whole 64-token chunks (the decode kernel copies
+  // whole chunks), so their rows are padded to a multiple of 64
+  const int Tp = (Tm + 63) / 64 * 64;
   const int act = d->dtype == KVQ_BF16 ? 2 : 4;
   memset(g, 0, sizeof *g);
   g->fmt = d->fmt; g->kb = d->key_bits; g->vb = d->value_bits; g->G = G;
@@ -111,17 +114,17 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
       break;
     case KVQ_FMT_AFFINE:
     case KVQ_FMT_SYMMETRIC:
-      set(KVQ_PLANE_K_CODES, Tm, D * d->key_bits / 8, 1);
-      set(KVQ_PLANE_K_SCALE, Tm, D / G, 2);
-      set(KVQ_PLANE_V_CODES, Tm, D * d->value_bits / 8, 1);
-      set(KVQ_PLANE_V_SCALE, Tm, D / G, 2);
+      set(KVQ_PLANE_K_CODES, Tp, D * d->key_bits / 8, 1);
+      set(KVQ_PLANE_K_SCALE, Tp, D / G, 2);
+      set(KVQ_PLANE_V_CODES, Tp, D * d->value_bits / 8, 1);
+      set(KVQ_PLANE_V_SCALE, Tp, D / G, 2);
       if (d->fmt == KVQ_FMT_AFFINE) {
-        set(KVQ_PLANE_K_ZERO, Tm, D / G, 2);
-        set(KVQ_PLANE_V_ZERO, Tm, D / G, 2);
+        set(KVQ_PLANE_K_ZERO, Tp, D / G, 2);
+        set(KVQ_PLANE_V_ZERO, Tp, D / G, 2);
       }
       break;
     case KVQ_FMT_KIVI: {
-      const int64_t nblk = (Tm + G - 1) / G;
+      const int64_t nblk = (Tp + G - 1) / G;
       set(KVQ_PLANE_K_CODES, nblk * G, D * d->key_bits / 8, 1);
       set(KVQ_PLANE_K_SCALE, nblk, D, 2);
       set(KVQ_PLANE_K_ZERO, nblk, D, 2);

@@ -97,6 +97,12 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
 // Decode split-K width for a cache geometry (fixed, independent of T).
 int decode_splits(const Geom& g);
 
+// Tensor-core split decode (attend_mma.cu): the formats it covers, and the
+// launch (partials to the workspace plane; the caller merges them).
+bool decode_mma_supported(const Geom& g);
+cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err,
+                              cudaStream_t s);
+
 // Token range of split `s` of `splits` over T tokens (tiles of `tile`).
 __host__ __device__ inline void split_range(int T, int splits, int s, int tile, int* ts,
                                             int* te) {

@@ -55,6 +55,10 @@ DECODE = [
     ("kvarn", "bf16", 1, 2, 4, 256, [128 + 64 * 2 + 9]),
     ("kvarn_small", "bf16", 2, 2, 4, 64, [40 + 32 * 3 + 31, 1]),
     ("kvarn_small", "f32", 1, 1, 2, 64, [20]),      # sinks only
+    ("affine4", "bf16", 1, 1, 16, 128, [777]),      # GQA group 16
+    ("sym2", "bf16", 3, 2, 6, 64, [65]),            # odd group, ragged chunk
+    ("kivi2", "bf16", 1, 1, 8, 64, [1000, 7]),      # chunks straddle the residual edge
+    ("affine2", "bf16", 2, 4, 8, 64, [4095, 1]),
 ]
 
 
