@@ -83,9 +83,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 __device__ __forceinline__ uint32_t pack_raw(uint16_t lo, uint16_t hi) {
   return (uint32_t)lo | ((uint32_t)hi << 16);
 }
-__device__ __forceinline__ float bf16_bits_to_float(uint32_t bits16) {
-  return __uint_as_float(bits16 << 16);
-}
 
 // Channel held by slot e (0..7) of a thread's 8-channel word in QK k-step s,
 // register half (0: a0/b0, 1: a2/b1), element j: see the LOP3 pairings.

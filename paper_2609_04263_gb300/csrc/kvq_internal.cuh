@@ -94,6 +94,15 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const int* pos_dev, float rope_base, int act,
                            void* const out[3], int* err, cudaStream_t s);
 
+// tcgen05 projection (project_tc.cu) for bf16 and more than 16 rows;
+// cudaErrorNotSupported if the head shapes do not tile.
+cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void* w,
+                              const void* const a[3], const void* const bm[3], const int r[3],
+                              float alpha_over_r, int Hq, int Hkv, int D, int pos0,
+                              const int* pos_dev, float rope_base, void* const out[3], int* err,
+                              cudaStream_t s);
+void rope_theta_table(float rope_base, int D, float* hi, float* lo);
+
 // Decode split-K width for a cache geometry (fixed, independent of T).
 int decode_splits(const Geom& g);
 

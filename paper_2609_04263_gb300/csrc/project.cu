@@ -22,7 +22,27 @@ struct ProjArgs {
   int B, L, d_in, Hq, Hkv, D, pos0, act;
   const int* pos_dev;   // if set, positions start at *pos_dev + pos0
   float alpha_over_r, rope_base;
+  // RoPE frequencies base^(-2i/D), i < D/2, computed in fp64 on the host and
+  // split into hi + lo floats
+  float theta_hi[128], theta_lo[128];
 };
+
+// cos and sin of pos * theta in fp32 to about 1e-7 absolute for positions
+// below 2^24: pos * theta_hi is formed exactly as p + e (FMA), reduced by
+// 2 pi in three parts (the first exact for multiples below 2^15), then the
+// small remainder goes to sincosf.
+__device__ __forceinline__ void rope_cos_sin(int pos, float th_hi, float th_lo, float* c,
+                                             float* s) {
+  const float x = (float)pos;
+  const float p = x * th_hi;
+  const float e = fmaf(x, th_hi, -p) + x * th_lo;
+  const float k = rintf(p * 0.15915494309189535f);          // 1 / (2 pi)
+  float r = fmaf(-k, 6.28125f, p);                            // 2 pi = 6.28125
+  r = fmaf(-k, 1.9353071795864769e-3f, r);                    //   + 1.9353072e-3
+  r = fmaf(-k, 1.0253132e-11f, r);                            //   + 1.0253e-11 (remainder)
+  r += e;
+  sincosf(r, s, c);
+}
 
 // One CTA: kMT rows of x times one head's D output columns.
 __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
@@ -123,9 +143,8 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
     float v = Y[i];
     if (rope) {
       const int half = D / 2, fi = d % half;
-      const double theta = pow((double)p.rope_base, -2.0 * fi / D);
-      const double ang = (double)(pos_base + l) * theta;
-      const float c = (float)cos(ang), s = (float)sin(ang);
+      float c, s;
+      rope_cos_sin(pos_base + l, p.theta_hi[fi], p.theta_lo[fi], &c, &s);
       if (d < half) v = Y[m * D + d] * c - Y[m * D + d + half] * s;
       else v = Y[m * D + d] * c + Y[m * D + d - half] * s;
     }
@@ -237,7 +256,9 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
 #pragma unroll
         for (int m = 0; m < MM; ++m) {
           if (m < M) {
-            const float* xr = xsm + m * K + k;
+            const float4* xr4 = reinterpret_cast<const float4*>(xsm + m * K + k);
+            const float4 xa = xr4[0], xb = xr4[1];
+            const float xr[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               acc1[m] += a[u][e] * xr[e];
@@ -273,9 +294,8 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
     const int b = lane / p.L, l = lane % p.L;
     if (proj < 2 && p.rope_base > 0.f) {
       const int pos = p.pos0 + (p.pos_dev ? *p.pos_dev : 0) + l;
-      const double theta = pow((double)p.rope_base, -2.0 * c / D);
-      const double ang = (double)pos * theta;
-      const float cs = (float)cos(ang), sn = (float)sin(ang);
+      float cs, sn;
+      rope_cos_sin(pos, p.theta_hi[c], p.theta_lo[c], &cs, &sn);
       const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
       y1 = o1;
       y2 = o2;
@@ -301,19 +321,35 @@ cudaError_t launch_skinny(const ProjArgs& p, cudaStream_t s) {
 
 }  // namespace
 
+// RoPE frequencies base^(-2i/D) for i < D/2 in fp64, split into hi + lo
+// floats (zeros elsewhere, or everywhere when base = 0).
+void rope_theta_table(float rope_base, int D, float* hi, float* lo) {
+  for (int i = 0; i < 128; ++i) {
+    const double th = i < D / 2 && rope_base > 0.f ? pow((double)rope_base, -2.0 * i / D) : 0.0;
+    hi[i] = (float)th;
+    lo[i] = (float)(th - (double)hi[i]);
+  }
+}
+
 cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const void* const a[3], const void* const bm[3], const int r[3],
                            float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                            const int* pos_dev, float rope_base, int act,
                            void* const out[3], int* err, cudaStream_t s) {
-  (void)err;
   ProjArgs p;
   p.x = x; p.w = w;
   for (int i = 0; i < 3; ++i) { p.a[i] = a[i]; p.bm[i] = bm[i]; p.r[i] = r[i]; p.out[i] = out[i]; }
   p.B = B; p.L = L; p.d_in = d_in; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.pos0 = pos0; p.act = act;
   p.pos_dev = pos_dev;
   p.alpha_over_r = alpha_over_r; p.rope_base = rope_base;
+  rope_theta_table(rope_base, D, p.theta_hi, p.theta_lo);
   const int M = B * L;
+  if (act == KVQ_BF16 && M > kSkinnyMaxM) {
+    cudaError_t e = launch_project_tc(x, B, L, d_in, w, a, bm, r, alpha_over_r, Hq, Hkv, D, pos0,
+                                      pos_dev, rope_base, out, err, s);
+    if (e != cudaErrorNotSupported) return e;
+    (void)cudaGetLastError();
+  }
   if (M <= kSkinnyMaxM && (size_t)M * d_in * 4 <= 160 * 1024 && d_in % 8 == 0)
     return act == KVQ_BF16 ? launch_skinny<__nv_bfloat16>(p, s) : launch_skinny<float>(p, s);
   const size_t sm = (size_t)(kMT * (kKC + 1) + 256 * (kKC + 1) + kMT * 64 + kMT * D) *

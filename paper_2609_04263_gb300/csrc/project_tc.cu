@@ -1,0 +1,447 @@
+// LoRA-adapted Q/K/V projection on the 5th-generation tensor cores (tcgen05),
+// for many rows (prefill).  Section 3, Eq. (1) and Eq. (lora), with the
+// adapter kept as an explicit rank-r branch (Section 3.4):
+//   y = x W_p^T + (alpha/r) (x A_p^T) B_p^T,   then RoPE on q and k.
+//
+// One CTA computes a 128 x BN tile of y inside one projection p (BN holds
+// whole heads).  Thread 0 streams K-slices of x, W and A_p with TMA
+// (128-byte swizzle) through a kStages-deep mbarrier ring; thread 32 issues
+// tcgen05.mma: x W^T accumulates in TMEM columns [0, BN), x A_p^T in columns
+// [BN, BN + RP).  Afterwards the 128 threads (one per row / TMEM lane) read
+// x A_p^T, scale it by alpha/r, round it to bf16 and write it to shared
+// memory as an MMA operand; one more MMA pass adds (alpha/r)(x A_p^T) B_p^T
+// into the main accumulator.  The epilogue reads the tile from TMEM, applies
+// rotate-half RoPE and stores head-major [B, H, L, D].  Every mbarrier wait is
+// bounded; a timeout sets the library's error word and the CTA still frees
+// its TMEM.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include <mutex>
+
+#include "kvq_internal.cuh"
+
+namespace kvq {
+
+// shared with project.cu
+void rope_theta_table(float rope_base, int D, float* hi, float* lo);
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;              // bf16 elements per 128-byte swizzle row
+constexpr int kStages = 3;
+constexpr int kThreads = 128;
+constexpr long kWaitLimit = 1L << 26;
+
+struct TcArgs {
+  void* out[3];
+  int B, L, M, D, Hq, Hkv;
+  int n_off[4];                 // first output column of q, k, v; total columns
+  int r[3], rp[3];              // ranks and ranks padded to 16
+  int pos0;
+  const int* pos_dev;
+  float alpha_over_r;
+  int rope;
+  int k_blocks;
+  int* err;
+  float theta_hi[128], theta_lo[128];
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, int count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (long i = 0; i < kWaitLimit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(smem_u32(dst)), "l"(map), "r"(c0), "r"(c1), "r"(smem_u32(bar)) : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
+// layout (rows of 128 bytes, 8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint64_t sw128_desc(const void* p) {
+  const uint64_t addr = smem_u32(p);
+  uint64_t d = 0;
+  d |= (addr >> 4) & 0x3FFFull;               // start address
+  d |= (uint64_t)1 << 16;                     // leading byte offset (unused for SW128 K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;           // stride byte offset: 8 rows x 128 B
+  d |= (uint64_t)1 << 46;                     // descriptor version (sm_100 family)
+  d |= (uint64_t)2 << 61;                     // layout: 128-byte swizzle
+  return d;
+}
+// Instruction descriptor: kind::f16 with bf16 A and B, fp32 accumulator,
+// both operands K-major, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                     uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+      ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float v[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void rope_cs(int pos, float th_hi, float th_lo, float* c, float* s) {
+  const float x = (float)pos;
+  const float p = x * th_hi;
+  const float e = fmaf(x, th_hi, -p) + x * th_lo;
+  const float k = rintf(p * 0.15915494309189535f);
+  float r = fmaf(-k, 6.28125f, p);
+  r = fmaf(-k, 1.9353071795864769e-3f, r);
+  r = fmaf(-k, 1.0253132e-11f, r);
+  r += e;
+  sincosf(r, s, c);
+}
+
+template <int BN>
+struct Smem {
+  static constexpr int A_B = BM * BK * 2;            // 16 KB
+  static constexpr int B_B = BN * BK * 2;            // up to 32 KB
+  static constexpr int LA_B = 64 * BK * 2;           // LoRA A slice, up to 64 ranks (8 KB)
+  static constexpr int STAGE_B = A_B + B_B + LA_B;
+  static constexpr int U_OFF = kStages * STAGE_B;    // (alpha/r) x A^T as bf16 operand
+  static constexpr int BP_OFF = U_OFF + BM * BK * 2; // B_p tile [BN][64 ranks]
+  static constexpr int TOTAL = BP_OFF + BN * BK * 2 + 1024;   // + alignment slack
+};
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
+                  const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_a1,
+                  const __grid_constant__ CUtensorMap tm_a2, const __grid_constant__ CUtensorMap tm_b0,
+                  const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_b2,
+                  const TcArgs args) {
+  using S = Smem<BN>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ uint64_t full_bar[kStages], empty_bar[kStages];
+  __shared__ uint64_t u_bar, bp_bar, acc_bar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int fail;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+  const int proj = n0 < args.n_off[1] ? 0 : n0 < args.n_off[2] ? 1 : 2;
+  const int r = args.r[proj], rp = args.rp[proj];
+  const CUtensorMap* tm_a = proj == 0 ? &tm_a0 : proj == 1 ? &tm_a1 : &tm_a2;
+  const CUtensorMap* tm_b = proj == 0 ? &tm_b0 : proj == 1 ? &tm_b1 : &tm_b2;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full_bar[i], 1);
+      mbar_init(&empty_bar[i], 1);
+    }
+    mbar_init(&u_bar, 1);
+    mbar_init(&bp_bar, 1);
+    mbar_init(&acc_bar, 1);
+    fail = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {   // TMEM: 512 columns (main BN + LoRA <= 64)
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;"
+                 ::"r"(smem_u32(&tmem_base)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+  const uint32_t tmem_u = tmem + BN;
+  const int KB = args.k_blocks;
+
+  if (threadIdx.x == 0) {
+    // ---------------- TMA producer ----------------
+    if (r > 0) {
+      mbar_expect_tx(&bp_bar, BN * BK * 2);
+      tma_load_2d(smem + S::BP_OFF, tm_b, 0, n0 - args.n_off[proj], &bp_bar);
+    }
+    for (int kb = 0; kb < KB; ++kb) {
+      const int s = kb % kStages;
+      if (kb >= kStages && !mbar_wait(&empty_bar[s], ((kb / kStages) - 1) & 1)) {
+        atomicOr(&fail, 1);
+        break;
+      }
+      unsigned char* st = smem + s * S::STAGE_B;
+      mbar_expect_tx(&full_bar[s], S::A_B + S::B_B + (r > 0 ? rp * BK * 2 : 0));
+      tma_load_2d(st, &tm_x, kb * BK, m0, &full_bar[s]);
+      tma_load_2d(st + S::A_B, &tm_w, kb * BK, n0, &full_bar[s]);
+      if (r > 0) tma_load_2d(st + S::A_B + S::B_B, tm_a, kb * BK, 0, &full_bar[s]);
+    }
+  } else if (threadIdx.x == 32) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t id_main = idesc_bf16(BM, BN);
+    const uint32_t id_u = idesc_bf16(BM, rp > 0 ? rp : 16);
+    bool ok = true;
+    for (int kb = 0; kb < KB; ++kb) {
+      const int s = kb % kStages;
+      if (!mbar_wait(&full_bar[s], (kb / kStages) & 1)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      unsigned char* st = smem + s * S::STAGE_B;
+#pragma unroll
+      for (int kk = 0; kk < BK / 16; ++kk) {
+        const uint64_t ad = sw128_desc(st + kk * 32);
+        umma(tmem, ad, sw128_desc(st + S::A_B + kk * 32), id_main, (kb | kk) != 0);
+        if (r > 0) umma(tmem_u, ad, sw128_desc(st + S::A_B + S::B_B + kk * 32), id_u, (kb | kk) != 0);
+      }
+      umma_commit(&empty_bar[s]);          // frees the stage when these MMAs finish
+    }
+    if (!ok) atomicOr(&fail, 1);
+    umma_commit(&u_bar);                   // all main-loop MMAs done
+  }
+  // ---------------- (alpha/r) x A^T -> bf16 operand in shared memory ----------
+  const bool u_ok = __syncthreads_and(mbar_wait(&u_bar, 0)) != 0;   // uniform
+  tc_fence_after();
+  const int row = warp * 32 + lane;            // TMEM lane = tile row
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  if (r > 0 && u_ok) {
+    unsigned char* us = smem + S::U_OFF;
+    for (int c0 = 0; c0 < rp; c0 += 16) {
+      float v[16];
+      tmem_ld16(tmem_u + lane_base + c0, v);
+      uint32_t w[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        w[i] = pack_bf16(v[2 * i] * args.alpha_over_r, v[2 * i + 1] * args.alpha_over_r);
+      // two 16-byte chunks (k = c0 .. c0+7, c0+8 .. c0+15) of row `row`,
+      // placed at chunk index c ^ (row % 8) of the 128-byte row
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int chunk = (c0 / 8 + h) ^ (row & 7);
+        *reinterpret_cast<uint4*>(us + row * 128 + chunk * 16) =
+            make_uint4(w[4 * h], w[4 * h + 1], w[4 * h + 2], w[4 * h + 3]);
+      }
+    }
+    // ranks rp .. 63 of the operand row are never read (the MMA uses K = rp)
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  tc_fence_before();
+  __syncthreads();
+  if (!u_ok && threadIdx.x == 0) atomicOr(&fail, 1);
+  if (threadIdx.x == 32) {
+    tc_fence_after();
+    if (r > 0 && u_ok && !fail) {
+      if (mbar_wait(&bp_bar, 0)) {
+        const uint32_t id_main = idesc_bf16(BM, BN);
+        for (int kk = 0; kk < rp / 16; ++kk)
+          umma(tmem, sw128_desc(smem + S::U_OFF + kk * 32),
+               sw128_desc(smem + S::BP_OFF + kk * 32), id_main, 1);
+      } else {
+        atomicOr(&fail, 1);
+      }
+    }
+    umma_commit(&acc_bar);
+  }
+  // ---------------- epilogue: RoPE and head-major store ----------------
+  const bool acc_wait = mbar_wait(&acc_bar, 0);
+  const bool good = __syncthreads_and(acc_wait) && !*reinterpret_cast<volatile int*>(&fail);
+  tc_fence_after();
+  const int m = m0 + row;
+  const bool active = m < args.M;                     // rows past M: load, do not store
+  if (good) {
+    const int D = args.D, half = D / 2;
+    const int mm = active ? m : 0;
+    const int b = mm / args.L, l = mm % args.L;
+    const int H = proj == 0 ? args.Hq : args.Hkv;
+    const int col0 = n0 - args.n_off[proj];           // first column within projection
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(args.out[proj]);
+    const bool rope = args.rope && proj < 2;
+    const int pos = args.pos0 + (args.pos_dev ? *args.pos_dev : 0) + l;
+    for (int j = 0; j < half; j += 16) {              // 16 frequencies at a time
+      float cs[16], sn[16];
+      if (rope) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          rope_cs(pos, args.theta_hi[j + i], args.theta_lo[j + i], &cs[i], &sn[i]);
+      }
+      for (int hc = 0; hc < BN; hc += D) {            // whole heads in the tile
+        const int head = (col0 + hc) / D;
+        __nv_bfloat16* orow = out + (((int64_t)b * H + head) * args.L + l) * D;
+        float x1[16], x2[16];
+        tmem_ld16(tmem + lane_base + hc + j, x1);
+        tmem_ld16(tmem + lane_base + hc + half + j, x2);
+        if (rope) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float a = x1[i], bb = x2[i];
+            x1[i] = a * cs[i] - bb * sn[i];
+            x2[i] = bb * cs[i] + a * sn[i];
+          }
+        }
+        if (!active) continue;
+        uint32_t w1[8], w2[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          w1[i] = pack_bf16(x1[2 * i], x1[2 * i + 1]);
+          w2[i] = pack_bf16(x2[2 * i], x2[2 * i + 1]);
+        }
+        uint4* d1 = reinterpret_cast<uint4*>(orow + j);
+        uint4* d2 = reinterpret_cast<uint4*>(orow + half + j);
+        d1[0] = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+        d1[1] = make_uint4(w1[4], w1[5], w1[6], w1[7]);
+        d2[0] = make_uint4(w2[0], w2[1], w2[2], w2[3]);
+        d2[1] = make_uint4(w2[4], w2[5], w2[6], w2[7]);
+      }
+    }
+  }
+  if (threadIdx.x == 0 && !good) atomicOr(args.err, 2);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host: tensor maps through the driver entry point (no libcuda link)
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2D bf16 tensor [rows][cols] (cols contiguous), box [box_rows][64 cols],
+// 128-byte swizzle; out-of-range elements read as zero.
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult res = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS;
+}
+
+template <int BN>
+cudaError_t launch_bn(const CUtensorMap maps[8], const TcArgs& a, cudaStream_t s) {
+  const int smem = Smem<BN>::TOTAL;
+  auto kern = project_tc_kernel<BN>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid(a.n_off[3] / BN, (a.M + BM - 1) / BM);
+  kern<<<grid, kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], maps[5],
+                                    maps[6], maps[7], a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+// Tile width for these head counts, or 0 if the tensor-core path does not
+// cover the shape (then the caller uses the SIMT kernel).
+int project_tc_tile(int Hq, int Hkv, int D, int d_in) {
+  if (d_in % 64) return 0;
+  const int nq = Hq * D, nk = Hkv * D;
+  for (int bn : {256, 128}) {
+    if (bn < D) continue;
+    if (nq % bn == 0 && nk % bn == 0) return bn;
+  }
+  return 0;
+}
+
+cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void* w,
+                              const void* const a[3], const void* const bm[3], const int r[3],
+                              float alpha_over_r, int Hq, int Hkv, int D, int pos0,
+                              const int* pos_dev, float rope_base, void* const out[3], int* err,
+                              cudaStream_t s) {
+  const int bn = project_tc_tile(Hq, Hkv, D, d_in);
+  if (!bn) return cudaErrorNotSupported;
+  TcArgs t;
+  const int M = B * L;
+  for (int i = 0; i < 3; ++i) {
+    t.out[i] = out[i];
+    t.r[i] = r[i];
+    t.rp[i] = (r[i] + 15) / 16 * 16;
+  }
+  t.B = B; t.L = L; t.M = M; t.D = D; t.Hq = Hq; t.Hkv = Hkv;
+  t.n_off[0] = 0; t.n_off[1] = Hq * D; t.n_off[2] = (Hq + Hkv) * D; t.n_off[3] = (Hq + 2 * Hkv) * D;
+  t.pos0 = pos0; t.pos_dev = pos_dev; t.alpha_over_r = alpha_over_r;
+  t.rope = rope_base > 0.f; t.k_blocks = d_in / 64; t.err = err;
+  rope_theta_table(rope_base, D, t.theta_hi, t.theta_lo);
+  CUtensorMap maps[8];
+  bool ok = make_map(&maps[0], x, M, d_in, BM) &&
+            make_map(&maps[1], w, (uint64_t)t.n_off[3], d_in, bn);
+  const int dout[3] = {Hq * D, Hkv * D, Hkv * D};
+  for (int p = 0; p < 3 && ok; ++p) {
+    if (r[p] > 0) {
+      ok = make_map(&maps[2 + p], a[p], r[p], d_in, t.rp[p]) &&
+           make_map(&maps[5 + p], bm[p], dout[p], r[p], bn);
+    } else {  // unused: any valid map
+      maps[2 + p] = maps[0];
+      maps[5 + p] = maps[0];
+    }
+  }
+  if (!ok) return cudaErrorInvalidValue;
+  return bn == 256 ? launch_bn<256>(maps, t, s) : launch_bn<128>(maps, t, s);
+}
+
+}  // namespace kvq

@@ -89,7 +89,7 @@ def test_create_view_and_host_validation(kvq):
         v = kvq.kvq_cache_view(h)
         ptrs = [v.ptr[i] for i in range(kvq.NUM_PLANES) if v.ptr[i]]
         assert all(fake <= p < fake + n and p % 256 == 0 for p in ptrs)
-        assert v.dims[0][2] == 100 and v.dims[0][3] == 32 and v.elem_bytes[0] == 1
+        assert v.dims[0][2] == 128 and v.dims[0][3] == 32 and v.elem_bytes[0] == 1  # rows padded to 64
         # capacity and argument errors are caught before any launch
         with pytest.raises(kvq.KvqError) as ei:
             kvq.kvq_append_pack(h, 1 << 33, 1 << 33, 101, 0)
