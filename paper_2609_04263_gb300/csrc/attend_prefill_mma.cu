@@ -1,0 +1,296 @@
+// Causal prefill attention over the packed cache on tensor cores (bf16
+// mma.sync), Sections 3.1-3.3: the L newest queries attend to the stored
+// reconstruction of every cached token.
+//
+// One CTA = (query tile, kv head, sequence).  Its ROWS rows are the g query
+// heads of the kv head times nq = ROWS / g consecutive queries, 16 rows per
+// warp, so every key/value tile is reconstructed once and shared by all g
+// heads.  Per KV tile of NT tokens: the CTA reconstructs K and V into shared
+// memory as bf16 (codes x fp16 scale + fp16 offset; full-precision windows
+// copied), then each warp computes S = Q K^T with ldmatrix-fed m16n8k16
+// MMAs, an online softmax in the log2 domain, and O += P V (V fragments via
+// ldmatrix.trans).  Query tiles are scheduled longest-first (causal work
+// grows with the position).
+#include <math.h>
+
+#include "kvq_internal.cuh"
+
+namespace kvq {
+namespace {
+
+template <int D>
+struct PCfg {
+  static constexpr int WARPS = D == 256 ? 4 : 8;
+  static constexpr int ROWS = WARPS * 16;
+  static constexpr int NT = D == 256 ? 32 : 64;      // tokens per KV tile
+  static constexpr int LDS = D + 8;                   // smem row stride (bf16), 16 B pad
+  static constexpr int Q_OFF = 0;
+  static constexpr int K_OFF = ROWS * LDS * 2;
+  static constexpr int V_OFF = K_OFF + NT * LDS * 2;
+  static constexpr int TOTAL = V_OFF + NT * LDS * 2;
+  static constexpr int THREADS = WARPS * 32;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t r[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t r[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Reconstruct channels 8c .. 8c+7 of token t (keys: which = 0) as 8 bf16.
+__device__ __forceinline__ uint4 deq8(const Geom& g, int which, int b, int h, int t, int c,
+                                      int T, int tq) {
+  if (t >= T) return make_uint4(0, 0, 0, 0);
+  const int G = g.G, bits = which ? g.vb : g.kb;
+  const int P_CODES = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int P_SCALE = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int P_ZERO = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int P_FULL = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+  const bool raw = g.fmt == KVQ_FMT_FLOAT || (g.fmt == KVQ_FMT_KIVI && t >= tq);
+  if (raw) {
+    const int slot = g.fmt == KVQ_FMT_KIVI ? t % g.ring : t;
+    return *reinterpret_cast<const uint4*>(
+        plane_ptr<__nv_bfloat16>(g, P_FULL, b, h, slot, 8 * c));
+  }
+  const uint8_t* row = plane_ptr<uint8_t>(g, P_CODES, b, h, t);
+  uint64_t w;
+  if (bits == 4) w = *reinterpret_cast<const uint32_t*>(row + 4 * c);
+  else if (bits == 2) w = *reinterpret_cast<const uint16_t*>(row + 2 * c);
+  else w = *reinterpret_cast<const uint64_t*>(row + 8 * c);
+  const unsigned mask = (1u << bits) - 1;
+  float v[8];
+  if (g.fmt == KVQ_FMT_KIVI && which == 0) {   // per channel: scale and zero per (block, d)
+    const uint4 su = *reinterpret_cast<const uint4*>(
+        plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t / G, 8 * c));
+    const uint4 zu = *reinterpret_cast<const uint4*>(
+        plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t / G, 8 * c));
+    const __half* s8 = reinterpret_cast<const __half*>(&su);
+    const __half* z8 = reinterpret_cast<const __half*>(&zu);
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      v[e] = (float)((w >> (e * bits)) & mask) * __half2float(s8[e]) + __half2float(z8[e]);
+  } else {
+    const int grp = (8 * c) / G;
+    const float s = __half2float(*plane_ptr<__half>(g, P_SCALE, b, h, t, grp));
+    float m;
+    if (g.fmt == KVQ_FMT_SYMMETRIC) m = -(float)(1 << (bits - 1)) * s;
+    else m = __half2float(*plane_ptr<__half>(g, P_ZERO, b, h, t, grp));
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = (float)((w >> (e * bits)) & mask) * s + m;
+  }
+  return make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
+                    pack_bf16(v[6], v[7]));
+}
+
+template <int D>
+__global__ void __launch_bounds__(PCfg<D>::THREADS)
+attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, float scale,
+                          __nv_bfloat16* __restrict__ out, int nq) {
+  using C = PCfg<D>;
+  constexpr int NT = C::NT, LDS = C::LDS, NTN = NT / 8;   // n-tiles of 8 tokens
+  extern __shared__ __align__(16) unsigned char smem[];
+  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem + C::Q_OFF);
+  __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem + C::K_OFF);
+  __nv_bfloat16* Vs = reinterpret_cast<__nv_bfloat16*>(smem + C::V_OFF);
+
+  const int nqt = gridDim.x;
+  const int qtile = nqt - 1 - blockIdx.x;             // longest first
+  const int hkv = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tid = lane & 3;
+  const int grp = g.Hq / g.H;
+  const int T = cache_tokens(g);
+  const int tq = g.fmt == KVQ_FMT_KIVI ? kivi_tq(T, g.R, g.G) : T;
+  const int q0 = qtile * nq;
+  const int nql = min(nq, L - q0);
+  const int pos_first = T - L + q0;
+  const int t_end = pos_first + nql;                  // keys [0, t_end)
+
+  // queries -> shared memory (zero rows beyond the heads or queries)
+  for (int i = threadIdx.x; i < C::ROWS * (D / 8); i += C::THREADS) {
+    const int r = i / (D / 8), c = i % (D / 8);
+    const int hl = r / nq, qi = r % nq;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (hl < grp && qi < nql)
+      v = *reinterpret_cast<const uint4*>(
+          q + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D + 8 * c);
+    *reinterpret_cast<uint4*>(Qs + r * LDS + 8 * c) = v;
+  }
+  // this thread's two rows: positions (or -1 for padding rows)
+  int pos[2];
+  for (int rr = 0; rr < 2; ++rr) {
+    const int r = warp * 16 + gid + 8 * rr;
+    const int hl = r / nq, qi = r % nq;
+    pos[rr] = (hl < grp && qi < nql) ? pos_first + qi : -1;
+  }
+  const int warp_pos_max = [&] {
+    int m = -1;
+    for (int i = 0; i < 16; ++i) {
+      const int r = warp * 16 + i;
+      const int hl = r / nq, qi = r % nq;
+      if (hl < grp && qi < nql) m = max(m, pos_first + qi);
+    }
+    return m;
+  }();
+  const float c2 = scale * 1.4426950408889634f;
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[D / 8][4];
+#pragma unroll
+  for (int j = 0; j < D / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+
+  for (int t0 = 0; t0 < t_end; t0 += NT) {
+    __syncthreads();                                  // previous tile consumed
+    for (int i = threadIdx.x; i < NT * (D / 8); i += C::THREADS) {
+      const int r = i / (D / 8), c = i % (D / 8);
+      *reinterpret_cast<uint4*>(Ks + r * LDS + 8 * c) = deq8(g, 0, b, hkv, t0 + r, c, T, tq);
+      *reinterpret_cast<uint4*>(Vs + r * LDS + 8 * c) = deq8(g, 1, b, hkv, t0 + r, c, T, tq);
+    }
+    __syncthreads();
+    if (warp_pos_max < t0) continue;                  // tile entirely in this warp's future
+    // ---- S = Q K^T ----
+    float s[NTN][4];
+#pragma unroll
+    for (int j = 0; j < NTN; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+      uint32_t a[4];
+      ldsm_x4(a, Qs + (warp * 16 + (lane & 15)) * LDS + 16 * ks + (lane >> 4) * 8);
+#pragma unroll
+      for (int np = 0; np < NTN / 2; ++np) {
+        uint32_t bq[4];
+        const int j = lane >> 3, i = lane & 7;
+        ldsm_x4(bq, Ks + ((2 * np + (j >> 1)) * 8 + i) * LDS + 16 * ks + (j & 1) * 8);
+        mma16816(s[2 * np], a, bq[0], bq[1]);
+        mma16816(s[2 * np + 1], a, bq[2], bq[3]);
+      }
+    }
+    // ---- mask, online softmax ----
+    const bool diag = t0 + NT - 1 > pos_first;         // some key may be in a row's future
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int j = 0; j < NTN; ++j)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int rr = i >> 1;
+        const int t = t0 + 8 * j + 2 * tid + (i & 1);
+        float v = s[j][i] * c2;
+        if (diag && t > pos[rr]) v = -INFINITY;
+        s[j][i] = v;
+        mx[rr] = fmaxf(mx[rr], v);
+      }
+    float alpha[2];
+#pragma unroll
+    for (int rr = 0; rr < 2; ++rr) {
+      mx[rr] = fmaxf(mx[rr], __shfl_xor_sync(0xffffffffu, mx[rr], 1));
+      mx[rr] = fmaxf(mx[rr], __shfl_xor_sync(0xffffffffu, mx[rr], 2));
+      const float mn = fmaxf(m_run[rr], mx[rr]);
+      alpha[rr] = mn == -INFINITY ? 1.f : exp2f(m_run[rr] - mn);
+      m_run[rr] = mn;
+      l_run[rr] *= alpha[rr];
+    }
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j) {
+      o[j][0] *= alpha[0]; o[j][1] *= alpha[0];
+      o[j][2] *= alpha[1]; o[j][3] *= alpha[1];
+    }
+    uint32_t pa[NT / 16][4];
+#pragma unroll
+    for (int j = 0; j < NTN; ++j) {
+      float p[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float mr = m_run[i >> 1];
+        p[i] = s[j][i] == -INFINITY ? 0.f : exp2f(s[j][i] - mr);
+        l_run[i >> 1] += p[i];
+      }
+      // A fragment of k-step j/2: n-tile 2k -> a0 (row gid), a1 (row gid+8);
+      // n-tile 2k+1 -> a2, a3
+      pa[j >> 1][(j & 1) * 2 + 0] = pack_bf16(p[0], p[1]);
+      pa[j >> 1][(j & 1) * 2 + 1] = pack_bf16(p[2], p[3]);
+    }
+    // ---- O += P V ----
+#pragma unroll
+    for (int kt = 0; kt < NT / 16; ++kt) {
+#pragma unroll
+      for (int nd = 0; nd < D / 8; nd += 2) {
+        uint32_t bv[4];
+        const int j = lane >> 3, i = lane & 7;
+        ldsm_x4_t(bv, Vs + (16 * kt + (j & 1) * 8 + i) * LDS + 8 * (nd + (j >> 1)));
+        mma16816(o[nd], pa[kt], bv[0], bv[1]);
+        mma16816(o[nd + 1], pa[kt], bv[2], bv[3]);
+      }
+    }
+  }
+  // ---- normalise and store ----
+#pragma unroll
+  for (int rr = 0; rr < 2; ++rr) {
+    l_run[rr] += __shfl_xor_sync(0xffffffffu, l_run[rr], 1);
+    l_run[rr] += __shfl_xor_sync(0xffffffffu, l_run[rr], 2);
+  }
+#pragma unroll
+  for (int rr = 0; rr < 2; ++rr) {
+    const int r = warp * 16 + gid + 8 * rr;
+    const int hl = r / nq, qi = r % nq;
+    if (hl >= grp || qi >= nql) continue;
+    const float inv = 1.f / l_run[rr];
+    __nv_bfloat16* orow = out + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D;
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j)
+      *reinterpret_cast<uint32_t*>(orow + 8 * j + 2 * tid) =
+          pack_bf16(o[j][2 * rr] * inv, o[j][2 * rr + 1] * inv);
+  }
+}
+
+template <int D>
+cudaError_t launch_d(const Geom& g, const void* q, int L, float scale, void* out,
+                     cudaStream_t s) {
+  using C = PCfg<D>;
+  const int grp = g.Hq / g.H;
+  const int nq = C::ROWS / grp;
+  auto kern = attend_prefill_mma_kernel<D>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       C::TOTAL);
+  if (e != cudaSuccess) return e;
+  dim3 grid((L + nq - 1) / nq, g.H, g.B);
+  kern<<<grid, C::THREADS, C::TOTAL, s>>>(g, reinterpret_cast<const __nv_bfloat16*>(q), L, scale,
+                                          reinterpret_cast<__nv_bfloat16*>(out), nq);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool prefill_mma_supported(const Geom& g) {
+  const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC ||
+                      g.fmt == KVQ_FMT_KIVI || g.fmt == KVQ_FMT_FLOAT;
+  const int grp = g.Hq / g.H;
+  const int rows = g.D == 256 ? 64 : 128;
+  return fmt_ok && g.act == KVQ_BF16 && grp <= rows &&
+         (g.D == 64 || g.D == 128 || g.D == 256);
+}
+
+cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale, void* out,
+                               cudaStream_t s) {
+  if (g.D == 64) return launch_d<64>(g, q, L, scale, out, s);
+  if (g.D == 128) return launch_d<128>(g, q, L, scale, out, s);
+  return launch_d<256>(g, q, L, scale, out, s);
+}
+
+}  // namespace kvq

@@ -109,6 +109,10 @@ int decode_splits(const Geom& g);
 // Tensor-core split decode (attend_mma.cu): the formats it covers, and the
 // launch (partials to the workspace plane; the caller merges them).
 bool decode_mma_supported(const Geom& g);
+// Tensor-core causal prefill (attend_prefill_mma.cu).
+bool prefill_mma_supported(const Geom& g);
+cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale, void* out,
+                               cudaStream_t s);
 cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err,
                               cudaStream_t s);
 

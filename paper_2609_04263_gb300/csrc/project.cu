@@ -158,8 +158,9 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
 // rows with 16-byte loads; x (all M rows) sits in shared memory.  The
 // rank-r branch: the CTA first forms (alpha/r) x A_p^T for its projection.
 // ---------------------------------------------------------------------------
-constexpr int kSkinnyWarps = 8;
+constexpr int kSkinnyWarps = 4;      // 3 CTAs per SM: one wave for up to 456 CTAs
 constexpr int kSkinnyMaxM = 16;
+constexpr int kSkinnyKIter = 8;      // 16-byte loads per row per lane in flight (2048 bf16)
 
 template <typename T>
 __device__ __forceinline__ void load8f(const T* p, float f[8]);
@@ -181,8 +182,36 @@ __device__ __forceinline__ void load8f<float>(const float* p, float f[8]) {
   f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
 }
 
-template <typename T, int MM>
-__global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjArgs p) {
+// Raw 8-element vector of activation type T (kept packed until used).
+template <typename T> struct Raw8;
+template <> struct Raw8<__nv_bfloat16> {
+  uint4 u;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) {
+    u = __ldg(reinterpret_cast<const uint4*>(p));
+  }
+  __device__ __forceinline__ void to_float(float f[8]) const {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 t = __bfloat1622float2(h[i]);
+      f[2 * i] = t.x;
+      f[2 * i + 1] = t.y;
+    }
+  }
+};
+template <> struct Raw8<float> {
+  float4 a, b;
+  __device__ __forceinline__ void load(const float* p) {
+    a = __ldg(reinterpret_cast<const float4*>(p));
+    b = __ldg(reinterpret_cast<const float4*>(p) + 1);
+  }
+  __device__ __forceinline__ void to_float(float f[8]) const {
+    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+  }
+};
+
+template <typename T, int MM, int KITER>
+__global__ void __launch_bounds__(kSkinnyWarps * 32, 3) project_skinny_kernel(ProjArgs p) {
   extern __shared__ float xsm[];             // [M][d_in] fp32, then U [M][64]
   const int M = p.B * p.L, D = p.D, K = p.d_in;
   const int half = D / 2;
@@ -195,29 +224,64 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
   const int r = p.r[proj];
   float* U = xsm + M * K;
   const T* x = reinterpret_cast<const T*>(p.x);
-  for (int i = threadIdx.x * 8; i < M * K; i += blockDim.x * 8) {
-    float f[8];
-    load8f<T>(x + i, f);
+  const int c = (pair0 + warp) % pairs_per_head;    // channel within the first half
+  const int n1 = hh * D + c, n2 = n1 + half;
+  const T* W = reinterpret_cast<const T*>(p.w);
+  const T* w1 = W + (int64_t)n1 * K;
+  const T* w2 = W + (int64_t)n2 * K;
+  // x -> shared memory (fp32): every thread issues all its loads, then stores
+  {
+    constexpr int XL = 8;                           // 16-byte loads per thread per round
+    for (int base = threadIdx.x * 8; base < M * K; base += blockDim.x * 8 * XL) {
+      Raw8<T> xv[XL];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) xsm[i + j] = f[j];
+      for (int u = 0; u < XL; ++u) {
+        const int i = base + u * blockDim.x * 8;
+        if (i < M * K) xv[u].load(x + i);
+      }
+#pragma unroll
+      for (int u = 0; u < XL; ++u) {
+        const int i = base + u * blockDim.x * 8;
+        if (i < M * K) {
+          float f[8];
+          xv[u].to_float(f);
+          *reinterpret_cast<float4*>(xsm + i) = make_float4(f[0], f[1], f[2], f[3]);
+          *reinterpret_cast<float4*>(xsm + i + 4) = make_float4(f[4], f[5], f[6], f[7]);
+        }
+      }
+    }
   }
   __syncthreads();
-  // (alpha/r) x A_p^T: warp w takes ranks w, w + 8, ...
+  // x A_p^T, one warp per rank: the row's 16-byte loads are all in flight
+  // (passes of KITER x 256 channels), then M dot products reduced by shuffles.
   if (r > 0) {
     const T* A = reinterpret_cast<const T*>(p.a[proj]);
     for (int j = warp; j < r; j += kSkinnyWarps) {
       float acc[MM];
 #pragma unroll
       for (int m = 0; m < MM; ++m) acc[m] = 0.f;
-      for (int k = lane * 8; k < K; k += 256) {
-        float a[8];
-        load8f<T>(A + (int64_t)j * K + k, a);
+      for (int kp = 0; kp < K; kp += KITER * 256) {
+        Raw8<T> av[KITER];
 #pragma unroll
-        for (int m = 0; m < MM; ++m) {
-          if (m < M) {
-            const float* xr = xsm + m * K + k;
+        for (int u = 0; u < KITER; ++u) {
+          const int k = kp + lane * 8 + u * 256;
+          if (k < K) av[u].load(A + (int64_t)j * K + k);
+        }
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc[m] += a[e] * xr[e];
+        for (int u = 0; u < KITER; ++u) {
+          const int k = kp + lane * 8 + u * 256;
+          if (k < K) {
+            float a[8];
+            av[u].to_float(a);
+#pragma unroll
+            for (int m = 0; m < MM; ++m) {
+              if (m < M) {
+                const float4* xr4 = reinterpret_cast<const float4*>(xsm + m * K + k);
+                const float4 xa = xr4[0], xb = xr4[1];
+                acc[m] += a[0] * xa.x + a[1] * xa.y + a[2] * xa.z + a[3] * xa.w +
+                          a[4] * xb.x + a[5] * xb.y + a[6] * xb.z + a[7] * xb.w;
+              }
+            }
           }
         }
       }
@@ -225,49 +289,47 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
       for (int m = 0; m < MM; ++m) {
         float v = acc[m];
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        if (lane == 0 && m < M) U[m * 64 + j] = v * p.alpha_over_r;
+        if (lane == 0 && m < M) U[m * 64 + j] = v;
       }
     }
   }
-  __syncthreads();
-  const int c = (pair0 + warp) % pairs_per_head;    // channel within the first half
-  const int n1 = hh * D + c, n2 = n1 + half;
-  const T* W = reinterpret_cast<const T*>(p.w);
-  const T* w1 = W + (int64_t)n1 * K;
-  const T* w2 = W + (int64_t)n2 * K;
+  // this warp's weight rows in passes of KITER x 256 channels: KITER 8-element
+  // loads per row per lane in flight together (the bulk of the bytes)
   float acc1[MM], acc2[MM];
 #pragma unroll
   for (int m = 0; m < MM; ++m) { acc1[m] = 0.f; acc2[m] = 0.f; }
-  constexpr int kUnroll = 4;
-  for (int k0 = lane * 8; k0 < K; k0 += 256 * kUnroll) {
-    float a[kUnroll][8], b[kUnroll][8];
+  for (int kp = 0; kp < K; kp += KITER * 256) {
+  Raw8<T> wa[KITER], wb[KITER];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int k = k0 + u * 256;
-      if (k < K) {
-        load8f<T>(w1 + k, a[u]);
-        load8f<T>(w2 + k, b[u]);
-      }
+  for (int u = 0; u < KITER; ++u) {
+    const int k = kp + lane * 8 + u * 256;
+    if (k < K) {
+      wa[u].load(w1 + k);
+      wb[u].load(w2 + k);
     }
+  }
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int k = k0 + u * 256;
-      if (k < K) {
+  for (int u = 0; u < KITER; ++u) {
+    const int k = kp + lane * 8 + u * 256;
+    if (k < K) {
+      float a[8], bq[8];
+      wa[u].to_float(a);
+      wb[u].to_float(bq);
 #pragma unroll
-        for (int m = 0; m < MM; ++m) {
-          if (m < M) {
-            const float4* xr4 = reinterpret_cast<const float4*>(xsm + m * K + k);
-            const float4 xa = xr4[0], xb = xr4[1];
-            const float xr[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+      for (int m = 0; m < MM; ++m) {
+        if (m < M) {
+          const float4* xr4 = reinterpret_cast<const float4*>(xsm + m * K + k);
+          const float4 xa = xr4[0], xb = xr4[1];
+          const float xr[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              acc1[m] += a[u][e] * xr[e];
-              acc2[m] += b[u][e] * xr[e];
-            }
+          for (int e = 0; e < 8; ++e) {
+            acc1[m] += a[e] * xr[e];
+            acc2[m] += bq[e] * xr[e];
           }
         }
       }
     }
+  }
   }
 #pragma unroll
   for (int m = 0; m < MM; ++m) {
@@ -276,6 +338,7 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
       acc2[m] += __shfl_xor_sync(0xffffffffu, acc2[m], o);
     }
   }
+  __syncthreads();                                  // U complete
   // rank-r up projection, RoPE, head-major store: lane m handles row m
   if (lane < M) {
     float y1 = 0.f, y2 = 0.f;
@@ -284,11 +347,18 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
       if (m == lane) { y1 = acc1[m]; y2 = acc2[m]; }
     if (r > 0) {
       const T* Bm = reinterpret_cast<const T*>(p.bm[proj]);
-      const int64_t b1 = ((int64_t)head * D + c) * r, b2 = ((int64_t)head * D + c + half) * r;
-      for (int j = 0; j < r; ++j) {
-        const float u = U[lane * 64 + j];
-        y1 += u * ld_act(Bm, b1 + j, p.act);
-        y2 += u * ld_act(Bm, b2 + j, p.act);
+      const T* b1 = Bm + ((int64_t)head * D + c) * r;
+      const T* b2 = Bm + ((int64_t)head * D + c + half) * r;
+      for (int j0 = 0; j0 < r; j0 += 8) {          // r is a multiple of 8
+        float f1[8], f2[8];
+        load8f<T>(b1 + j0, f1);
+        load8f<T>(b2 + j0, f2);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float uu = U[lane * 64 + j0 + e] * p.alpha_over_r;
+          y1 += uu * f1[e];
+          y2 += uu * f2[e];
+        }
       }
     }
     const int b = lane / p.L, l = lane % p.L;
@@ -300,19 +370,192 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32) project_skinny_kernel(ProjA
       y1 = o1;
       y2 = o2;
     }
-    const int H = proj == 0 ? p.Hq : proj == 1 ? p.Hkv : p.Hkv;
+    const int H = proj == 0 ? p.Hq : p.Hkv;
     const int64_t base = (((int64_t)b * H + head) * p.L + l) * D;
     st_act(p.out[proj], base + c, y1, p.act);
     st_act(p.out[proj], base + c + half, y2, p.act);
   }
 }
 
+// ---------------------------------------------------------------------------
+// Few rows (M = B * L <= 16, the decode step), bf16: weight streaming on
+// mma.sync.  One CTA per RoPE pair-tile: weight rows hD + c0 + i and their
+// partners hD + D/2 + c0 + i (i < 8) of one head, plus the rank rows of A_p.
+// x is the MMA's A operand (tokens as rows, zero-padded to 16); weight rows
+// are B operands (n = 8 rows).  Within each 32-channel chunk the MMA k index
+// is permuted so that a thread's operand is one 16-byte load: thread t holds
+// channels 8t .. 8t+7, words 2s and 2s+1 feed k-step s.  The 8 warps split
+// the channels; partial tiles are summed through shared memory, then the
+// rank-r up-projection, RoPE and the head-major store follow.
+// ---------------------------------------------------------------------------
+constexpr int kDecWarps = 8;
+constexpr int kDecMaxNt = 2 + 8;          // 2 weight tiles + up to 64 ranks / 8
+
+__device__ __forceinline__ void mma16816_p(float c[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                           uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+template <int M16, int NT>   // M16: x rows held (8 or 16); NT: 2 + rank tiles
+__global__ void __launch_bounds__(kDecWarps * 32)
+project_decode_mma_kernel(ProjArgs p) {
+  extern __shared__ __align__(16) unsigned char dsm[];
+  const int M = p.B * p.L, D = p.D, K = p.d_in;
+  const int half = D / 2;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tid = lane & 3;
+  const int tiles_per_head = half / 8;
+  const int hh = blockIdx.x / tiles_per_head;               // stacked head index
+  const int c0 = (blockIdx.x % tiles_per_head) * 8;
+  const int proj = hh < p.Hq ? 0 : hh < p.Hq + p.Hkv ? 1 : 2;
+  const int head = proj == 0 ? hh : proj == 1 ? hh - p.Hq : hh - p.Hq - p.Hkv;
+  const int r = p.r[proj];
+  const int nt_used = 2 + r / 8;                            // r is a multiple of 8
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(dsm);   // [M16][K]
+  float* red = reinterpret_cast<float*>(dsm + (size_t)M16 * K * 2);   // [warps][NT][32][4]
+  float* fin = red + kDecWarps * NT * 128;                  // [NT][16 m][8 n]
+  const __nv_bfloat16* x = reinterpret_cast<const __nv_bfloat16*>(p.x);
+  const __nv_bfloat16* W = reinterpret_cast<const __nv_bfloat16*>(p.w);
+  const __nv_bfloat16* A = reinterpret_cast<const __nv_bfloat16*>(p.a[proj]);
+
+  // x -> shared memory (rows >= M zero)
+  for (int i = threadIdx.x * 8; i < M16 * K; i += blockDim.x * 8) {
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (i < M * K) v = __ldg(reinterpret_cast<const uint4*>(x + i));
+    *reinterpret_cast<uint4*>(xs + i) = v;
+  }
+  // B-operand row pointers of this thread (row gid of each n-tile)
+  const __nv_bfloat16* brow[NT];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    if (nt == 0) brow[nt] = W + ((int64_t)hh * D + c0 + gid) * K;
+    else if (nt == 1) brow[nt] = W + ((int64_t)hh * D + half + c0 + gid) * K;
+    else brow[nt] = A + (int64_t)((nt - 2) * 8 + gid) * K;   // valid only for nt < nt_used
+  }
+  __syncthreads();
+  float acc[NT][4];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+  const int chunks = K / 32;
+  const int per = (chunks + kDecWarps - 1) / kDecWarps;
+  const int ch0 = warp * per, ch1 = min(chunks, ch0 + per);
+  constexpr int U = 4;                                       // chunks in flight per pass
+  for (int cb = ch0; cb < ch1; cb += U) {
+    uint4 bw[U][NT];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+        if (cb + u < ch1 && nt < nt_used)
+          bw[u][nt] = __ldg(reinterpret_cast<const uint4*>(brow[nt] + (cb + u) * 32 + 8 * tid));
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (cb + u >= ch1) break;
+      const int k = (cb + u) * 32 + 8 * tid;
+      const uint4 xa = *reinterpret_cast<const uint4*>(xs + gid * K + k);
+      uint4 xb = make_uint4(0, 0, 0, 0);
+      if (M16 == 16) xb = *reinterpret_cast<const uint4*>(xs + (gid + 8) * K + k);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        if (nt < nt_used) {
+          mma16816_p(acc[nt], xa.x, xb.x, xa.y, xb.y, bw[u][nt].x, bw[u][nt].y);
+          mma16816_p(acc[nt], xa.z, xb.z, xa.w, xb.w, bw[u][nt].z, bw[u][nt].w);
+        }
+      }
+    }
+  }
+  // sum the warps' partial tiles: fragment element i of lane -> (m, n)
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt)
+    *reinterpret_cast<float4*>(red + ((warp * NT + nt) * 32 + lane) * 4) =
+        make_float4(acc[nt][0], acc[nt][1], acc[nt][2], acc[nt][3]);
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < nt_used * 128; idx += blockDim.x) {
+    const int nt = idx / 128, e = idx % 128, ln = e / 4, i = e % 4;
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kDecWarps; ++w) sum += red[((w * NT + nt) * 32 + ln) * 4 + i];
+    const int m = (ln >> 2) + 8 * (i >> 1), n = 2 * (ln & 3) + (i & 1);
+    fin[(nt * 16 + m) * 8 + n] = sum;
+  }
+  __syncthreads();
+  // (alpha/r) (x A^T) B^T, RoPE, store: thread per (row m, channel i)
+  const int m = threadIdx.x >> 3, i = threadIdx.x & 7;
+  if (m < M) {
+    float y1 = fin[(0 * 16 + m) * 8 + i], y2 = fin[(1 * 16 + m) * 8 + i];
+    if (r > 0) {
+      const __nv_bfloat16* Bm = reinterpret_cast<const __nv_bfloat16*>(p.bm[proj]);
+      const __nv_bfloat16* b1 = Bm + ((int64_t)head * D + c0 + i) * r;
+      const __nv_bfloat16* b2 = Bm + ((int64_t)head * D + half + c0 + i) * r;
+      for (int j0 = 0; j0 < r; j0 += 8) {
+        const uint4 u1 = __ldg(reinterpret_cast<const uint4*>(b1 + j0));
+        const uint4 u2 = __ldg(reinterpret_cast<const uint4*>(b2 + j0));
+        const __nv_bfloat16* e1 = reinterpret_cast<const __nv_bfloat16*>(&u1);
+        const __nv_bfloat16* e2 = reinterpret_cast<const __nv_bfloat16*>(&u2);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const int j = j0 + e;
+          const float uu = fin[((2 + j / 8) * 16 + m) * 8 + (j & 7)] * p.alpha_over_r;
+          y1 += uu * __bfloat162float(e1[e]);
+          y2 += uu * __bfloat162float(e2[e]);
+        }
+      }
+    }
+    const int b = m / p.L, l = m % p.L;
+    const int c = c0 + i;
+    if (proj < 2 && p.rope_base > 0.f) {
+      const int pos = p.pos0 + (p.pos_dev ? *p.pos_dev : 0) + l;
+      float cs, sn;
+      rope_cos_sin(pos, p.theta_hi[c], p.theta_lo[c], &cs, &sn);
+      const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
+      y1 = o1;
+      y2 = o2;
+    }
+    const int H = proj == 0 ? p.Hq : p.Hkv;
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[proj]);
+    const int64_t base = (((int64_t)b * H + head) * p.L + l) * D;
+    out[base + c] = __float2bfloat16_rn(y1);
+    out[base + c + half] = __float2bfloat16_rn(y2);
+  }
+}
+
+template <int M16, int NT>
+cudaError_t launch_decode_mma_nt(const ProjArgs& p, cudaStream_t s) {
+  const size_t sm = (size_t)M16 * p.d_in * 2 + (size_t)kDecWarps * NT * 128 * 4 +
+                    (size_t)NT * 128 * 4;
+  auto kern = project_decode_mma_kernel<M16, NT>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  const int tiles = (p.Hq + 2 * p.Hkv) * (p.D / 16);
+  kern<<<tiles, kDecWarps * 32, sm, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_mma(const ProjArgs& p, cudaStream_t s) {
+  const int M = p.B * p.L;
+  const int rmax = max(p.r[0], max(p.r[1], p.r[2]));
+  const int nt = 2 + rmax / 8;
+  if (M <= 8) {
+    if (nt <= 4) return launch_decode_mma_nt<8, 4>(p, s);
+    return launch_decode_mma_nt<8, kDecMaxNt>(p, s);
+  }
+  if (nt <= 4) return launch_decode_mma_nt<16, 4>(p, s);
+  return launch_decode_mma_nt<16, kDecMaxNt>(p, s);
+}
+
 template <typename T>
 cudaError_t launch_skinny(const ProjArgs& p, cudaStream_t s) {
   const int M = p.B * p.L;
   const int pairs = (p.Hq + 2 * p.Hkv) * p.D / 2;
-  const size_t sm = ((size_t)M * p.d_in + (size_t)M * 64) * sizeof(float);
-  auto kern = M <= 4 ? project_skinny_kernel<T, 4> : project_skinny_kernel<T, kSkinnyMaxM>;
+  const size_t sm = ((size_t)M * p.d_in + (size_t)kSkinnyMaxM * 64) * sizeof(float);
+  // fp32 weights take twice the registers: half the loads per pass
+  constexpr int KI = sizeof(T) == 2 ? kSkinnyKIter : kSkinnyKIter / 2;
+  auto kern = M <= 4 ? project_skinny_kernel<T, 4, KI>
+            : M <= 8 ? project_skinny_kernel<T, 8, KI> : project_skinny_kernel<T, kSkinnyMaxM, KI>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   kern<<<pairs / kSkinnyWarps, kSkinnyWarps * 32, sm, s>>>(p);
@@ -350,7 +593,9 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
     if (e != cudaErrorNotSupported) return e;
     (void)cudaGetLastError();
   }
-  if (M <= kSkinnyMaxM && (size_t)M * d_in * 4 <= 160 * 1024 && d_in % 8 == 0)
+  if (act == KVQ_BF16 && M <= 16 && d_in % 32 == 0 && (size_t)16 * d_in * 2 <= 160 * 1024)
+    return launch_decode_mma(p, s);
+  if (M <= kSkinnyMaxM && (size_t)M * d_in * 4 <= 120 * 1024 && d_in % 64 == 0)
     return act == KVQ_BF16 ? launch_skinny<__nv_bfloat16>(p, s) : launch_skinny<float>(p, s);
   const size_t sm = (size_t)(kMT * (kKC + 1) + 256 * (kKC + 1) + kMT * 64 + kMT * D) *
                     sizeof(float);

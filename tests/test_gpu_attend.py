@@ -84,6 +84,9 @@ PREFILL = [
     ("kivi_r0", "bf16", 1, 1, 4, 64, [0], 70),
     ("kvarn", "bf16", 1, 2, 4, 256, [100], 200),
     ("kvarn_small", "bf16", 1, 2, 2, 64, [0], 150),
+    ("affine4", "bf16", 1, 1, 16, 64, [0], 130),     # GQA 16: 8 queries per CTA
+    ("sym4", "bf16", 2, 1, 6, 128, [37], 90),        # group 6 does not divide the rows
+    ("affine4", "bf16", 1, 1, 2, 256, [50], 333),
 ]
 
 
