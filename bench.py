@@ -134,6 +134,7 @@ class Runner:
         self.o_dec = e(B, Hq, 1, D)
         self.graph = None
         self.events = None
+        self.eager = False
 
     # one layer's calls ----------------------------------------------------
     def _project(self, l, x, out):
@@ -208,7 +209,10 @@ class Runner:
     def decode(self):
         for s in range(self.wl.decode):
             self.xs.copy_(self.x_dec[s])
-            self.graph.replay()
+            if self.eager:
+                self.decode_step_eager()
+            else:
+                self.graph.replay()
 
     def job(self, phase_events=None):
         self.reset()
@@ -436,6 +440,15 @@ def main():
     ap.add_argument("--impl", default="kvq", choices=["kvq", "reference"])
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    # smaller runs for profiler launch lists (not for reported numbers)
+    ap.add_argument("--decode-steps", type=int, default=None,
+                    help="decode steps per job (default: the workload's)")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="attention layers (default: the workload's)")
+    ap.add_argument("--eager-decode", action="store_true",
+                    help="launch decode steps directly instead of replaying a graph")
+    ap.add_argument("--timed-only", action="store_true",
+                    help="skip the per-kernel, end-to-end and CPU passes")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":
@@ -450,9 +463,16 @@ def main():
     device = f"cuda:{local}"
     torch.cuda.set_device(device)
     wl = synth.WORKLOADS[args.workload]
+    import dataclasses
+    if args.decode_steps is not None:
+        wl = dataclasses.replace(wl, decode=args.decode_steps)
+    if args.layers is not None:
+        wl = dataclasses.replace(wl, layers=args.layers)
     peaks, peak_kind = load_peaks()
     run = Runner(wl, device)
-    run.capture()
+    run.eager = args.eager_decode
+    if not run.eager:
+        run.capture()
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=device)
 
     for _ in range(max(args.warmup, 3)):
@@ -480,6 +500,13 @@ def main():
     tokens_per_step = wl.batch * (wl.prefill + wl.decode)
     value = world * tokens_per_step * args.steps / total_s
     decode_tps = wl.batch * wl.decode / (statistics.mean(dec_ms) / 1000.0)
+
+    if args.timed_only:
+        if rank == 0:
+            print(json.dumps({"timed_only": True, "ms_per_step": statistics.mean(step_ms),
+                              "workload": wl.name, "decode": wl.decode,
+                              "eager_decode": run.eager}), flush=True)
+        return
 
     # ---- per-kernel durations ---------------------------------------------
     # Prefill kernels run for milliseconds: CUDA events around each eager

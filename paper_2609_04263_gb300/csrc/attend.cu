@@ -266,10 +266,7 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
   if (decode && decode_mma_supported(g)) {
     int* err = device_error_word();
     if (!err) return cudaErrorInvalidDevice;
-    cudaError_t e = launch_decode_mma(g, q, scale, err, s);
-    if (e != cudaSuccess) return e;
-    combine_kernel<<<dim3(g.Hq, g.B), 64, 0, s>>>(g, g.splits, out);
-    return cudaGetLastError();
+    return launch_decode_mma(g, q, scale, err, out, s);
   }
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));

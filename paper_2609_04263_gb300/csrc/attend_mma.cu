@@ -1,6 +1,9 @@
 // Split-K flash-decode over the packed cache on tensor cores (bf16 mma.sync).
 //
-// One CTA = (split of the tokens, kv head, sequence); 4 warps.  The split's
+// One CTA = (split of the tokens, kv head, sequence); 4 warps.  Each CTA
+// writes its split's partial (m, l, o) to the workspace; the last CTA of a
+// (sequence, kv head) to finish (an arrival counter, no waiting) merges them
+// by log-sum-exp into the output.  The split's
 // tokens stream through shared memory in 64-token chunks: one thread issues
 // TMA bulk copies (codes and fp16 metadata of the chunk) on an mbarrier ring
 // of kStages buffers; each warp then takes one 16-token tile of the chunk.
@@ -111,12 +114,14 @@ struct Cfg {
 
 template <int D, int BITS, int FMT>
 __global__ void __launch_bounds__(kWarps * 32)
-attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err) {
+attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err,
+                         __nv_bfloat16* __restrict__ out) {
   using C = Cfg<D, BITS, FMT>;
   constexpr int NG = C::NG, KSTEP = C::KSTEP, NT_PV = C::NT_PV;
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint64_t full_bar[kStages];
   __shared__ float red_m[kWarps][16], red_l[kWarps][16];
+  __shared__ int last_cta;
 
   const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -523,10 +528,59 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
                  (((int64_t)b * g.Hq + hkv * grp + row) * kMaxSplits + split) * (D + kWsStride);
     wsr[c] = val;
   }
+  // ---- the last split CTA of this (sequence, kv head) merges all splits ----
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned prev = atomicAdd(&g.counters[b * g.H + hkv], 1u);
+    last_cta = prev == (unsigned)g.splits - 1;
+  }
+  __syncthreads();
+  if (!last_cta) return;
+  __threadfence();
+  const float* wbase = reinterpret_cast<const float*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
+                       ((int64_t)b * g.Hq + hkv * grp) * kMaxSplits * (D + kWsStride);
+  // per row: split weights exp(m_s - M) / sum_s exp(m_s - M) l_s in shared
+  // memory (reusing the pipeline buffers), then each output sums over splits
+  // with 8 independent loads in flight
+  float* fw = reinterpret_cast<float*>(smem);          // [16][kMaxSplits]
+  const int S = g.splits;
+  for (int row = warp; row < grp; row += kWarps) {
+    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride);
+    const float m = lane < S ? __ldcg(w + lane * (D + kWsStride)) : -INFINITY;
+    const float l = lane < S ? __ldcg(w + lane * (D + kWsStride) + 1) : 0.f;
+    float M = m;
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float f = m == -INFINITY ? 0.f : expf(m - M);
+    float L = f * l;
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (lane < kMaxSplits) fw[row * kMaxSplits + lane] = L > 0.f ? f / L : 0.f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < grp * (D / 2); i += blockDim.x) {
+    const int row = i / (D / 2), d = 2 * (i % (D / 2));
+    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride) + 2 + d;
+    float2 v[kMaxSplits];
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp)
+      v[sp] = sp < S ? __ldcg(reinterpret_cast<const float2*>(w + sp * (D + kWsStride)))
+                     : make_float2(0.f, 0.f);
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp) {
+      const float f = sp < S ? fw[row * kMaxSplits + sp] : 0.f;
+      a0 += f * v[sp].x;
+      a1 += f * v[sp].y;
+    }
+    *reinterpret_cast<__nv_bfloat162*>(out + ((int64_t)b * g.Hq + hkv * grp + row) * D + d) =
+        __floats2bfloat162_rn(a0, a1);
+  }
+  if (threadIdx.x == 0) g.counters[b * g.H + hkv] = 0;   // ready for the next call
 }
 
 template <int D, int BITS, int FMT>
-cudaError_t launch_one(const Geom& g, const void* q, float scale, int* err, cudaStream_t s) {
+cudaError_t launch_one(const Geom& g, const void* q, float scale, int* err, void* out,
+                       cudaStream_t s) {
   using C = Cfg<D, BITS, FMT>;
   const size_t sm_pipe = (size_t)kStages * C::STAGE_B;
   const size_t sm_out = (size_t)kWarps * 16 * D * sizeof(float);
@@ -535,16 +589,19 @@ cudaError_t launch_one(const Geom& g, const void* q, float scale, int* err, cuda
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   kern<<<dim3(g.splits, g.H, g.B), kWarps * 32, sm, s>>>(
-      g, reinterpret_cast<const __nv_bfloat16*>(q), scale, err);
+      g, reinterpret_cast<const __nv_bfloat16*>(q), scale, err,
+      reinterpret_cast<__nv_bfloat16*>(out));
   return cudaGetLastError();
 }
 
 template <int D, int BITS>
-cudaError_t launch_fmt(const Geom& g, const void* q, float scale, int* err, cudaStream_t s) {
+cudaError_t launch_fmt(const Geom& g, const void* q, float scale, int* err, void* out,
+                       cudaStream_t s) {
   switch (g.fmt) {
-    case KVQ_FMT_AFFINE: return launch_one<D, BITS, KVQ_FMT_AFFINE>(g, q, scale, err, s);
-    case KVQ_FMT_SYMMETRIC: return launch_one<D, BITS, KVQ_FMT_SYMMETRIC>(g, q, scale, err, s);
-    case KVQ_FMT_KIVI: return launch_one<D, BITS, KVQ_FMT_KIVI>(g, q, scale, err, s);
+    case KVQ_FMT_AFFINE: return launch_one<D, BITS, KVQ_FMT_AFFINE>(g, q, scale, err, out, s);
+    case KVQ_FMT_SYMMETRIC:
+      return launch_one<D, BITS, KVQ_FMT_SYMMETRIC>(g, q, scale, err, out, s);
+    case KVQ_FMT_KIVI: return launch_one<D, BITS, KVQ_FMT_KIVI>(g, q, scale, err, out, s);
   }
   return cudaErrorNotSupported;
 }
@@ -557,12 +614,12 @@ bool decode_mma_supported(const Geom& g) {
          (g.D == 64 || g.D == 128) && g.Hq / g.H <= 16;
 }
 
-cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err,
+cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err, void* out,
                               cudaStream_t s) {
-  if (g.D == 64) return g.kb == 4 ? launch_fmt<64, 4>(g, q, scale, err, s)
-                                  : launch_fmt<64, 2>(g, q, scale, err, s);
-  return g.kb == 4 ? launch_fmt<128, 4>(g, q, scale, err, s)
-                   : launch_fmt<128, 2>(g, q, scale, err, s);
+  if (g.D == 64) return g.kb == 4 ? launch_fmt<64, 4>(g, q, scale, err, out, s)
+                                  : launch_fmt<64, 2>(g, q, scale, err, out, s);
+  return g.kb == 4 ? launch_fmt<128, 4>(g, q, scale, err, out, s)
+                   : launch_fmt<128, 2>(g, q, scale, err, out, s);
 }
 
 }  // namespace kvq

@@ -160,7 +160,7 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     }
   }
   g->splits = decode_splits(*g);
-  size_t total = sizeof(CacheState);   // device state block at offset 0
+  size_t total = state_region_bytes(B, H);   // device state + split counters at offset 0
   static_assert(sizeof(CacheState) == 256, "state block is 256 bytes");
   for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
     off[i] = 0;
@@ -209,7 +209,7 @@ int* device_error_word() {
 // (stream-ordered, so it can be captured with the calls that follow).
 cudaError_t ensure_cache_init(kvq_cache* c, cudaStream_t s) {
   if (!c->need_init) return cudaSuccess;
-  cudaError_t e = cudaMemsetAsync(c->g.state, 0, sizeof(CacheState), s);
+  cudaError_t e = cudaMemsetAsync(c->g.state, 0, state_region_bytes(c->g.B, c->g.H), s);
   if (e == cudaSuccess) c->need_init = false;
   return e;
 }
@@ -268,6 +268,7 @@ kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t by
   c->T = 0;
   c->need_init = true;
   c->g.state = reinterpret_cast<CacheState*>(c->base);
+  c->g.counters = reinterpret_cast<uint32_t*>(c->base + sizeof(CacheState));
   for (int i = 0; i < KVQ_NUM_PLANES; ++i)
     c->g.pl[i].p = c->g.pl[i].rows ? c->base + off[i] : nullptr;
   *out = c;

@@ -43,6 +43,7 @@ struct Geom {
   int32_t ring;          // KIVI: R + G residual slots
   int32_t splits;        // decode split-K width (fixed per cache)
   CacheState* state;
+  uint32_t* counters;    // [B][Hkv] split arrival counters (zeroed with the state)
   Plane pl[KVQ_NUM_PLANES];
 };
 
@@ -113,7 +114,7 @@ bool decode_mma_supported(const Geom& g);
 bool prefill_mma_supported(const Geom& g);
 cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale, void* out,
                                cudaStream_t s);
-cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err,
+cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err, void* out,
                               cudaStream_t s);
 
 // Token range of split `s` of `splits` over T tokens (tiles of `tile`).
@@ -159,6 +160,12 @@ __device__ __forceinline__ int cache_tokens(const Geom& g) {
 
 // Device address of the library's error word (set up once per device).
 int* device_error_word();
+
+// Bytes of the device state region at the start of a cache buffer: the
+// CacheState block, then one split arrival counter per (sequence, kv head).
+inline size_t state_region_bytes(int B, int H) {
+  return sizeof(CacheState) + (((size_t)B * H * 4 + 255) & ~size_t(255));
+}
 
 // Floats of split-K partials a decode over this geometry addresses:
 // [B][Hq][kMaxSplits][D + kWsStride].
