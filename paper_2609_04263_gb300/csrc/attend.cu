@@ -122,6 +122,8 @@ __device__ void dequant_tile(const Geom& g, int which, int b, int h, int t0, int
 __global__ void __launch_bounds__(kThreads)
 attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
                       int nq, int splits, int decode, float inv_sqrt_d) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   const int T = cache_tokens(g);
   const int D = g.D, grp = g.Hq / g.H;
@@ -231,6 +233,8 @@ attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
 // Merge the split partials of one (b, q head): o = sum_s e^(m_s - M) o_s /
 // sum_s e^(m_s - M) l_s.
 __global__ void combine_kernel(Geom g, int splits, void* out) {
+  pdl_wait();
+  pdl_trigger();
   const int hq = blockIdx.x, b = blockIdx.y;
   const int D = g.D;
   const float* w = ws_row(g, b, hq);
@@ -289,11 +293,11 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
   if (e != cudaSuccess) return e;
   const int nqt = (L + nq - 1) / nq;
   dim3 grid(nqt * splits, g.H, g.B);
-  attend_generic_kernel<<<grid, kThreads, sm, s>>>(g, q, L, scale, out, nq, splits,
+  launch_pdl(attend_generic_kernel, dim3(grid), dim3(kThreads), sm, s, g, q, L, scale, out, nq, splits,
                                                    decode ? 1 : 0, inv_sqrt_d);
   e = cudaGetLastError();
   if (e != cudaSuccess || !decode) return e;
-  combine_kernel<<<dim3(g.Hq, g.B), 64, 0, s>>>(g, splits, out);
+  launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, splits, out);
   return cudaGetLastError();
 }
 

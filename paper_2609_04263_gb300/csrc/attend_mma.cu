@@ -79,6 +79,25 @@ __device__ __forceinline__ uint32_t magic2(uint32_t x, uint32_t mask) {
   asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "r"(mask), "r"(kMagic));
   return r;
 }
+// (x & mask) | 0x64006400: two codes as fp16 (1024 + c)
+constexpr uint32_t kMagicH = 0x64006400u;
+__device__ __forceinline__ uint32_t magic2h(uint32_t x, uint32_t mask) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "r"(mask), "r"(kMagicH));
+  return r;
+}
+__device__ __forceinline__ void mma16816_f16(float c[4], const uint32_t a[4], uint32_t b0,
+                                             uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -116,6 +135,8 @@ template <int D, int BITS, int FMT>
 __global__ void __launch_bounds__(kWarps * 32)
 attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err,
                          __nv_bfloat16* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   using C = Cfg<D, BITS, FMT>;
   constexpr int NG = C::NG, KSTEP = C::KSTEP, NT_PV = C::NT_PV;
   extern __shared__ __align__(128) unsigned char smem[];
@@ -157,7 +178,9 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
       qsum[gq][r] += __shfl_xor_sync(0xffffffffu, qsum[gq][r], 1);
       qsum[gq][r] += __shfl_xor_sync(0xffffffffu, qsum[gq][r], 2);
     }
-  auto build_q = [&](uint32_t (&dst)[KSTEP][4], const float (*mul)[8]) {
+  // dst = bf16(q * mul); lo (if given) = bf16 of the remainder, so that
+  // hi + lo carries about 16 significant bits of q * mul
+  auto build_q = [&](uint32_t (&dst)[KSTEP][4], const float (*mul)[8], uint32_t (*lo)[4]) {
     // mul[gq][e]: per-channel factor of this thread's channels (KIVI block
     // scales), or nullptr
     for (int gq = 0; gq < NG; ++gq)
@@ -171,11 +194,16 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
               v0 *= mul[gq][e0];
               v1 *= mul[gq][e1];
             }
-            dst[ks][half * 2 + r] = pack_bf16(v0, v1);
+            const __nv_bfloat162 hb = __floats2bfloat162_rn(v0, v1);
+            dst[ks][half * 2 + r] = *reinterpret_cast<const uint32_t*>(&hb);
+            if (lo) {
+              const float2 hf = __bfloat1622float2(hb);
+              lo[ks][half * 2 + r] = pack_bf16(v0 - hf.x, v1 - hf.y);
+            }
           }
       }
   };
-  build_q(qa, nullptr);
+  build_q(qa, nullptr, nullptr);
 
   // ---- running softmax state and accumulators -----------------------------
   float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
@@ -299,17 +327,19 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
         float mul[NG][8];
         for (int gq = 0; gq < NG; ++gq)
           for (int e = 0; e < 8; ++e) mul[gq][e] = __half2float(ksc[32 * gq + 8 * tid + e]);
-        uint32_t qk[KSTEP][4];
-        build_q(qk, mul);
-        // constant: sum_d q_d m_d - 128 sum_d q'_d (q' as rounded into the MMA)
+        uint32_t qk[KSTEP][4], ql[KSTEP][4];
+        build_q(qk, mul, ql);
+        // constant: sum_d q_d m_d - 128 sum_d q'_d, q' = hi + lo as fed to the MMAs
         float cst[2] = {0.f, 0.f};
         for (int gq = 0; gq < NG; ++gq)
           for (int e = 0; e < 8; ++e) {
             const float mz = __half2float(kze[32 * gq + 8 * tid + e]);
             for (int r = 0; r < 2; ++r) {
               const float qr = qv[r][gq][e];
-              const float qs = __bfloat162float(__float2bfloat16_rn(qr * mul[gq][e]));
-              cst[r] += qr * mz - 128.f * qs;
+              const float qx = qr * mul[gq][e];
+              const float qh = __bfloat162float(__float2bfloat16_rn(qx));
+              const float ql2 = __bfloat162float(__float2bfloat16_rn(qx - qh));
+              cst[r] += qr * mz - 128.f * (qh + ql2);
             }
           }
         for (int r = 0; r < 2; ++r) {
@@ -326,9 +356,11 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
               const uint32_t v = *reinterpret_cast<const uint16_t*>(row + 8 * gq + 2 * tid);
               w = v | (v << 14);
             }
-            for (int s = 0; s < 2; ++s)
-              mma16816(acc, qk[2 * gq + s], magic2(w >> (8 * s), kmask),
-                       magic2(w >> (8 * s + 4), kmask));
+            for (int s = 0; s < 2; ++s) {
+              const uint32_t b0 = magic2(w >> (8 * s), kmask), b1 = magic2(w >> (8 * s + 4), kmask);
+              mma16816(acc, qk[2 * gq + s], b0, b1);
+              mma16816(acc, ql[2 * gq + s], b0, b1);
+            }
           }
           sacc[nt][0] = acc[0] + cst[0];
           sacc[nt][1] = acc[1] + cst[0];
@@ -411,21 +443,21 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
                 : FMT == KVQ_FMT_SYMMETRIC ? -(float)zbias * sc : __half2float(vze[rr * NG + gv]);
           }
           // p is indexed [nt][2r + cc]; token tok[i]: nt = i >> 1, cc = i & 1.
-          // The MMA sees bf16(p s) (c + 128); the offset term removes exactly
-          // 128 bf16(p s) and adds p m.
+          // The fp16 MMA sees fp16(p s) (c + 1024); the offset term removes
+          // exactly 1024 fp16(p s) and adds p m.
           float ps[2][4];
           for (int nt = 0; nt < 2; ++nt)
             for (int i = 0; i < 4; ++i)
-              ps[nt][i] = __bfloat162float(__float2bfloat16_rn(p[nt][i] * sv[2 * nt + (i & 1)]));
+              ps[nt][i] = __half2float(__float2half_rn(p[nt][i] * sv[2 * nt + (i & 1)]));
           uint32_t a[4];
-          a[0] = pack_bf16(ps[0][0], ps[0][1]);
-          a[1] = pack_bf16(ps[0][2], ps[0][3]);
-          a[2] = pack_bf16(ps[1][0], ps[1][1]);
-          a[3] = pack_bf16(ps[1][2], ps[1][3]);
+          a[0] = pack_f16(ps[0][0], ps[0][1]);
+          a[1] = pack_f16(ps[0][2], ps[0][3]);
+          a[2] = pack_f16(ps[1][0], ps[1][1]);
+          a[3] = pack_f16(ps[1][2], ps[1][3]);
           for (int r = 0; r < 2; ++r)
             for (int nt = 0; nt < 2; ++nt)
               for (int cc = 0; cc < 2; ++cc)
-                cterm[r][gv] += p[nt][2 * r + cc] * mz[2 * nt + cc] - 128.f * ps[nt][2 * r + cc];
+                cterm[r][gv] += p[nt][2 * r + cc] * mz[2 * nt + cc] - 1024.f * ps[nt][2 * r + cc];
           // B: codes of tokens (2tid, 2tid+1) and (2tid+8, 2tid+9) at channels
           // 32 gv + 4 gid + jj, jj = 0..3 (one n-tile per jj)
           uint32_t cw[4];
@@ -436,15 +468,15 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
           }
           const uint32_t x01 = cw[0] | (cw[1] << 16), x23 = cw[2] | (cw[3] << 16);
           for (int jj = 0; jj < 4; ++jj)
-            mma16816(o[4 * gv + jj], a, magic2(x01 >> (BITS * jj), kmask),
-                     magic2(x23 >> (BITS * jj), kmask));
+            mma16816_f16(o[4 * gv + jj], a, magic2h(x01 >> (BITS * jj), kmask),
+                         magic2h(x23 >> (BITS * jj), kmask));
         }
-      } else {  // full-precision values
+      } else {  // full-precision values (bf16 -> fp16 for the fp16 MMA)
         uint32_t a[4];
-        a[0] = pack_bf16(p[0][0], p[0][1]);
-        a[1] = pack_bf16(p[0][2], p[0][3]);
-        a[2] = pack_bf16(p[1][0], p[1][1]);
-        a[3] = pack_bf16(p[1][2], p[1][3]);
+        a[0] = pack_f16(p[0][0], p[0][1]);
+        a[1] = pack_f16(p[0][2], p[0][3]);
+        a[2] = pack_f16(p[1][0], p[1][1]);
+        a[3] = pack_f16(p[1][2], p[1][3]);
         for (int gv = 0; gv < NG; ++gv) {
           uint2 vw[4];
           for (int i = 0; i < 4; ++i) {
@@ -457,10 +489,10 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
           }
           for (int jj = 0; jj < 4; ++jj) {
             auto el = [&](int i) {
-              const uint16_t* e = reinterpret_cast<const uint16_t*>(&vw[i]);
-              return e[jj];
+              const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&vw[i]);
+              return __bfloat162float(e[jj]);
             };
-            mma16816(o[4 * gv + jj], a, pack_raw(el(0), el(1)), pack_raw(el(2), el(3)));
+            mma16816_f16(o[4 * gv + jj], a, pack_f16(el(0), el(1)), pack_f16(el(2), el(3)));
           }
         }
       }
@@ -588,7 +620,7 @@ cudaError_t launch_one(const Geom& g, const void* q, float scale, int* err, void
   auto kern = attend_decode_mma_kernel<D, BITS, FMT>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
-  kern<<<dim3(g.splits, g.H, g.B), kWarps * 32, sm, s>>>(
+  launch_pdl(kern, dim3(dim3(g.splits, g.H, g.B)), dim3(kWarps * 32), sm, s, 
       g, reinterpret_cast<const __nv_bfloat16*>(q), scale, err,
       reinterpret_cast<__nv_bfloat16*>(out));
   return cudaGetLastError();

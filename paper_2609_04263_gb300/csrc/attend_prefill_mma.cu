@@ -6,9 +6,12 @@
 // heads of the kv head times nq = ROWS / g consecutive queries, 16 rows per
 // warp, so every key/value tile is reconstructed once and shared by all g
 // heads.  Per KV tile of NT tokens: the CTA reconstructs K and V into shared
-// memory as bf16 (codes x fp16 scale + fp16 offset; full-precision windows
-// copied), then each warp computes S = Q K^T with ldmatrix-fed m16n8k16
-// MMAs, an online softmax in the log2 domain, and O += P V (V fragments via
+// memory (codes x fp16 scale + fp16 offset; full-precision windows copied):
+// K as a bf16 high part plus a bf16 remainder, so that Q K^T (two bf16 MMAs
+// per tile) carries about 16 significant bits of K (with real activations the
+// logits are large and a bf16-rounded K would move them visibly); V in fp16.
+// Each warp computes S = Q K^T with ldmatrix-fed m16n8k16 MMAs, an online
+// softmax in the log2 domain, and O += P V in fp16 (V fragments via
 // ldmatrix.trans).  Query tiles are scheduled longest-first (causal work
 // grows with the position).
 #include <math.h>
@@ -25,9 +28,13 @@ struct PCfg {
   static constexpr int NT = D == 256 ? 32 : 64;      // tokens per KV tile
   static constexpr int LDS = D + 8;                   // smem row stride (bf16), 16 B pad
   static constexpr int Q_OFF = 0;
-  static constexpr int K_OFF = ROWS * LDS * 2;
-  static constexpr int V_OFF = K_OFF + NT * LDS * 2;
+  static constexpr int K_OFF = ROWS * LDS * 2;          // bf16 high part of K
+  static constexpr int KL_OFF = K_OFF + NT * LDS * 2;   // bf16 remainder K - K_hi
+  static constexpr int V_OFF = KL_OFF + NT * LDS * 2;   // fp16 V
   static constexpr int TOTAL = V_OFF + NT * LDS * 2;
+  // KVarN: fp32 rows of one reconstructed tile before the inverse Hadamard
+  static constexpr int SCR_OFF = TOTAL;
+  static constexpr int TOTAL_KVARN = SCR_OFF + NT * D * 4;
   static constexpr int THREADS = WARPS * 32;
 };
 
@@ -50,15 +57,49 @@ __device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+__device__ __forceinline__ void mma16816_f16(float c[4], const uint32_t a[4], uint32_t b0,
+                                             uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+// Store 8 reconstructed values: keys as bf16 high part + bf16 remainder
+// (about 16 significant bits), values as fp16.
+__device__ __forceinline__ void store_k8(const float v[8], __nv_bfloat16* hi, __nv_bfloat16* lo) {
+  uint32_t h[4], l[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const __nv_bfloat162 hb = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    const float2 hf = __bfloat1622float2(hb);
+    h[i] = *reinterpret_cast<const uint32_t*>(&hb);
+    l[i] = pack_bf16(v[2 * i] - hf.x, v[2 * i + 1] - hf.y);
+  }
+  *reinterpret_cast<uint4*>(hi) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4*>(lo) = make_uint4(l[0], l[1], l[2], l[3]);
+}
+__device__ __forceinline__ void store_v8(const float v[8], __half* dst) {
+  *reinterpret_cast<uint4*>(dst) = make_uint4(pack_f16(v[0], v[1]), pack_f16(v[2], v[3]),
+                                              pack_f16(v[4], v[5]), pack_f16(v[6], v[7]));
+}
 
-// Reconstruct channels 8c .. 8c+7 of token t (keys: which = 0) as 8 bf16.
-__device__ __forceinline__ uint4 deq8(const Geom& g, int which, int b, int h, int t, int c,
-                                      int T, int tq) {
-  if (t >= T) return make_uint4(0, 0, 0, 0);
+// Reconstruct channels 8c .. 8c+7 of token t (keys: which = 0) in fp32.
+__device__ __forceinline__ void deq8(const Geom& g, int which, int b, int h, int t, int c,
+                                     int T, int tq, float v[8]) {
+  if (t >= T) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    return;
+  }
   const int G = g.G, bits = which ? g.vb : g.kb;
   const int P_CODES = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
   const int P_SCALE = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
@@ -67,8 +108,12 @@ __device__ __forceinline__ uint4 deq8(const Geom& g, int which, int b, int h, in
   const bool raw = g.fmt == KVQ_FMT_FLOAT || (g.fmt == KVQ_FMT_KIVI && t >= tq);
   if (raw) {
     const int slot = g.fmt == KVQ_FMT_KIVI ? t % g.ring : t;
-    return *reinterpret_cast<const uint4*>(
+    const uint4 u = *reinterpret_cast<const uint4*>(
         plane_ptr<__nv_bfloat16>(g, P_FULL, b, h, slot, 8 * c));
+    const __nv_bfloat16* e8 = reinterpret_cast<const __nv_bfloat16*>(&u);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = __bfloat162float(e8[e]);
+    return;
   }
   const uint8_t* row = plane_ptr<uint8_t>(g, P_CODES, b, h, t);
   uint64_t w;
@@ -76,7 +121,6 @@ __device__ __forceinline__ uint4 deq8(const Geom& g, int which, int b, int h, in
   else if (bits == 2) w = *reinterpret_cast<const uint16_t*>(row + 2 * c);
   else w = *reinterpret_cast<const uint64_t*>(row + 8 * c);
   const unsigned mask = (1u << bits) - 1;
-  float v[8];
   if (g.fmt == KVQ_FMT_KIVI && which == 0) {   // per channel: scale and zero per (block, d)
     const uint4 su = *reinterpret_cast<const uint4*>(
         plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t / G, 8 * c));
@@ -96,20 +140,93 @@ __device__ __forceinline__ uint4 deq8(const Geom& g, int which, int b, int h, in
 #pragma unroll
     for (int e = 0; e < 8; ++e) v[e] = (float)((w >> (e * bits)) & mask) * s + m;
   }
-  return make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
-                    pack_bf16(v[6], v[7]));
+}
+
+// KVarN: reconstruct tokens [t0, t0 + NT) into dst [NT][LDS] bf16.  Sinks and
+// staged tokens are copied; coded tokens are r_t c_j (s code + m) in the
+// rotated basis, rotated back by the normalised Hadamard (its own inverse) in
+// fp32 in `scr` [NT][D].
+template <int D, int NT, int THREADS>
+__device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T,
+                           __nv_bfloat16* khi, __nv_bfloat16* klo, __half* vdst, int lds,
+                           float* scr, float inv_sqrt_d) {
+  const int G = g.G, bits = which ? g.vb : g.kb, S = g.S;
+  const int nbq = kvarn_nblocks(T, S, G) * G;
+  const int P_CODES = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int P_SCALE = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int P_ZERO = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int P_FULL = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+  const int P_PEND = which ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
+  const int P_ROW = which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW;
+  const int P_COL = which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL;
+  const unsigned mask = (1u << bits) - 1;
+  for (int i = threadIdx.x; i < NT * (D / 8); i += THREADS) {
+    const int r = i / (D / 8), c = i % (D / 8), t = t0 + r;
+    float* sr = scr + r * D + 8 * c;
+    if (t >= T) {
+      for (int e = 0; e < 8; ++e) sr[e] = 0.f;
+    } else if (t < S || t - S >= nbq) {
+      const __nv_bfloat16* src = t < S
+          ? plane_ptr<__nv_bfloat16>(g, P_FULL, b, h, t, 8 * c)
+          : plane_ptr<__nv_bfloat16>(g, P_PEND, b, h, (t - S) % G, 8 * c);
+      const uint4 u = *reinterpret_cast<const uint4*>(src);
+      const __nv_bfloat16* e8 = reinterpret_cast<const __nv_bfloat16*>(&u);
+      for (int e = 0; e < 8; ++e) sr[e] = __bfloat162float(e8[e]);
+    } else {
+      const int qi = t - S;
+      const uint8_t* row = plane_ptr<uint8_t>(g, P_CODES, b, h, qi);
+      uint64_t w;
+      if (bits == 4) w = *reinterpret_cast<const uint32_t*>(row + 4 * c);
+      else if (bits == 2) w = *reinterpret_cast<const uint16_t*>(row + 2 * c);
+      else w = *reinterpret_cast<const uint64_t*>(row + 8 * c);
+      const int grp = (8 * c) / G;
+      const float sc = __half2float(*plane_ptr<__half>(g, P_SCALE, b, h, qi, grp));
+      const float mz = __half2float(*plane_ptr<__half>(g, P_ZERO, b, h, qi, grp));
+      const float rr = __half2float(*plane_ptr<__half>(g, P_ROW, b, h, 0, qi));
+      const uint4 cu = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, P_COL, b, h, qi / G, 8 * c));
+      const __half* c8 = reinterpret_cast<const __half*>(&cu);
+      for (int e = 0; e < 8; ++e)
+        sr[e] = rr * __half2float(c8[e]) * ((float)((w >> (e * bits)) & mask) * sc + mz);
+    }
+  }
+  __syncthreads();
+  // inverse rotation of the coded rows (butterflies h = 1 .. D/2, then 1/sqrt(D))
+  for (int hs = 1; hs < D; hs <<= 1) {
+    for (int p = threadIdx.x; p < NT * D / 2; p += THREADS) {
+      const int r = p / (D / 2), k = p % (D / 2), t = t0 + r;
+      if (t < S || t - S >= nbq || t >= T) continue;
+      const int j = (k / hs) * 2 * hs + (k % hs);
+      const float a = scr[r * D + j], c = scr[r * D + j + hs];
+      scr[r * D + j] = a + c;
+      scr[r * D + j + hs] = a - c;
+    }
+    __syncthreads();
+  }
+  for (int i = threadIdx.x; i < NT * (D / 8); i += THREADS) {
+    const int r = i / (D / 8), c = i % (D / 8), t = t0 + r;
+    const float f = (t >= S && t - S < nbq && t < T) ? inv_sqrt_d : 1.f;
+    const float* sr = scr + r * D + 8 * c;
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = sr[e] * f;
+    if (which == 0) store_k8(v, khi + r * lds + 8 * c, klo + r * lds + 8 * c);
+    else store_v8(v, vdst + r * lds + 8 * c);
+  }
 }
 
 template <int D>
 __global__ void __launch_bounds__(PCfg<D>::THREADS)
 attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, float scale,
-                          __nv_bfloat16* __restrict__ out, int nq) {
+                          __nv_bfloat16* __restrict__ out, int nq, float inv_sqrt_d) {
+  pdl_wait();
+  pdl_trigger();
   using C = PCfg<D>;
   constexpr int NT = C::NT, LDS = C::LDS, NTN = NT / 8;   // n-tiles of 8 tokens
   extern __shared__ __align__(16) unsigned char smem[];
   __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem + C::Q_OFF);
   __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem + C::K_OFF);
-  __nv_bfloat16* Vs = reinterpret_cast<__nv_bfloat16*>(smem + C::V_OFF);
+  __nv_bfloat16* Kl = reinterpret_cast<__nv_bfloat16*>(smem + C::KL_OFF);
+  __half* Vs = reinterpret_cast<__half*>(smem + C::V_OFF);
 
   const int nqt = gridDim.x;
   const int qtile = nqt - 1 - blockIdx.x;             // longest first
@@ -158,10 +275,20 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
 
   for (int t0 = 0; t0 < t_end; t0 += NT) {
     __syncthreads();                                  // previous tile consumed
-    for (int i = threadIdx.x; i < NT * (D / 8); i += C::THREADS) {
-      const int r = i / (D / 8), c = i % (D / 8);
-      *reinterpret_cast<uint4*>(Ks + r * LDS + 8 * c) = deq8(g, 0, b, hkv, t0 + r, c, T, tq);
-      *reinterpret_cast<uint4*>(Vs + r * LDS + 8 * c) = deq8(g, 1, b, hkv, t0 + r, c, T, tq);
+    if (g.fmt == KVQ_FMT_KVARN) {
+      float* scr = reinterpret_cast<float*>(smem + C::SCR_OFF);
+      kvarn_tile<D, NT, C::THREADS>(g, 0, b, hkv, t0, T, Ks, Kl, Vs, LDS, scr, inv_sqrt_d);
+      __syncthreads();
+      kvarn_tile<D, NT, C::THREADS>(g, 1, b, hkv, t0, T, Ks, Kl, Vs, LDS, scr, inv_sqrt_d);
+    } else {
+      for (int i = threadIdx.x; i < NT * (D / 8); i += C::THREADS) {
+        const int r = i / (D / 8), c = i % (D / 8);
+        float v[8];
+        deq8(g, 0, b, hkv, t0 + r, c, T, tq, v);
+        store_k8(v, Ks + r * LDS + 8 * c, Kl + r * LDS + 8 * c);
+        deq8(g, 1, b, hkv, t0 + r, c, T, tq, v);
+        store_v8(v, Vs + r * LDS + 8 * c);
+      }
     }
     __syncthreads();
     if (warp_pos_max < t0) continue;                  // tile entirely in this warp's future
@@ -175,11 +302,15 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
       ldsm_x4(a, Qs + (warp * 16 + (lane & 15)) * LDS + 16 * ks + (lane >> 4) * 8);
 #pragma unroll
       for (int np = 0; np < NTN / 2; ++np) {
-        uint32_t bq[4];
+        uint32_t bq[4], bl[4];
         const int j = lane >> 3, i = lane & 7;
-        ldsm_x4(bq, Ks + ((2 * np + (j >> 1)) * 8 + i) * LDS + 16 * ks + (j & 1) * 8);
+        const int off = ((2 * np + (j >> 1)) * 8 + i) * LDS + 16 * ks + (j & 1) * 8;
+        ldsm_x4(bq, Ks + off);
+        ldsm_x4(bl, Kl + off);
         mma16816(s[2 * np], a, bq[0], bq[1]);
         mma16816(s[2 * np + 1], a, bq[2], bq[3]);
+        mma16816(s[2 * np], a, bl[0], bl[1]);
+        mma16816(s[2 * np + 1], a, bl[2], bl[3]);
       }
     }
     // ---- mask, online softmax ----
@@ -223,8 +354,8 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
       }
       // A fragment of k-step j/2: n-tile 2k -> a0 (row gid), a1 (row gid+8);
       // n-tile 2k+1 -> a2, a3
-      pa[j >> 1][(j & 1) * 2 + 0] = pack_bf16(p[0], p[1]);
-      pa[j >> 1][(j & 1) * 2 + 1] = pack_bf16(p[2], p[3]);
+      pa[j >> 1][(j & 1) * 2 + 0] = pack_f16(p[0], p[1]);
+      pa[j >> 1][(j & 1) * 2 + 1] = pack_f16(p[2], p[3]);
     }
     // ---- O += P V ----
 #pragma unroll
@@ -234,8 +365,8 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
         uint32_t bv[4];
         const int j = lane >> 3, i = lane & 7;
         ldsm_x4_t(bv, Vs + (16 * kt + (j & 1) * 8 + i) * LDS + 8 * (nd + (j >> 1)));
-        mma16816(o[nd], pa[kt], bv[0], bv[1]);
-        mma16816(o[nd + 1], pa[kt], bv[2], bv[3]);
+        mma16816_f16(o[nd], pa[kt], bv[0], bv[1]);
+        mma16816_f16(o[nd + 1], pa[kt], bv[2], bv[3]);
       }
     }
   }
@@ -266,12 +397,14 @@ cudaError_t launch_d(const Geom& g, const void* q, int L, float scale, void* out
   const int grp = g.Hq / g.H;
   const int nq = C::ROWS / grp;
   auto kern = attend_prefill_mma_kernel<D>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       C::TOTAL);
+  const int smem = g.fmt == KVQ_FMT_KVARN ? C::TOTAL_KVARN : C::TOTAL;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
+  const float inv_sqrt_d = (float)(1.0 / sqrt((double)D));
   dim3 grid((L + nq - 1) / nq, g.H, g.B);
-  kern<<<grid, C::THREADS, C::TOTAL, s>>>(g, reinterpret_cast<const __nv_bfloat16*>(q), L, scale,
-                                          reinterpret_cast<__nv_bfloat16*>(out), nq);
+  launch_pdl(kern, dim3(grid), dim3(C::THREADS), (size_t)smem, s, g,
+             reinterpret_cast<const __nv_bfloat16*>(q), L, scale,
+             reinterpret_cast<__nv_bfloat16*>(out), nq, inv_sqrt_d);
   return cudaGetLastError();
 }
 
@@ -279,7 +412,7 @@ cudaError_t launch_d(const Geom& g, const void* q, int L, float scale, void* out
 
 bool prefill_mma_supported(const Geom& g) {
   const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC ||
-                      g.fmt == KVQ_FMT_KIVI || g.fmt == KVQ_FMT_FLOAT;
+                      g.fmt == KVQ_FMT_KIVI || g.fmt == KVQ_FMT_FLOAT || g.fmt == KVQ_FMT_KVARN;
   const int grp = g.Hq / g.H;
   const int rows = g.D == 256 ? 64 : 128;
   return fmt_ok && g.act == KVQ_BF16 && grp <= rows &&

@@ -8,6 +8,8 @@
 #include <cuda_fp16.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/kvq.h"
 
 namespace kvq {
@@ -79,6 +81,32 @@ __device__ __forceinline__ float ld_act(const void* p, int64_t i, int act) {
 __device__ __forceinline__ void st_act(void* p, int64_t i, float v, int act) {
   if (act == KVQ_BF16) reinterpret_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
   else reinterpret_cast<float*>(p)[i] = v;
+}
+
+// Programmatic dependent launch: every kernel of the library is launched with
+// programmatic stream serialization, so the next grid can be resident while
+// the previous one drains.  pdl_wait() (first statement of every kernel)
+// blocks until the preceding grid has completed and its memory is visible;
+// pdl_trigger() lets the next grid start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 // Host-side launchers (each defined in the translation unit of its kernels).

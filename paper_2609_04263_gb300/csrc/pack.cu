@@ -82,6 +82,8 @@ __device__ __forceinline__ int sym_code(float x, float s, int bits) {
 // ---------------------------------------------------------------------------
 __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
                                      int final_kernel) {
+  pdl_wait();
+  pdl_trigger();
   bool ok;
   const int T0 = append_begin(g, L, &ok);
   const int which = kivi ? 1 : blockIdx.y;
@@ -163,6 +165,8 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
 // slot (t - S) mod G).  Always the final kernel of an append.
 // ---------------------------------------------------------------------------
 __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
+  pdl_wait();
+  pdl_trigger();
   bool ok;
   const int T0 = append_begin(g, L, &ok);
   const int T1 = T0 + L;
@@ -217,6 +221,8 @@ __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
 // this append completes (grid sized for the most an append of L can flush).
 // ---------------------------------------------------------------------------
 __global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float smem[];
   bool ok;
   const int T0 = append_begin(g, L, &ok);
@@ -263,6 +269,8 @@ __global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
 // k|v).  Sums follow the stride-halving pairwise tree in fp32.
 // ---------------------------------------------------------------------------
 __global__ void kvarn_block_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float smem[];
   bool ok;
   const int T0 = append_begin(g, L, &ok);
@@ -393,14 +401,14 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
   cudaError_t e;
   switch (g.fmt) {
     case KVQ_FMT_FLOAT:
-      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     case KVQ_FMT_AFFINE:
     case KVQ_FMT_SYMMETRIC: {
       const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
       const int64_t units = (int64_t)g.B * g.H * L * (g.D / g.G);
       const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
-      pack_pertoken_kernel<<<dim3(grid_for(threads, 256), 2), 256, 0, s>>>(g, L, sk, sv, sym, 0, 1);
+      launch_pdl(pack_pertoken_kernel, dim3(dim3(grid_for(threads, 256), 2)), dim3(256), 0, s, g, L, sk, sv, sym, 0, 1);
       return cudaGetLastError();
     }
     case KVQ_FMT_KIVI: {
@@ -410,11 +418,11 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       e = cudaFuncSetAttribute(kivi_key_flush_kernel,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
       if (e != cudaSuccess) return e;
-      kivi_key_flush_kernel<<<dim3(max_blocks, g.B * g.H), 128, sm, s>>>(g, L, sk);
+      launch_pdl(kivi_key_flush_kernel, dim3(dim3(max_blocks, g.B * g.H)), dim3(128), sm, s, g, L, sk);
       const int64_t units = (int64_t)g.B * g.H * max_blocks * g.G * (g.D / g.G);
       const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
-      pack_pertoken_kernel<<<dim3(grid_for(threads, 256), 1), 256, 0, s>>>(g, L, sk, sv, 0, 1, 0);
-      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      launch_pdl(pack_pertoken_kernel, dim3(dim3(grid_for(threads, 256), 1)), dim3(256), 0, s, g, L, sk, sv, 0, 1, 0);
+      launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     }
     case KVQ_FMT_KVARN: {
@@ -425,8 +433,8 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       if (e != cudaSuccess) return e;
       sk.ring_plane = KVQ_PLANE_K_PEND; sk.ring_off = g.S; sk.ring_rows = g.G;
       sv.ring_plane = KVQ_PLANE_V_PEND; sv.ring_off = g.S; sv.ring_rows = g.G;
-      kvarn_block_kernel<<<dim3(max_blocks, g.B * g.H, 2), 256, sm, s>>>(g, L, sk, sv, inv_sqrt_d);
-      store_full_kernel<<<dim3(grid_for(full_threads, 256), 2), 256, 0, s>>>(g, L, k, v);
+      launch_pdl(kvarn_block_kernel, dim3(dim3(max_blocks, g.B * g.H, 2)), dim3(256), sm, s, g, L, sk, sv, inv_sqrt_d);
+      launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     }
   }

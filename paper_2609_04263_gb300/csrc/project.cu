@@ -46,6 +46,8 @@ __device__ __forceinline__ void rope_cos_sin(int pos, float th_hi, float th_lo, 
 
 // One CTA: kMT rows of x times one head's D output columns.
 __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   const int D = p.D, M = p.B * p.L;
   const int hh = blockIdx.y;                 // stacked head index over q, k, v
@@ -212,6 +214,8 @@ template <> struct Raw8<float> {
 
 template <typename T, int MM, int KITER>
 __global__ void __launch_bounds__(kSkinnyWarps * 32, 3) project_skinny_kernel(ProjArgs p) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float xsm[];             // [M][d_in] fp32, then U [M][64]
   const int M = p.B * p.L, D = p.D, K = p.d_in;
   const int half = D / 2;
@@ -403,6 +407,8 @@ __device__ __forceinline__ void mma16816_p(float c[4], uint32_t a0, uint32_t a1,
 template <int M16, int NT>   // M16: x rows held (8 or 16); NT: 2 + rank tiles
 __global__ void __launch_bounds__(kDecWarps * 32)
 project_decode_mma_kernel(ProjArgs p) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(16) unsigned char dsm[];
   const int M = p.B * p.L, D = p.D, K = p.d_in;
   const int half = D / 2;
@@ -531,7 +537,7 @@ cudaError_t launch_decode_mma_nt(const ProjArgs& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   const int tiles = (p.Hq + 2 * p.Hkv) * (p.D / 16);
-  kern<<<tiles, kDecWarps * 32, sm, s>>>(p);
+  launch_pdl(kern, dim3(tiles), dim3(kDecWarps * 32), sm, s, p);
   return cudaGetLastError();
 }
 
@@ -558,7 +564,7 @@ cudaError_t launch_skinny(const ProjArgs& p, cudaStream_t s) {
             : M <= 8 ? project_skinny_kernel<T, 8, KI> : project_skinny_kernel<T, kSkinnyMaxM, KI>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
-  kern<<<pairs / kSkinnyWarps, kSkinnyWarps * 32, sm, s>>>(p);
+  launch_pdl(kern, dim3(pairs / kSkinnyWarps), dim3(kSkinnyWarps * 32), sm, s, p);
   return cudaGetLastError();
 }
 
@@ -603,7 +609,7 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   dim3 grid((M + kMT - 1) / kMT, Hq + 2 * Hkv);
-  project_simt_kernel<<<grid, kThreads, sm, s>>>(p);
+  launch_pdl(project_simt_kernel, dim3(grid), dim3(kThreads), sm, s, p);
   return cudaGetLastError();
 }
 

@@ -165,6 +165,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
                   const __grid_constant__ CUtensorMap tm_a2, const __grid_constant__ CUtensorMap tm_b0,
                   const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_b2,
                   const TcArgs args) {
+  pdl_wait();
+  pdl_trigger();
   using S = Smem<BN>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -389,7 +391,7 @@ cudaError_t launch_bn(const CUtensorMap maps[8], const TcArgs& a, cudaStream_t s
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_off[3] / BN, (a.M + BM - 1) / BM);
-  kern<<<grid, kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], maps[5],
+  launch_pdl(kern, dim3(grid), dim3(kThreads), smem, s, maps[0], maps[1], maps[2], maps[3], maps[4], maps[5],
                                     maps[6], maps[7], a);
   return cudaGetLastError();
 }
