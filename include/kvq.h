@@ -213,6 +213,25 @@ kvq_status kvq_attend_decode(kvq_cache* cache, const void* q, int n_q_heads,
                              float softmax_scale, void* out, void* stream);
 
 /*
+ * One decode step of one layer: kvq_project_lora of the new token (x [B][1]
+ * [d_in], positions continue the cache), kvq_append_pack of its key and value,
+ * then kvq_attend_decode of its query (Sections 3-3.3).  q, k, v receive the
+ * projections ([B][Hq][1][D], [B][Hkv][1][D] x 2); out [B][Hq][1][D].  B and
+ * the head counts are the cache's.  For bf16 affine/symmetric caches with
+ * 2/4-bit codes, G = 32, head_dim 64/128 and B <= 16 the three steps run as
+ * one cooperative kernel with one CTA per SM (grid-wide barriers between the
+ * phases, bounded waits); other caches run the three calls in order.  The
+ * results are the same either way.  Like kvq_attend_decode it uses the
+ * cache's workspace, so calls on one cache must not overlap.
+ */
+kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void* w_qkv,
+                           const void* a_q, const void* b_q, int r_q,
+                           const void* a_k, const void* b_k, int r_k,
+                           const void* a_v, const void* b_v, int r_v,
+                           float alpha_over_r, float rope_base, float softmax_scale,
+                           void* q, void* k, void* v, void* out, void* stream);
+
+/*
  * kvq_attend_decode for callers that cannot allocate device memory.  (No
  * counterpart in the paper: this is a deployment variant of the decode step.)
  *

@@ -80,6 +80,27 @@ class Cache:
         kvq.kvq_attend_decode(self.handle, _ptr(q), q.shape[1], scale, _ptr(out), _stream())
         return out
 
+    def decode_step(self, x, w_qkv, lora, alpha_over_r, rope_base, qkv=None, out=None,
+                    scale=None):
+        """Project the new token x [B,1,d_in], append its key/value and attend:
+        returns (q, k, v), out."""
+        d = self.desc
+        B, D = d.batch, d.head_dim
+        if qkv is None:
+            qkv = (torch.empty(B, d.q_heads, 1, D, dtype=x.dtype, device=x.device),
+                   torch.empty(B, d.kv_heads, 1, D, dtype=x.dtype, device=x.device),
+                   torch.empty(B, d.kv_heads, 1, D, dtype=x.dtype, device=x.device))
+        out = torch.empty(B, d.q_heads, 1, D, dtype=x.dtype, device=x.device) if out is None else out
+        scale = 1.0 / math.sqrt(D) if scale is None else scale
+        args = []
+        for p in "qkv":
+            ab = lora.get(p)
+            args += [None, None, 0] if ab is None else [_ptr(ab[0]), _ptr(ab[1]), ab[0].shape[0]]
+        kvq.kvq_decode_step(self.handle, _ptr(x), x.shape[-1], _ptr(w_qkv), *args, alpha_over_r,
+                            rope_base, scale, _ptr(qkv[0]), _ptr(qkv[1]), _ptr(qkv[2]), _ptr(out),
+                            _stream())
+        return qkv, out
+
     def planes(self) -> dict:
         """name -> tensor view [B, H, rows, cols] of each present plane."""
         v = kvq.kvq_cache_view(self.handle)

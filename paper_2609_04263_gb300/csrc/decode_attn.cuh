@@ -1,0 +1,640 @@
+// Device code of the split-K decode attention (shared by the standalone
+// kernel in attend_mma.cu and the fused decode step in decode_step.cu).
+#pragma once
+
+#include <math.h>
+
+#include "kvq_internal.cuh"
+
+namespace kvq {
+namespace dattn {
+// Split-K flash-decode over the packed cache on tensor cores (bf16 mma.sync).
+//
+// One CTA = (split of the tokens, kv head, sequence); 4 warps.  Each CTA
+// writes its split's partial (m, l, o) to the workspace; the last CTA of a
+// (sequence, kv head) to finish (an arrival counter, no waiting) merges them
+// by log-sum-exp into the output.  The split's
+// tokens stream through shared memory in 64-token chunks: one thread issues
+// TMA bulk copies (codes and fp16 metadata of the chunk) on an mbarrier ring
+// of kStages buffers; each warp then takes one 16-token tile of the chunk.
+//
+// Scores: S[h][t] = sum_d q[h][d] k_hat[t][d] with the g = Hq/Hkv query heads
+// of the kv head as the MMA rows (zero-padded to 16) and tokens as columns.
+// Codes enter the MMA as exact bf16 integers: (0x4300 | c) is the bf16 value
+// 128 + c, built two at a time by one LOP3.  With per-token groups,
+//   q . k_hat = sum_groups s_g (q_g . (c_g + 128)) + (m_g - 128 s_g) sum(q_g),
+// so each group keeps its own accumulator and the scale and offset are applied
+// per token after the MMA.  KIVI keys (one scale per block and channel) fold
+// the scale into q instead: q' = q * s_blk, split into bf16 hi + lo.  Values
+// run through fp16 MMAs with codes as (0x6400 | c) = 1024 + c:
+//   O[h][d] += sum_t fp16(p s)[h][t] (c + 1024)[t][d] + sum_t (p m - 1024 fp16(p s)).
+//
+// The MMA's k index may map to any channel as long as q and k agree, and its
+// output columns to any channel as long as the store undoes it; the mappings
+// below make each thread's codes one contiguous word per group.
+
+constexpr int kCT = 64;          // tokens per chunk (4 tiles of 16)
+constexpr int kStages = 4;
+constexpr int kWarps = 4;
+constexpr uint32_t kMagic = 0x43004300u;
+constexpr long kWaitLimit = 1L << 24;   // bounded mbarrier polling
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_inval(uint64_t* bar) {
+  asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, int count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Bounded wait; returns false (and the caller flags an error) on timeout.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (long i = 0; i < kWaitLimit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// (x & mask) | 0x43004300: two codes as bf16 (128 + c)
+__device__ __forceinline__ uint32_t magic2(uint32_t x, uint32_t mask) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "r"(mask), "r"(kMagic));
+  return r;
+}
+// (x & mask) | 0x64006400: two codes as fp16 (1024 + c)
+constexpr uint32_t kMagicH = 0x64006400u;
+__device__ __forceinline__ uint32_t magic2h(uint32_t x, uint32_t mask) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "r"(mask), "r"(kMagicH));
+  return r;
+}
+__device__ __forceinline__ void mma16816_f16(float c[4], const uint32_t a[4], uint32_t b0,
+                                             uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t pack_raw(uint16_t lo, uint16_t hi) {
+  return (uint32_t)lo | ((uint32_t)hi << 16);
+}
+
+// Channel held by slot e (0..7) of a thread's 8-channel word in QK k-step s,
+// register half (0: a0/b0, 1: a2/b1), element j: see the LOP3 pairings.
+template <int BITS>
+__device__ __forceinline__ int qk_chan(int s, int half, int j) {
+  if (BITS == 4) return 2 * s + half + 4 * j;     // pairs (n0,n4),(n1,n5),(n2,n6),(n3,n7)
+  return 4 * s + 2 * half + j;                     // pairs (c0,c1),(c2,c3),(c4,c5),(c6,c7)
+}
+
+template <int D, int BITS, int FMT>
+struct Cfg {
+  static constexpr int NG = D / 32;                 // quantization groups (G = 32)
+  static constexpr int KSTEP = D / 16;
+  static constexpr int CODE_B = D * BITS / 8;       // code bytes per token
+  static constexpr int NT_PV = D / 8;               // PV n-tiles
+  // shared memory per stage
+  static constexpr int KC_OFF = 0;
+  static constexpr int VC_OFF = KC_OFF + kCT * CODE_B;
+  static constexpr int KS_OFF = VC_OFF + kCT * CODE_B;            // K scale (per token or block)
+  static constexpr int KMETA_B = FMT == KVQ_FMT_KIVI ? (kCT / 32) * D * 2 : kCT * NG * 2;
+  static constexpr int KZ_OFF = KS_OFF + KMETA_B;
+  static constexpr int VS_OFF = KZ_OFF + KMETA_B;
+  static constexpr int VZ_OFF = VS_OFF + kCT * NG * 2;
+  static constexpr int STAGE_B = ((VZ_OFF + kCT * NG * 2) + 127) / 128 * 128;
+};
+
+// One split of one (sequence, kv head): blockIdx-independent, so a fused
+// kernel can run several per CTA.  T = tokens stored (read by the caller).
+// smem: the dynamic buffer of at least attn_smem_bytes<D, BITS, FMT>().
+template <int D, int BITS, int FMT>
+__device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q, float scale,
+                             int* err, __nv_bfloat16* __restrict__ out, int split, int hkv, int b,
+                             int T, unsigned char* smem) {
+  using C = Cfg<D, BITS, FMT>;
+  constexpr int NG = C::NG, KSTEP = C::KSTEP, NT_PV = C::NT_PV;
+  __shared__ uint64_t full_bar[kStages];
+  __shared__ float red_m[kWarps][16], red_l[kWarps][16];
+  __shared__ int last_cta;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tid = lane & 3;
+  int ts, te;
+  split_range(T, g.splits, split, kCT, &ts, &te);
+  const int grp = g.Hq / g.H;
+  const int tq = FMT == KVQ_FMT_KIVI ? kivi_tq(T, g.R, 32) : T;   // coded tokens [0, tq)
+  const float l2e = 1.4426950408889634f;
+  const float qk_scale = scale * l2e;                 // scores in log2 units
+
+  // ---- query fragments (rows = heads gid, gid + 8) and per-group sums -----
+  uint32_t qa[KSTEP][4];
+  float qsum[NG][2];
+  float qv[2][NG][8];                                 // this thread's 8 channels per group
+  for (int r = 0; r < 2; ++r) {
+    const int hl = gid + 8 * r;
+    for (int gq = 0; gq < NG; ++gq) {
+      float s = 0.f;
+      for (int e = 0; e < 8; ++e) {
+        float v = 0.f;
+        if (hl < grp)
+          v = __bfloat162float(q[((int64_t)b * g.Hq + hkv * grp + hl) * D + 32 * gq + 8 * tid + e]);
+        qv[r][gq][e] = v;
+        s += v;
+      }
+      qsum[gq][r] = s;       // partial over this thread's 8 channels
+    }
+  }
+  for (int gq = 0; gq < NG; ++gq)
+    for (int r = 0; r < 2; ++r) {
+      qsum[gq][r] += __shfl_xor_sync(0xffffffffu, qsum[gq][r], 1);
+      qsum[gq][r] += __shfl_xor_sync(0xffffffffu, qsum[gq][r], 2);
+    }
+  // dst = bf16(q * mul); lo (if given) = bf16 of the remainder, so that
+  // hi + lo carries about 16 significant bits of q * mul
+  auto build_q = [&](uint32_t (&dst)[KSTEP][4], const float (*mul)[8], uint32_t (*lo)[4]) {
+    // mul[gq][e]: per-channel factor of this thread's channels (KIVI block
+    // scales), or nullptr
+    for (int gq = 0; gq < NG; ++gq)
+      for (int s = 0; s < 2; ++s) {
+        const int ks = 2 * gq + s;
+        for (int half = 0; half < 2; ++half)
+          for (int r = 0; r < 2; ++r) {
+            const int e0 = qk_chan<BITS>(s, half, 0), e1 = qk_chan<BITS>(s, half, 1);
+            float v0 = qv[r][gq][e0], v1 = qv[r][gq][e1];
+            if (mul) {
+              v0 *= mul[gq][e0];
+              v1 *= mul[gq][e1];
+            }
+            const __nv_bfloat162 hb = __floats2bfloat162_rn(v0, v1);
+            dst[ks][half * 2 + r] = *reinterpret_cast<const uint32_t*>(&hb);
+            if (lo) {
+              const float2 hf = __bfloat1622float2(hb);
+              lo[ks][half * 2 + r] = pack_bf16(v0 - hf.x, v1 - hf.y);
+            }
+          }
+      }
+  };
+  build_q(qa, nullptr, nullptr);
+
+  // ---- running softmax state and accumulators -----------------------------
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[NT_PV][4];
+  for (int j = 0; j < NT_PV; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  float cterm[2][NG];
+  for (int gq = 0; gq < NG; ++gq) cterm[0][gq] = cterm[1][gq] = 0.f;
+
+  // ---- chunk pipeline ------------------------------------------------------
+  const int nchunks = te > ts ? (te - ts + kCT - 1) / kCT : 0;
+  const bool leader = threadIdx.x == 0;
+  if (leader)
+    for (int i = 0; i < kStages; ++i) mbar_init(&full_bar[i], 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+
+  auto issue = [&](int chunk) {
+    const int stage = chunk % kStages;
+    unsigned char* st = smem + stage * C::STAGE_B;
+    const int c0 = ts + chunk * kCT;
+    int nq = min(kCT, tq - c0);                 // coded tokens of the chunk
+    if (nq <= 0) {                              // nothing coded: arrive with no bytes
+      mbar_expect_tx(&full_bar[stage], 0);
+      return;
+    }
+    nq = (nq + 3) & ~3;                         // 16-byte multiples (planes padded)
+    const uint32_t code_bytes = nq * C::CODE_B;
+    const uint32_t kmeta = FMT == KVQ_FMT_KIVI ? ((nq + 31) / 32) * D * 2 : nq * NG * 2;
+    const uint32_t vmeta = nq * NG * 2;
+    const bool zero_planes = FMT != KVQ_FMT_SYMMETRIC;
+    uint32_t total = 2 * code_bytes + kmeta + vmeta;
+    if (zero_planes) total += kmeta + vmeta;
+    mbar_expect_tx(&full_bar[stage], total);
+    bulk_g2s(st + C::KC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, c0), code_bytes,
+             &full_bar[stage]);
+    bulk_g2s(st + C::VC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
+             &full_bar[stage]);
+    if (FMT == KVQ_FMT_KIVI) {
+      bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
+               &full_bar[stage]);
+      bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
+               &full_bar[stage]);
+    } else {
+      bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,
+               &full_bar[stage]);
+      if (zero_planes)
+        bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0), kmeta,
+                 &full_bar[stage]);
+    }
+    bulk_g2s(st + C::VS_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, c0), vmeta,
+             &full_bar[stage]);
+    if (zero_planes)
+      bulk_g2s(st + C::VZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, c0), vmeta,
+               &full_bar[stage]);
+  };
+  if (leader)
+    for (int c = 0; c < min(kStages, nchunks); ++c) issue(c);
+
+  bool timed_out = false;
+  const uint32_t kmask = BITS == 4 ? 0x000F000Fu : 0x00030003u;
+  const int zbias = FMT == KVQ_FMT_SYMMETRIC ? (1 << (BITS - 1)) : 0;
+
+  int chunk = 0;
+  for (; chunk < nchunks; ++chunk) {
+    const int stage = chunk % kStages;
+    const bool ok = mbar_wait(&full_bar[stage], (chunk / kStages) & 1);
+    if (__syncthreads_or(!ok)) {        // the same decision in every thread
+      timed_out = true;
+      break;
+    }
+    const unsigned char* st = smem + stage * C::STAGE_B;
+    const int c0 = ts + chunk * kCT;
+    const int t0 = c0 + 16 * warp;                   // this warp's tile
+    const int tile_off = 16 * warp;                  // row offset within the chunk
+    if (warp < kWarps && t0 < te) {                  // extra warps (fused kernel) idle
+      const bool coded = t0 < tq;
+      float sacc[2][4];                              // S for n-tiles 0, 1 (tokens t0 + 8nt + col)
+      // ---------------- scores ----------------
+      if (coded && FMT != KVQ_FMT_KIVI) {
+        float acc[NG][2][4];
+        for (int gq = 0; gq < NG; ++gq)
+          for (int nt = 0; nt < 2; ++nt) acc[gq][nt][0] = acc[gq][nt][1] = acc[gq][nt][2] = acc[gq][nt][3] = 0.f;
+        for (int nt = 0; nt < 2; ++nt) {
+          const unsigned char* row = st + C::KC_OFF + (tile_off + 8 * nt + gid) * C::CODE_B;
+          for (int gq = 0; gq < NG; ++gq) {
+            uint32_t w;
+            if (BITS == 4) w = *reinterpret_cast<const uint32_t*>(row + 16 * gq + 4 * tid);
+            else {
+              const uint32_t v = *reinterpret_cast<const uint16_t*>(row + 8 * gq + 2 * tid);
+              w = v | (v << 14);
+            }
+            for (int s = 0; s < 2; ++s) {
+              const uint32_t b0 = magic2(w >> (BITS == 4 ? 8 * s : 8 * s), kmask);
+              const uint32_t b1 = magic2(w >> (BITS == 4 ? 8 * s + 4 : 8 * s + 4), kmask);
+              mma16816(acc[gq][nt], qa[2 * gq + s], b0, b1);
+            }
+          }
+        }
+        // apply per-token scale and offset: columns 2tid, 2tid+1 of each n-tile
+        const __half* ksc = reinterpret_cast<const __half*>(st + C::KS_OFF);
+        const __half* kze = reinterpret_cast<const __half*>(st + C::KZ_OFF);
+        for (int nt = 0; nt < 2; ++nt)
+          for (int cc = 0; cc < 2; ++cc) {
+            const int rr = tile_off + 8 * nt + 2 * tid + cc;     // row within chunk
+            float s0 = 0.f, s1 = 0.f;
+            for (int gq = 0; gq < NG; ++gq) {
+              const float sc = __half2float(ksc[rr * NG + gq]);
+              const float mz = FMT == KVQ_FMT_SYMMETRIC ? -(float)zbias * sc
+                                                       : __half2float(kze[rr * NG + gq]);
+              const float off = mz - 128.f * sc;
+              s0 += sc * acc[gq][nt][cc] + off * qsum[gq][0];
+              s1 += sc * acc[gq][nt][2 + cc] + off * qsum[gq][1];
+            }
+            sacc[nt][cc] = s0;
+            sacc[nt][2 + cc] = s1;
+          }
+      } else if (coded) {  // KIVI: per-channel block scale folded into q
+        const int blk_row = (tile_off) / 32;            // block within the chunk
+        const __half* ksc = reinterpret_cast<const __half*>(st + C::KS_OFF) + blk_row * D;
+        const __half* kze = reinterpret_cast<const __half*>(st + C::KZ_OFF) + blk_row * D;
+        float mul[NG][8];
+        for (int gq = 0; gq < NG; ++gq)
+          for (int e = 0; e < 8; ++e) mul[gq][e] = __half2float(ksc[32 * gq + 8 * tid + e]);
+        uint32_t qk[KSTEP][4], ql[KSTEP][4];
+        build_q(qk, mul, ql);
+        // constant: sum_d q_d m_d - 128 sum_d q'_d, q' = hi + lo as fed to the MMAs
+        float cst[2] = {0.f, 0.f};
+        for (int gq = 0; gq < NG; ++gq)
+          for (int e = 0; e < 8; ++e) {
+            const float mz = __half2float(kze[32 * gq + 8 * tid + e]);
+            for (int r = 0; r < 2; ++r) {
+              const float qr = qv[r][gq][e];
+              const float qx = qr * mul[gq][e];
+              const float qh = __bfloat162float(__float2bfloat16_rn(qx));
+              const float ql2 = __bfloat162float(__float2bfloat16_rn(qx - qh));
+              cst[r] += qr * mz - 128.f * (qh + ql2);
+            }
+          }
+        for (int r = 0; r < 2; ++r) {
+          cst[r] += __shfl_xor_sync(0xffffffffu, cst[r], 1);
+          cst[r] += __shfl_xor_sync(0xffffffffu, cst[r], 2);
+        }
+        for (int nt = 0; nt < 2; ++nt) {
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+          const unsigned char* row = st + C::KC_OFF + (tile_off + 8 * nt + gid) * C::CODE_B;
+          for (int gq = 0; gq < NG; ++gq) {
+            uint32_t w;
+            if (BITS == 4) w = *reinterpret_cast<const uint32_t*>(row + 16 * gq + 4 * tid);
+            else {
+              const uint32_t v = *reinterpret_cast<const uint16_t*>(row + 8 * gq + 2 * tid);
+              w = v | (v << 14);
+            }
+            for (int s = 0; s < 2; ++s) {
+              const uint32_t b0 = magic2(w >> (8 * s), kmask), b1 = magic2(w >> (8 * s + 4), kmask);
+              mma16816(acc, qk[2 * gq + s], b0, b1);
+              mma16816(acc, ql[2 * gq + s], b0, b1);
+            }
+          }
+          sacc[nt][0] = acc[0] + cst[0];
+          sacc[nt][1] = acc[1] + cst[0];
+          sacc[nt][2] = acc[2] + cst[1];
+          sacc[nt][3] = acc[3] + cst[1];
+        }
+      } else {  // full-precision tokens (KIVI residual ring)
+        for (int nt = 0; nt < 2; ++nt) {
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+          const int t = t0 + 8 * nt + gid;
+          const bool ok = t < te;
+          const int slot = t % g.ring;
+          const __nv_bfloat16* krow =
+              plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, hkv, ok ? slot : 0);
+          for (int gq = 0; gq < NG; ++gq) {
+            uint4 u = ok ? *reinterpret_cast<const uint4*>(krow + 32 * gq + 8 * tid)
+                         : make_uint4(0, 0, 0, 0);
+            const uint16_t* e = reinterpret_cast<const uint16_t*>(&u);
+            for (int s = 0; s < 2; ++s) {
+              const uint32_t b0 = pack_raw(e[qk_chan<BITS>(s, 0, 0)], e[qk_chan<BITS>(s, 0, 1)]);
+              const uint32_t b1 = pack_raw(e[qk_chan<BITS>(s, 1, 0)], e[qk_chan<BITS>(s, 1, 1)]);
+              mma16816(acc, qa[2 * gq + s], b0, b1);
+            }
+          }
+          for (int i = 0; i < 4; ++i) sacc[nt][i] = acc[i];
+        }
+      }
+      // ---------------- online softmax (log2 domain) ----------------
+      float mx[2] = {-INFINITY, -INFINITY};
+      for (int nt = 0; nt < 2; ++nt)
+        for (int cc = 0; cc < 2; ++cc) {
+          const int t = t0 + 8 * nt + 2 * tid + cc;
+          for (int r = 0; r < 2; ++r) {
+            float v = sacc[nt][2 * r + cc] * qk_scale;
+            if (t >= te) v = -INFINITY;
+            sacc[nt][2 * r + cc] = v;
+            mx[r] = fmaxf(mx[r], v);
+          }
+        }
+      float alpha[2];
+      for (int r = 0; r < 2; ++r) {
+        mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+        mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+        const float mn = fmaxf(m_run[r], mx[r]);
+        alpha[r] = mn == -INFINITY ? 1.f : exp2f(m_run[r] - mn);
+        m_run[r] = mn;
+        l_run[r] *= alpha[r];
+      }
+      for (int j = 0; j < NT_PV; ++j) {
+        o[j][0] *= alpha[0]; o[j][1] *= alpha[0];
+        o[j][2] *= alpha[1]; o[j][3] *= alpha[1];
+      }
+      for (int gq = 0; gq < NG; ++gq) {
+        cterm[0][gq] *= alpha[0];
+        cterm[1][gq] *= alpha[1];
+      }
+      float p[2][4];
+      for (int nt = 0; nt < 2; ++nt)
+        for (int i = 0; i < 4; ++i) {
+          const int r = i >> 1;
+          const float v = sacc[nt][i];
+          p[nt][i] = v == -INFINITY ? 0.f : exp2f(v - m_run[r]);
+          l_run[r] += p[nt][i];
+        }
+      // ---------------- P V ----------------
+      // A fragment: a0 = (row gid, tokens 2tid, 2tid+1) = p[0][0..1], a1 = row
+      // gid+8 = p[0][2..3], a2 = tokens 2tid+8, +9 = p[1][0..1], a3 = p[1][2..3].
+      const int tok[4] = {2 * tid, 2 * tid + 1, 2 * tid + 8, 2 * tid + 9};
+      if (coded) {
+        const __half* vsc = reinterpret_cast<const __half*>(st + C::VS_OFF);
+        const __half* vze = reinterpret_cast<const __half*>(st + C::VZ_OFF);
+        for (int gv = 0; gv < NG; ++gv) {
+          float sv[4], mz[4];
+          for (int i = 0; i < 4; ++i) {
+            const int rr = tile_off + tok[i];
+            const bool ok = t0 + tok[i] < te;
+            const float sc = ok ? __half2float(vsc[rr * NG + gv]) : 0.f;
+            sv[i] = sc;
+            mz[i] = !ok ? 0.f
+                : FMT == KVQ_FMT_SYMMETRIC ? -(float)zbias * sc : __half2float(vze[rr * NG + gv]);
+          }
+          // p is indexed [nt][2r + cc]; token tok[i]: nt = i >> 1, cc = i & 1.
+          // The fp16 MMA sees fp16(p s) (c + 1024); the offset term removes
+          // exactly 1024 fp16(p s) and adds p m.
+          float ps[2][4];
+          for (int nt = 0; nt < 2; ++nt)
+            for (int i = 0; i < 4; ++i)
+              ps[nt][i] = __half2float(__float2half_rn(p[nt][i] * sv[2 * nt + (i & 1)]));
+          uint32_t a[4];
+          a[0] = pack_f16(ps[0][0], ps[0][1]);
+          a[1] = pack_f16(ps[0][2], ps[0][3]);
+          a[2] = pack_f16(ps[1][0], ps[1][1]);
+          a[3] = pack_f16(ps[1][2], ps[1][3]);
+          for (int r = 0; r < 2; ++r)
+            for (int nt = 0; nt < 2; ++nt)
+              for (int cc = 0; cc < 2; ++cc)
+                cterm[r][gv] += p[nt][2 * r + cc] * mz[2 * nt + cc] - 1024.f * ps[nt][2 * r + cc];
+          // B: codes of tokens (2tid, 2tid+1) and (2tid+8, 2tid+9) at channels
+          // 32 gv + 4 gid + jj, jj = 0..3 (one n-tile per jj)
+          uint32_t cw[4];
+          for (int i = 0; i < 4; ++i) {
+            const unsigned char* row = st + C::VC_OFF + (tile_off + tok[i]) * C::CODE_B;
+            cw[i] = BITS == 4 ? *reinterpret_cast<const uint16_t*>(row + 16 * gv + 2 * gid)
+                              : *reinterpret_cast<const uint8_t*>(row + 8 * gv + gid);
+          }
+          const uint32_t x01 = cw[0] | (cw[1] << 16), x23 = cw[2] | (cw[3] << 16);
+          for (int jj = 0; jj < 4; ++jj)
+            mma16816_f16(o[4 * gv + jj], a, magic2h(x01 >> (BITS * jj), kmask),
+                         magic2h(x23 >> (BITS * jj), kmask));
+        }
+      } else {  // full-precision values (bf16 -> fp16 for the fp16 MMA)
+        uint32_t a[4];
+        a[0] = pack_f16(p[0][0], p[0][1]);
+        a[1] = pack_f16(p[0][2], p[0][3]);
+        a[2] = pack_f16(p[1][0], p[1][1]);
+        a[3] = pack_f16(p[1][2], p[1][3]);
+        for (int gv = 0; gv < NG; ++gv) {
+          uint2 vw[4];
+          for (int i = 0; i < 4; ++i) {
+            const int t = t0 + tok[i];
+            const bool ok = t < te;
+            const __nv_bfloat16* vrow =
+                plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, hkv, ok ? t % g.ring : 0);
+            vw[i] = ok ? *reinterpret_cast<const uint2*>(vrow + 32 * gv + 4 * gid)
+                       : make_uint2(0, 0);
+          }
+          for (int jj = 0; jj < 4; ++jj) {
+            auto el = [&](int i) {
+              const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&vw[i]);
+              return __bfloat162float(e[jj]);
+            };
+            mma16816_f16(o[4 * gv + jj], a, pack_f16(el(0), el(1)), pack_f16(el(2), el(3)));
+          }
+        }
+      }
+    }
+    __syncthreads();                                  // every warp is done with the stage
+    if (leader && chunk + kStages < nchunks) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      issue(chunk + kStages);
+    }
+  }
+  if (timed_out) {
+    // flag the error, then drain (again bounded) the copies still in flight
+    if (threadIdx.x == 0) {
+      atomicOr(err, 1);
+      for (int c = chunk + 1; c < min(nchunks, chunk + kStages); ++c)
+        mbar_wait(&full_bar[c % kStages], (c / kStages) & 1);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+      for (int i = 0; i < kStages; ++i) mbar_inval(&full_bar[i]);
+    __syncthreads();
+    return;
+  }
+  // ---- finish: reduce l and the offset terms over the 4 lanes of a row ----
+  for (int r = 0; r < 2; ++r) {
+    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 1);
+    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 2);
+    for (int gv = 0; gv < NG; ++gv) {
+      cterm[r][gv] += __shfl_xor_sync(0xffffffffu, cterm[r][gv], 1);
+      cterm[r][gv] += __shfl_xor_sync(0xffffffffu, cterm[r][gv], 2);
+    }
+  }
+  // o columns: n-tile j = 4 gv + jj holds channels 32 gv + 4 col + jj at
+  // columns col = 2tid, 2tid + 1
+  float* osm = reinterpret_cast<float*>(smem);        // [kWarps][16][D]
+  __syncthreads();
+  if (warp < kWarps) {
+    for (int j = 0; j < NT_PV; ++j) {
+      const int gv = j >> 2, jj = j & 3;
+      for (int i = 0; i < 4; ++i) {
+        const int row = gid + 8 * (i >> 1), col = 2 * tid + (i & 1);
+        const int d = 32 * gv + 4 * col + jj;
+        osm[(warp * 16 + row) * D + d] = o[j][i] + cterm[i >> 1][gv];
+      }
+    }
+  }
+  if (warp < kWarps && tid == 0) {
+    red_m[warp][gid] = m_run[0];
+    red_m[warp][gid + 8] = m_run[1];
+    red_l[warp][gid] = l_run[0];
+    red_l[warp][gid + 8] = l_run[1];
+  }
+  __syncthreads();
+  // merge the warps and write the split's partial (m in natural-log units)
+  for (int i = threadIdx.x; i < grp * (D + kWsStride); i += blockDim.x) {
+    const int row = i / (D + kWsStride), c = i % (D + kWsStride);
+    float M = -INFINITY;
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w][row]);
+    float val = 0.f;
+    if (c == 0) {
+      val = M == -INFINITY ? -INFINITY : M / l2e;
+    } else {
+      for (int w = 0; w < kWarps; ++w) {
+        const float mw = red_m[w][row];
+        if (mw == -INFINITY) continue;
+        const float f = exp2f(mw - M);
+        val += f * (c == 1 ? red_l[w][row] : osm[(w * 16 + row) * D + c - 2]);
+      }
+    }
+    float* wsr = reinterpret_cast<float*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
+                 (((int64_t)b * g.Hq + hkv * grp + row) * kMaxSplits + split) * (D + kWsStride);
+    wsr[c] = val;
+  }
+  // ---- the last split CTA of this (sequence, kv head) merges all splits ----
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned prev = atomicAdd(&g.counters[b * g.H + hkv], 1u);
+    last_cta = prev == (unsigned)g.splits - 1;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0)                       // all copies were consumed: retire the barriers
+    for (int i = 0; i < kStages; ++i) mbar_inval(&full_bar[i]);
+  if (!last_cta) {
+    __syncthreads();
+    return;
+  }
+  __threadfence();
+  const float* wbase = reinterpret_cast<const float*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
+                       ((int64_t)b * g.Hq + hkv * grp) * kMaxSplits * (D + kWsStride);
+  // per row: split weights exp(m_s - M) / sum_s exp(m_s - M) l_s in shared
+  // memory (reusing the pipeline buffers), then each output sums over splits
+  // with 8 independent loads in flight
+  float* fw = reinterpret_cast<float*>(smem);          // [16][kMaxSplits]
+  const int S = g.splits;
+  for (int row = warp; row < grp; row += blockDim.x >> 5) {
+    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride);
+    const float m = lane < S ? __ldcg(w + lane * (D + kWsStride)) : -INFINITY;
+    const float l = lane < S ? __ldcg(w + lane * (D + kWsStride) + 1) : 0.f;
+    float M = m;
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float f = m == -INFINITY ? 0.f : expf(m - M);
+    float L = f * l;
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (lane < kMaxSplits) fw[row * kMaxSplits + lane] = L > 0.f ? f / L : 0.f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < grp * (D / 2); i += blockDim.x) {
+    const int row = i / (D / 2), d = 2 * (i % (D / 2));
+    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride) + 2 + d;
+    float2 v[kMaxSplits];
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp)
+      v[sp] = sp < S ? __ldcg(reinterpret_cast<const float2*>(w + sp * (D + kWsStride)))
+                     : make_float2(0.f, 0.f);
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp) {
+      const float f = sp < S ? fw[row * kMaxSplits + sp] : 0.f;
+      a0 += f * v[sp].x;
+      a1 += f * v[sp].y;
+    }
+    *reinterpret_cast<__nv_bfloat162*>(out + ((int64_t)b * g.Hq + hkv * grp + row) * D + d) =
+        __floats2bfloat162_rn(a0, a1);
+  }
+  if (threadIdx.x == 0) g.counters[b * g.H + hkv] = 0;   // ready for the next call
+  __syncthreads();
+}
+
+template <int D, int BITS, int FMT>
+__host__ __device__ constexpr size_t attn_smem_bytes() {
+  using C = Cfg<D, BITS, FMT>;
+  return (size_t)kStages * C::STAGE_B > (size_t)kWarps * 16 * D * sizeof(float)
+             ? (size_t)kStages * C::STAGE_B : (size_t)kWarps * 16 * D * sizeof(float);
+}
+
+
+}  // namespace dattn
+}  // namespace kvq

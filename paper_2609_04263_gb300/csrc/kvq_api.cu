@@ -424,6 +424,63 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
   return KVQ_OK;
 }
 
+kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void* w_qkv,
+                           const void* a_q, const void* b_q, int r_q,
+                           const void* a_k, const void* b_k, int r_k,
+                           const void* a_v, const void* b_v, int r_v,
+                           float alpha_over_r, float rope_base, float softmax_scale,
+                           void* q, void* k, void* v, void* out, void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  const Geom& g = cache->g;
+  if (!out) return fail(KVQ_ERR_ARG, "out is NULL");
+  if (misaligned(out)) return fail(KVQ_ERR_ARG, "out must be 16-byte aligned");
+  if (!(softmax_scale > 0.f)) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
+  if (cache->T + 1 > g.Tmax)
+    return fail(KVQ_ERR_CAPACITY, "decode step on a full cache (%d tokens)", cache->T);
+  const int r[3] = {r_q, r_k, r_v};
+  const void* a[3] = {a_q, a_k, a_v};
+  const void* bm[3] = {b_q, b_k, b_v};
+  if (g.act == KVQ_BF16 && decode_step_supported(g, d_in, r)) {
+    // same validation as the separate calls
+    kvq_status st = KVQ_OK;
+    if (d_in <= 0 || d_in % 64) st = fail(KVQ_ERR_SHAPE, "d_in %d must be a multiple of 64", d_in);
+    if (!x || !w_qkv || !q || !k || !v) st = fail(KVQ_ERR_ARG, "NULL tensor pointer");
+    if (st == KVQ_OK && (misaligned(x) || misaligned(w_qkv) || misaligned(q) || misaligned(k) ||
+                         misaligned(v)))
+      st = fail(KVQ_ERR_ARG, "tensor pointers must be 16-byte aligned");
+    for (int p = 0; p < 3 && st == KVQ_OK; ++p) {
+      if (r[p] < 0 || r[p] % 8) st = fail(KVQ_ERR_SHAPE, "bf16 rank %d not a multiple of 8", r[p]);
+      else if (r[p] > 0 && (!a[p] || !bm[p])) st = fail(KVQ_ERR_ARG, "rank %d but NULL factor", r[p]);
+      else if (r[p] > 0 && (misaligned(a[p]) || misaligned(bm[p])))
+        st = fail(KVQ_ERR_ARG, "LoRA factors must be 16-byte aligned");
+    }
+    if (st != KVQ_OK) return st;
+    const void* aa[3] = {r_q ? a_q : nullptr, r_k ? a_k : nullptr, r_v ? a_v : nullptr};
+    const void* bb[3] = {r_q ? b_q : nullptr, r_k ? b_k : nullptr, r_v ? b_v : nullptr};
+    int* err = device_error_word();
+    if (!err) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = ensure_init(cache, s);
+    void* qkv[3] = {q, k, v};
+    if (e == cudaSuccess)
+      e = launch_decode_step(g, x, d_in, w_qkv, aa, bb, r, alpha_over_r, rope_base, softmax_scale,
+                             qkv, out, err, s);
+    if (e != cudaErrorNotSupported) {
+      if (e != cudaSuccess) return cuda_fail(e, "kvq_decode_step launch");
+      cache->T += 1;
+      return KVQ_OK;
+    }
+    (void)cudaGetLastError();
+  }
+  // general path: the three calls in sequence
+  kvq_status st = kvq_project_lora(x, g.B, 1, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v,
+                                   r_v, alpha_over_r, g.Hq, g.H, g.D, 0, cache, rope_base, g.act,
+                                   q, k, v, stream);
+  if (st == KVQ_OK) st = kvq_append_pack(cache, k, v, 1, stream);
+  if (st == KVQ_OK) st = kvq_attend_decode(cache, q, g.Hq, softmax_scale, out, stream);
+  return st;
+}
+
 kvq_status kvq_device_status(void* stream, int* out) {
   if (!out) return fail(KVQ_ERR_ARG, "out is NULL");
   int* p = device_error_word();

@@ -132,6 +132,14 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               cudaStream_t s);
 void rope_theta_table(float rope_base, int D, float* hi, float* lo);
 
+// Fused decode step (decode_step.cu): projection of the new token, append,
+// decode attention in one cooperative kernel.
+bool decode_step_supported(const Geom& g, int d_in, const int r[3]);
+cudaError_t launch_decode_step(const Geom& g, const void* x, int d_in, const void* w,
+                               const void* const a[3], const void* const bm[3], const int r[3],
+                               float alpha_over_r, float rope_base, float scale,
+                               void* const qkv[3], void* out, int* err, cudaStream_t s);
+
 // Decode split-K width for a cache geometry (fixed, independent of T).
 int decode_splits(const Geom& g);
 

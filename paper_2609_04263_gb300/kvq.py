@@ -67,6 +67,10 @@ _SIGS = {
     "kvq_device_status": (c_int, [c_void_p, ctypes.POINTER(c_int)]),
     "kvq_attend_decode_noalloc": (c_int, [c_void_p, c_void_p, c_int, c_float, c_void_p,
                                           c_void_p]),
+    "kvq_decode_step": (c_int, [c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p, c_int,
+                                c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_float,
+                                c_float, c_float, c_void_p, c_void_p, c_void_p, c_void_p,
+                                c_void_p]),
 }
 
 _lib = None
@@ -166,6 +170,14 @@ def kvq_attend_decode_noalloc(handle, q, n_q_heads, softmax_scale, out, stream) 
     device memory instead of the cache's workspace (nothing is allocated)."""
     _check(lib().kvq_attend_decode_noalloc(c_void_p(handle), c_void_p(q), n_q_heads,
                                            softmax_scale, c_void_p(out), c_void_p(stream or 0)))
+
+
+def kvq_decode_step(handle, x, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,
+                    alpha_over_r, rope_base, softmax_scale, q, k, v, out, stream) -> None:
+    P = lambda t: c_void_p(t or 0)
+    _check(lib().kvq_decode_step(c_void_p(handle), P(x), d_in, P(w_qkv), P(a_q), P(b_q), r_q,
+                                 P(a_k), P(b_k), r_k, P(a_v), P(b_v), r_v, alpha_over_r,
+                                 rope_base, softmax_scale, P(q), P(k), P(v), P(out), P(stream)))
 
 
 def kvq_device_status(stream=0) -> int:
