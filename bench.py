@@ -5,8 +5,8 @@ workload (22 layers, batch 4, hidden 2048, 32 query / 4 KV heads, head_dim 64,
 4-bit affine cache with groups of 32, rank-16 LoRA on Q, K and V): reset the
 caches, prefill 2048 tokens per sequence (LoRA Q/K/V projection with RoPE,
 quantize-and-pack append, causal prefill attention, per layer), then 256 decode
-steps (projection, append, split-K decode attention, per layer; one captured
-CUDA graph per decode step).  `value` is tokens processed per second
+steps (projection, append, split-K decode attention: one fused kvq_decode_step
+kernel per layer; one captured CUDA graph per decode step).  `value` is tokens processed per second
 (batch x (prefill + decode) tokens per step); the decode phase alone, pack
 bandwidth and projection TFLOP/s are reported beside it.
 
@@ -86,6 +86,14 @@ def decode_attn_bytes(wl, T):
     return B * H * T * code_bytes_per_token(wl) + 2 * B * Hq * D * 2
 
 
+def decode_step_bytes(wl, T):
+    """HBM bytes of one fused decode step of one layer: the projection's
+    weights, factors, input and q/k/v outputs, the new token's packed codes,
+    the cache read by attention over T tokens and its output."""
+    B, H = wl.batch, wl.n_kv_heads
+    return proj_bytes(wl, B) + B * H * code_bytes_per_token(wl) + decode_attn_bytes(wl, T)
+
+
 def prefill_attn_flops(wl, L, T):
     """Causal: query l (position T - L + l) sees T - L + l + 1 keys; QK^T and
     PV each 2 D flops per visible key."""
@@ -135,6 +143,10 @@ class Runner:
         self.graph = None
         self.events = None
         self.eager = False
+        # decode steps through kvq_decode_step (one fused kernel per layer
+        # where the cache format allows) unless separate calls are asked for
+        self.separate = False
+        self.fused = self.caches[0].decode_step_fused(wl.d_in, self.layers[0][1])
 
     # one layer's calls ----------------------------------------------------
     def _project(self, l, x, out):
@@ -165,6 +177,17 @@ class Runner:
                 timer("attend_prefill", 1)
 
     def decode_step_eager(self, timer=None):
+        if not self.separate:
+            wl = self.wl
+            for l, c in enumerate(self.caches):
+                w, lora = self.layers[l]
+                if timer:
+                    timer("decode_step", 0)
+                c.decode_step(self.xs, w, lora, wl.alpha_over_r, wl.rope_base, qkv=self.dec,
+                              out=self.o_dec)
+                if timer:
+                    timer("decode_step", 1)
+            return
         for l, c in enumerate(self.caches):
             if timer:
                 timer("project_decode", 0)
@@ -179,6 +202,13 @@ class Runner:
             c.attend_decode(q, out=self.o_dec)
             if timer:
                 timer("attend_decode", 1)
+
+    def decode_step_layers(self):
+        wl = self.wl
+        for l, c in enumerate(self.caches):
+            w, lora = self.layers[l]
+            c.decode_step(self.xs, w, lora, wl.alpha_over_r, wl.rope_base, qkv=self.dec,
+                          out=self.o_dec)
 
     # the three decode call classes, each over all layers (for timing)
     def decode_project_layers(self):
@@ -225,13 +255,25 @@ class Runner:
         if phase_events:
             phase_events[2].record()
 
+    def decode_path(self):
+        if self.separate:
+            return "three calls per layer (project, append, attend)"
+        return ("kvq_decode_step: one fused kernel per layer" if self.fused else
+                "kvq_decode_step: three kernels per layer")
+
     def launches_per_step(self):
+        """Kernels the library launches in one whole-job step."""
         wl = self.wl
         append = {synth.FMT_FLOAT: 1, synth.FMT_AFFINE: 1, synth.FMT_SYMMETRIC: 1,
                   synth.FMT_KIVI: 3, synth.FMT_KVARN: 2}[wl.fmt]
+        # decode attention merges its splits in its last CTA on the
+        # tensor-core path (bf16, affine/symmetric/KIVI), else in a second kernel
+        attend = 1 if (wl.dtype == "bf16" and wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC,
+                                                         synth.FMT_KIVI)
+                       and wl.head_dim in (64, 128)) else 2
         prefill = wl.layers * (1 + append + 1)
-        decode = wl.decode * wl.layers * (1 + append + 2)
-        return prefill + decode
+        per_layer = 1 if (self.fused and not self.separate) else 1 + append + attend
+        return prefill + wl.decode * wl.layers * per_layer
 
 
 class EventTimer:
@@ -447,6 +489,8 @@ def main():
                     help="attention layers (default: the workload's)")
     ap.add_argument("--eager-decode", action="store_true",
                     help="launch decode steps directly instead of replaying a graph")
+    ap.add_argument("--separate-decode", action="store_true",
+                    help="decode through the three separate calls, not kvq_decode_step")
     ap.add_argument("--timed-only", action="store_true",
                     help="skip the per-kernel, end-to-end and CPU passes")
     args = ap.parse_args()
@@ -471,6 +515,7 @@ def main():
     peaks, peak_kind = load_peaks()
     run = Runner(wl, device)
     run.eager = args.eager_decode
+    run.separate = args.separate_decode
     if not run.eager:
         run.capture()
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=device)
@@ -505,7 +550,8 @@ def main():
         if rank == 0:
             print(json.dumps({"timed_only": True, "ms_per_step": statistics.mean(step_ms),
                               "workload": wl.name, "decode": wl.decode,
-                              "eager_decode": run.eager}), flush=True)
+                              "eager_decode": run.eager, "decode_path": run.decode_path()}),
+              flush=True)
         return
 
     # ---- per-kernel durations ---------------------------------------------
@@ -520,20 +566,25 @@ def main():
     mean_ms = timer.mean_ms()
     run.xs.copy_(run.x_dec[0])
     reps = 10
-    T_prof = wl.prefill + 2 + reps          # cache length during the attention replays
-    for name, fn in (("project_decode", run.decode_project_layers),
-                     ("append_decode", run.decode_append_layers),
-                     ("attend_decode", run.decode_attend_layers)):
-        mean_ms[name] = graph_time_ms(fn, reps) / wl.layers
-    T_dec = T_prof
+    n_dec = wl.layers * wl.decode
     work = {
         "project": ("tensor", proj_flops(wl, wl.batch * wl.prefill), wl.layers),
         "attend_prefill": ("tensor", prefill_attn_flops(wl, wl.prefill, wl.prefill), wl.layers),
         "append": ("hbm", pack_bytes(wl, wl.prefill), wl.layers),
-        "project_decode": ("hbm", proj_bytes(wl, wl.batch), wl.layers * wl.decode),
-        "append_decode": ("hbm", pack_bytes(wl, 1), wl.layers * wl.decode),
-        "attend_decode": ("hbm", decode_attn_bytes(wl, T_dec), wl.layers * wl.decode),
     }
+    if run.separate:
+        for name, fn in (("project_decode", run.decode_project_layers),
+                         ("append_decode", run.decode_append_layers),
+                         ("attend_decode", run.decode_attend_layers)):
+            mean_ms[name] = graph_time_ms(fn, reps) / wl.layers
+        T_dec = wl.prefill + 2 + reps          # cache length during the attention replays
+        work["project_decode"] = ("hbm", proj_bytes(wl, wl.batch), n_dec)
+        work["append_decode"] = ("hbm", pack_bytes(wl, 1), n_dec)
+        work["attend_decode"] = ("hbm", decode_attn_bytes(wl, T_dec), n_dec)
+    else:
+        mean_ms["decode_step"] = graph_time_ms(run.decode_step_layers, reps) / wl.layers
+        T_dec = wl.prefill + 2 + reps // 2     # mean cache length over the timed replays
+        work["decode_step"] = ("hbm", decode_step_bytes(wl, T_dec), n_dec)
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)
     bound, amount, _ = work[dominant]
@@ -597,6 +648,7 @@ def main():
                 "lora_rank": wl.rank, "tokens_per_step": tokens_per_step,
                 "l2": "flushed (256 MiB write) between timed steps; job working set > L2",
                 "parallelism": f"replicas x{world}",
+                "decode_path": run.decode_path(),
             },
             "phases": {"prefill_ms": statistics.mean(pre_ms), "decode_ms": statistics.mean(dec_ms),
                        "decode_tokens_per_s": decode_tps,

@@ -232,6 +232,13 @@ kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void
                            void* q, void* k, void* v, void* out, void* stream);
 
 /*
+ * 1 when kvq_decode_step on `cache` with this d_in and these LoRA ranks runs
+ * as the one fused kernel, 0 when it runs the three separate calls, -1 when
+ * cache is NULL.  Launches nothing.
+ */
+int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, int r_v);
+
+/*
  * kvq_attend_decode for callers that cannot allocate device memory.  (No
  * counterpart in the paper: this is a deployment variant of the decode step.)
  *

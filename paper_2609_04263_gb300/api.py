@@ -101,6 +101,12 @@ class Cache:
                             _stream())
         return qkv, out
 
+    def decode_step_fused(self, d_in, lora) -> bool:
+        """Whether decode_step with this d_in and these LoRA factors runs as
+        one fused kernel."""
+        r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
+        return kvq.kvq_decode_step_fused(self.handle, d_in, *r)
+
     def planes(self) -> dict:
         """name -> tensor view [B, H, rows, cols] of each present plane."""
         v = kvq.kvq_cache_view(self.handle)

@@ -13,8 +13,11 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
   pdl_wait();
   pdl_trigger();
   extern __shared__ __align__(128) unsigned char smem[];
-  decode_split<D, BITS, FMT>(g, q, scale, err, out, blockIdx.x, blockIdx.y, blockIdx.z,
-                             cache_tokens(g), smem);
+  __shared__ uint64_t bars[kStages];
+  const int grp = g.Hq / g.H;
+  decode_split<D, BITS, FMT, kStages, kWarps>(
+      g, q + ((int64_t)blockIdx.z * g.Hq + blockIdx.y * grp) * D, scale, err, out, blockIdx.x,
+      g.splits, kMaxSplits, blockIdx.y, blockIdx.z, cache_tokens(g), smem, bars, false);
 }
 
 template <int D, int BITS, int FMT>

@@ -73,6 +73,22 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
 
+// Tagged words: a float in the low half, the writer's launch tag in the high
+// half, stored and loaded as one 64-bit access, so a reader that sees its own
+// launch's tag also sees that launch's value (no fence or flag needed).
+constexpr long kPollLimit = 1L << 20;   // polls of one L2 round trip: about a second
+__device__ __forceinline__ void st_tagged(uint64_t* p, float v, uint32_t tag) {
+  const uint64_t w = (uint64_t)__float_as_uint(v) | ((uint64_t)tag << 32);
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_tagged(const uint64_t* p) {
+  uint64_t w;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
+  return w;
+}
+__device__ __forceinline__ float tagged_value(uint64_t w) { return __uint_as_float((uint32_t)w); }
+__device__ __forceinline__ bool tag_is(uint64_t w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
+
 __device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32_t b0,
                                          uint32_t b1) {
   asm volatile(
@@ -139,25 +155,171 @@ struct Cfg {
   static constexpr int STAGE_B = ((VZ_OFF + kCT * NG * 2) + 127) / 128 * 128;
 };
 
+// Token range of one split: [ts, te), coded tokens [0, tq), chunks of kCT.
+struct SplitPlan {
+  int ts, te, tq, nchunks;
+};
+template <int FMT>
+__device__ __forceinline__ SplitPlan split_plan(const Geom& g, int T, int splits, int split) {
+  SplitPlan p;
+  split_range(T, splits, split, kCT, &p.ts, &p.te);
+  p.tq = FMT == KVQ_FMT_KIVI ? kivi_tq(T, g.R, 32) : T;
+  p.nchunks = p.te > p.ts ? (p.te - p.ts + kCT - 1) / kCT : 0;
+  return p;
+}
+
+// Copies of one chunk (codes and fp16 metadata) into stage chunk % STAGES.
+// One thread calls it.
+template <int D, int BITS, int FMT, int STAGES>
+__device__ void split_issue(const Geom& g, int b, int hkv, const SplitPlan& sp, int chunk,
+                            unsigned char* smem, uint64_t* bars) {
+  using C = Cfg<D, BITS, FMT>;
+  constexpr int NG = C::NG;
+  const int stage = chunk % STAGES;
+  unsigned char* st = smem + stage * C::STAGE_B;
+  const int c0 = sp.ts + chunk * kCT;
+  int nq = min(kCT, sp.tq - c0);              // coded tokens of the chunk
+  if (nq <= 0) {                              // nothing coded: arrive with no bytes
+    mbar_expect_tx(&bars[stage], 0);
+    return;
+  }
+  nq = (nq + 3) & ~3;                         // 16-byte multiples (planes padded)
+  const uint32_t code_bytes = nq * C::CODE_B;
+  const uint32_t kmeta = FMT == KVQ_FMT_KIVI ? ((nq + 31) / 32) * D * 2 : nq * NG * 2;
+  const uint32_t vmeta = nq * NG * 2;
+  const bool zero_planes = FMT != KVQ_FMT_SYMMETRIC;
+  uint32_t total = 2 * code_bytes + kmeta + vmeta;
+  if (zero_planes) total += kmeta + vmeta;
+  mbar_expect_tx(&bars[stage], total);
+  bulk_g2s(st + C::KC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, c0), code_bytes,
+           &bars[stage]);
+  bulk_g2s(st + C::VC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
+           &bars[stage]);
+  if (FMT == KVQ_FMT_KIVI) {
+    bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
+             &bars[stage]);
+    bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
+             &bars[stage]);
+  } else {
+    bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,
+             &bars[stage]);
+    if (zero_planes)
+      bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0), kmeta,
+               &bars[stage]);
+  }
+  bulk_g2s(st + C::VS_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, c0), vmeta,
+           &bars[stage]);
+  if (zero_planes)
+    bulk_g2s(st + C::VZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, c0), vmeta,
+             &bars[stage]);
+}
+
+// Initialise the stage barriers and issue the first STAGES chunks of a split.
+// Every thread of the CTA calls it.
+template <int D, int BITS, int FMT, int STAGES>
+__device__ void split_prologue(const Geom& g, int b, int hkv, const SplitPlan& sp,
+                               unsigned char* smem, uint64_t* bars) {
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < STAGES; ++i) mbar_init(&bars[i], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    for (int c = 0; c < min(STAGES, sp.nchunks); ++c)
+      split_issue<D, BITS, FMT, STAGES>(g, b, hkv, sp, c, smem, bars);
+  }
+  __syncthreads();
+}
+
+// Merge the tagged split partials of the query heads of kv head hkv of
+// sequence b into out, polling each word until it carries `tag`.  Each
+// output pair takes m, l and its two values from every split in one pass.
+template <int D>
+__device__ void merge_tagged(const Geom& g, __nv_bfloat16* __restrict__ out, int b, int hkv,
+                             int grp, int S, int sstride, uint32_t tag, int* err) {
+  const uint64_t* wbase = reinterpret_cast<const uint64_t*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
+                          ((int64_t)b * g.Hq + hkv * grp) * sstride * (D + kWsStride);
+  constexpr int SB = 16;
+  for (int i = threadIdx.x; i < grp * (D / 2); i += blockDim.x) {
+    const int row = i / (D / 2), d = 2 * (i % (D / 2));
+    const uint64_t* w = wbase + (int64_t)row * sstride * (D + kWsStride);
+    float M = -INFINITY, L = 0.f, a0 = 0.f, a1 = 0.f;
+    for (int s0 = 0; s0 < S; s0 += SB) {
+      float ms[SB], ls[SB], v0[SB], v1[SB];
+      for (long it = 0;; ++it) {
+        bool ok = true;
+#pragma unroll
+        for (int k = 0; k < SB; ++k) {
+          const int sp = s0 + k;
+          ms[k] = -INFINITY;
+          ls[k] = v0[k] = v1[k] = 0.f;
+          if (sp < S) {
+            const uint64_t* ws = w + sp * (D + kWsStride);
+            const uint64_t wm = ld_tagged(ws), wl = ld_tagged(ws + 1);
+            const uint64_t w0 = ld_tagged(ws + 2 + d), w1 = ld_tagged(ws + 3 + d);
+            ok = ok && tag_is(wm, tag) && tag_is(wl, tag) && tag_is(w0, tag) && tag_is(w1, tag);
+            ms[k] = tagged_value(wm);
+            ls[k] = tagged_value(wl);
+            v0[k] = tagged_value(w0);
+            v1[k] = tagged_value(w1);
+          }
+        }
+        if (ok) break;
+        if (it > kPollLimit) {
+          atomicOr(err, 2);
+          break;
+        }
+      }
+      float Mb = M;
+#pragma unroll
+      for (int k = 0; k < SB; ++k) Mb = fmaxf(Mb, ms[k]);
+      if (Mb == -INFINITY) continue;
+      const float r = M == -INFINITY ? 0.f : expf(M - Mb);
+      L *= r;
+      a0 *= r;
+      a1 *= r;
+#pragma unroll
+      for (int k = 0; k < SB; ++k) {
+        const float f = ms[k] == -INFINITY ? 0.f : expf(ms[k] - Mb);
+        L += f * ls[k];
+        a0 += f * v0[k];
+        a1 += f * v1[k];
+      }
+      M = Mb;
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    *reinterpret_cast<__nv_bfloat162*>(out + ((int64_t)b * g.Hq + hkv * grp + row) * D + d) =
+        __floats2bfloat162_rn(a0 * inv, a1 * inv);
+  }
+}
+
 // One split of one (sequence, kv head): blockIdx-independent, so a fused
-// kernel can run several per CTA.  T = tokens stored (read by the caller).
-// smem: the dynamic buffer of at least attn_smem_bytes<D, BITS, FMT>().
-template <int D, int BITS, int FMT>
-__device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q, float scale,
-                             int* err, __nv_bfloat16* __restrict__ out, int split, int hkv, int b,
-                             int T, unsigned char* smem) {
+// kernel can run several per CTA.  T = tokens stored (read by the caller);
+// `splits` splits share the tokens.  qg: the query rows of the kv head's
+// query heads (row hl at qg + hl D, global or shared memory).  The CTA has
+// NW warps (a multiple of 4): each step takes NW / 4 chunks, one 16-token
+// tile per warp.  smem: at least attn_smem_bytes<D, BITS, FMT, STAGES, NW>()
+// bytes; full_bar: STAGES mbarriers in shared memory.  With `prologue_done`
+// the caller already ran split_prologue (to start the copies early).  The
+// split partials of query head (b, h) sit in the workspace at element
+// ((b Hq + h) sstride + split) (D + 2) (sstride >= splits).  With tag == 0
+// they are floats and the last split CTA to arrive (an atomic counter)
+// merges; otherwise they are tagged words and the CTA called with `merger`
+// polls the other splits' words and merges.
+template <int D, int BITS, int FMT, int STAGES, int NW>
+__device__ void decode_split(const Geom& g, const __nv_bfloat16* qg, float scale, int* err,
+                             __nv_bfloat16* __restrict__ out, int split, int splits, int sstride,
+                             int hkv, int b, int T, unsigned char* smem, uint64_t* full_bar,
+                             bool prologue_done, uint32_t tag = 0, bool merger = false) {
   using C = Cfg<D, BITS, FMT>;
   constexpr int NG = C::NG, KSTEP = C::KSTEP, NT_PV = C::NT_PV;
-  __shared__ uint64_t full_bar[kStages];
-  __shared__ float red_m[kWarps][16], red_l[kWarps][16];
+  constexpr int GCH = NW / kWarps;                    // chunks per step
+  static_assert(NW % kWarps == 0 && STAGES >= GCH, "warps cover whole chunks");
+  __shared__ float red_m[NW][16], red_l[NW][16], wsc[NW][16];
   __shared__ int last_cta;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gid = lane >> 2, tid = lane & 3;
-  int ts, te;
-  split_range(T, g.splits, split, kCT, &ts, &te);
+  const SplitPlan sp = split_plan<FMT>(g, T, splits, split);
+  const int ts = sp.ts, te = sp.te, tq = sp.tq;
   const int grp = g.Hq / g.H;
-  const int tq = FMT == KVQ_FMT_KIVI ? kivi_tq(T, g.R, 32) : T;   // coded tokens [0, tq)
   const float l2e = 1.4426950408889634f;
   const float qk_scale = scale * l2e;                 // scores in log2 units
 
@@ -168,13 +330,16 @@ __device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q,
   for (int r = 0; r < 2; ++r) {
     const int hl = gid + 8 * r;
     for (int gq = 0; gq < NG; ++gq) {
+      uint4 u = make_uint4(0, 0, 0, 0);
+      if (hl < grp) u = *reinterpret_cast<const uint4*>(qg + hl * D + 32 * gq + 8 * tid);
+      const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&u);
       float s = 0.f;
-      for (int e = 0; e < 8; ++e) {
-        float v = 0.f;
-        if (hl < grp)
-          v = __bfloat162float(q[((int64_t)b * g.Hq + hkv * grp + hl) * D + 32 * gq + 8 * tid + e]);
-        qv[r][gq][e] = v;
-        s += v;
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __bfloat1622float2(h2[e]);
+        qv[r][gq][2 * e] = f.x;
+        qv[r][gq][2 * e + 1] = f.y;
+        s += f.x;
+        s += f.y;
       }
       qsum[gq][r] = s;       // partial over this thread's 8 channels
     }
@@ -219,72 +384,28 @@ __device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q,
   for (int gq = 0; gq < NG; ++gq) cterm[0][gq] = cterm[1][gq] = 0.f;
 
   // ---- chunk pipeline ------------------------------------------------------
-  const int nchunks = te > ts ? (te - ts + kCT - 1) / kCT : 0;
+  const int nchunks = sp.nchunks;
   const bool leader = threadIdx.x == 0;
-  if (leader)
-    for (int i = 0; i < kStages; ++i) mbar_init(&full_bar[i], 1);
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  __syncthreads();
-
-  auto issue = [&](int chunk) {
-    const int stage = chunk % kStages;
-    unsigned char* st = smem + stage * C::STAGE_B;
-    const int c0 = ts + chunk * kCT;
-    int nq = min(kCT, tq - c0);                 // coded tokens of the chunk
-    if (nq <= 0) {                              // nothing coded: arrive with no bytes
-      mbar_expect_tx(&full_bar[stage], 0);
-      return;
-    }
-    nq = (nq + 3) & ~3;                         // 16-byte multiples (planes padded)
-    const uint32_t code_bytes = nq * C::CODE_B;
-    const uint32_t kmeta = FMT == KVQ_FMT_KIVI ? ((nq + 31) / 32) * D * 2 : nq * NG * 2;
-    const uint32_t vmeta = nq * NG * 2;
-    const bool zero_planes = FMT != KVQ_FMT_SYMMETRIC;
-    uint32_t total = 2 * code_bytes + kmeta + vmeta;
-    if (zero_planes) total += kmeta + vmeta;
-    mbar_expect_tx(&full_bar[stage], total);
-    bulk_g2s(st + C::KC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, c0), code_bytes,
-             &full_bar[stage]);
-    bulk_g2s(st + C::VC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
-             &full_bar[stage]);
-    if (FMT == KVQ_FMT_KIVI) {
-      bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
-               &full_bar[stage]);
-      bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
-               &full_bar[stage]);
-    } else {
-      bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,
-               &full_bar[stage]);
-      if (zero_planes)
-        bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0), kmeta,
-                 &full_bar[stage]);
-    }
-    bulk_g2s(st + C::VS_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, c0), vmeta,
-             &full_bar[stage]);
-    if (zero_planes)
-      bulk_g2s(st + C::VZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, c0), vmeta,
-               &full_bar[stage]);
-  };
-  if (leader)
-    for (int c = 0; c < min(kStages, nchunks); ++c) issue(c);
+  if (!prologue_done) split_prologue<D, BITS, FMT, STAGES>(g, b, hkv, sp, smem, full_bar);
 
   bool timed_out = false;
   const uint32_t kmask = BITS == 4 ? 0x000F000Fu : 0x00030003u;
   const int zbias = FMT == KVQ_FMT_SYMMETRIC ? (1 << (BITS - 1)) : 0;
 
+  const int wchunk = warp / kWarps;                  // chunk of the step this warp takes
+  const int tile_off = 16 * (warp % kWarps);         // its tile's row offset in the chunk
   int chunk = 0;
-  for (; chunk < nchunks; ++chunk) {
-    const int stage = chunk % kStages;
-    const bool ok = mbar_wait(&full_bar[stage], (chunk / kStages) & 1);
+  for (; chunk < nchunks; chunk += GCH) {
+    const int my = chunk + wchunk;
+    bool ok = true;
+    if (my < nchunks) ok = mbar_wait(&full_bar[my % STAGES], (my / STAGES) & 1);
     if (__syncthreads_or(!ok)) {        // the same decision in every thread
       timed_out = true;
       break;
     }
-    const unsigned char* st = smem + stage * C::STAGE_B;
-    const int c0 = ts + chunk * kCT;
-    const int t0 = c0 + 16 * warp;                   // this warp's tile
-    const int tile_off = 16 * warp;                  // row offset within the chunk
-    if (warp < kWarps && t0 < te) {                  // extra warps (fused kernel) idle
+    const unsigned char* st = smem + (my % STAGES) * C::STAGE_B;
+    const int t0 = ts + my * kCT + tile_off;         // this warp's tile
+    if (my < nchunks && t0 < te) {
       const bool coded = t0 < tq;
       float sacc[2][4];                              // S for n-tiles 0, 1 (tokens t0 + 8nt + col)
       // ---------------- scores ----------------
@@ -503,22 +624,25 @@ __device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q,
         }
       }
     }
-    __syncthreads();                                  // every warp is done with the stage
-    if (leader && chunk + kStages < nchunks) {
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      issue(chunk + kStages);
+    __syncthreads();                                  // every warp is done with the stages
+    if (leader && chunk + STAGES < nchunks) {
+      // shared: the stages were read by generic loads; global: in the fused
+      // step a chunk may hold rows stored earlier in the same kernel
+      asm volatile("fence.proxy.async;" ::: "memory");
+      for (int j = 0; j < GCH && chunk + j + STAGES < nchunks; ++j)
+        split_issue<D, BITS, FMT, STAGES>(g, b, hkv, sp, chunk + j + STAGES, smem, full_bar);
     }
   }
   if (timed_out) {
     // flag the error, then drain (again bounded) the copies still in flight
     if (threadIdx.x == 0) {
       atomicOr(err, 1);
-      for (int c = chunk + 1; c < min(nchunks, chunk + kStages); ++c)
-        mbar_wait(&full_bar[c % kStages], (c / kStages) & 1);
+      for (int c = chunk; c < min(nchunks, chunk + STAGES); ++c)
+        mbar_wait(&full_bar[c % STAGES], (c / STAGES) & 1);
     }
     __syncthreads();
     if (threadIdx.x == 0)
-      for (int i = 0; i < kStages; ++i) mbar_inval(&full_bar[i]);
+      for (int i = 0; i < STAGES; ++i) mbar_inval(&full_bar[i]);
     __syncthreads();
     return;
   }
@@ -533,106 +657,130 @@ __device__ void decode_split(const Geom& g, const __nv_bfloat16* __restrict__ q,
   }
   // o columns: n-tile j = 4 gv + jj holds channels 32 gv + 4 col + jj at
   // columns col = 2tid, 2tid + 1
-  float* osm = reinterpret_cast<float*>(smem);        // [kWarps][16][D]
+  constexpr int OS = D + 1;                           // odd row stride: no bank conflicts
+  float* osm = reinterpret_cast<float*>(smem);        // [NW][16][OS]
   __syncthreads();
-  if (warp < kWarps) {
-    for (int j = 0; j < NT_PV; ++j) {
-      const int gv = j >> 2, jj = j & 3;
-      for (int i = 0; i < 4; ++i) {
-        const int row = gid + 8 * (i >> 1), col = 2 * tid + (i & 1);
-        const int d = 32 * gv + 4 * col + jj;
-        osm[(warp * 16 + row) * D + d] = o[j][i] + cterm[i >> 1][gv];
-      }
+  for (int j = 0; j < NT_PV; ++j) {
+    const int gv = j >> 2, jj = j & 3;
+    for (int i = 0; i < 4; ++i) {
+      const int row = gid + 8 * (i >> 1), col = 2 * tid + (i & 1);
+      const int d = 32 * gv + 4 * col + jj;
+      osm[(warp * 16 + row) * OS + d] = o[j][i] + cterm[i >> 1][gv];
     }
   }
-  if (warp < kWarps && tid == 0) {
+  if (tid == 0) {
     red_m[warp][gid] = m_run[0];
     red_m[warp][gid + 8] = m_run[1];
     red_l[warp][gid] = l_run[0];
     red_l[warp][gid + 8] = l_run[1];
   }
   __syncthreads();
+  // per row: the warps' weights exp2(m_w - M), M = max_w m_w (0 for empty warps)
+  if (threadIdx.x < 16) {
+    const int row = threadIdx.x;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w][row]);
+#pragma unroll
+    for (int w = 0; w < NW; ++w)
+      wsc[w][row] = red_m[w][row] == -INFINITY ? 0.f : exp2f(red_m[w][row] - M);
+  }
+  __syncthreads();
   // merge the warps and write the split's partial (m in natural-log units)
   for (int i = threadIdx.x; i < grp * (D + kWsStride); i += blockDim.x) {
     const int row = i / (D + kWsStride), c = i % (D + kWsStride);
-    float M = -INFINITY;
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w][row]);
     float val = 0.f;
     if (c == 0) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w][row]);
       val = M == -INFINITY ? -INFINITY : M / l2e;
+    } else if (c == 1) {
+#pragma unroll
+      for (int w = 0; w < NW; ++w) val += wsc[w][row] * red_l[w][row];
     } else {
-      for (int w = 0; w < kWarps; ++w) {
-        const float mw = red_m[w][row];
-        if (mw == -INFINITY) continue;
-        const float f = exp2f(mw - M);
-        val += f * (c == 1 ? red_l[w][row] : osm[(w * 16 + row) * D + c - 2]);
-      }
+#pragma unroll
+      for (int w = 0; w < NW; ++w) val += wsc[w][row] * osm[(w * 16 + row) * OS + c - 2];
     }
-    float* wsr = reinterpret_cast<float*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
-                 (((int64_t)b * g.Hq + hkv * grp + row) * kMaxSplits + split) * (D + kWsStride);
-    wsr[c] = val;
+    const int64_t wi = (((int64_t)b * g.Hq + hkv * grp + row) * sstride + split) * (D + kWsStride) + c;
+    if (tag) st_tagged(reinterpret_cast<uint64_t*>(g.pl[KVQ_PLANE_WORKSPACE].p) + wi, val, tag);
+    else reinterpret_cast<float*>(g.pl[KVQ_PLANE_WORKSPACE].p)[wi] = val;
+  }
+  if (tag) {
+    // tagged partials: the merger polls them; everyone else is done
+    __syncthreads();
+    if (threadIdx.x == 0)
+      for (int i = 0; i < STAGES; ++i) mbar_inval(&full_bar[i]);
+    if (merger) merge_tagged<D>(g, out, b, hkv, grp, splits, sstride, tag, err);
+    __syncthreads();
+    return;
   }
   // ---- the last split CTA of this (sequence, kv head) merges all splits ----
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
     const unsigned prev = atomicAdd(&g.counters[b * g.H + hkv], 1u);
-    last_cta = prev == (unsigned)g.splits - 1;
+    last_cta = prev == (unsigned)splits - 1;
   }
   __syncthreads();
   if (threadIdx.x == 0)                       // all copies were consumed: retire the barriers
-    for (int i = 0; i < kStages; ++i) mbar_inval(&full_bar[i]);
+    for (int i = 0; i < STAGES; ++i) mbar_inval(&full_bar[i]);
   if (!last_cta) {
     __syncthreads();
     return;
   }
   __threadfence();
   const float* wbase = reinterpret_cast<const float*>(g.pl[KVQ_PLANE_WORKSPACE].p) +
-                       ((int64_t)b * g.Hq + hkv * grp) * kMaxSplits * (D + kWsStride);
-  // per row: split weights exp(m_s - M) / sum_s exp(m_s - M) l_s in shared
-  // memory (reusing the pipeline buffers), then each output sums over splits
-  // with 8 independent loads in flight
-  float* fw = reinterpret_cast<float*>(smem);          // [16][kMaxSplits]
-  const int S = g.splits;
-  for (int row = warp; row < grp; row += blockDim.x >> 5) {
-    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride);
-    const float m = lane < S ? __ldcg(w + lane * (D + kWsStride)) : -INFINITY;
-    const float l = lane < S ? __ldcg(w + lane * (D + kWsStride) + 1) : 0.f;
-    float M = m;
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float f = m == -INFINITY ? 0.f : expf(m - M);
-    float L = f * l;
-    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    if (lane < kMaxSplits) fw[row * kMaxSplits + lane] = L > 0.f ? f / L : 0.f;
-  }
-  __syncthreads();
+                       ((int64_t)b * g.Hq + hkv * grp) * sstride * (D + kWsStride);
+  // each output pair loads the m, l and values of all splits of its row in
+  // one pass (blocks of 16 splits, rescaled online), then normalises
+  const int S = splits;
+  constexpr int SB = 16;
   for (int i = threadIdx.x; i < grp * (D / 2); i += blockDim.x) {
     const int row = i / (D / 2), d = 2 * (i % (D / 2));
-    const float* w = wbase + (int64_t)row * kMaxSplits * (D + kWsStride) + 2 + d;
-    float2 v[kMaxSplits];
+    const float* w = wbase + (int64_t)row * sstride * (D + kWsStride);
+    float M = -INFINITY, L = 0.f, a0 = 0.f, a1 = 0.f;
+    for (int s0 = 0; s0 < S; s0 += SB) {
+      float ms[SB], ls[SB];
+      float2 v[SB];
 #pragma unroll
-    for (int sp = 0; sp < kMaxSplits; ++sp)
-      v[sp] = sp < S ? __ldcg(reinterpret_cast<const float2*>(w + sp * (D + kWsStride)))
-                     : make_float2(0.f, 0.f);
-    float a0 = 0.f, a1 = 0.f;
+      for (int k = 0; k < SB; ++k) {
+        const int sp = s0 + k;
+        const float* ws = w + sp * (D + kWsStride);
+        ms[k] = sp < S ? __ldcg(ws) : -INFINITY;
+        ls[k] = sp < S ? __ldcg(ws + 1) : 0.f;
+        v[k] = sp < S ? __ldcg(reinterpret_cast<const float2*>(ws + 2 + d)) : make_float2(0.f, 0.f);
+      }
+      float Mb = M;
 #pragma unroll
-    for (int sp = 0; sp < kMaxSplits; ++sp) {
-      const float f = sp < S ? fw[row * kMaxSplits + sp] : 0.f;
-      a0 += f * v[sp].x;
-      a1 += f * v[sp].y;
+      for (int k = 0; k < SB; ++k) Mb = fmaxf(Mb, ms[k]);
+      if (Mb == -INFINITY) continue;
+      const float r = M == -INFINITY ? 0.f : expf(M - Mb);
+      L *= r;
+      a0 *= r;
+      a1 *= r;
+#pragma unroll
+      for (int k = 0; k < SB; ++k) {
+        const float f = ms[k] == -INFINITY ? 0.f : expf(ms[k] - Mb);
+        L += f * ls[k];
+        a0 += f * v[k].x;
+        a1 += f * v[k].y;
+      }
+      M = Mb;
     }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
     *reinterpret_cast<__nv_bfloat162*>(out + ((int64_t)b * g.Hq + hkv * grp + row) * D + d) =
-        __floats2bfloat162_rn(a0, a1);
+        __floats2bfloat162_rn(a0 * inv, a1 * inv);
   }
   if (threadIdx.x == 0) g.counters[b * g.H + hkv] = 0;   // ready for the next call
   __syncthreads();
 }
 
-template <int D, int BITS, int FMT>
+template <int D, int BITS, int FMT, int STAGES = kStages, int NW = kWarps>
 __host__ __device__ constexpr size_t attn_smem_bytes() {
   using C = Cfg<D, BITS, FMT>;
-  return (size_t)kStages * C::STAGE_B > (size_t)kWarps * 16 * D * sizeof(float)
-             ? (size_t)kStages * C::STAGE_B : (size_t)kWarps * 16 * D * sizeof(float);
+  return (size_t)STAGES * C::STAGE_B > (size_t)NW * 16 * (D + 1) * sizeof(float)
+             ? (size_t)STAGES * C::STAGE_B : (size_t)NW * 16 * (D + 1) * sizeof(float);
 }
 
 

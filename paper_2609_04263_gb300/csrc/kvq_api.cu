@@ -176,6 +176,8 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
   g->pl[KVQ_PLANE_WORKSPACE].cols = D + kWsStride;
   g->pl[KVQ_PLANE_WORKSPACE].elem = 4;
   total = align256(total + (size_t)B * d->q_heads * kMaxSplits * (D + kWsStride) * 4);
+  // epoch block of the fused decode step (256 bytes, never reset)
+  total += 256;
   *st = KVQ_OK;
   return total;
 }
@@ -209,7 +211,15 @@ int* device_error_word() {
 // (stream-ordered, so it can be captured with the calls that follow).
 cudaError_t ensure_cache_init(kvq_cache* c, cudaStream_t s) {
   if (!c->need_init) return cudaSuccess;
-  cudaError_t e = cudaMemsetAsync(c->g.state, 0, state_region_bytes(c->g.B, c->g.H), s);
+  cudaError_t e = cudaSuccess;
+  if (c->need_clear) {
+    // once per buffer: the workspace (whose tagged words the fused decode
+    // step matches against its epoch) and the epoch block after it
+    char* ws = static_cast<char*>(c->g.pl[KVQ_PLANE_WORKSPACE].p);
+    e = cudaMemsetAsync(ws, 0, reinterpret_cast<char*>(c->g.epoch) + 256 - ws, s);
+    if (e == cudaSuccess) c->need_clear = false;
+  }
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->g.state, 0, state_region_bytes(c->g.B, c->g.H), s);
   if (e == cudaSuccess) c->need_init = false;
   return e;
 }
@@ -267,8 +277,10 @@ kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t by
   c->bytes = bytes;
   c->T = 0;
   c->need_init = true;
+  c->need_clear = true;
   c->g.state = reinterpret_cast<CacheState*>(c->base);
   c->g.counters = reinterpret_cast<uint32_t*>(c->base + sizeof(CacheState));
+  c->g.epoch = reinterpret_cast<uint32_t*>(c->base + need - 256);
   for (int i = 0; i < KVQ_NUM_PLANES; ++i)
     c->g.pl[i].p = c->g.pl[i].rows ? c->base + off[i] : nullptr;
   *out = c;
@@ -479,6 +491,12 @@ kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void
   if (st == KVQ_OK) st = kvq_append_pack(cache, k, v, 1, stream);
   if (st == KVQ_OK) st = kvq_attend_decode(cache, q, g.Hq, softmax_scale, out, stream);
   return st;
+}
+
+int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, int r_v) {
+  if (!cache) return -1;
+  const int r[3] = {r_q, r_k, r_v};
+  return cache->g.act == KVQ_BF16 && decode_step_supported(cache->g, d_in, r) ? 1 : 0;
 }
 
 kvq_status kvq_device_status(void* stream, int* out) {

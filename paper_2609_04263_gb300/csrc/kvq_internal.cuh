@@ -46,6 +46,7 @@ struct Geom {
   int32_t splits;        // decode split-K width (fixed per cache)
   CacheState* state;
   uint32_t* counters;    // [B][Hkv] split arrival counters (zeroed with the state)
+  uint32_t* epoch;       // launch counter of the fused decode step; kept across resets
   Plane pl[KVQ_NUM_PLANES];
 };
 
@@ -224,6 +225,7 @@ struct kvq_cache {
   size_t bytes;
   int T;            // host mirror of the device token count
   bool need_init;   // device state not yet zeroed since create/reset
+  bool need_clear;  // workspace and epoch not yet zeroed since create
 };
 
 namespace kvq {

@@ -71,6 +71,7 @@ _SIGS = {
                                 c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_float,
                                 c_float, c_float, c_void_p, c_void_p, c_void_p, c_void_p,
                                 c_void_p]),
+    "kvq_decode_step_fused": (c_int, [c_void_p, c_int, c_int, c_int, c_int]),
 }
 
 _lib = None
@@ -178,6 +179,11 @@ def kvq_decode_step(handle, x, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b
     _check(lib().kvq_decode_step(c_void_p(handle), P(x), d_in, P(w_qkv), P(a_q), P(b_q), r_q,
                                  P(a_k), P(b_k), r_k, P(a_v), P(b_v), r_v, alpha_over_r,
                                  rope_base, softmax_scale, P(q), P(k), P(v), P(out), P(stream)))
+
+
+def kvq_decode_step_fused(handle, d_in, r_q, r_k, r_v) -> bool:
+    """True when kvq_decode_step with these shapes runs as one fused kernel."""
+    return lib().kvq_decode_step_fused(c_void_p(handle), d_in, r_q, r_k, r_v) == 1
 
 
 def kvq_device_status(stream=0) -> int:
