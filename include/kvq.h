@@ -218,11 +218,16 @@ kvq_status kvq_attend_decode(kvq_cache* cache, const void* q, int n_q_heads,
  * then kvq_attend_decode of its query (Sections 3-3.3).  q, k, v receive the
  * projections ([B][Hq][1][D], [B][Hkv][1][D] x 2); out [B][Hq][1][D].  B and
  * the head counts are the cache's.  For bf16 affine/symmetric caches with
- * 2/4-bit codes, G = 32, head_dim 64/128 and B <= 16 the three steps run as
- * one cooperative kernel with one CTA per SM (grid-wide barriers between the
- * phases, bounded waits); other caches run the three calls in order.  The
- * results are the same either way.  Like kvq_attend_decode it uses the
- * cache's workspace, so calls on one cache must not overlap.
+ * 2/4-bit codes, G = 32, head_dim 64/128, B <= 16, d_in a multiple of 256 and
+ * ranks that are multiples of 8 up to 64 (kvq_decode_step_fused tells) the
+ * three steps run as one cooperative kernel with one CTA per SM, whose CTAs
+ * hand results to one another through the cache's workspace with bounded
+ * waits; other shapes run the three calls in order.  Both give the same codes
+ * for the same k and v and agree to bf16 rounding.  Like kvq_attend_decode
+ * it uses the cache's workspace, so calls on one cache must not overlap.
+ * The fused kernel starts reading w_qkv and the LoRA factors before the work
+ * queued before it on `stream` has finished (programmatic dependent launch):
+ * that work must not write them.
  */
 kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void* w_qkv,
                            const void* a_q, const void* b_q, int r_q,

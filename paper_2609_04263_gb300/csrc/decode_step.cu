@@ -349,45 +349,23 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
   CacheState* st = g.state;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gid = lane >> 2, tid = lane & 3;
-  // tokens before this step and the launch epoch: read once (thread 0) and
-  // shared, so that both reads are complete before this CTA arrives on the
-  // counter below
-  __shared__ int s_T0;
-  __shared__ uint32_t s_epoch;
+  // ---- before the dependency wait: read-only inputs only (weights) ---------
+  // The weight units and the LoRA up-projection rows do not depend on the
+  // preceding kernel on the stream, so their copies start while it drains
+  // (programmatic dependent launch); everything else waits for it.
   if (threadIdx.x == 0) {
-    s_T0 = *reinterpret_cast<volatile int32_t*>(&st->tokens);
-    s_epoch = *reinterpret_cast<volatile uint32_t*>(g.epoch);
     for (int i = 0; i < a.nslot; ++i) dattn::mbar_init(&ubar[i], 1);
     dattn::mbar_init(&bbar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
-  const int T0 = s_T0;
-  const uint32_t epoch = s_epoch;
-  const uint32_t tag = 0xFFC00000u | ((epoch + 1) & 0x003FFFFFu);   // a NaN no arithmetic makes
-  const bool room = T0 >= 0 && T0 + 1 <= g.Tmax;
-  const int T = T0 + 1;
-  const int M = g.B;
-  unsigned char* ring = sm;
-  unsigned char* asmem = sm + a.att_off;
-  unsigned char* xs = sm + a.xs_off;
-  uint64_t* part = reinterpret_cast<uint64_t*>(g.pl[KVQ_PLANE_WORKSPACE].p) + a.part_off;
-
-  // ---- entry: start the copies -------------------------------------------
   const int u_begin = (int)((int64_t)blockIdx.x * a.units / gridDim.x);
   const int n_local = (int)((int64_t)(blockIdx.x + 1) * a.units / gridDim.x) - u_begin;
   const int unitb = unit_bytes(a.ks), rstride = 2 * a.ks + 64;
+  unsigned char* ring = sm;
   for (int i = warp; i < min(n_local, a.nslot); i += kWarpsF)
     issue_unit(a, u_begin + i, ring + (i % a.nslot) * unitb, &ubar[i % a.nslot], lane);
   const int items3 = a.splits * g.H * g.B;
-  const bool attend_here = room && (int)blockIdx.x < items3;
-  int early = 0;                           // attention chunks issued ahead of the split
-  if (attend_here) {
-    const int rest = blockIdx.x / a.splits;
-    const dattn::SplitPlan sp = dattn::split_plan<FMT>(g, T, a.splits, blockIdx.x % a.splits);
-    dattn::split_prologue<D, BITS, FMT, AST>(g, rest / g.H, rest % g.H, sp, asmem, abar);
-    early = min(AST, sp.nchunks);
-  }
   const int grp = g.Hq / g.H;
   // LoRA up-projection rows of this CTA's first item (its kv head's query
   // heads, key and value) into shared memory
@@ -413,6 +391,36 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
       asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
                    ::"l"(reinterpret_cast<const char*>(a.bm[p]) + lo), "r"((uint32_t)(hi - lo))
                    : "memory");
+  }
+  pdl_trigger();
+  pdl_wait();
+
+  // tokens before this step and the launch epoch: read once (thread 0) and
+  // shared, so that both reads are complete before this CTA arrives on the
+  // counter below
+  __shared__ int s_T0;
+  __shared__ uint32_t s_epoch;
+  if (threadIdx.x == 0) {
+    s_T0 = *reinterpret_cast<volatile int32_t*>(&st->tokens);
+    s_epoch = *reinterpret_cast<volatile uint32_t*>(g.epoch);
+  }
+  __syncthreads();
+  const int T0 = s_T0;
+  const uint32_t epoch = s_epoch;
+  const uint32_t tag = 0xFFC00000u | ((epoch + 1) & 0x003FFFFFu);   // a NaN no arithmetic makes
+  const bool room = T0 >= 0 && T0 + 1 <= g.Tmax;
+  const int T = T0 + 1;
+  const int M = g.B;
+  unsigned char* asmem = sm + a.att_off;
+  unsigned char* xs = sm + a.xs_off;
+  uint64_t* part = reinterpret_cast<uint64_t*>(g.pl[KVQ_PLANE_WORKSPACE].p) + a.part_off;
+  const bool attend_here = room && (int)blockIdx.x < items3;
+  int early = 0;                           // attention chunks issued ahead of the split
+  if (attend_here) {
+    const int rest = blockIdx.x / a.splits;
+    const dattn::SplitPlan sp = dattn::split_plan<FMT>(g, T, a.splits, blockIdx.x % a.splits);
+    dattn::split_prologue<D, BITS, FMT, AST>(g, rest / g.H, rest % g.H, sp, asmem, abar);
+    early = min(AST, sp.nchunks);
   }
   for (int i = threadIdx.x * 8; i < M * a.d_in; i += blockDim.x * 8) {
     const int m = i / a.d_in, k = i - m * a.d_in;
@@ -627,12 +635,20 @@ cudaError_t launch_step(StepArgs& a, const int r[3], cudaStream_t s) {
   cfg.blockDim = dim3(kWarpsF * 32);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a);
+  cfg.numAttrs = 2;
+  e = cudaLaunchKernelEx(&cfg, kern, a);
+  if (e != cudaSuccess) {                  // without the early start
+    (void)cudaGetLastError();
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, a);
+  }
+  return e;
 }
 
 template <int D>
