@@ -42,6 +42,25 @@ PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+TRAFFIC_PATH = os.path.join(ROOT, "profiles", "roofline_traffic.json")
+
+
+def measured_traffic(kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu record, or None
+    when there is none or the kernel's sources changed since it was taken."""
+    import hashlib
+    try:
+        with open(TRAFFIC_PATH) as f:
+            rec = json.load(f)[kernel]
+        h = hashlib.sha256()
+        for name in rec["sources"]:
+            with open(os.path.join(ROOT, name), "rb") as f:
+                h.update(f.read())
+    except (OSError, KeyError, ValueError):
+        return None
+    return rec["dram_bytes_per_launch"] if h.hexdigest() == rec["sources_sha256"] else None
+
+
 def load_peaks():
     try:
         with open(PEAKS_PATH) as f:
@@ -658,7 +677,8 @@ def main():
                          "peak": peak, "unit": unit, "frac": round(achieved / peak, 4),
                          "peak_source": f"{peak_kind} "
                                         f"({'bf16_tflops_sustained' if bound == 'tensor' else 'hbm_gbs'})",
-                         "traffic": None},
+                         "traffic": measured_traffic(dominant),
+                         "algorithmic_bytes" if bound == "hbm" else "algorithmic_flops": amount},
             "kernels": kernels,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
