@@ -266,6 +266,11 @@ int decode_splits(const Geom& g) {
 
 cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
                           bool decode, cudaStream_t s) {
+  if (!decode && prefill_tc_supported(g)) {
+    int* err = device_error_word();
+    if (!err) return cudaErrorInvalidDevice;
+    return launch_prefill_tc(g, q, L, scale, out, err, s);
+  }
   if (!decode && prefill_mma_supported(g)) return launch_prefill_mma(g, q, L, scale, out, s);
   if (decode && decode_mma_supported(g)) {
     int* err = device_error_word();
