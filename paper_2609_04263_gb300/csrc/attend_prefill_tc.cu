@@ -52,37 +52,47 @@ __device__ __forceinline__ int sw128(int r, int c) {
   return (r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4);
 }
 
-// The stored state of one token of an affine/symmetric cache (G = 32, D = 64):
-// code rows of K and V and their fp16 scales (and offsets).
+// What one producer thread loads per tile (affine/symmetric cache, G = 32,
+// D = 64): the K code row of its token with the token's fp16 scales (and
+// offsets), and, for its block of V (8 tokens x 8 channels), each token's
+// code word of those channels with the scale (and offset) of their group.
 template <int BITS>
 struct TokenCodes {
-  uint4 kc[BITS / 2], vc[BITS / 2];    // D * BITS / 8 bytes each
-  uint32_t ks, kz, vs, vz;             // two fp16 per word (groups 0, 1)
+  uint4 kc[BITS / 2];                  // D * BITS / 8 bytes
+  uint32_t ks, kz;                     // two fp16 per word (groups 0, 1)
+  uint32_t vw[8];                      // 8 codes of channels 8dc .. 8dc+7, per token
+  __half vs[8], vz[8];
 };
 
 template <int BITS, bool SYM>
-__device__ __forceinline__ void load_token(const Geom& g, int b, int h, int t, int T,
-                                           TokenCodes<BITS>& r) {
-  if (t >= T) {                       // beyond the cache: reconstructs as zeros
+__device__ __forceinline__ void load_token(const Geom& g, int b, int h, int t, int vt0, int dc,
+                                           int T, TokenCodes<BITS>& r) {
+  if (t < T) {
+    const uint4* kc = reinterpret_cast<const uint4*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t));
 #pragma unroll
-    for (int i = 0; i < BITS / 2; ++i) r.kc[i] = r.vc[i] = make_uint4(0, 0, 0, 0);
-    r.ks = r.kz = r.vs = r.vz = 0;
-    return;
-  }
-  const uint4* kc = reinterpret_cast<const uint4*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t));
-  const uint4* vc = reinterpret_cast<const uint4*>(plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t));
+    for (int i = 0; i < BITS / 2; ++i) r.kc[i] = __ldg(kc + i);
+    r.ks = __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t)));
+    r.kz = SYM ? 0u
+               : __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t)));
+  } else {                            // beyond the cache: reconstructs as zeros
 #pragma unroll
-  for (int i = 0; i < BITS / 2; ++i) {
-    r.kc[i] = __ldg(kc + i);
-    r.vc[i] = __ldg(vc + i);
+    for (int i = 0; i < BITS / 2; ++i) r.kc[i] = make_uint4(0, 0, 0, 0);
+    r.ks = r.kz = 0;
   }
-  r.ks = __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t)));
-  r.vs = __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, t)));
-  if (!SYM) {
-    r.kz = __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t)));
-    r.vz = __ldg(reinterpret_cast<const uint32_t*>(plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, t)));
-  } else {
-    r.kz = r.vz = 0;
+  const __half hz = __float2half_rn(0.f);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int tv = vt0 + i;
+    if (tv < T) {
+      const uint8_t* row = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, tv);
+      r.vw[i] = BITS == 4 ? __ldg(reinterpret_cast<const uint32_t*>(row) + dc)
+                          : (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(row) + dc);
+      r.vs[i] = __ldg(plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, tv, dc >> 2));
+      r.vz[i] = SYM ? hz : __ldg(plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, tv, dc >> 2));
+    } else {
+      r.vw[i] = 0;
+      r.vs[i] = r.vz[i] = hz;
+    }
   }
 }
 
@@ -180,15 +190,16 @@ attend_prefill_tc_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, flo
 
   if (warp >= 4 && warp < 8) {
     // ---------------- producers: reconstruct K and V tiles ----------------
-    const int t = threadIdx.x - 128;                  // token within the tile
+    const int t = threadIdx.x - 128;                  // K: token t of the tile
+    const int dc = t & 7, tb = t >> 3;                // V: channels 8dc.., tokens 8tb..
     TokenCodes<BITS> cur, nxt;
-    if (ntiles > 0) load_token<BITS, SYM>(g, b, hkv, t, T, cur);
+    if (ntiles > 0) load_token<BITS, SYM>(g, b, hkv, t, 8 * tb, dc, T, cur);
     for (int j = 0; j < ntiles; ++j) {
       const int bf = j & 1;
-      if (j + 1 < ntiles) load_token<BITS, SYM>(g, b, hkv, (j + 1) * kTok + t, T, nxt);
+      if (j + 1 < ntiles)
+        load_token<BITS, SYM>(g, b, hkv, (j + 1) * kTok + t, (j + 1) * kTok + 8 * tb, dc, T, nxt);
       if (j >= 2 && !mbar_wait_or_abort(&kv_free[bf], ((j - 2) >> 1) & 1, abort)) break;
       unsigned char* kv = smem + S::KV_OFF + bf * S::KV_B;
-      unsigned char* vt = kv + S::VT + (t >> 6) * 8192 + (t & 7) * 2;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         float v[8];
@@ -204,11 +215,24 @@ attend_prefill_tc_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, flo
         }
         *reinterpret_cast<uint4*>(kv + S::KH + sw128(t, c)) = make_uint4(h[0], h[1], h[2], h[3]);
         *reinterpret_cast<uint4*>(kv + S::KL + sw128(t, c)) = make_uint4(l[0], l[1], l[2], l[3]);
-        recon8<BITS, SYM>(cur.vc, cur.vs, cur.vz, c, v);
-        // V^T: row d = 8c + e, token t along K (atom t / 64)
+      }
+      // V^T block: rows d = 8dc + e, tokens 8tb .. 8tb+7 (one 16-byte chunk each)
+      {
+        float vv[8][8];                               // [token][channel]
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float s = __half2float(cur.vs[i]);
+          const float m = SYM ? -(float)(1 << (BITS - 1)) * s : __half2float(cur.vz[i]);
+          constexpr unsigned mask = (1u << BITS) - 1;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) vv[i][e] = (float)((cur.vw[i] >> (e * BITS)) & mask) * s + m;
+        }
+        unsigned char* vt = kv + S::VT + (tb >> 3) * 8192;
 #pragma unroll
         for (int e = 0; e < 8; ++e)
-          *reinterpret_cast<__half*>(vt + sw128(8 * c + e, (t & 63) >> 3)) = __float2half_rn(v[e]);
+          *reinterpret_cast<uint4*>(vt + sw128(8 * dc + e, tb & 7)) =
+              make_uint4(pack_h2(vv[0][e], vv[1][e]), pack_h2(vv[2][e], vv[3][e]),
+                         pack_h2(vv[4][e], vv[5][e]), pack_h2(vv[6][e], vv[7][e]));
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_arrive(&kv_full[bf]);
@@ -273,6 +297,7 @@ attend_prefill_tc_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, flo
           break;
         }
         tc_fence_after();
+        const bool full = t0 + kTok - 1 <= pos;         // no key of the tile is masked
         // two passes over the scores in TMEM: the row max, then exp2 and P
         const uint32_t srow = tmem + lane_base + bf * kTok;
         float mx = -INFINITY;
@@ -282,10 +307,16 @@ attend_prefill_tc_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, flo
           tmem_ld16_nowait(srow + c0, sr);
           tmem_ld16_nowait(srow + c0 + 16, sr + 16);
           tmem_wait_ld();
+          if (full) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (t0 + c0 + i <= pos) mx = fmaxf(mx, __uint_as_float(sr[i]) * c2);
+            for (int i = 0; i < 32; ++i) mx = fmaxf(mx, __uint_as_float(sr[i]));
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (t0 + c0 + i <= pos) mx = fmaxf(mx, __uint_as_float(sr[i]));
+          }
         }
+        mx *= c2;                                      // (c2 > 0: the max commutes)
         const float m_new = fmaxf(m, mx);
         alpha = m_new == -INFINITY ? 1.f : exp2f(m - m_new);
         float sum = 0.f;
@@ -302,7 +333,8 @@ attend_prefill_tc_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, flo
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               const int i = 8 * c + e;
-              p[e] = t0 + c0 + i <= pos ? exp2f(__uint_as_float(sr[i]) * c2 - m_new) : 0.f;
+              const float x = exp2f(fmaf(__uint_as_float(sr[i]), c2, -m_new));
+              p[e] = full || t0 + c0 + i <= pos ? x : 0.f;
               sum += p[e];
             }
             const int ch = (c0 >> 3) + c;               // chunk 0..15 along the tile
