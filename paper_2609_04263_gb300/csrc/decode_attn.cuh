@@ -406,7 +406,9 @@ __device__ void decode_split(const Geom& g, const __nv_bfloat16* qg, float scale
     const unsigned char* st = smem + (my % STAGES) * C::STAGE_B;
     const int t0 = ts + my * kCT + tile_off;         // this warp's tile
     if (my < nchunks && t0 < te) {
-      const bool coded = t0 < tq;
+      // every token of an affine/symmetric cache is coded; KIVI keeps the
+      // newest tokens in full precision
+      const bool coded = FMT != KVQ_FMT_KIVI || t0 < tq;
       float sacc[2][4];                              // S for n-tiles 0, 1 (tokens t0 + 8nt + col)
       // ---------------- scores ----------------
       if (coded && FMT != KVQ_FMT_KIVI) {

@@ -24,10 +24,11 @@ struct ProjArgs {
   float theta_hi[128], theta_lo[128];
 };
 
-// cos and sin of pos * theta in fp32 to about 1e-7 absolute for positions
-// below 2^24: pos * theta_hi is formed exactly as p + e (FMA), reduced by
-// 2 pi in three parts (the first exact for multiples below 2^15), then the
-// small remainder goes to sincosf.
+// cos and sin of pos * theta in fp32 for positions below 2^24: pos * theta_hi
+// is formed exactly as p + e (FMA), reduced by 2 pi in three parts (the first
+// exact for multiples below 2^15) to |r| <= pi, where the hardware __sincosf
+// is accurate to about 2^-21 absolute (far below the bf16 rounding of the
+// outputs) without the large-argument path of sincosf.
 __device__ __forceinline__ void rope_cos_sin(int pos, float th_hi, float th_lo, float* c,
                                              float* s) {
   const float x = (float)pos;
@@ -38,7 +39,7 @@ __device__ __forceinline__ void rope_cos_sin(int pos, float th_hi, float th_lo, 
   r = fmaf(-k, 1.9353071795864769e-3f, r);                    //   + 1.9353072e-3
   r = fmaf(-k, 1.0253132e-11f, r);                            //   + 1.0253e-11 (remainder)
   r += e;
-  sincosf(r, s, c);
+  __sincosf(r, s, c);
 }
 
 // ---------------------------------------------------------------------------
