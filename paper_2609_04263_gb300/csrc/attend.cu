@@ -95,13 +95,14 @@ __device__ void dequant_tile(const Geom& g, int which, int b, int h, int t0, int
     }
     dst[r * ld + d] = val;
   }
-  if (g.fmt == KVQ_FMT_KVARN) {
-    // rotate the quantized rows back to the original basis (H is its own inverse)
+  if (g.fmt == KVQ_FMT_KVARN && !(t0 >= g.S && t0 + n <= g.S + nbq)) {
+    // KVarN is attended in the rotated basis (the coded rows are stored
+    // rotated): rotate the full-precision rows (sinks, staged) forward
     __syncthreads();
     for (int hs = 1; hs < D; hs <<= 1) {
       for (int p = threadIdx.x; p < n * D / 2; p += blockDim.x) {
         const int r = p / (D / 2), k = p % (D / 2), t = t0 + r;
-        if (t < g.S || t - g.S >= nbq) continue;
+        if (t >= T || (t >= g.S && t - g.S < nbq)) continue;
         const int j = (k / hs) * 2 * hs + (k % hs);
         float a = dst[r * ld + j], c = dst[r * ld + j + hs];
         dst[r * ld + j] = a + c;
@@ -111,9 +112,27 @@ __device__ void dequant_tile(const Geom& g, int which, int b, int h, int t0, int
     }
     for (int i = threadIdx.x; i < n * D; i += blockDim.x) {
       const int r = i / D, t = t0 + r;
-      if (t >= g.S && t - g.S < nbq) dst[r * ld + i % D] *= inv_sqrt_d;
+      if (t < T && !(t >= g.S && t - g.S < nbq)) dst[r * ld + i % D] *= inv_sqrt_d;
     }
   }
+}
+
+// Normalised Hadamard transform of `rows` rows of D values at x [rows][ld]
+// (the whole CTA; H / sqrt(D) is its own inverse).
+__device__ void rotate_rows(float* x, int rows, int D, int ld, float inv_sqrt_d) {
+  __syncthreads();
+  for (int hs = 1; hs < D; hs <<= 1) {
+    for (int p = threadIdx.x; p < rows * D / 2; p += blockDim.x) {
+      const int r = p / (D / 2), k = p % (D / 2);
+      const int j = (k / hs) * 2 * hs + (k % hs);
+      const float a = x[r * ld + j], c = x[r * ld + j + hs];
+      x[r * ld + j] = a + c;
+      x[r * ld + j + hs] = a - c;
+    }
+    __syncthreads();
+  }
+  for (int i = threadIdx.x; i < rows * D; i += blockDim.x) x[(i / D) * ld + i % D] *= inv_sqrt_d;
+  __syncthreads();
 }
 
 // One CTA: `rows` = g heads x nq queries of one (b, kv head), over the tokens
@@ -161,6 +180,8 @@ attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
     lrow[r] = 0.f;
   }
   __syncthreads();
+  const bool kvarn = g.fmt == KVQ_FMT_KVARN;
+  if (kvarn) rotate_rows(qs, rows, D, D, inv_sqrt_d);     // queries into the rotated basis
   for (int t0 = ts; t0 < te; t0 += kTile) {
     const int n = min(kTile, te - t0);
     dequant_tile(g, 0, b, hkv, t0, n, T, Kt, ldk, inv_sqrt_d);
@@ -211,6 +232,7 @@ attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
     }
     __syncthreads();
   }
+  if (kvarn) rotate_rows(acc, rows, D, D, inv_sqrt_d);    // output back to the original basis
   if (decode) {
     for (int i = threadIdx.x; i < rows * (D + kWsStride); i += blockDim.x) {
       const int r = i / (D + kWsStride), c = i % (D + kWsStride);

@@ -35,7 +35,11 @@ struct PCfg {
   static constexpr int TOTAL = V_OFF + NT * LDS * 2;
   // KVarN: fp32 rows of one reconstructed tile before the inverse Hadamard
   static constexpr int SCR_OFF = TOTAL;
-  static constexpr int TOTAL_KVARN = SCR_OFF + NT * D * 4;
+  // KVarN: fp32 scratch for rotating full-precision tiles, then the bf16
+  // remainder of the rotated queries
+  static constexpr int QL_OFF = SCR_OFF + NT * D * 4;
+  static constexpr int TOTAL_KVARN = QL_OFF + ROWS * LDS * 2;
+  static_assert(QL_OFF - K_OFF >= ROWS * D * 4, "rotated output fits the K/V area");
   static constexpr int THREADS = WARPS * 32;
 };
 
@@ -93,10 +97,38 @@ __device__ __forceinline__ void store_v8(const float v[8], __half* dst) {
                                               pack_f16(v[4], v[5]), pack_f16(v[6], v[7]));
 }
 
-// KVarN: reconstruct tokens [t0, t0 + NT) into dst [NT][LDS] bf16.  Sinks and
-// staged tokens are copied; coded tokens are r_t c_j (s code + m) in the
-// rotated basis, rotated back by the normalised Hadamard (its own inverse) in
-// fp32 in `scr` [NT][D].
+// In-warp normalised Hadamard transform of one row of D values held as
+// x[i] = row[lane + 32 i]: butterflies (a + b, a - b) for h = 1 .. D/2 (lanes,
+// then slots), then 1/sqrt(D).  H / sqrt(D) is symmetric and orthonormal, so
+// it is its own inverse and q . k = (H q) . (H k) / D.
+template <int D>
+__device__ __forceinline__ void fwht_warp(float (&x)[D / 32], int lane, float inv_sqrt_d) {
+  constexpr int NS = D / 32;
+#pragma unroll
+  for (int h = 1; h < 32; h <<= 1)
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const float y = __shfl_xor_sync(0xffffffffu, x[i], h);
+      x[i] = (lane & h) ? y - x[i] : x[i] + y;
+    }
+#pragma unroll
+  for (int hs = 1; hs < NS; hs <<= 1)
+#pragma unroll
+    for (int i = 0; i < NS; ++i)
+      if (!(i & hs)) {
+        const float a = x[i], c = x[i + hs];
+        x[i] = a + c;
+        x[i + hs] = a - c;
+      }
+#pragma unroll
+  for (int i = 0; i < NS; ++i) x[i] *= inv_sqrt_d;
+}
+
+// KVarN, attended in the rotated basis: tokens [t0, t0 + NT) into dst [NT][LDS]
+// bf16.  Coded tokens are stored rotated (Section 3.1: r_t c_j (s code + m)),
+// so they are reconstructed as they are; sinks and staged tokens are stored
+// in the original basis and are rotated forward here (fp32 butterflies in
+// `scr` [NT][D]).  The queries are rotated once and the output rotated back.
 template <int D, int NT, int THREADS>
 __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T,
                            __nv_bfloat16* khi, __nv_bfloat16* klo, __half* vdst, int lds,
@@ -111,18 +143,23 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
   const int P_ROW = which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW;
   const int P_COL = which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL;
   const unsigned mask = (1u << bits) - 1;
+  // a tile with full-precision rows goes through the scratch and is rotated
+  const bool all_coded = t0 >= S && t0 + NT <= S + nbq && t0 + NT <= T;
   for (int i = threadIdx.x; i < NT * (D / 8); i += THREADS) {
     const int r = i / (D / 8), c = i % (D / 8), t = t0 + r;
-    float* sr = scr + r * D + 8 * c;
+    float v[8];
+    const bool coded = t < T && t >= S && t - S < nbq;
     if (t >= T) {
-      for (int e = 0; e < 8; ++e) sr[e] = 0.f;
-    } else if (t < S || t - S >= nbq) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    } else if (!coded) {
       const __nv_bfloat16* src = t < S
           ? plane_ptr<__nv_bfloat16>(g, P_FULL, b, h, t, 8 * c)
           : plane_ptr<__nv_bfloat16>(g, P_PEND, b, h, (t - S) % G, 8 * c);
       const uint4 u = *reinterpret_cast<const uint4*>(src);
       const __nv_bfloat16* e8 = reinterpret_cast<const __nv_bfloat16*>(&u);
-      for (int e = 0; e < 8; ++e) sr[e] = __bfloat162float(e8[e]);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = __bfloat162float(e8[e]);
     } else {
       const int qi = t - S;
       const uint8_t* row = plane_ptr<uint8_t>(g, P_CODES, b, h, qi);
@@ -136,16 +173,26 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
       const float rr = __half2float(*plane_ptr<__half>(g, P_ROW, b, h, 0, qi));
       const uint4 cu = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, P_COL, b, h, qi / G, 8 * c));
       const __half* c8 = reinterpret_cast<const __half*>(&cu);
+#pragma unroll
       for (int e = 0; e < 8; ++e)
-        sr[e] = rr * __half2float(c8[e]) * ((float)((w >> (e * bits)) & mask) * sc + mz);
+        v[e] = rr * __half2float(c8[e]) * ((float)((w >> (e * bits)) & mask) * sc + mz);
+    }
+    if (all_coded) {
+      if (which == 0) store_k8(v, khi + r * lds + 8 * c, klo + r * lds + 8 * c);
+      else store_v8(v, vdst + r * lds + 8 * c);
+    } else {
+      float* sr = scr + r * D + 8 * c;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) sr[e] = v[e];
     }
   }
+  if (all_coded) return;
   __syncthreads();
-  // inverse rotation of the coded rows (butterflies h = 1 .. D/2, then 1/sqrt(D))
+  // forward rotation of the full-precision rows (butterflies h = 1 .. D/2)
   for (int hs = 1; hs < D; hs <<= 1) {
     for (int p = threadIdx.x; p < NT * D / 2; p += THREADS) {
       const int r = p / (D / 2), k = p % (D / 2), t = t0 + r;
-      if (t < S || t - S >= nbq || t >= T) continue;
+      if (t >= T || (t >= S && t - S < nbq)) continue;
       const int j = (k / hs) * 2 * hs + (k % hs);
       const float a = scr[r * D + j], c = scr[r * D + j + hs];
       scr[r * D + j] = a + c;
@@ -155,7 +202,7 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
   }
   for (int i = threadIdx.x; i < NT * (D / 8); i += THREADS) {
     const int r = i / (D / 8), c = i % (D / 8), t = t0 + r;
-    const float f = (t >= S && t - S < nbq && t < T) ? inv_sqrt_d : 1.f;
+    const float f = (t < T && !(t >= S && t - S < nbq)) ? inv_sqrt_d : 1.f;
     const float* sr = scr + r * D + 8 * c;
     float v[8];
 #pragma unroll
@@ -201,6 +248,24 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
       v = *reinterpret_cast<const uint4*>(
           q + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D + 8 * c);
     *reinterpret_cast<uint4*>(Qs + r * LDS + 8 * c) = v;
+  }
+  const bool kvarn = g.fmt == KVQ_FMT_KVARN;
+  __nv_bfloat16* Ql = reinterpret_cast<__nv_bfloat16*>(smem + C::QL_OFF);
+  if (kvarn) {
+    // rotate the query rows: high part in Qs, bf16 remainder in Ql
+    __syncthreads();
+    for (int r = warp; r < C::ROWS; r += C::WARPS) {
+      float x[D / 32];
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) x[i] = __bfloat162float(Qs[r * LDS + lane + 32 * i]);
+      fwht_warp<D>(x, lane, inv_sqrt_d);
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) {
+        const __nv_bfloat16 hb = __float2bfloat16_rn(x[i]);
+        Qs[r * LDS + lane + 32 * i] = hb;
+        Ql[r * LDS + lane + 32 * i] = __float2bfloat16_rn(x[i] - __bfloat162float(hb));
+      }
+    }
   }
   // this thread's two rows: positions (or -1 for padding rows)
   int pos[2];
@@ -249,8 +314,10 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
     for (int j = 0; j < NTN; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
-      uint32_t a[4];
-      ldsm_x4(a, Qs + (warp * 16 + (lane & 15)) * LDS + 16 * ks + (lane >> 4) * 8);
+      uint32_t a[4], al[4];
+      const int qoff = (warp * 16 + (lane & 15)) * LDS + 16 * ks + (lane >> 4) * 8;
+      ldsm_x4(a, Qs + qoff);
+      if (kvarn) ldsm_x4(al, Ql + qoff);
 #pragma unroll
       for (int np = 0; np < NTN / 2; ++np) {
         uint32_t bq[4], bl[4];
@@ -262,6 +329,10 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
         mma16816(s[2 * np + 1], a, bq[2], bq[3]);
         mma16816(s[2 * np], a, bl[0], bl[1]);
         mma16816(s[2 * np + 1], a, bl[2], bl[3]);
+        if (kvarn) {
+          mma16816(s[2 * np], al, bq[0], bq[1]);
+          mma16816(s[2 * np + 1], al, bq[2], bq[3]);
+        }
       }
     }
     // ---- mask, online softmax ----
@@ -326,6 +397,35 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
   for (int rr = 0; rr < 2; ++rr) {
     l_run[rr] += __shfl_xor_sync(0xffffffffu, l_run[rr], 1);
     l_run[rr] += __shfl_xor_sync(0xffffffffu, l_run[rr], 2);
+  }
+  if (kvarn) {
+    // normalised rotated rows -> fp32 shared memory (the K/V area), then each
+    // warp rotates rows back and stores them
+    float* os = reinterpret_cast<float*>(smem + C::K_OFF);   // [ROWS][D]
+    __syncthreads();
+#pragma unroll
+    for (int rr = 0; rr < 2; ++rr) {
+      const int r = warp * 16 + gid + 8 * rr;
+      const float inv = l_run[rr] > 0.f ? 1.f / l_run[rr] : 0.f;
+#pragma unroll
+      for (int j = 0; j < D / 8; ++j) {
+        os[r * D + 8 * j + 2 * tid] = o[j][2 * rr] * inv;
+        os[r * D + 8 * j + 2 * tid + 1] = o[j][2 * rr + 1] * inv;
+      }
+    }
+    __syncthreads();
+    for (int r = warp; r < C::ROWS; r += C::WARPS) {
+      const int hl = r / nq, qi = r % nq;
+      if (hl >= grp || qi >= nql) continue;
+      float x[D / 32];
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) x[i] = os[r * D + lane + 32 * i];
+      fwht_warp<D>(x, lane, inv_sqrt_d);
+      __nv_bfloat16* orow = out + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D;
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) orow[lane + 32 * i] = __float2bfloat16_rn(x[i]);
+    }
+    return;
   }
 #pragma unroll
   for (int rr = 0; rr < 2; ++rr) {
