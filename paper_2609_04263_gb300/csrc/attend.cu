@@ -277,6 +277,232 @@ __global__ void combine_kernel(Geom g, int splits, void* out) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// KVarN decode attention in the rotated basis (Section 3.1: coded tokens are
+// stored as r_t c_j (s code + m) after the normalised Hadamard rotation).
+// One CTA = (split, kv head, sequence), 8 warps, each warp a contiguous part
+// of the split; lane l holds channels [NS l, NS l + NS), NS = D / 32.  The
+// queries are rotated once (in registers); a coded token's score is
+//   r_t (s_t sum_j q'_j code_j + m_t sum_j q'_j),  q' = q_rot c_block,
+// refolded when the token block changes (a lane's channels lie in one group);
+// sinks and staged tokens are rotated forward in registers.  The values
+// accumulate in the rotated basis; the split's output is rotated back before
+// its (m, l, o) partial goes to the workspace, which combine_kernel merges.
+// ---------------------------------------------------------------------------
+template <int D>
+__device__ __forceinline__ void fwht_contig(float (&x)[D / 32], int lane, float inv_sqrt_d) {
+  constexpr int NS = D / 32;
+#pragma unroll
+  for (int h = 1; h < NS; h <<= 1)
+#pragma unroll
+    for (int i = 0; i < NS; ++i)
+      if (!(i & h)) {
+        const float a = x[i], c = x[i + h];
+        x[i] = a + c;
+        x[i + h] = a - c;
+      }
+#pragma unroll
+  for (int lh = 1; lh < 32; lh <<= 1)
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const float y = __shfl_xor_sync(0xffffffffu, x[i], lh);
+      x[i] = (lane & lh) ? y - x[i] : x[i] + y;
+    }
+#pragma unroll
+  for (int i = 0; i < NS; ++i) x[i] *= inv_sqrt_d;
+}
+
+// NS codes of `bits` bits of this lane's channels from a packed row
+__device__ __forceinline__ uint32_t lane_codes(const uint8_t* row, int lane, int ns, int bits) {
+  const int bit = ns * bits * lane;
+  return __ldg(reinterpret_cast<const uint32_t*>(row) + (bit >> 5)) >> (bit & 31);
+}
+
+template <int D, int GM>
+__global__ void __launch_bounds__(256)
+attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale,
+                           float inv_sqrt_d) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int NS = D / 32;
+  extern __shared__ float ksm[];                 // [8 warps][GM][D + 2]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, hkv = blockIdx.y, b = blockIdx.z;
+  const int grp = g.Hq / g.H, G = g.G, S = g.S;
+  const int T = cache_tokens(g);
+  const int nbq = kvarn_nblocks(T, S, G) * G;
+  int ts, te;
+  split_range(T, g.splits, split, G, &ts, &te);
+  const float c2 = scale * 1.4426950408889634f;   // scores in log2 units
+  // rotated queries, pre-scaled
+  float qr[GM][NS];
+#pragma unroll
+  for (int h = 0; h < GM; ++h) {
+    float x[NS];
+    const bool live = h < grp;
+    const __nv_bfloat16* src = q + ((int64_t)b * g.Hq + hkv * grp + (live ? h : 0)) * D + NS * lane;
+#pragma unroll
+    for (int i = 0; i < NS; ++i) x[i] = live ? __bfloat162float(src[i]) : 0.f;
+    fwht_contig<D>(x, lane, inv_sqrt_d);
+#pragma unroll
+    for (int i = 0; i < NS; ++i) qr[h][i] = x[i] * c2;
+  }
+  float m[GM], l[GM], o[GM][NS];
+#pragma unroll
+  for (int h = 0; h < GM; ++h) {
+    m[h] = -INFINITY;
+    l[h] = 0.f;
+#pragma unroll
+    for (int i = 0; i < NS; ++i) o[h][i] = 0.f;
+  }
+  const int per = (te - ts + 7) / 8;
+  const int w0 = ts + warp * per, w1 = min(te, w0 + per);
+  const int kb = g.kb, vb = g.vb;
+  const unsigned kmask = (1u << kb) - 1, vmask = (1u << vb) - 1;
+  const int grpc = NS * lane / G;                   // this lane's channel group
+  float qp[GM][NS], qs[GM];                         // q' = q_rot c_block and its lane sum
+  float cv[NS];                                     // value column scales of the block
+  int cur_blk = -1;
+  for (int t = w0; t < w1; ++t) {
+    float kv[NS], vv[NS];
+    const bool coded = t >= S && t - S < nbq;
+    float dot[GM];
+    if (coded) {
+      const int qi = t - S, blk = qi / G;
+      if (blk != cur_blk) {                         // refold the block's column scales
+        cur_blk = blk;
+        const __half* ck = plane_ptr<__half>(g, KVQ_PLANE_K_COL, b, hkv, blk, NS * lane);
+        const __half* cvp = plane_ptr<__half>(g, KVQ_PLANE_V_COL, b, hkv, blk, NS * lane);
+#pragma unroll
+        for (int i = 0; i < NS; ++i) {
+          const float c = __half2float(ck[i]);
+          cv[i] = __half2float(cvp[i]);
+#pragma unroll
+          for (int h = 0; h < GM; ++h) qp[h][i] = qr[h][i] * c;
+        }
+#pragma unroll
+        for (int h = 0; h < GM; ++h) {
+          float a = 0.f;
+#pragma unroll
+          for (int i = 0; i < NS; ++i) a += qp[h][i];
+          qs[h] = a;
+        }
+      }
+      const uint32_t wk = lane_codes(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, qi), lane, NS, kb);
+      const uint32_t wv = lane_codes(plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, qi), lane, NS, vb);
+      const float ks = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, qi, grpc));
+      const float kz = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, qi, grpc));
+      const float kr = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_ROW, b, hkv, 0, qi));
+      const float vs = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, qi, grpc));
+      const float vz = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, qi, grpc));
+      const float vr = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_ROW, b, hkv, 0, qi));
+#pragma unroll
+      for (int h = 0; h < GM; ++h) {
+        float a = 0.f;
+#pragma unroll
+        for (int i = 0; i < NS; ++i) a += qp[h][i] * (float)((wk >> (i * kb)) & kmask);
+        dot[h] = kr * (ks * a + kz * qs[h]);
+      }
+#pragma unroll
+      for (int i = 0; i < NS; ++i) vv[i] = vr * cv[i] * ((float)((wv >> (i * vb)) & vmask) * vs + vz);
+    } else {                                        // sink or staged: rotate forward
+      const __nv_bfloat16* kp = t < S
+          ? plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, hkv, t, NS * lane)
+          : plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_PEND, b, hkv, (t - S) % G, NS * lane);
+      const __nv_bfloat16* vp = t < S
+          ? plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, hkv, t, NS * lane)
+          : plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_PEND, b, hkv, (t - S) % G, NS * lane);
+#pragma unroll
+      for (int i = 0; i < NS; ++i) {
+        kv[i] = __bfloat162float(kp[i]);
+        vv[i] = __bfloat162float(vp[i]);
+      }
+      fwht_contig<D>(kv, lane, inv_sqrt_d);
+      fwht_contig<D>(vv, lane, inv_sqrt_d);
+#pragma unroll
+      for (int h = 0; h < GM; ++h) {
+        float a = 0.f;
+#pragma unroll
+        for (int i = 0; i < NS; ++i) a += qr[h][i] * kv[i];
+        dot[h] = a;
+      }
+    }
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      float sc = dot[h];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sc += __shfl_xor_sync(0xffffffffu, sc, off);
+      const float mn = fmaxf(m[h], sc);
+      const float alpha = exp2f(m[h] - mn);         // m = -inf at first: alpha = 0
+      const float p = exp2f(sc - mn);
+      m[h] = mn;
+      l[h] = l[h] * alpha + p;
+#pragma unroll
+      for (int i = 0; i < NS; ++i) o[h][i] = o[h][i] * alpha + p * vv[i];
+    }
+  }
+  // ---- merge the warps, rotate back, write the split's partial ----
+  float* red = ksm;                                  // [8][GM][D + 2]
+#pragma unroll
+  for (int h = 0; h < GM; ++h) {
+    float* rw = red + (warp * GM + h) * (D + 2);
+    if (lane == 0) {
+      rw[0] = m[h];
+      rw[1] = l[h];
+    }
+#pragma unroll
+    for (int i = 0; i < NS; ++i) rw[2 + NS * lane + i] = o[h][i];
+  }
+  __syncthreads();
+  for (int h = warp; h < grp; h += 8) {
+    float M = -INFINITY;
+    for (int w = 0; w < 8; ++w) M = fmaxf(M, red[(w * GM + h) * (D + 2)]);
+    float L = 0.f, x[NS];
+#pragma unroll
+    for (int i = 0; i < NS; ++i) x[i] = 0.f;
+    for (int w = 0; w < 8; ++w) {
+      const float* rw = red + (w * GM + h) * (D + 2);
+      if (rw[0] == -INFINITY) continue;
+      const float f = exp2f(rw[0] - M);
+      L += f * rw[1];
+#pragma unroll
+      for (int i = 0; i < NS; ++i) x[i] += f * rw[2 + NS * lane + i];
+    }
+    fwht_contig<D>(x, lane, inv_sqrt_d);
+    float* wsr = ws_row(g, b, hkv * grp + h) + (int64_t)split * (D + kWsStride);
+    if (lane == 0) {
+      wsr[0] = M == -INFINITY ? -INFINITY : M * 0.6931471805599453f;   // natural-log units
+      wsr[1] = L;
+    }
+#pragma unroll
+    for (int i = 0; i < NS; ++i) wsr[2 + NS * lane + i] = x[i];
+  }
+}
+
+template <int D>
+cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, cudaStream_t s) {
+  const int grp = g.Hq / g.H;
+  const float inv_sqrt_d = (float)(1.0 / sqrt((double)D));
+  dim3 grid(g.splits, g.H, g.B);
+  auto run = [&](auto kern, int gm) {
+    const size_t sm = (size_t)8 * gm * (D + 2) * sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    launch_pdl(kern, dim3(grid), dim3(256), sm, s, g, reinterpret_cast<const __nv_bfloat16*>(q),
+               scale, inv_sqrt_d);
+    return cudaGetLastError();
+  };
+  if (grp <= 2) return run(attend_kvarn_decode_kernel<D, 2>, 2);
+  if (grp <= 4) return run(attend_kvarn_decode_kernel<D, 4>, 4);
+  return run(attend_kvarn_decode_kernel<D, 8>, 8);
+}
+
+bool kvarn_decode_supported(const Geom& g) {
+  return g.fmt == KVQ_FMT_KVARN && g.act == KVQ_BF16 && (g.D == 64 || g.D == 128 || g.D == 256) &&
+         g.Hq / g.H <= 8 && (g.kb == 2 || g.kb == 4) && (g.vb == 2 || g.vb == 4) &&
+         g.G >= g.D / 32 && g.G % (g.D / 32) == 0;
+}
+
 }  // namespace
 
 int decode_splits(const Geom& g) {
@@ -298,6 +524,14 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
     int* err = device_error_word();
     if (!err) return cudaErrorInvalidDevice;
     return launch_decode_mma(g, q, scale, err, out, s);
+  }
+  if (decode && kvarn_decode_supported(g)) {
+    cudaError_t e = g.D == 64 ? launch_kvarn_d<64>(g, q, scale, s)
+                  : g.D == 128 ? launch_kvarn_d<128>(g, q, scale, s)
+                               : launch_kvarn_d<256>(g, q, scale, s);
+    if (e != cudaSuccess) return e;
+    launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, g.splits, out);
+    return cudaGetLastError();
   }
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));
