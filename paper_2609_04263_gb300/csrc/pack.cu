@@ -384,6 +384,164 @@ __global__ void kvarn_block_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float in
   }
 }
 
+// The same block transform with warps instead of CTA-wide steps (D = 64/128/
+// 256, G = 32/64).  Every floating-point operation and its order are those of
+// kvarn_block_kernel (and of the reference definition): Hadamard stages
+// h = 1 .. D/2 with explicit fp32 add/sub, the stride-halving pairwise trees
+// for the row and column sums of squares, IEEE sqrt and division.  A warp
+// owns whole rows for the Hadamard and the row statistics (lane l holds
+// channels l + 32 i: the upper tree levels add slots in registers, the last
+// five add lanes by xor-shuffle); a thread owns a whole column for the column
+// statistics (the tree in registers).  Two CTA barriers per iteration.
+template <int D, int G>
+__global__ void __launch_bounds__(256)
+kvarn_block_fast_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int NS = D / 32, NG = D / G;
+  extern __shared__ float smem[];
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
+  const int n0 = kvarn_nblocks(T0, g.S, G), n1 = kvarn_nblocks(T0 + L, g.S, G);
+  const int blk = n0 + blockIdx.x;
+  if (!ok || blk >= n1) return;
+  const int which = blockIdx.z;
+  TokSrc src = which ? sv : sk;
+  src.T0 = T0;
+  const int bits = which ? g.vb : g.kb;
+  float* y = smem;                                // [G][D]
+  float* rsc = y + G * D;                         // [G] row scales
+  float* csc = rsc + G;                           // [D] column scales
+  uint8_t* cs = reinterpret_cast<uint8_t*>(csc + D);   // [G][D] codes
+  const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
+  const int q0 = blk * G, t0 = g.S + q0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // load and rotate: a warp per row
+  for (int r = warp; r < G; r += 8) {
+    float x[NS];
+    const void* sb;
+    const int64_t e = tok_elem(g, src, b, h, t0 + r, &sb);
+#pragma unroll
+    for (int i = 0; i < NS; ++i) x[i] = ld_act(sb, e + lane + 32 * i, g.act);
+#pragma unroll
+    for (int hh = 1; hh < 32; hh <<= 1)
+#pragma unroll
+      for (int i = 0; i < NS; ++i) {
+        const float o = __shfl_xor_sync(0xffffffffu, x[i], hh);
+        x[i] = (lane & hh) ? __fsub_rn(o, x[i]) : __fadd_rn(x[i], o);
+      }
+#pragma unroll
+    for (int hs = 1; hs < NS; hs <<= 1)
+#pragma unroll
+      for (int i = 0; i < NS; ++i)
+        if (!(i & hs)) {
+          const float a = x[i], c = x[i + hs];
+          x[i] = __fadd_rn(a, c);
+          x[i + hs] = __fsub_rn(a, c);
+        }
+#pragma unroll
+    for (int i = 0; i < NS; ++i) y[r * D + lane + 32 * i] = __fmul_rn(x[i], inv_sqrt_d);
+    if (lane == 0) rsc[r] = 1.f;
+  }
+  for (int j = threadIdx.x; j < D; j += blockDim.x) csc[j] = 1.f;
+  __syncthreads();
+  const float inv_d = 1.f / (float)D, inv_g = 1.f / (float)G;
+  for (int it = 0; it < g.iters; ++it) {
+    // rows
+    for (int r = warp; r < G; r += 8) {
+      float x[NS], a[NS];
+#pragma unroll
+      for (int i = 0; i < NS; ++i) {
+        x[i] = y[r * D + lane + 32 * i];
+        a[i] = __fmul_rn(x[i], x[i]);
+      }
+#pragma unroll
+      for (int ns = NS / 2; ns >= 1; ns >>= 1)
+#pragma unroll
+        for (int i = 0; i < ns; ++i) a[i] = __fadd_rn(a[i], a[i + ns]);
+#pragma unroll
+      for (int n = 16; n >= 1; n >>= 1) a[0] = __fadd_rn(a[0], __shfl_xor_sync(0xffffffffu, a[0], n));
+      const float sum = __shfl_sync(0xffffffffu, a[0], 0);
+      const float sg = fmaxf(__fsqrt_rn(__fmul_rn(sum, inv_d)), 1e-8f);
+      if (lane == 0) rsc[r] = __fmul_rn(rsc[r], sg);
+#pragma unroll
+      for (int i = 0; i < NS; ++i) y[r * D + lane + 32 * i] = __fdiv_rn(x[i], sg);
+    }
+    __syncthreads();
+    // columns: a thread per column
+    for (int j = threadIdx.x; j < D; j += blockDim.x) {
+      float col[G], a[G];
+#pragma unroll
+      for (int r = 0; r < G; ++r) {
+        col[r] = y[r * D + j];
+        a[r] = __fmul_rn(col[r], col[r]);
+      }
+#pragma unroll
+      for (int n = G / 2; n >= 1; n >>= 1)
+#pragma unroll
+        for (int r = 0; r < n; ++r) a[r] = __fadd_rn(a[r], a[r + n]);
+      const float sg = fmaxf(__fsqrt_rn(__fmul_rn(a[0], inv_g)), 1e-8f);
+      csc[j] = __fmul_rn(csc[j], sg);
+#pragma unroll
+      for (int r = 0; r < G; ++r) y[r * D + j] = __fdiv_rn(col[r], sg);
+    }
+    __syncthreads();
+  }
+  // grouped affine along D (groups of G channels)
+  const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int row_plane = which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW;
+  const int col_plane = which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL;
+  for (int p = threadIdx.x; p < G * NG; p += blockDim.x) {
+    const int r = p / NG, gq = p % NG;
+    const float* row = y + r * D + gq * G;
+    float mn = row[0], mx = row[0];
+    for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
+    const float sc = affine_scale(mn, mx, bits);
+    for (int j = 0; j < G; ++j) cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, bits);
+    *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
+    *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
+  }
+  for (int r = threadIdx.x; r < G; r += blockDim.x)
+    *plane_ptr<__half>(g, row_plane, b, h, 0, q0 + r) = __float2half_rn(rsc[r]);
+  for (int j = threadIdx.x; j < D; j += blockDim.x)
+    *plane_ptr<__half>(g, col_plane, b, h, blk, j) = __float2half_rn(csc[j]);
+  __syncthreads();
+  const int per = 8 / bits, row_bytes = D * bits / 8;
+  for (int i = threadIdx.x; i < G * row_bytes; i += blockDim.x) {
+    const int r = i / row_bytes, j = i % row_bytes;
+    unsigned byte = 0;
+    for (int e = 0; e < per; ++e) byte |= (unsigned)cs[r * D + j * per + e] << (e * bits);
+    plane_ptr<uint8_t>(g, codes_plane, b, h, q0 + r)[j] = (uint8_t)byte;
+  }
+}
+
+template <int D, int G>
+cudaError_t launch_kvarn_fast(const Geom& g, int max_blocks, int L, const TokSrc& sk,
+                              const TokSrc& sv, float inv_sqrt_d, cudaStream_t s) {
+  const size_t sm = (size_t)G * D * 4 + (size_t)(G + D) * 4 + (size_t)G * D;
+  auto kern = kvarn_block_fast_kernel<D, G>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  launch_pdl(kern, dim3(dim3(max_blocks, g.B * g.H, 2)), dim3(256), sm, s, g, L, sk, sv, inv_sqrt_d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_kvarn_blocks(const Geom& g, int max_blocks, int L, const TokSrc& sk,
+                                const TokSrc& sv, float inv_sqrt_d, cudaStream_t s) {
+  if (g.G == 32) {
+    if (g.D == 64) return launch_kvarn_fast<64, 32>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+    if (g.D == 128) return launch_kvarn_fast<128, 32>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+    if (g.D == 256) return launch_kvarn_fast<256, 32>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+  } else if (g.G == 64) {
+    if (g.D == 64) return launch_kvarn_fast<64, 64>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+    if (g.D == 128) return launch_kvarn_fast<128, 64>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+    if (g.D == 256) return launch_kvarn_fast<256, 64>(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+  }
+  return cudaErrorNotSupported;
+}
+
 int grid_for(int64_t threads_needed, int block) {
   int64_t n = (threads_needed + block - 1) / block;
   int64_t cap = (int64_t)num_sms() * 8;
@@ -433,7 +591,13 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       if (e != cudaSuccess) return e;
       sk.ring_plane = KVQ_PLANE_K_PEND; sk.ring_off = g.S; sk.ring_rows = g.G;
       sv.ring_plane = KVQ_PLANE_V_PEND; sv.ring_off = g.S; sv.ring_rows = g.G;
-      launch_pdl(kvarn_block_kernel, dim3(dim3(max_blocks, g.B * g.H, 2)), dim3(256), sm, s, g, L, sk, sv, inv_sqrt_d);
+      e = launch_kvarn_blocks(g, max_blocks, L, sk, sv, inv_sqrt_d, s);
+      if (e == cudaErrorNotSupported) {
+        (void)cudaGetLastError();
+        launch_pdl(kvarn_block_kernel, dim3(dim3(max_blocks, g.B * g.H, 2)), dim3(256), sm, s, g, L, sk, sv, inv_sqrt_d);
+      } else if (e != cudaSuccess) {
+        return e;
+      }
       launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     }
