@@ -45,13 +45,15 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 TRAFFIC_PATH = os.path.join(ROOT, "profiles", "roofline_traffic.json")
 
 
-def measured_traffic(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu record, or None
-    when there is none or the kernel's sources changed since it was taken."""
+def measured_traffic(workload, kernel, variant=""):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu
+    record (keyed "workload/kernel[/variant]"), or None when there is none or
+    the kernel's sources changed since it was taken."""
     import hashlib
+    key = f"{workload}/{kernel}" + (f"/{variant}" if variant else "")
     try:
         with open(TRAFFIC_PATH) as f:
-            rec = json.load(f)[kernel]
+            rec = json.load(f)[key]
         h = hashlib.sha256()
         for name in rec["sources"]:
             with open(os.path.join(ROOT, name), "rb") as f:
@@ -279,6 +281,10 @@ class Runner:
             return "three calls per layer (project, append, attend)"
         return ("kvq_decode_step: one fused kernel per layer" if self.fused else
                 "kvq_decode_step: three kernels per layer")
+
+    def traffic_variant(self):
+        """Which decode-step implementation the per-kernel "decode_step" times."""
+        return "separate" if self.separate else ("fused" if self.fused else "three_kernels")
 
     def launches_per_step(self):
         """Kernels the library launches in one whole-job step."""
@@ -677,7 +683,9 @@ def main():
                          "peak": peak, "unit": unit, "frac": round(achieved / peak, 4),
                          "peak_source": f"{peak_kind} "
                                         f"({'bf16_tflops_sustained' if bound == 'tensor' else 'hbm_gbs'})",
-                         "traffic": measured_traffic(dominant),
+                         "traffic": measured_traffic(
+                             wl.name, dominant,
+                             run.traffic_variant() if dominant == "decode_step" else ""),
                          "algorithmic_bytes" if bound == "hbm" else "algorithmic_flops": amount},
             "kernels": kernels,
             "cpu_baseline": cpu,
