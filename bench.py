@@ -97,14 +97,40 @@ def proj_bytes(wl, M):
     return 2 * (w + lora + M * wl.d_in + M * wl.n_out)
 
 
+def coded_bytes_per_token(wl):
+    """Packed bytes per coded token and KV head, with KVarN's fp16 row scale and
+    its share of the per-block fp16 column scales (keys and values)."""
+    extra = 2 * (2 + 2 * wl.head_dim // wl.group_size) if wl.fmt == synth.FMT_KVARN else 0
+    return code_bytes_per_token(wl) + extra
+
+
+def cache_read_bytes(wl, T):
+    """HBM bytes a decode attention reads from one (sequence, KV head) holding
+    T tokens: coded tokens plus the full-precision windows (KIVI residual,
+    KVarN sinks and staged tokens) in the activation dtype."""
+    G = wl.group_size
+    full = 2 * wl.head_dim * (2 if wl.dtype == "bf16" else 4)
+    if wl.fmt == synth.FMT_FLOAT:
+        return T * full
+    coded = coded_bytes_per_token(wl)
+    if wl.fmt == synth.FMT_KIVI:
+        tq = G * (max(T - wl.residual_tokens, 0) // G)
+        return tq * coded + (T - tq) * full
+    if wl.fmt == synth.FMT_KVARN:
+        s = min(T, wl.sink_tokens)
+        tq = G * ((T - s) // G)
+        return tq * coded + (T - tq) * full
+    return T * coded
+
+
 def pack_bytes(wl, L):
     B, H, D = wl.batch, wl.n_kv_heads, wl.head_dim
-    return B * H * L * (2 * D * 2 + code_bytes_per_token(wl))
+    return B * H * L * (2 * D * 2 + coded_bytes_per_token(wl))
 
 
 def decode_attn_bytes(wl, T):
     B, H, Hq, D = wl.batch, wl.n_kv_heads, wl.n_q_heads, wl.head_dim
-    return B * H * T * code_bytes_per_token(wl) + 2 * B * Hq * D * 2
+    return B * H * cache_read_bytes(wl, T) + 2 * B * Hq * D * 2
 
 
 def decode_step_bytes(wl, T):
@@ -394,6 +420,28 @@ def graph_time_ms(fn, reps):
     return a.elapsed_time(b) / reps
 
 
+def cold_graph_time_ms(fn, reps, flush):
+    """Mean device time of one call of `fn` replayed from a captured graph,
+    with L2 flushed before each timed replay (outside the events)."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        fn()
+    torch.cuda.synchronize()
+    g.replay()
+    ms = []
+    for _ in range(reps):
+        l2_flush(flush)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        ms.append(a.elapsed_time(b))
+    return statistics.mean(ms)
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle (the reported baseline and the reference arm)
 # ---------------------------------------------------------------------------
@@ -610,6 +658,16 @@ def main():
         mean_ms["decode_step"] = graph_time_ms(run.decode_step_layers, reps) / wl.layers
         T_dec = wl.prefill + 2 + reps // 2     # mean cache length over the timed replays
         work["decode_step"] = ("hbm", decode_step_bytes(wl, T_dec), n_dec)
+    # the packed-cache decode attention alone (kvq_attend_decode over every
+    # layer's cache, L2 flushed before each timed replay), against HBM
+    att_ms = cold_graph_time_ms(run.decode_attend_layers, reps, flush) / wl.layers
+    T_att = run.caches[0].sync()
+    att_bytes = decode_attn_bytes(wl, T_att)
+    att_rate = att_bytes / (att_ms / 1000.0) / 1e9
+    decode_attention = {"mean_ms": round(att_ms, 5), "tokens": T_att,
+                        "algorithmic_bytes": att_bytes, "achieved": round(att_rate, 3),
+                        "unit": "GB/s", "frac": round(att_rate / peaks["hbm_gbs"], 4),
+                        "l2": "flushed before each replay of all layers' calls"}
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)
     bound, amount, _ = work[dominant]
@@ -688,6 +746,7 @@ def main():
                              run.traffic_variant() if dominant == "decode_step" else ""),
                          "algorithmic_bytes" if bound == "hbm" else "algorithmic_flops": amount},
             "kernels": kernels,
+            "decode_attention": decode_attention,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},

@@ -513,13 +513,23 @@ int decode_splits(const Geom& g) {
 }
 
 cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
-                          bool decode, cudaStream_t s) {
+                          bool decode, int t_hint, cudaStream_t s) {
   if (!decode && prefill_tc_supported(g)) {
     int* err = device_error_word();
     if (!err) return cudaErrorInvalidDevice;
     return launch_prefill_tc(g, q, L, scale, out, err, s);
   }
   if (!decode && prefill_mma_supported(g)) return launch_prefill_mma(g, q, L, scale, out, s);
+  // the streaming decode pays off once every CTA streams a few stages; short
+  // caches keep the split kernel (both read T on the device and are exact
+  // for any T, so a captured graph stays correct as the cache grows)
+  const int64_t blocks = (int64_t)g.B * g.H * ((t_hint + 31) / 32);
+  if (decode && decode_stream_supported(g) &&
+      (!decode_mma_supported(g) || blocks >= 16 * (int64_t)decode_stream_ctas(g))) {
+    int* err = device_error_word();
+    if (!err) return cudaErrorInvalidDevice;
+    return launch_decode_stream(g, q, scale, err, out, s);
+  }
   if (decode && decode_mma_supported(g)) {
     int* err = device_error_word();
     if (!err) return cudaErrorInvalidDevice;

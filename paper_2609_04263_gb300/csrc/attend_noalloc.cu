@@ -80,7 +80,7 @@ extern "C" kvq_status kvq_attend_decode_noalloc(kvq_cache* cache, const void* q,
                                          cudaGetErrorString(e));
   Geom g = cache->g;                        // same kernels, partials in the static array
   g.pl[KVQ_PLANE_WORKSPACE].p = scratch;
-  e = launch_attend(g, q, 1, softmax_scale, out, true, s);
+  e = launch_attend(g, q, 1, softmax_scale, out, true, cache->T, s);
   if (e != cudaSuccess) return set_error(KVQ_ERR_CUDA, "kvq_attend_decode_noalloc launch: %s",
                                          cudaGetErrorString(e));
   return KVQ_OK;

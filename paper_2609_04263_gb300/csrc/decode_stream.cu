@@ -1,0 +1,823 @@
+// Streaming split-K decode attention over the packed cache (§3.1 cache
+// formats, §3.2-3.3 attention over the stored reconstruction, L = 1).
+//
+// Persistent CTAs, one per SM: the (sequence, kv head, 32-token block) space
+// is flattened head-major and cut into one contiguous range per CTA, so every
+// CTA streams the same number of blocks whatever B, Hkv and T are.  One
+// producer warp copies each block (codes and fp16 metadata) with
+// cp.async.bulk into a deep ring of shared-memory stages (full/empty
+// mbarriers, bounded waits); eight consumer warps take the ring's blocks in
+// turn.  A warp keeps a running softmax state per kv head; where the CTA's
+// range crosses into the next head, its warps hand their partials to a
+// shared-memory slot, the last of them merges the slot, and where a head
+// spans several CTAs the last CTA to finish it (an arrival counter) merges
+// their partials from the workspace.  No CTA ever waits on another.
+//
+// Tensor-core layout (mma.sync m16n8k16): tokens are the MMA rows and the
+// g = Hq / Hkv query heads of the kv head its columns, so GQA heads share
+// every code that is unpacked.
+//   scores   S^T[t][h] = sum_d k_hat[t][d] q[h][d]
+//     A = key codes as exact bf16 integers (0x4300 | c) = 128 + c, B = q.
+//     Per-token groups: one accumulator per group, then
+//       S = sum_g s_tg acc_g + (m_tg - 128 s_tg) sum_{d in g} q_d.
+//     KIVI keys (one scale per 32-token block and channel): B = q * s_blk as
+//     bf16 high + low parts (two MMAs); the 128 of the codes is removed with
+//     an MMA over a constant operand, and sum_d q_d m_d is added per block.
+//   softmax  in base 2 with the softmax scale folded in; P goes to fp16 and
+//     movmatrix transposes each 8x8 tile into the B operand of P V.
+//   values   O^T[d][h] = sum_t v_hat[t][d] p[h][t]
+//     A = value codes as exact fp16 integers (0x6400 | c) = 1024 + c,
+//     B = fp16(p) * s_tg (the group's per-token scale), so
+//       O = MMA(codes + 1024, P s) - 1024 MMA(1, P s) + MMA(m, P):
+//     the bias and the per-token offsets m are two small MMAs (rows = groups).
+// KIVI's newest tokens (its full-precision residual ring) are read from
+// global memory as bf16 rows in the same layout.
+#include "decode_attn.cuh"
+
+namespace kvq {
+namespace {
+using namespace dattn;
+
+constexpr int kBT = 32;            // tokens per block (one KIVI key block)
+constexpr int kSB = 8;             // blocks per ring stage (copied together)
+constexpr int kNW = 8;             // consumer warps
+constexpr int kThreads = (kNW + 1) * 32;
+constexpr int kMaxStages = 64;
+constexpr int kSmemMax = 227 * 1024;
+constexpr long kSpin = 1L << 22;   // bounded shared-memory polls
+
+template <int D, int KB, int VB, int FMT>
+struct SCfg {
+  static constexpr int NG = D / 32;                    // groups of 32 channels
+  static constexpr int KS_STEPS = D / 16;              // MMA k-steps over channels
+  static constexpr int MT = D / 16;                    // P V m-tiles (channels)
+  static constexpr bool KIVI = FMT == KVQ_FMT_KIVI;
+  static constexpr bool SYM = FMT == KVQ_FMT_SYMMETRIC;
+  static constexpr int KCB = D * KB / 8, VCB = D * VB / 8;   // code bytes per token
+  // per block: K metadata (KIVI: one row of D per block; else per token), V metadata
+  static constexpr int KMETA = KIVI ? D * 2 : kBT * NG * 2;
+  static constexpr int VMETA = kBT * NG * 2;
+  // a stage holds kSB consecutive blocks, each plane contiguous over them
+  static constexpr int KC = 0;
+  static constexpr int VC = KC + kSB * kBT * KCB;
+  static constexpr int KS = VC + kSB * kBT * VCB;
+  static constexpr int KZ = KS + kSB * KMETA;
+  static constexpr int VS = KZ + (SYM ? 0 : kSB * KMETA);
+  static constexpr int VZ = VS + kSB * VMETA;
+  static constexpr int STAGE = (VZ + (SYM ? 0 : kSB * VMETA) + 127) / 128 * 128;
+};
+
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+__device__ __forceinline__ uint32_t hmul2u(uint32_t a, uint32_t b) {
+  __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&a), *reinterpret_cast<const __half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+__device__ __forceinline__ uint32_t h2u(__half lo, __half hi) {
+  return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
+}
+__device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// First block index of CTA c when N blocks are cut into P ranges.
+__device__ __forceinline__ int64_t range_start(int64_t c, int64_t N, int P) { return c * N / P; }
+// The CTA whose range holds block x.
+__device__ __forceinline__ int cta_of(int64_t x, int64_t N, int P) {
+  int c = (int)(x * P / N);
+  while (c + 1 < P && range_start(c + 1, N, P) <= x) ++c;
+  while (c > 0 && range_start(c, N, P) > x) --c;
+  return c;
+}
+
+// Shared-memory layout after the ring: one partial slot per consumer warp
+// (grp rows of m, l and D outputs), the merge scratch, then the barriers.
+struct Merge {
+  float m[kMaxSplits][8];   // partials' m (log2 units), then their weights
+  float l[kMaxSplits][8];
+  float M[8], L[8];
+  int last;
+  int pad;
+};
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kNW * 32) : "memory");
+}
+// Two tokens' fp16 metadata of group gq packed as (token a, token b), from
+// each token's NG values loaded as 32-bit words.
+__device__ __forceinline__ uint32_t pair_group(uint32_t wa, uint32_t wb, int gq) {
+  return __byte_perm(wa, wb, (gq & 1) ? 0x7632 : 0x5410);
+}
+
+template <int D, int KB, int VB, int FMT>
+__global__ void __launch_bounds__(kThreads, 1)
+decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err,
+                     __nv_bfloat16* __restrict__ out, int ns) {
+  using C = SCfg<D, KB, VB, FMT>;
+  constexpr int NG = C::NG, KSS = C::KS_STEPS, MT = C::MT;
+  extern __shared__ __align__(128) unsigned char smem[];
+  pdl_wait();
+  pdl_trigger();
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tid = lane & 3;
+  const int grp = g.Hq / g.H;
+  const int PW = grp * (D + 2);                      // floats of one warp's partial
+  float* slot = reinterpret_cast<float*>(smem + (size_t)ns * C::STAGE);   // [kNW][PW]
+  Merge* mg = reinterpret_cast<Merge*>(slot + kNW * PW);
+  uint64_t* full = reinterpret_cast<uint64_t*>(mg + 1);
+  uint64_t* empty = full + ns;
+
+  const int T = cache_tokens(g);
+  const int BH = g.B * g.H;
+  const int nb = (T + kBT - 1) / kBT;                // blocks per head
+  const int64_t N = (int64_t)BH * nb;
+  if (N == 0) {                                      // nothing stored: zero output
+    if (blockIdx.x == 0)
+      for (int i = threadIdx.x; i < g.B * g.Hq * D; i += blockDim.x) out[i] = __float2bfloat16(0.f);
+    return;
+  }
+  const int P = N < (int64_t)gridDim.x ? (int)N : (int)gridDim.x;
+  if ((int)blockIdx.x >= P) return;
+  const int64_t k0 = range_start(blockIdx.x, N, P), k1 = range_start(blockIdx.x + 1, N, P);
+  const int nblk = (int)(k1 - k0);
+  const int tq = C::KIVI ? kivi_tq(T, g.R, 32) : T;  // coded tokens
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < ns; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kSB);                     // one arrival per block
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  // ------------------------------------------------------------------ producer
+  if (warp == kNW) {
+    const int nst = (nblk + kSB - 1) / kSB;          // stages
+    int head = (int)(k0 / nb), blk = (int)(k0 % nb); // first block of the next stage
+    int s = 0;
+    for (; s < nst; ++s) {
+      const int st = s % ns;
+      bool ok = true;
+      if (s >= ns && lane == 0) ok = mbar_wait(&empty[st], ((s / ns) - 1) & 1);
+      if (!__shfl_sync(0xffffffffu, ok, 0)) {
+        if (lane == 0) atomicOr(err, 1);
+        break;
+      }
+      // split the stage's blocks into runs of one head's coded blocks; in
+      // pass p, lane 6 r + c issues copy c of run 5 p + r (every lane walks
+      // the same blocks, so the bookkeeping stays in registers)
+      const int nbs = min(kSB, nblk - s * kSB);
+      const int h_st = head, b_st = blk;             // the stage's first block
+      unsigned char* sp = smem + (size_t)st * C::STAGE;
+      int nrun = 0;
+      uint32_t total = 0;
+      for (int pass = 0; pass == 0 || pass * 5 < nrun; ++pass) {
+        const int myr = pass * 5 + lane / 6, myc = lane % 6;
+        int hh = h_st, bb = b_st, cnt = 0, r_head = 0, r_blk = 0, r_n = 0, r_sub = 0;
+        int p_head = -1, p_end = -1;                 // end of the current run
+#pragma unroll
+        for (int i = 0; i < kSB; ++i) {
+          if (i < nbs && bb * kBT < tq) {
+            if (!(hh == p_head && bb == p_end)) {    // a new run starts here
+              if (cnt == myr) { r_head = hh; r_blk = bb; r_sub = i; }
+              ++cnt;
+            }
+            if (cnt - 1 == myr) ++r_n;
+            if (pass == 0) {
+              // bytes of the block (the last coded block of a head may be
+              // partial: whole 4-token groups are copied)
+              const int nt = (min(kBT, tq - bb * kBT) + 3) & ~3;
+              total += nt * (C::KCB + C::VCB) + (C::SYM ? 1 : 2) * nt * NG * 2;
+              total += C::KIVI ? 2 * D * 2 : (C::SYM ? 1 : 2) * nt * NG * 2;
+            }
+            p_head = hh;
+            p_end = bb + 1;
+          }
+          if (i < nbs && ++bb == nb) { bb = 0; ++hh; }
+        }
+        if (pass == 0) {
+          nrun = cnt;
+          head = hh;                                 // first block of the next stage
+          blk = bb;
+          if (lane == 0) mbar_expect_tx(&full[st], total);   // 0: nothing to copy
+          __syncwarp();
+        }
+        if (lane < 30 && myr < nrun && (!C::SYM || myc < 4)) {
+          const int t0 = r_blk * kBT;
+          const int n4 = (min(r_n * kBT, tq - t0) + 3) & ~3;
+          const int tsub = r_sub * kBT;              // first token slot in the stage
+          // plane rows of head h: plane_ptr(g, plane, 0, h, row) addresses (b, hkv) = h
+          const uint8_t* src;
+          unsigned char* dst;
+          uint32_t bytes;
+          if (myc == 0) {
+            src = plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, 0, r_head, t0);
+            dst = sp + C::KC + tsub * C::KCB;
+            bytes = n4 * C::KCB;
+          } else if (myc == 1) {
+            src = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, 0, r_head, t0);
+            dst = sp + C::VC + tsub * C::VCB;
+            bytes = n4 * C::VCB;
+          } else if (myc == 2 || myc == 4) {
+            const int pl = myc == 2 ? KVQ_PLANE_K_SCALE : KVQ_PLANE_K_ZERO;
+            src = reinterpret_cast<const uint8_t*>(
+                plane_ptr<__half>(g, pl, 0, r_head, C::KIVI ? r_blk : t0));
+            dst = sp + (myc == 2 ? C::KS : C::KZ) + r_sub * C::KMETA;
+            bytes = C::KIVI ? r_n * D * 2 : n4 * NG * 2;
+          } else {
+            const int pl = myc == 3 ? KVQ_PLANE_V_SCALE : KVQ_PLANE_V_ZERO;
+            src = reinterpret_cast<const uint8_t*>(plane_ptr<__half>(g, pl, 0, r_head, t0));
+            dst = sp + (myc == 3 ? C::VS : C::VZ) + r_sub * C::VMETA;
+            bytes = n4 * NG * 2;
+          }
+          bulk_g2s(dst, src, bytes, &full[st]);
+        }
+      }
+    }
+    // keep the CTA alive until the last copies have landed (the consumers
+    // wait for them too, unless they gave up on a timeout)
+    if (lane == 0)
+      for (int i = max(0, s - ns); i < s; ++i)
+        if (!mbar_wait(&full[i % ns], (i / ns) & 1)) atomicOr(err, 1);
+    return;
+  }
+
+  // ------------------------------------------------------------------ consumers
+  const float c2 = scale * 1.4426950408889634f;      // scores in log2 units
+  const uint32_t kmask = KB == 4 ? 0x000F000Fu : 0x00030003u;
+  const uint32_t vmask = VB == 4 ? 0x000F000Fu : 0x00030003u;
+  const int zb = C::SYM ? (1 << (KB - 1)) : 0;       // symmetric key code bias
+  const int zbv = C::SYM ? (1 << (VB - 1)) : 0;
+  const __half kbias = __float2half_rn(1024.f + (float)zbv);
+  const uint32_t kbias2 = h2u(kbias, kbias);
+  const int tc = threadIdx.x;                        // 0 .. kNW * 32 - 1
+  float* wsb = reinterpret_cast<float*>(g.pl[KVQ_PLANE_WORKSPACE].p);
+
+  int b = 0, hkv = 0;
+  bool bad = false;                                  // a wait timed out: stop computing
+  uint32_t qb[KSS][2];                               // B fragments of q (head gid)
+  float qs[NG][2];                                   // per-group sum of q, heads 2tid, 2tid+1
+  float m_run[2], l_run[2];
+  float o[MT][4], bias[NG][4], offa[4];
+
+  // q of the head: thread (gid, tid) holds head gid, channels 32 gq + 8 tid + e
+  auto load_q = [&]() {
+    const __nv_bfloat16* qh = q + ((int64_t)b * g.Hq + hkv * grp) * D;
+#pragma unroll
+    for (int gq = 0; gq < NG; ++gq) {
+      uint4 u = make_uint4(0, 0, 0, 0);
+      if (gid < grp) u = *reinterpret_cast<const uint4*>(qh + gid * D + 32 * gq + 8 * tid);
+      const uint16_t* e = reinterpret_cast<const uint16_t*>(&u);
+#pragma unroll
+      for (int sub = 0; sub < 2; ++sub) {
+        qb[2 * gq + sub][0] = pack_raw(e[qk_chan<KB>(sub, 0, 0)], e[qk_chan<KB>(sub, 0, 1)]);
+        qb[2 * gq + sub][1] = pack_raw(e[qk_chan<KB>(sub, 1, 0)], e[qk_chan<KB>(sub, 1, 1)]);
+      }
+      const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+      float s = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h2[i]);
+        s += f.x + f.y;
+      }
+      s += __shfl_xor_sync(0xffffffffu, s, 1);
+      s += __shfl_xor_sync(0xffffffffu, s, 2);       // head gid, group gq
+      qs[gq][0] = __shfl_sync(0xffffffffu, s, 4 * (2 * tid));
+      qs[gq][1] = __shfl_sync(0xffffffffu, s, 4 * (2 * tid + 1));
+    }
+    m_run[0] = m_run[1] = -INFINITY;
+    l_run[0] = l_run[1] = 0.f;
+#pragma unroll
+    for (int i = 0; i < MT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+#pragma unroll
+    for (int i = 0; i < NG; ++i) bias[i][0] = bias[i][1] = bias[i][2] = bias[i][3] = 0.f;
+    offa[0] = offa[1] = offa[2] = offa[3] = 0.f;
+  };
+
+  // one 32-token block: scores, online softmax, P V
+  auto process = [&](const unsigned char* sp, int sub_blk, int t0, int nv, bool coded) {
+    const unsigned char* kcp = sp + C::KC + sub_blk * kBT * C::KCB;
+    const unsigned char* vcp = sp + C::VC + sub_blk * kBT * C::VCB;
+    const unsigned char* ksp = sp + C::KS + sub_blk * C::KMETA;
+    const unsigned char* kzp = sp + C::KZ + sub_blk * C::KMETA;
+    const unsigned char* vsp = sp + C::VS + sub_blk * C::VMETA;
+    const unsigned char* vzp = sp + C::VZ + sub_blk * C::VMETA;
+    float S[2][4];
+    if (coded && !C::KIVI) {
+      float acc[NG][2][4];
+#pragma unroll
+      for (int gq = 0; gq < NG; ++gq)
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) acc[gq][mt][0] = acc[gq][mt][1] = acc[gq][mt][2] = acc[gq][mt][3] = 0.f;
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        const unsigned char* r0 = kcp + (16 * mt + gid) * C::KCB;
+        const unsigned char* r1 = r0 + 8 * C::KCB;
+#pragma unroll
+        for (int gq = 0; gq < NG; ++gq) {
+          uint32_t w0, w1;
+          if (KB == 4) {
+            w0 = *reinterpret_cast<const uint32_t*>(r0 + 16 * gq + 4 * tid);
+            w1 = *reinterpret_cast<const uint32_t*>(r1 + 16 * gq + 4 * tid);
+          } else {
+            const uint32_t v0 = *reinterpret_cast<const uint16_t*>(r0 + 8 * gq + 2 * tid);
+            const uint32_t v1 = *reinterpret_cast<const uint16_t*>(r1 + 8 * gq + 2 * tid);
+            w0 = v0 | (v0 << 14);
+            w1 = v1 | (v1 << 14);
+          }
+#pragma unroll
+          for (int sub = 0; sub < 2; ++sub) {
+            uint32_t a[4];
+            a[0] = magic2(w0 >> (8 * sub), kmask);
+            a[1] = magic2(w1 >> (8 * sub), kmask);
+            a[2] = magic2(w0 >> (8 * sub + 4), kmask);
+            a[3] = magic2(w1 >> (8 * sub + 4), kmask);
+            mma16816(acc[gq][mt], a, qb[2 * gq + sub][0], qb[2 * gq + sub][1]);
+          }
+        }
+      }
+      const __half* ksc = reinterpret_cast<const __half*>(ksp);
+      const __half* kze = reinterpret_cast<const __half*>(kzp);
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int t = 16 * mt + gid + 8 * r;
+          float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+          for (int gq = 0; gq < NG; gq += 2) {
+            const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(ksc + t * NG + gq));
+            float2 mz;
+            if (C::SYM) mz = make_float2(-(float)zb * sc.x, -(float)zb * sc.y);
+            else mz = __half22float2(*reinterpret_cast<const __half2*>(kze + t * NG + gq));
+            const float off0 = mz.x - 128.f * sc.x, off1 = mz.y - 128.f * sc.y;
+            s0 += sc.x * acc[gq][mt][2 * r] + off0 * qs[gq][0];
+            s1 += sc.x * acc[gq][mt][2 * r + 1] + off0 * qs[gq][1];
+            s0 += sc.y * acc[gq + 1][mt][2 * r] + off1 * qs[gq + 1][0];
+            s1 += sc.y * acc[gq + 1][mt][2 * r + 1] + off1 * qs[gq + 1][1];
+          }
+          const bool valid = t < nv;
+          S[mt][2 * r] = valid ? s0 * c2 : -INFINITY;
+          S[mt][2 * r + 1] = valid ? s1 * c2 : -INFINITY;
+        }
+    } else if (coded) {  // KIVI keys: B = q * s_blk (scaled) as bf16 high + low parts
+      const __half* ksc = reinterpret_cast<const __half*>(ksp);
+      const __half* kze = reinterpret_cast<const __half*>(kzp);
+      uint32_t qh[KSS][2], ql[KSS][2];
+      float qm = 0.f;                                // sum_d q_d m_d over this thread's channels
+#pragma unroll
+      for (int gq = 0; gq < NG; ++gq) {
+        const uint4 su = *reinterpret_cast<const uint4*>(ksc + 32 * gq + 8 * tid);
+        const uint4 zu = *reinterpret_cast<const uint4*>(kze + 32 * gq + 8 * tid);
+        const __half* sv = reinterpret_cast<const __half*>(&su);
+        const __half* zv = reinterpret_cast<const __half*>(&zu);
+#pragma unroll
+        for (int sub = 0; sub < 2; ++sub)
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            const int e0 = qk_chan<KB>(sub, hf, 0), e1 = qk_chan<KB>(sub, hf, 1);
+            const uint32_t qw = qb[2 * gq + sub][hf];
+            const float2 qq = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw));
+            const float x0 = qq.x * __half2float(sv[e0]);
+            const float x1 = qq.y * __half2float(sv[e1]);
+            const uint32_t hw = pack_bf16(x0, x1);
+            const float2 hv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hw));
+            qh[2 * gq + sub][hf] = hw;
+            ql[2 * gq + sub][hf] = pack_bf16(x0 - hv.x, x1 - hv.y);
+            qm += qq.x * __half2float(zv[e0]) + qq.y * __half2float(zv[e1]);
+          }
+      }
+      qm += __shfl_xor_sync(0xffffffffu, qm, 1);
+      qm += __shfl_xor_sync(0xffffffffu, qm, 2);     // head gid
+      // the codes enter as 128 + c: the same MMA over a constant 128 operand
+      // gives the 128 sum(hi + lo) to remove, per head, as the tensor core sums it
+      float bh[4] = {0.f, 0.f, 0.f, 0.f}, bl[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint32_t a128[4] = {kMagic, kMagic, kMagic, kMagic};
+#pragma unroll
+      for (int ks = 0; ks < KSS; ++ks) {
+        mma16816(bh, a128, qh[ks][0], qh[ks][1]);
+        mma16816(bl, a128, ql[ks][0], ql[ks][1]);
+      }
+      const float cs0 = __shfl_sync(0xffffffffu, qm, 4 * (2 * tid)) - (bh[0] + bl[0]);
+      const float cs1 = __shfl_sync(0xffffffffu, qm, 4 * (2 * tid + 1)) - (bh[1] + bl[1]);
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        float acc[2][4];                             // [high, low]
+#pragma unroll
+        for (int k = 0; k < 2; ++k) acc[k][0] = acc[k][1] = acc[k][2] = acc[k][3] = 0.f;
+        const unsigned char* r0 = kcp + (16 * mt + gid) * C::KCB;
+        const unsigned char* r1 = r0 + 8 * C::KCB;
+#pragma unroll
+        for (int gq = 0; gq < NG; ++gq) {
+          uint32_t w0, w1;
+          if (KB == 4) {
+            w0 = *reinterpret_cast<const uint32_t*>(r0 + 16 * gq + 4 * tid);
+            w1 = *reinterpret_cast<const uint32_t*>(r1 + 16 * gq + 4 * tid);
+          } else {
+            const uint32_t v0 = *reinterpret_cast<const uint16_t*>(r0 + 8 * gq + 2 * tid);
+            const uint32_t v1 = *reinterpret_cast<const uint16_t*>(r1 + 8 * gq + 2 * tid);
+            w0 = v0 | (v0 << 14);
+            w1 = v1 | (v1 << 14);
+          }
+#pragma unroll
+          for (int sub = 0; sub < 2; ++sub) {
+            uint32_t a[4];
+            a[0] = magic2(w0 >> (8 * sub), kmask);
+            a[1] = magic2(w1 >> (8 * sub), kmask);
+            a[2] = magic2(w0 >> (8 * sub + 4), kmask);
+            a[3] = magic2(w1 >> (8 * sub + 4), kmask);
+            mma16816(acc[0], a, qh[2 * gq + sub][0], qh[2 * gq + sub][1]);
+            mma16816(acc[1], a, ql[2 * gq + sub][0], ql[2 * gq + sub][1]);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const bool valid = 16 * mt + gid + 8 * r < nv;
+          const float v0 = acc[0][2 * r] + acc[1][2 * r];
+          const float v1 = acc[0][2 * r + 1] + acc[1][2 * r + 1];
+          S[mt][2 * r] = valid ? (v0 + cs0) * c2 : -INFINITY;
+          S[mt][2 * r + 1] = valid ? (v1 + cs1) * c2 : -INFINITY;
+        }
+      }
+    } else {  // full-precision keys (KIVI residual ring), read from global memory
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        const int ta = t0 + 16 * mt + gid, tb = ta + 8;
+        const __nv_bfloat16* ka = plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, hkv, ta < t0 + nv ? ta % g.ring : 0);
+        const __nv_bfloat16* kb = plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, hkv, tb < t0 + nv ? tb % g.ring : 0);
+#pragma unroll
+        for (int gq = 0; gq < NG; ++gq) {
+          const uint4 ua = ta < t0 + nv ? *reinterpret_cast<const uint4*>(ka + 32 * gq + 8 * tid) : make_uint4(0, 0, 0, 0);
+          const uint4 ub = tb < t0 + nv ? *reinterpret_cast<const uint4*>(kb + 32 * gq + 8 * tid) : make_uint4(0, 0, 0, 0);
+          const uint16_t* ea = reinterpret_cast<const uint16_t*>(&ua);
+          const uint16_t* eb = reinterpret_cast<const uint16_t*>(&ub);
+#pragma unroll
+          for (int sub = 0; sub < 2; ++sub) {
+            uint32_t a[4];
+            a[0] = pack_raw(ea[qk_chan<KB>(sub, 0, 0)], ea[qk_chan<KB>(sub, 0, 1)]);
+            a[1] = pack_raw(eb[qk_chan<KB>(sub, 0, 0)], eb[qk_chan<KB>(sub, 0, 1)]);
+            a[2] = pack_raw(ea[qk_chan<KB>(sub, 1, 0)], ea[qk_chan<KB>(sub, 1, 1)]);
+            a[3] = pack_raw(eb[qk_chan<KB>(sub, 1, 0)], eb[qk_chan<KB>(sub, 1, 1)]);
+            mma16816(acc, a, qb[2 * gq + sub][0], qb[2 * gq + sub][1]);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const bool valid = 16 * mt + gid + 8 * r < nv;
+          S[mt][2 * r] = valid ? acc[2 * r] * c2 : -INFINITY;
+          S[mt][2 * r + 1] = valid ? acc[2 * r + 1] * c2 : -INFINITY;
+        }
+      }
+    }
+
+    // --------------------------------------------------------------- softmax
+    float mx[2];
+#pragma unroll
+    for (int jh = 0; jh < 2; ++jh) {
+      mx[jh] = fmaxf(fmaxf(S[0][jh], S[0][2 + jh]), fmaxf(S[1][jh], S[1][2 + jh]));
+      mx[jh] = fmaxf(mx[jh], __shfl_xor_sync(0xffffffffu, mx[jh], 4));
+      mx[jh] = fmaxf(mx[jh], __shfl_xor_sync(0xffffffffu, mx[jh], 8));
+      mx[jh] = fmaxf(mx[jh], __shfl_xor_sync(0xffffffffu, mx[jh], 16));
+    }
+    float alpha[2];
+#pragma unroll
+    for (int jh = 0; jh < 2; ++jh) {
+      const float mn = fmaxf(m_run[jh], mx[jh]);
+      alpha[jh] = m_run[jh] == -INFINITY ? 0.f : exp2f(m_run[jh] - mn);
+      m_run[jh] = mn;
+      l_run[jh] *= alpha[jh];
+    }
+    if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
+#pragma unroll
+      for (int i = 0; i < MT; ++i) {
+        o[i][0] *= alpha[0]; o[i][1] *= alpha[1];
+        o[i][2] *= alpha[0]; o[i][3] *= alpha[1];
+      }
+#pragma unroll
+      for (int i = 0; i < NG; ++i) {
+        bias[i][0] *= alpha[0]; bias[i][1] *= alpha[1];
+        bias[i][2] *= alpha[0]; bias[i][3] *= alpha[1];
+      }
+      offa[0] *= alpha[0]; offa[1] *= alpha[1];
+      offa[2] *= alpha[0]; offa[3] *= alpha[1];
+    }
+    uint32_t pb[2][2];                               // B fragments of P^T per 16-token step
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      float p[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        p[i] = exp2f(S[mt][i] - m_run[i & 1]);       // exp2(-inf) = 0
+        l_run[i & 1] += p[i];
+      }
+      pb[mt][0] = movmatrix_t(pack_f16(p[0], p[1]));
+      pb[mt][1] = movmatrix_t(pack_f16(p[2], p[3]));
+    }
+
+    // ------------------------------------------------------------------- P V
+    if (coded) {
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        int tk[4];
+        uint32_t vsw[4][(NG + 1) / 2];               // per token: NG fp16 scales as words
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          tk[i] = 16 * mt + 2 * tid + (i & 1) + 8 * (i >> 1);
+          const bool v = tk[i] < nv;
+          const uint32_t* src = reinterpret_cast<const uint32_t*>(vsp + tk[i] * NG * 2);
+#pragma unroll
+          for (int w = 0; w < (NG + 1) / 2; ++w) vsw[i][w] = v ? src[w] : 0u;
+        }
+        if (!C::SYM) {                               // offsets: rows = groups
+          uint32_t a[4] = {0u, 0u, 0u, 0u};
+          if (gid < NG) {
+            const uint16_t* vz = reinterpret_cast<const uint16_t*>(vzp);
+            uint32_t z[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) z[i] = tk[i] < nv ? vz[tk[i] * NG + gid] : 0u;
+            a[0] = z[0] | (z[1] << 16);
+            a[2] = z[2] | (z[3] << 16);
+          }
+          mma16816_f16(offa, a, pb[mt][0], pb[mt][1]);
+        }
+#pragma unroll
+        for (int gq = 0; gq < NG; ++gq) {
+          const uint32_t s01 = pair_group(vsw[0][gq >> 1], vsw[1][gq >> 1], gq);
+          const uint32_t s89 = pair_group(vsw[2][gq >> 1], vsw[3][gq >> 1], gq);
+          const uint32_t b0 = hmul2u(pb[mt][0], s01), b1 = hmul2u(pb[mt][1], s89);
+          const unsigned char* vc = vcp;
+          uint32_t x01, x89;
+          if (VB == 4) {
+            x01 = (uint32_t)*reinterpret_cast<const uint16_t*>(vc + tk[0] * C::VCB + 16 * gq + 2 * gid) |
+                  ((uint32_t)*reinterpret_cast<const uint16_t*>(vc + tk[1] * C::VCB + 16 * gq + 2 * gid) << 16);
+            x89 = (uint32_t)*reinterpret_cast<const uint16_t*>(vc + tk[2] * C::VCB + 16 * gq + 2 * gid) |
+                  ((uint32_t)*reinterpret_cast<const uint16_t*>(vc + tk[3] * C::VCB + 16 * gq + 2 * gid) << 16);
+          } else {
+            x01 = (uint32_t)vc[tk[0] * C::VCB + 8 * gq + gid] | ((uint32_t)vc[tk[1] * C::VCB + 8 * gq + gid] << 16);
+            x89 = (uint32_t)vc[tk[2] * C::VCB + 8 * gq + gid] | ((uint32_t)vc[tk[3] * C::VCB + 8 * gq + gid] << 16);
+          }
+          constexpr int SH = VB == 4 ? 4 : 2;        // bits between consecutive channels
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            uint32_t a[4];
+            a[0] = magic2h(x01 >> (2 * SH * u), vmask);
+            a[1] = magic2h(x01 >> (2 * SH * u + SH), vmask);
+            a[2] = magic2h(x89 >> (2 * SH * u), vmask);
+            a[3] = magic2h(x89 >> (2 * SH * u + SH), vmask);
+            mma16816_f16(o[2 * gq + u], a, b0, b1);
+          }
+          const uint32_t ab[4] = {kbias2, kbias2, kbias2, kbias2};
+          mma16816_f16(bias[gq], ab, b0, b1);
+        }
+      }
+    } else {  // full-precision values
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        const __nv_bfloat16* vr[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int t = t0 + 16 * mt + 2 * tid + (i & 1) + 8 * (i >> 1);
+          vr[i] = t < t0 + nv ? plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, hkv, t % g.ring) : nullptr;
+        }
+#pragma unroll
+        for (int gq = 0; gq < NG; ++gq) {
+          uint2 vw[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            vw[i] = vr[i] ? *reinterpret_cast<const uint2*>(vr[i] + 32 * gq + 4 * gid) : make_uint2(0, 0);
+          auto el = [&](int i, int c) {
+            const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&vw[i]);
+            return __bfloat162float(e[c]);
+          };
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            uint32_t a[4];
+            a[0] = pack_f16(el(0, 2 * u), el(1, 2 * u));
+            a[1] = pack_f16(el(0, 2 * u + 1), el(1, 2 * u + 1));
+            a[2] = pack_f16(el(2, 2 * u), el(3, 2 * u));
+            a[3] = pack_f16(el(2, 2 * u + 1), el(3, 2 * u + 1));
+            mma16816_f16(o[2 * gq + u], a, pb[mt][0], pb[mt][1]);
+          }
+        }
+      }
+    }
+  };
+
+  // ------------------------------------------------------ head segments
+  // The CTA's range crosses heads hfirst..hlast.  Every consumer warp runs
+  // every segment (warps without blocks in it only join the merge), so the
+  // named barriers below are reached by all of them.
+  const int hfirst = (int)(k0 / nb), hlast = (int)((k1 - 1) / nb);
+  for (int hd = hfirst; hd <= hlast; ++hd) {
+    const int64_t hs = (int64_t)hd * nb;
+    const int a = (int)(max(k0, hs) - k0), e = (int)(min(k1, hs + nb) - k0);
+    b = hd / g.H;
+    hkv = hd % g.H;
+    const int jst = a + ((warp - a) % kNW + kNW) % kNW;   // first block of this warp
+    const bool mine = jst < e;
+    if (mine) load_q();
+    for (int j = jst; j < e && !bad; j += kNW) {
+      const int sj = j / kSB, st = sj % ns;
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&full[st], (sj / ns) & 1);
+      if (!__shfl_sync(0xffffffffu, ok, 0)) {
+        if (lane == 0) atomicOr(err, 1);
+        bad = true;
+        break;
+      }
+      const int t0 = (int)(k0 + j - hs) * kBT;
+      process(smem + (size_t)st * C::STAGE, j % kSB, t0, min(kBT, T - t0), t0 < tq);
+      __syncwarp();
+      if (lane == 0) mbar_arrive1(&empty[st]);
+    }
+    if (mine) {
+      // fold the bias and offset terms into O; reduce l over the rows
+#pragma unroll
+      for (int gq = 0; gq < NG; ++gq) {
+        const float f0 = __shfl_sync(0xffffffffu, offa[0], 4 * gq + tid) - bias[gq][0];
+        const float f1 = __shfl_sync(0xffffffffu, offa[1], 4 * gq + tid) - bias[gq][1];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          o[2 * gq + u][0] += f0;
+          o[2 * gq + u][1] += f1;
+          o[2 * gq + u][2] += f0;
+          o[2 * gq + u][3] += f1;
+        }
+      }
+#pragma unroll
+      for (int jh = 0; jh < 2; ++jh) {
+        l_run[jh] += __shfl_xor_sync(0xffffffffu, l_run[jh], 4);
+        l_run[jh] += __shfl_xor_sync(0xffffffffu, l_run[jh], 8);
+        l_run[jh] += __shfl_xor_sync(0xffffffffu, l_run[jh], 16);
+        if (bad) m_run[jh] = -INFINITY;
+      }
+    }
+    consumer_sync();                                 // the previous merge is done with the slots
+    if (mine) {
+      float* ws = slot + warp * PW;
+#pragma unroll
+      for (int i = 0; i < MT; ++i) {
+        const int d0 = 32 * (i >> 1) + 4 * gid + 2 * (i & 1);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int h = 2 * tid + (r & 1);
+          if (h < grp) ws[h * (D + 2) + 2 + d0 + (r >> 1)] = o[i][r];
+        }
+      }
+      if (gid == 0)
+#pragma unroll
+        for (int jh = 0; jh < 2; ++jh)
+          if (2 * tid + jh < grp) {
+            ws[(2 * tid + jh) * (D + 2)] = m_run[jh];
+            ws[(2 * tid + jh) * (D + 2) + 1] = l_run[jh];
+          }
+    }
+    consumer_sync();
+    // merge the warps' partials: warps (a + i) % kNW, i < np, hold this head
+    const int np = min(kNW, e - a);
+    if (tc < grp) {
+      float M = -INFINITY;
+      for (int i = 0; i < np; ++i) M = fmaxf(M, slot[((a + i) % kNW) * PW + tc * (D + 2)]);
+      float L = 0.f;
+      for (int i = 0; i < np; ++i) {
+        const float* pp = slot + ((a + i) % kNW) * PW + tc * (D + 2);
+        const float w = pp[0] == -INFINITY ? 0.f : exp2f(pp[0] - M);
+        mg->m[i][tc] = w;
+        L += w * pp[1];
+      }
+      mg->M[tc] = M;
+      mg->L[tc] = L;
+    }
+    consumer_sync();
+    const int c0 = cta_of(hs, N, P), c1 = cta_of(hs + nb - 1, N, P);
+    const int nct = c1 - c0 + 1;
+    if (nct > kMaxSplits) {                          // the host sizes the grid so this cannot happen
+      if (tc == 0) atomicOr(err, 4);
+      continue;
+    }
+    const int64_t orow0 = (int64_t)b * g.Hq + hkv * grp;
+    for (int idx = tc; idx < grp * D; idx += kNW * 32) {
+      const int h = idx / D, d = idx % D;
+      float acc = 0.f;
+      for (int i = 0; i < np; ++i) acc += mg->m[i][h] * slot[((a + i) % kNW) * PW + h * (D + 2) + 2 + d];
+      if (nct == 1) {
+        const float L = mg->L[h];
+        out[(orow0 + h) * D + d] = __float2bfloat16(L > 0.f ? acc / L : 0.f);
+      } else {
+        wsb[((orow0 + h) * kMaxSplits + (blockIdx.x - c0)) * (D + kWsStride) + 2 + d] = acc;
+      }
+    }
+    if (nct == 1) continue;
+    if (tc < grp) {
+      float* wr = wsb + ((orow0 + tc) * kMaxSplits + (blockIdx.x - c0)) * (D + kWsStride);
+      wr[0] = mg->M[tc];
+      wr[1] = mg->L[tc];
+    }
+    // the last CTA of this head merges all of its CTAs' partials
+    consumer_sync();
+    if (tc == 0) {
+      __threadfence();
+      mg->last = atomicAdd(&g.counters[hd], 1u) == (unsigned)nct - 1;
+    }
+    consumer_sync();
+    if (!mg->last) continue;
+    __threadfence();
+    if (tc < grp * nct) {
+      const int h = tc / nct, i = tc % nct;
+      const float* wr = wsb + ((orow0 + h) * kMaxSplits + i) * (D + kWsStride);
+      mg->m[i][h] = __ldcg(wr);
+      mg->l[i][h] = __ldcg(wr + 1);
+    }
+    consumer_sync();
+    if (tc < grp) {
+      float M = -INFINITY;
+      for (int i = 0; i < nct; ++i) M = fmaxf(M, mg->m[i][tc]);
+      float L = 0.f;
+      for (int i = 0; i < nct; ++i) {
+        const float w = mg->m[i][tc] == -INFINITY ? 0.f : exp2f(mg->m[i][tc] - M);
+        mg->m[i][tc] = w;
+        L += w * mg->l[i][tc];
+      }
+      mg->L[tc] = L;
+    }
+    consumer_sync();
+    for (int idx = tc; idx < grp * D; idx += kNW * 32) {
+      const int h = idx / D, d = idx % D;
+      const float* wr = wsb + (orow0 + h) * kMaxSplits * (D + kWsStride) + 2 + d;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int i = 0; i < nct; ++i) acc += mg->m[i][h] * __ldcg(wr + i * (D + kWsStride));
+      const float L = mg->L[h];
+      out[(orow0 + h) * D + d] = __float2bfloat16(L > 0.f ? acc / L : 0.f);
+    }
+    if (tc == 0) g.counters[hd] = 0;                 // ready for the next call
+  }
+}
+
+template <int D, int KB, int VB, int FMT>
+size_t stream_smem(int grp, int* ns) {
+  using C = SCfg<D, KB, VB, FMT>;
+  const size_t fixed = (size_t)kNW * grp * (D + 2) * 4 + sizeof(Merge);
+  int n = (int)((kSmemMax - fixed) / (C::STAGE + 16));
+  if (n > kMaxStages) n = kMaxStages;
+  *ns = n;
+  return (size_t)n * C::STAGE + fixed + (size_t)2 * n * 8;
+}
+
+template <int D, int KB, int VB, int FMT>
+cudaError_t launch_t(const Geom& g, const void* q, float scale, int* err, void* out,
+                     cudaStream_t s) {
+  const int grp = g.Hq / g.H;
+  int ns = 0;
+  const size_t sm = stream_smem<D, KB, VB, FMT>(grp, &ns);
+  auto kern = decode_stream_kernel<D, KB, VB, FMT>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  launch_pdl(kern, dim3(decode_stream_ctas(g)), dim3(kThreads), sm, s, g,
+             reinterpret_cast<const __nv_bfloat16*>(q), scale, err,
+             reinterpret_cast<__nv_bfloat16*>(out), ns);
+  return cudaGetLastError();
+}
+
+template <int D, int BITS>
+cudaError_t launch_fmt(const Geom& g, const void* q, float scale, int* err, void* out,
+                       cudaStream_t s) {
+  switch (g.fmt) {
+    case KVQ_FMT_AFFINE: return launch_t<D, BITS, BITS, KVQ_FMT_AFFINE>(g, q, scale, err, out, s);
+    case KVQ_FMT_SYMMETRIC: return launch_t<D, BITS, BITS, KVQ_FMT_SYMMETRIC>(g, q, scale, err, out, s);
+    case KVQ_FMT_KIVI: return launch_t<D, BITS, BITS, KVQ_FMT_KIVI>(g, q, scale, err, out, s);
+  }
+  return cudaErrorNotSupported;
+}
+
+}  // namespace
+
+// CTAs of the streaming decode: one per SM, at most 15 per (sequence, kv head)
+// so that a head never spans more CTAs than its kMaxSplits workspace rows.
+int decode_stream_ctas(const Geom& g) {
+  const int bh = g.B * g.H;
+  int p = num_sms();
+  if (p > 15 * bh) p = 15 * bh;
+  return p < 1 ? 1 : p;
+}
+
+bool decode_stream_supported(const Geom& g) {
+  const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC || g.fmt == KVQ_FMT_KIVI;
+  return fmt_ok && g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb && (g.kb == 2 || g.kb == 4) &&
+         (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
+}
+
+cudaError_t launch_decode_stream(const Geom& g, const void* q, float scale, int* err, void* out,
+                                 cudaStream_t s) {
+  if (g.D == 64) return g.kb == 4 ? launch_fmt<64, 4>(g, q, scale, err, out, s)
+                                  : launch_fmt<64, 2>(g, q, scale, err, out, s);
+  return g.kb == 4 ? launch_fmt<128, 4>(g, q, scale, err, out, s)
+                   : launch_fmt<128, 2>(g, q, scale, err, out, s);
+}
+
+}  // namespace kvq

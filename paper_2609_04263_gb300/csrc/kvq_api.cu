@@ -373,7 +373,8 @@ static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_
                 cache->T);
   if (!(scale > 0.f) || scale != scale) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
   cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
-  if (e == cudaSuccess) e = launch_attend(cache->g, q, L, scale, out, decode, (cudaStream_t)stream);
+  if (e == cudaSuccess) e = launch_attend(cache->g, q, L, scale, out, decode, cache->T,
+                                            (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_attend launch");
   return KVQ_OK;
 }

@@ -114,8 +114,10 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 // They return cudaGetLastError() of their launches.
 // All launchers read the token count from g.state on the device.
 cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cudaStream_t s);
+// t_hint: the host's count of stored tokens, used only to choose between
+// decode kernels (the kernels read the count from the device).
 cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
-                          bool decode, cudaStream_t s);
+                          bool decode, int t_hint, cudaStream_t s);
 // pos_dev: if non-NULL, positions start at *pos_dev + pos0 (a cache's token
 // count read on the device), else at pos0.
 cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
@@ -156,6 +158,12 @@ cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale,
                                cudaStream_t s);
 cudaError_t launch_decode_mma(const Geom& g, const void* q, float scale, int* err, void* out,
                               cudaStream_t s);
+// Streaming persistent decode (decode_stream.cu): the formats it covers, its
+// grid size, and the launch (it merges its own partials).
+bool decode_stream_supported(const Geom& g);
+int decode_stream_ctas(const Geom& g);
+cudaError_t launch_decode_stream(const Geom& g, const void* q, float scale, int* err, void* out,
+                                 cudaStream_t s);
 
 // Token range of split `s` of `splits` over T tokens (tiles of `tile`).
 __host__ __device__ inline void split_range(int T, int splits, int s, int tile, int* ts,

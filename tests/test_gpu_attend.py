@@ -59,6 +59,13 @@ DECODE = [
     ("sym2", "bf16", 3, 2, 6, 64, [65]),            # odd group, ragged chunk
     ("kivi2", "bf16", 1, 1, 8, 64, [1000, 7]),      # chunks straddle the residual edge
     ("affine2", "bf16", 2, 4, 8, 64, [4095, 1]),
+    # shapes large enough for the streaming decode (>= 16 blocks of 32 tokens
+    # per CTA); many short heads put up to 8 heads in one ring stage
+    ("affine4", "bf16", 160, 16, 32, 64, [20]),
+    ("sym2", "bf16", 100, 16, 32, 64, [40]),         # two blocks per head, the second partial
+    ("kivi2", "bf16", 160, 16, 64, 128, [31]),       # residual only: nothing coded
+    ("kivi2", "bf16", 8, 8, 32, 128, [1297, 3]),     # heads spanning several CTAs
+    ("affine2", "bf16", 4, 8, 64, 128, [2500]),      # GQA 8, D 128
 ]
 
 
