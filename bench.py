@@ -667,7 +667,8 @@ def main():
     decode_attention = {"mean_ms": round(att_ms, 5), "tokens": T_att,
                         "algorithmic_bytes": att_bytes, "achieved": round(att_rate, 3),
                         "unit": "GB/s", "frac": round(att_rate / peaks["hbm_gbs"], 4),
-                        "l2": "flushed before each replay of all layers' calls"}
+                        "l2": "flushed before each replay of all layers' calls",
+                        "traffic": measured_traffic(wl.name, "decode_attention")}
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)
     bound, amount, _ = work[dominant]
