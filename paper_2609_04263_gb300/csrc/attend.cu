@@ -506,8 +506,10 @@ bool kvarn_decode_supported(const Geom& g) {
 }  // namespace
 
 int decode_splits(const Geom& g) {
+  // the split kernels fit two CTAs per SM: round down so that every split of
+  // every (sequence, kv head) runs in the first wave
   const int bh = g.B * g.H;
-  int s = (2 * num_sms() + bh - 1) / bh;
+  int s = 2 * num_sms() / bh;
   if (s > kMaxSplits) s = kMaxSplits;
   return s < 1 ? 1 : s;
 }
