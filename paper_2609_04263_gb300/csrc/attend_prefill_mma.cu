@@ -213,7 +213,7 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
 }
 
 template <int D>
-__global__ void __launch_bounds__(PCfg<D>::THREADS)
+__global__ void __launch_bounds__(PCfg<D>::THREADS, D == 128 ? 2 : 1)
 attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, float scale,
                           __nv_bfloat16* __restrict__ out, int nq, float inv_sqrt_d) {
   pdl_wait();
