@@ -26,7 +26,8 @@ template <int D>
 struct PCfg {
   static constexpr int WARPS = D == 256 ? 4 : 8;
   static constexpr int ROWS = WARPS * 16;
-  static constexpr int NT = D == 256 ? 32 : 64;      // tokens per KV tile
+  // tokens per KV tile (16 at D = 256: two CTAs fit an SM)
+  static constexpr int NT = D == 256 ? 16 : 64;
   static constexpr int LDS = D + 8;                   // smem row stride (bf16), 16 B pad
   static constexpr int Q_OFF = 0;
   static constexpr int K_OFF = ROWS * LDS * 2;          // bf16 high part of K
@@ -39,7 +40,7 @@ struct PCfg {
   // remainder of the rotated queries
   static constexpr int QL_OFF = SCR_OFF + NT * D * 4;
   static constexpr int TOTAL_KVARN = QL_OFF + ROWS * LDS * 2;
-  static_assert(QL_OFF - K_OFF >= ROWS * D * 4, "rotated output fits the K/V area");
+  static_assert(QL_OFF - K_OFF >= WARPS * 8 * D * 4, "half of each warp's output fits the K/V area");
   static constexpr int THREADS = WARPS * 32;
 };
 
@@ -213,7 +214,7 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
 }
 
 template <int D>
-__global__ void __launch_bounds__(PCfg<D>::THREADS, D == 128 ? 2 : 1)
+__global__ void __launch_bounds__(PCfg<D>::THREADS, D >= 128 ? 2 : 1)
 attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, float scale,
                           __nv_bfloat16* __restrict__ out, int nq, float inv_sqrt_d) {
   pdl_wait();
@@ -399,31 +400,32 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
     l_run[rr] += __shfl_xor_sync(0xffffffffu, l_run[rr], 2);
   }
   if (kvarn) {
-    // normalised rotated rows -> fp32 shared memory (the K/V area), then each
-    // warp rotates rows back and stores them
-    float* os = reinterpret_cast<float*>(smem + C::K_OFF);   // [ROWS][D]
-    __syncthreads();
+    // normalised rotated rows -> fp32 shared memory (each warp its own 8
+    // rows of the K/V area at a time), then the warp rotates them back
+    float* os = reinterpret_cast<float*>(smem + C::K_OFF) + warp * 8 * D;   // [8][D]
+    __syncthreads();                                  // every warp is done with K and V
 #pragma unroll
     for (int rr = 0; rr < 2; ++rr) {
-      const int r = warp * 16 + gid + 8 * rr;
       const float inv = l_run[rr] > 0.f ? 1.f / l_run[rr] : 0.f;
 #pragma unroll
       for (int j = 0; j < D / 8; ++j) {
-        os[r * D + 8 * j + 2 * tid] = o[j][2 * rr] * inv;
-        os[r * D + 8 * j + 2 * tid + 1] = o[j][2 * rr + 1] * inv;
+        os[gid * D + 8 * j + 2 * tid] = o[j][2 * rr] * inv;
+        os[gid * D + 8 * j + 2 * tid + 1] = o[j][2 * rr + 1] * inv;
       }
-    }
-    __syncthreads();
-    for (int r = warp; r < C::ROWS; r += C::WARPS) {
-      const int hl = r / nq, qi = r % nq;
-      if (hl >= grp || qi >= nql) continue;
-      float x[D / 32];
+      __syncwarp();
+      for (int k = 0; k < 8; ++k) {
+        const int r = warp * 16 + 8 * rr + k;
+        const int hl = r / nq, qi = r % nq;
+        if (hl >= grp || qi >= nql) continue;
+        float x[D / 32];
 #pragma unroll
-      for (int i = 0; i < D / 32; ++i) x[i] = os[r * D + lane + 32 * i];
-      fwht_warp<D>(x, lane, inv_sqrt_d);
-      __nv_bfloat16* orow = out + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D;
+        for (int i = 0; i < D / 32; ++i) x[i] = os[k * D + lane + 32 * i];
+        fwht_warp<D>(x, lane, inv_sqrt_d);
+        __nv_bfloat16* orow = out + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D;
 #pragma unroll
-      for (int i = 0; i < D / 32; ++i) orow[lane + 32 * i] = __float2bfloat16_rn(x[i]);
+        for (int i = 0; i < D / 32; ++i) orow[lane + 32 * i] = __float2bfloat16_rn(x[i]);
+      }
+      __syncwarp();                                   // the rows are read before the next half
     }
     return;
   }
