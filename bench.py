@@ -312,6 +312,19 @@ class Runner:
         """Which decode-step implementation the per-kernel "decode_step" times."""
         return "separate" if self.separate else ("fused" if self.fused else "three_kernels")
 
+    def kvarn_streamed(self):
+        """Whether KVarN decode attention at the prefill length takes the
+        tensor-core kernel over the coded tokens (the library's size rule)."""
+        wl = self.wl
+        if wl.fmt != synth.FMT_KVARN or wl.dtype != "bf16" or (wl.key_bits, wl.value_bits) != (4, 2):
+            return False
+        if (wl.head_dim, wl.group_size) not in ((256, 64), (64, 32)):
+            return False
+        bh = wl.batch * wl.n_kv_heads
+        ctas = min(torch.cuda.get_device_properties(0).multi_processor_count, 15 * bh)
+        coded = max(wl.prefill - wl.sink_tokens, 0) // wl.group_size * wl.group_size
+        return bh * (coded // 32) >= 16 * ctas
+
     def launches_per_step(self):
         """Kernels the library launches in one whole-job step."""
         wl = self.wl
@@ -322,6 +335,8 @@ class Runner:
         attend = 1 if (wl.dtype == "bf16" and wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC,
                                                          synth.FMT_KIVI)
                        and wl.head_dim in (64, 128)) else 2
+        if self.kvarn_streamed():
+            attend = 3          # coded tokens, sinks and staged tokens, combine
         prefill = wl.layers * (1 + append + 1)
         per_layer = 1 if (self.fused and not self.separate) else 1 + append + attend
         return prefill + wl.decode * wl.layers * per_layer

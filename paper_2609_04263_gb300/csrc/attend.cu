@@ -253,25 +253,27 @@ attend_generic_kernel(Geom g, const void* q, int L, float scale, void* out,
 }
 
 // Merge the split partials of one (b, q head): o = sum_s e^(m_s - M) o_s /
-// sum_s e^(m_s - M) l_s.
-__global__ void combine_kernel(Geom g, int splits, void* out) {
+// sum_s e^(m_s - M) l_s over slots 0 .. splits-1, and slot `extra` if >= 0.
+__global__ void combine_kernel(Geom g, int splits, int extra, void* out) {
   pdl_wait();
   pdl_trigger();
   const int hq = blockIdx.x, b = blockIdx.y;
   const int D = g.D;
   const float* w = ws_row(g, b, hq);
+  const int n = splits + (extra >= 0 ? 1 : 0);
+  auto row = [&](int i) { return w + (int64_t)(i < splits ? i : extra) * (D + kWsStride); };
   float M = -INFINITY;
-  for (int s = 0; s < splits; ++s) M = fmaxf(M, w[s * (D + kWsStride)]);
+  for (int i = 0; i < n; ++i) M = fmaxf(M, row(i)[0]);
   float Lsum = 0.f;
-  for (int s = 0; s < splits; ++s) {
-    const float m = w[s * (D + kWsStride)];
-    if (m != -INFINITY) Lsum += expf(m - M) * w[s * (D + kWsStride) + 1];
+  for (int i = 0; i < n; ++i) {
+    const float m = row(i)[0];
+    if (m != -INFINITY) Lsum += expf(m - M) * row(i)[1];
   }
   for (int d = threadIdx.x; d < D; d += blockDim.x) {
     float o = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      const float m = w[s * (D + kWsStride)];
-      if (m != -INFINITY) o += expf(m - M) * w[s * (D + kWsStride) + 2 + d];
+    for (int i = 0; i < n; ++i) {
+      const float m = row(i)[0];
+      if (m != -INFINITY) o += expf(m - M) * row(i)[2 + d];
     }
     st_act(out, ((int64_t)b * g.Hq + hq) * D + d, o / Lsum, g.act);
   }
@@ -321,7 +323,7 @@ __device__ __forceinline__ uint32_t lane_codes(const uint8_t* row, int lane, int
 template <int D, int GM>
 __global__ void __launch_bounds__(256)
 attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale,
-                           float inv_sqrt_d) {
+                           float inv_sqrt_d, int full_only) {
   pdl_wait();
   pdl_trigger();
   constexpr int NS = D / 32;
@@ -331,8 +333,11 @@ attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float sc
   const int grp = g.Hq / g.H, G = g.G, S = g.S;
   const int T = cache_tokens(g);
   const int nbq = kvarn_nblocks(T, S, G) * G;
+  // full_only: the splits share the full-precision tokens alone (sinks, then
+  // staged), indexed f = 0 .. T - nbq - 1 and mapped to token f or f + nbq
   int ts, te;
-  split_range(T, g.splits, split, G, &ts, &te);
+  if (full_only) split_range(T - nbq, g.splits, split, 1, &ts, &te);
+  else split_range(T, g.splits, split, G, &ts, &te);
   const float c2 = scale * 1.4426950408889634f;   // scores in log2 units
   // rotated queries, pre-scaled
   float qr[GM][NS];
@@ -363,7 +368,8 @@ attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float sc
   float qp[GM][NS], qs[GM];                         // q' = q_rot c_block and its lane sum
   float cv[NS];                                     // value column scales of the block
   int cur_blk = -1;
-  for (int t = w0; t < w1; ++t) {
+  for (int f = w0; f < w1; ++f) {
+    const int t = full_only && f >= S ? f + nbq : f;
     float kv[NS], vv[NS];
     const bool coded = t >= S && t - S < nbq;
     float dot[GM];
@@ -480,7 +486,7 @@ attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float sc
 }
 
 template <int D>
-cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, cudaStream_t s) {
+cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, int full_only, cudaStream_t s) {
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)D));
   dim3 grid(g.splits, g.H, g.B);
@@ -489,7 +495,7 @@ cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, cudaStream
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     launch_pdl(kern, dim3(grid), dim3(256), sm, s, g, reinterpret_cast<const __nv_bfloat16*>(q),
-               scale, inv_sqrt_d);
+               scale, inv_sqrt_d, full_only);
     return cudaGetLastError();
   };
   if (grp <= 2) return run(attend_kvarn_decode_kernel<D, 2>, 2);
@@ -510,7 +516,7 @@ int decode_splits(const Geom& g) {
   // every (sequence, kv head) runs in the first wave
   const int bh = g.B * g.H;
   int s = 2 * num_sms() / bh;
-  if (s > kMaxSplits) s = kMaxSplits;
+  if (s > kMaxSplits - 1) s = kMaxSplits - 1;     // the last slot is reserved (KVarN)
   return s < 1 ? 1 : s;
 }
 
@@ -538,11 +544,23 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
     return launch_decode_mma(g, q, scale, err, out, s);
   }
   if (decode && kvarn_decode_supported(g)) {
-    cudaError_t e = g.D == 64 ? launch_kvarn_d<64>(g, q, scale, s)
-                  : g.D == 128 ? launch_kvarn_d<128>(g, q, scale, s)
-                               : launch_kvarn_d<256>(g, q, scale, s);
+    // long caches: the coded tokens on tensor cores (one partial per head in
+    // the reserved slot), the sinks and staged tokens in the split kernel
+    const int64_t coded = (int64_t)g.B * g.H * (kvarn_nblocks(t_hint, g.S, g.G) * g.G / 32);
+    const bool streamed = decode_stream_kvarn_supported(g) &&
+                          coded >= 16 * (int64_t)decode_stream_ctas(g);
+    if (streamed) {
+      int* err = device_error_word();
+      if (!err) return cudaErrorInvalidDevice;
+      cudaError_t e = launch_decode_stream_kvarn(g, q, scale, err, s);
+      if (e != cudaSuccess) return e;
+    }
+    cudaError_t e = g.D == 64 ? launch_kvarn_d<64>(g, q, scale, streamed, s)
+                  : g.D == 128 ? launch_kvarn_d<128>(g, q, scale, streamed, s)
+                               : launch_kvarn_d<256>(g, q, scale, streamed, s);
     if (e != cudaSuccess) return e;
-    launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, g.splits, out);
+    launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, g.splits,
+               streamed ? kMaxSplits - 1 : -1, out);
     return cudaGetLastError();
   }
   const int grp = g.Hq / g.H;
@@ -570,7 +588,7 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
                                                    decode ? 1 : 0, inv_sqrt_d);
   e = cudaGetLastError();
   if (e != cudaSuccess || !decode) return e;
-  launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, splits, out);
+  launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, splits, -1, out);
   return cudaGetLastError();
 }
 

@@ -33,18 +33,12 @@
 // KIVI's newest tokens (its full-precision residual ring) are read from
 // global memory as bf16 rows in the same layout.
 #include "decode_attn.cuh"
+#include "stream_common.cuh"
 
 namespace kvq {
 namespace {
 using namespace dattn;
-
-constexpr int kBT = 32;            // tokens per block (one KIVI key block)
-constexpr int kSB = 8;             // blocks per ring stage (copied together)
-constexpr int kNW = 8;             // consumer warps
-constexpr int kThreads = (kNW + 1) * 32;
-constexpr int kMaxStages = 64;
-constexpr int kSmemMax = 227 * 1024;
-constexpr long kSpin = 1L << 22;   // bounded shared-memory polls
+using namespace stream;
 
 template <int D, int KB, int VB, int FMT>
 struct SCfg {
@@ -67,44 +61,6 @@ struct SCfg {
   static constexpr int STAGE = (VZ + (SYM ? 0 : kSB * VMETA) + 127) / 128 * 128;
 };
 
-__device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
-  uint32_t d;
-  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
-  return d;
-}
-__device__ __forceinline__ uint32_t hmul2u(uint32_t a, uint32_t b) {
-  __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&a), *reinterpret_cast<const __half2*>(&b));
-  return *reinterpret_cast<uint32_t*>(&r);
-}
-__device__ __forceinline__ uint32_t h2u(__half lo, __half hi) {
-  return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
-}
-__device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-// First block index of CTA c when N blocks are cut into P ranges.
-__device__ __forceinline__ int64_t range_start(int64_t c, int64_t N, int P) { return c * N / P; }
-// The CTA whose range holds block x.
-__device__ __forceinline__ int cta_of(int64_t x, int64_t N, int P) {
-  int c = (int)(x * P / N);
-  while (c + 1 < P && range_start(c + 1, N, P) <= x) ++c;
-  while (c > 0 && range_start(c, N, P) > x) --c;
-  return c;
-}
-
-// Shared-memory layout after the ring: one partial slot per consumer warp
-// (grp rows of m, l and D outputs), the merge scratch, then the barriers.
-struct Merge {
-  float m[kMaxSplits][8];   // partials' m (log2 units), then their weights
-  float l[kMaxSplits][8];
-  float M[8], L[8];
-  int last;
-  int pad;
-};
-__device__ __forceinline__ void consumer_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kNW * 32) : "memory");
-}
 // Two tokens' fp16 metadata of group gq packed as (token a, token b), from
 // each token's NG values loaded as 32-bit words.
 __device__ __forceinline__ uint32_t pair_group(uint32_t wa, uint32_t wb, int gq) {

@@ -164,6 +164,11 @@ bool decode_stream_supported(const Geom& g);
 int decode_stream_ctas(const Geom& g);
 cudaError_t launch_decode_stream(const Geom& g, const void* q, float scale, int* err, void* out,
                                  cudaStream_t s);
+// Streaming KVarN decode over the coded tokens (decode_stream_kvarn.cu): it
+// leaves each head's partial in workspace slot kMaxSplits - 1 for the combine.
+bool decode_stream_kvarn_supported(const Geom& g);
+cudaError_t launch_decode_stream_kvarn(const Geom& g, const void* q, float scale, int* err,
+                                       cudaStream_t s);
 
 // Token range of split `s` of `splits` over T tokens (tiles of `tile`).
 __host__ __device__ inline void split_range(int T, int splits, int s, int tile, int* ts,

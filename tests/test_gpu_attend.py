@@ -66,6 +66,10 @@ DECODE = [
     ("kivi2", "bf16", 160, 16, 64, 128, [31]),       # residual only: nothing coded
     ("kivi2", "bf16", 8, 8, 32, 128, [1297, 3]),     # heads spanning several CTAs
     ("affine2", "bf16", 4, 8, 64, 128, [2500]),      # GQA 8, D 128
+    # KVarN long enough for the streaming kernel over the coded tokens (the
+    # sinks and staged tokens go through the split kernel, then one combine)
+    ("kvarn", "bf16", 8, 8, 16, 256, [1500]),
+    ("kvarn_small", "bf16", 16, 8, 32, 64, [700, 1]),
 ]
 
 
