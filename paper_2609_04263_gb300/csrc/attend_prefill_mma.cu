@@ -213,7 +213,74 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
   }
 }
 
-template <int D>
+// KIVI with BITS-bit keys and values: tokens [t0, t0 + NT) into the K high /
+// remainder and V tiles.  A thread keeps one 8-channel chunk for all of its
+// tokens, so the keys' per-channel block scales and offsets (one row per 32
+// tokens) are loaded once per block, and the plane rows are addressed from
+// per-head bases.  Tokens from tq on are the full-precision residual ring.
+template <int D, int BITS, int NT, int THREADS>
+__device__ __forceinline__ void kivi_tile(const Geom& g, int b, int h, int t0, int T, int tq,
+                                          __nv_bfloat16* khi, __nv_bfloat16* klo, __half* vdst,
+                                          int lds) {
+  constexpr int CH = D / 8;
+  constexpr int RSTEP = THREADS / CH;                 // token step between a thread's items
+  static_assert(THREADS % CH == 0 && NT % RSTEP == 0, "whole tokens per pass");
+  constexpr unsigned mask = (1u << BITS) - 1;
+  const int c = threadIdx.x % CH, r0 = threadIdx.x / CH;
+  int cur_blk = -1;
+  uint4 su = make_uint4(0, 0, 0, 0), zu = make_uint4(0, 0, 0, 0);   // block scales, offsets (fp16)
+#pragma unroll 1
+  for (int k = 0; k < NT / RSTEP; ++k) {
+    const int r = r0 + k * RSTEP, t = t0 + r;
+    float kv[8], vv[8];
+    if (t >= T) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) kv[e] = vv[e] = 0.f;
+    } else if (t >= tq) {
+      const int slot = t % g.ring;
+      const uint4 ku = *reinterpret_cast<const uint4*>(plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, h, slot, 8 * c));
+      const uint4 vu = *reinterpret_cast<const uint4*>(plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, h, slot, 8 * c));
+      const __nv_bfloat16* k8 = reinterpret_cast<const __nv_bfloat16*>(&ku);
+      const __nv_bfloat16* v8 = reinterpret_cast<const __nv_bfloat16*>(&vu);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        kv[e] = __bfloat162float(k8[e]);
+        vv[e] = __bfloat162float(v8[e]);
+      }
+    } else {
+      const int blk = t / 32;
+      if (blk != cur_blk) {                           // the keys' block scales of these channels
+        cur_blk = blk;
+        su = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, 8 * c));
+        zu = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, 8 * c));
+      }
+      const uint8_t* kr = plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t) + (BITS == 4 ? 4 : 2) * c;
+      const uint8_t* vr = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t) + (BITS == 4 ? 4 : 2) * c;
+      const uint32_t kw = BITS == 4 ? *reinterpret_cast<const uint32_t*>(kr)
+                                    : *reinterpret_cast<const uint16_t*>(kr);
+      const uint32_t vw = BITS == 4 ? *reinterpret_cast<const uint32_t*>(vr)
+                                    : *reinterpret_cast<const uint16_t*>(vr);
+      const float vs = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, t, c / 4));
+      const float vz = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, t, c / 4));
+      const __half2* s2 = reinterpret_cast<const __half2*>(&su);
+      const __half2* z2 = reinterpret_cast<const __half2*>(&zu);
+#pragma unroll
+      for (int e2 = 0; e2 < 4; ++e2) {
+        const float2 sf = __half22float2(s2[e2]), zf = __half22float2(z2[e2]);
+        kv[2 * e2] = (float)((kw >> (2 * e2 * BITS)) & mask) * sf.x + zf.x;
+        kv[2 * e2 + 1] = (float)((kw >> ((2 * e2 + 1) * BITS)) & mask) * sf.y + zf.y;
+        vv[2 * e2] = (float)((vw >> (2 * e2 * BITS)) & mask) * vs + vz;
+        vv[2 * e2 + 1] = (float)((vw >> ((2 * e2 + 1) * BITS)) & mask) * vs + vz;
+      }
+    }
+    store_k8(kv, khi + r * lds + 8 * c, klo + r * lds + 8 * c);
+    store_v8(vv, vdst + r * lds + 8 * c);
+  }
+}
+
+// KIVIB: 0 = any format (tiles through deq8 or kvarn_tile); 2 or 4 = a KIVI
+// cache with KIVIB-bit keys and values (tiles through kivi_tile).
+template <int D, int KIVIB>
 __global__ void __launch_bounds__(PCfg<D>::THREADS, D >= 128 ? 2 : 1)
 attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, float scale,
                           __nv_bfloat16* __restrict__ out, int nq, float inv_sqrt_d) {
@@ -250,7 +317,7 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
           q + (((int64_t)b * g.Hq + hkv * grp + hl) * L + q0 + qi) * D + 8 * c);
     *reinterpret_cast<uint4*>(Qs + r * LDS + 8 * c) = v;
   }
-  const bool kvarn = g.fmt == KVQ_FMT_KVARN;
+  const bool kvarn = KIVIB == 0 && g.fmt == KVQ_FMT_KVARN;
   __nv_bfloat16* Ql = reinterpret_cast<__nv_bfloat16*>(smem + C::QL_OFF);
   if (kvarn) {
     // rotate the query rows: high part in Qs, bf16 remainder in Ql
@@ -292,7 +359,9 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
 
   for (int t0 = 0; t0 < t_end; t0 += NT) {
     __syncthreads();                                  // previous tile consumed
-    if (g.fmt == KVQ_FMT_KVARN) {
+    if (KIVIB != 0) {
+      kivi_tile<D, KIVIB == 0 ? 2 : KIVIB, NT, C::THREADS>(g, b, hkv, t0, T, tq, Ks, Kl, Vs, LDS);
+    } else if (g.fmt == KVQ_FMT_KVARN) {
       float* scr = reinterpret_cast<float*>(smem + C::SCR_OFF);
       kvarn_tile<D, NT, C::THREADS>(g, 0, b, hkv, t0, T, Ks, Kl, Vs, LDS, scr, inv_sqrt_d);
       __syncthreads();
@@ -449,7 +518,9 @@ cudaError_t launch_d(const Geom& g, const void* q, int L, float scale, void* out
   using C = PCfg<D>;
   const int grp = g.Hq / g.H;
   const int nq = C::ROWS / grp;
-  auto kern = attend_prefill_mma_kernel<D>;
+  auto kern = g.fmt == KVQ_FMT_KIVI && g.kb == g.vb && g.kb == 2 ? attend_prefill_mma_kernel<D, 2>
+            : g.fmt == KVQ_FMT_KIVI && g.kb == g.vb && g.kb == 4 ? attend_prefill_mma_kernel<D, 4>
+                                                                 : attend_prefill_mma_kernel<D, 0>;
   const int smem = g.fmt == KVQ_FMT_KVARN ? C::TOTAL_KVARN : C::TOTAL;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
