@@ -213,6 +213,55 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
   }
 }
 
+// KVarN tile whose tokens are all coded (stored rotated: r_t c_j (s code + m)),
+// keys and values in one pass.  A thread keeps one 8-channel chunk for all
+// of its tokens; the tile lies inside one column-scale block (NT divides the
+// block length G and the sinks end on a tile boundary), so the chunk's
+// column scales are loaded once.
+template <int D, int NT, int THREADS>
+__device__ __forceinline__ void kvarn_tile_coded(const Geom& g, int b, int h, int t0,
+                                                 __nv_bfloat16* khi, __nv_bfloat16* klo,
+                                                 __half* vdst, int lds) {
+  constexpr int CH = D / 8;
+  constexpr int RSTEP = THREADS / CH;
+  static_assert(THREADS % CH == 0 && NT % RSTEP == 0, "whole tokens per pass");
+  const int c = threadIdx.x % CH, r0 = threadIdx.x / CH;
+  const int kb = g.kb, vb = g.vb, grp = (8 * c) / g.G;
+  const unsigned kmask = (1u << kb) - 1, vmask = (1u << vb) - 1;
+  const int blk = (t0 - g.S) / g.G;
+  const uint4 kcu = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, KVQ_PLANE_K_COL, b, h, blk, 8 * c));
+  const uint4 vcu = *reinterpret_cast<const uint4*>(plane_ptr<__half>(g, KVQ_PLANE_V_COL, b, h, blk, 8 * c));
+#pragma unroll 1
+  for (int k = 0; k < NT / RSTEP; ++k) {
+    const int r = r0 + k * RSTEP, qi = t0 + r - g.S;
+    const uint8_t* krow = plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, qi);
+    const uint8_t* vrow = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, qi);
+    const uint32_t kw = kb == 4 ? *reinterpret_cast<const uint32_t*>(krow + 4 * c)
+                                : *reinterpret_cast<const uint16_t*>(krow + 2 * c);
+    const uint32_t vw = vb == 4 ? *reinterpret_cast<const uint32_t*>(vrow + 4 * c)
+                                : *reinterpret_cast<const uint16_t*>(vrow + 2 * c);
+    const float ks = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, qi, grp));
+    const float kz = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, qi, grp));
+    const float vs = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, qi, grp));
+    const float vz = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, qi, grp));
+    const float kr = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_K_ROW, b, h, 0, qi));
+    const float vr = __half2float(*plane_ptr<__half>(g, KVQ_PLANE_V_ROW, b, h, 0, qi));
+    const __half2* kc2 = reinterpret_cast<const __half2*>(&kcu);
+    const __half2* vc2 = reinterpret_cast<const __half2*>(&vcu);
+    float kv[8], vv[8];
+#pragma unroll
+    for (int e2 = 0; e2 < 4; ++e2) {
+      const float2 kc = __half22float2(kc2[e2]), vc = __half22float2(vc2[e2]);
+      kv[2 * e2] = kr * kc.x * ((float)((kw >> (2 * e2 * kb)) & kmask) * ks + kz);
+      kv[2 * e2 + 1] = kr * kc.y * ((float)((kw >> ((2 * e2 + 1) * kb)) & kmask) * ks + kz);
+      vv[2 * e2] = vr * vc.x * ((float)((vw >> (2 * e2 * vb)) & vmask) * vs + vz);
+      vv[2 * e2 + 1] = vr * vc.y * ((float)((vw >> ((2 * e2 + 1) * vb)) & vmask) * vs + vz);
+    }
+    store_k8(kv, khi + r * lds + 8 * c, klo + r * lds + 8 * c);
+    store_v8(vv, vdst + r * lds + 8 * c);
+  }
+}
+
 // KIVI with BITS-bit keys and values: tokens [t0, t0 + NT) into the K high /
 // remainder and V tiles.  A thread keeps one 8-channel chunk for all of its
 // tokens, so the keys' per-channel block scales and offsets (one row per 32
@@ -361,6 +410,9 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
     __syncthreads();                                  // previous tile consumed
     if (KIVIB != 0) {
       kivi_tile<D, KIVIB == 0 ? 2 : KIVIB, NT, C::THREADS>(g, b, hkv, t0, T, tq, Ks, Kl, Vs, LDS);
+    } else if (D != 128 && g.fmt == KVQ_FMT_KVARN && t0 >= g.S && t0 + NT <= T &&
+               t0 + NT <= g.S + kvarn_nblocks(T, g.S, g.G) * g.G && g.G % NT == 0 && g.S % NT == 0) {
+      kvarn_tile_coded<D, NT, C::THREADS>(g, b, hkv, t0, Ks, Kl, Vs, LDS);
     } else if (g.fmt == KVQ_FMT_KVARN) {
       float* scr = reinterpret_cast<float*>(smem + C::SCR_OFF);
       kvarn_tile<D, NT, C::THREADS>(g, 0, b, hkv, t0, T, Ks, Kl, Vs, LDS, scr, inv_sqrt_d);
