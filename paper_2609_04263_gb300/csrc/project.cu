@@ -427,6 +427,11 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
     if (e != cudaErrorNotSupported) return e;
     (void)cudaGetLastError();
   }
+  if (act == KVQ_BF16 && M <= 16 && d_in % 64 == 0) {
+    cudaError_t e = launch_project_decode_stream(p, err, s);
+    if (e != cudaErrorNotSupported) return e;
+    (void)cudaGetLastError();
+  }
   if (act == KVQ_BF16 && M <= 16 && d_in % 32 == 0 && (size_t)16 * d_in * 2 <= 160 * 1024)
     return launch_decode_mma(p, s);
   if (M <= kSkinnyMaxM && (size_t)M * d_in * 4 <= 120 * 1024 && d_in % 64 == 0)

@@ -51,6 +51,14 @@ CASES = [
     ("bf16", 1, 130, 256, 4, 2, 128, (64, 0, 8), 0, 500000.0),
     ("bf16", 3, 5, 384, 2, 2, 256, (0, 32, 32), 900, 10000.0),
     ("bf16", 4, 1, 512, 8, 2, 64, (16, 16, 16), 2048, 10000.0),
+    # decode shapes of the weight-streaming kernel: 8B-like (16 rows, 4096
+    # channels, ranges spanning projections), 12B-like (a ragged last stage,
+    # D = 256), a two-chunk last stage with 8- and 64-rank factors and one
+    # CTA per pair-tile, and 24/8/40-rank factors (part-filled U tiles)
+    ("bf16", 16, 1, 4096, 32, 8, 128, (16, 16, 16), 8200, 500000.0),
+    ("bf16", 4, 1, 3840, 16, 8, 256, (32, 32, 32), 8700, 10000.0),
+    ("bf16", 1, 1, 2112, 4, 1, 64, (8, 0, 64), 3, 10000.0),
+    ("bf16", 2, 4, 1024, 6, 2, 64, (24, 8, 40), 0, 10000.0),
     ("bf16", 1, 64, 256, 4, 4, 64, (0, 0, 0), 0, 0.0),
     ("f32", 1, 96, 256, 4, 4, 64, (8, 8, 8), 0, 10000.0),
     ("f32", 1, 1, 256, 4, 4, 64, (8, 8, 8), 511, 10000.0),
