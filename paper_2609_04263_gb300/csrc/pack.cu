@@ -53,8 +53,23 @@ __device__ __forceinline__ void load8(const void* base, int64_t e, int act, floa
 __device__ __forceinline__ float affine_scale(float mn, float mx, int bits) {
   return fmaxf(__fdiv_rn(__fsub_rn(mx, mn), (float)((1 << bits) - 1)), 1e-8f);
 }
+// rint(a / s) where the quotient is first rounded to fp32 (both roundings to
+// nearest even), which is how the cache format defines a code.  __fdividef is
+// within 2 ulp of a / s for s in the normal range; when its result q lies
+// farther than 2^-14 from the half-integer between its two neighbouring
+// integers (and |q| < 64, where 2 ulp < 2^-17), the exact quotient and its
+// fp32 rounding lie on the same side of that representable half-integer
+// (rounding is monotone), so all three round to the same integer.  Otherwise
+// (near a tie, or NaN / out of range) the IEEE quotient is formed.
+__device__ __forceinline__ float rint_quot(float a, float s) {
+  const float q = __fdividef(a, s);
+  const float d = fabsf(q - (floorf(q) + 0.5f));
+  if (d > 0x1p-14f && fabsf(q) < 64.f) return rintf(q);
+  return rintf(__fdiv_rn(a, s));
+}
+
 __device__ __forceinline__ int affine_code(float x, float mn, float s, int bits) {
-  float c = rintf(__fdiv_rn(__fsub_rn(x, mn), s));
+  float c = rint_quot(__fsub_rn(x, mn), s);
   c = fminf(fmaxf(c, 0.f), (float)((1 << bits) - 1));
   return (int)c;
 }
@@ -65,7 +80,7 @@ __device__ __forceinline__ float sym_scale(float amax, int bits) {
 }
 __device__ __forceinline__ int sym_code(float x, float s, int bits) {
   const float qmax = (float)((1 << (bits - 1)) - 1);
-  float q = rintf(__fdiv_rn(x, s));
+  float q = rint_quot(x, s);
   q = fminf(fmaxf(q, -qmax), qmax);
   return (int)q + (1 << (bits - 1));
 }
@@ -77,8 +92,8 @@ __device__ __forceinline__ int sym_code(float x, float s, int bits) {
 // codes LSB-first into one 16/32/64-bit store.  blockIdx.y selects keys (0)
 // or values (1).  kivi = 1: code the values of the KIVI blocks that this
 // append completes (tokens [q0, q1), read from the residual ring or the
-// input); else code the new tokens [T0, T0 + L).  max_tok bounds the token
-// count for the grid-stride loop.
+// input); else code the new tokens [T0, T0 + L).  A grid-stride loop over
+// 8-element chunks with 32-bit indices (the host bounds the chunk count).
 // ---------------------------------------------------------------------------
 __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
                                      int final_kernel) {
@@ -96,30 +111,29 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
     TokSrc src = which ? sv : sk;
     src.T0 = T0;
     const int bits = which ? g.vb : g.kb;
-    const int lpg = g.G / 8;                 // lanes per group
-    const int gpw = 32 / lpg;                // groups per warp pass
+    const int lpg = g.G / 8;                 // lanes per group (a power of two)
     const int lane = threadIdx.x & 31;
-    const int sub = lane / lpg, li = lane % lpg;
-    const int groups_per_tok = g.D / g.G;
-    const int64_t ntok = (int64_t)(t_end - t_begin);
-    const int64_t units = (int64_t)g.B * g.H * ntok * groups_per_tok;
+    const int cpt = g.D / 8;                 // 8-element chunks per token (a power of two)
+    const int ntok = t_end - t_begin;
+    const int cpr = ntok * cpt;              // chunks per (b, h) row
+    const int total = g.B * g.H * cpr;       // below 2^31 (checked by the host)
     const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
     const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
     const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
-    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (int64_t base = warp * gpw; base < units; base += nwarps * gpw) {
-      const int64_t u = base + sub;
-      const bool live = u < units;
-      const int64_t uu = live ? u : units - 1;
-      const int grp = (int)(uu % groups_per_tok);
-      int64_t rest = uu / groups_per_tok;
-      const int t = t_begin + (int)(rest % ntok);
-      rest /= ntok;
-      const int h = (int)(rest % g.H);
-      const int b = (int)(rest / g.H);
+    const int stride = gridDim.x * blockDim.x;
+    // chunk i = ((b H + h) ntok + token) cpt + c8; a warp covers 32
+    // consecutive chunks, so a group's lanes are consecutive and aligned
+    for (int i0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < total; i0 += stride) {
+      const int i = i0 + lane;
+      const bool live = i < total;
+      const int ii = live ? i : total - 1;
+      const int row = ii / cpr, rem = ii - row * cpr;
+      const int tt = rem / cpt, c8 = rem & (cpt - 1);
+      const int b = row / g.H, h = row - b * g.H;
+      const int t = t_begin + tt;
+      const int grp = c8 / lpg, li = c8 & (lpg - 1);
       const void* sb;
-      const int64_t e = tok_elem(g, src, b, h, t, &sb) + grp * g.G + li * 8;
+      const int64_t e = tok_elem(g, src, b, h, t, &sb) + c8 * 8;
       float v[8];
       load8(sb, e, g.act, v);
       float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
@@ -145,7 +159,7 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
       }
       if (!live) continue;
       uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
-      const int byte0 = (grp * g.G + li * 8) * bits / 8;
+      const int byte0 = c8 * bits;
       if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
       else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
       else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
@@ -174,36 +188,37 @@ __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
     const int which = blockIdx.y;
     const void* x = which ? v : k;
     const int es = g.act == KVQ_BF16 ? 2 : 4;
-    const int vec_per_tok = g.D * es / 16;
-    const int64_t total = (int64_t)g.B * g.H * L * vec_per_tok;
-    int lo = T0;        // first token that goes to a full-precision plane
-    if (g.fmt == KVQ_FMT_KIVI) lo = max(T0, kivi_tq(T1, g.R, g.G));
-    const int pend_lo = g.S + kvarn_nblocks(T1, g.S, g.G) * g.G;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-      const int vi = (int)(i % vec_per_tok);
-      int64_t rest = i / vec_per_tok;
-      const int t = T0 + (int)(rest % L);
-      rest /= L;
-      const int h = (int)(rest % g.H), b = (int)(rest / g.H);
+    const int vec_per_tok = g.D * es / 16;          // a power of two
+    // the tokens that go to a full-precision plane: [a0, a1) and [c0, c1)
+    int a0 = T0, a1 = T1, c0 = T1, c1 = T1;
+    if (g.fmt == KVQ_FMT_KIVI) {
+      a0 = max(T0, kivi_tq(T1, g.R, g.G));
+    } else if (g.fmt == KVQ_FMT_KVARN) {
+      const int pend_lo = g.S + kvarn_nblocks(T1, g.S, g.G) * g.G;
+      a1 = max(T0, min(T1, g.S));
+      c0 = min(max(T0, pend_lo), T1);
+    }
+    const int na = a1 - a0, n = na + (c1 - c0);
+    const int total = g.B * g.H * n * vec_per_tok;   // below 2^31 (checked by the host)
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+      const int vi = i & (vec_per_tok - 1);
+      const int rest = i / vec_per_tok;
+      const int row = rest / n, j = rest - row * n;
+      const int h = row % g.H, b = row / g.H;
+      const int t = j < na ? a0 + j : c0 + (j - na);
       int plane, slot;
       if (g.fmt == KVQ_FMT_FLOAT) {
         plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
         slot = t;
       } else if (g.fmt == KVQ_FMT_KIVI) {
-        if (t < lo) continue;
         plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
         slot = t % g.ring;
-      } else {  // KVARN
-        if (t < g.S) {
-          plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
-          slot = t;
-        } else if (t >= pend_lo) {
-          plane = which ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
-          slot = (t - g.S) % g.G;
-        } else {
-          continue;
-        }
+      } else if (t < g.S) {                       // KVarN sinks
+        plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+        slot = t;
+      } else {                                    // KVarN staging ring
+        plane = which ? KVQ_PLANE_V_PEND : KVQ_PLANE_K_PEND;
+        slot = (t - g.S) % g.G;
       }
       const uint4* src = reinterpret_cast<const uint4*>(
           reinterpret_cast<const char*>(x) + ((((int64_t)b * g.H + h) * L + (t - T0)) * g.D) * es);
@@ -218,9 +233,13 @@ __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
 
 // ---------------------------------------------------------------------------
 // KIVI keys: one group per (G-token block, channel).  One CTA per block that
-// this append completes (grid sized for the most an append of L can flush).
+// this append completes (grid sized for the most an append of L can flush):
+// the block's G x D keys come in as 8-element vectors (residual ring or
+// input) into shared memory, a thread per channel finds its min / max and
+// codes its G values, and each output word of a token's packed row is
+// gathered from the byte codes and stored whole.
 // ---------------------------------------------------------------------------
-__global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
+__global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ float smem[];
@@ -235,11 +254,16 @@ __global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
   uint8_t* cs = reinterpret_cast<uint8_t*>(xs + G * D); // [G][D]
   const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
   const int t0 = blk * G;
-  for (int i = threadIdx.x; i < G * D; i += blockDim.x) {
-    const int r = i / D, d = i % D;
+  const int cpt = D / 8;
+  for (int i = threadIdx.x; i < G * cpt; i += blockDim.x) {
+    const int r = i / cpt, c8 = i - r * cpt;
     const void* sb;
-    int64_t e = tok_elem(g, src, b, h, t0 + r, &sb);
-    xs[i] = ld_act(sb, e + d, g.act);
+    const int64_t e = tok_elem(g, src, b, h, t0 + r, &sb) + c8 * 8;
+    float v[8];
+    load8(sb, e, g.act, v);
+    float4* dst = reinterpret_cast<float4*>(xs + r * D + c8 * 8);
+    dst[0] = make_float4(v[0], v[1], v[2], v[3]);
+    dst[1] = make_float4(v[4], v[5], v[6], v[7]);
   }
   __syncthreads();
   for (int d = threadIdx.x; d < D; d += blockDim.x) {
@@ -254,12 +278,14 @@ __global__ void kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
     *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
   }
   __syncthreads();
-  const int per = 8 / bits, row_bytes = D * bits / 8;
-  for (int i = threadIdx.x; i < G * row_bytes; i += blockDim.x) {
-    const int r = i / row_bytes, j = i % row_bytes;
-    unsigned byte = 0;
-    for (int e = 0; e < per; ++e) byte |= (unsigned)cs[r * D + j * per + e] << (e * bits);
-    plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r)[j] = (uint8_t)byte;
+  // 32-bit words of packed codes, LSB first: 32 / bits channels per word
+  const int cpw = 32 / bits, wpr = D / cpw;
+  for (int i = threadIdx.x; i < G * wpr; i += blockDim.x) {
+    const int r = i / wpr, w = i - r * wpr;
+    const uint8_t* c = cs + r * D + w * cpw;
+    uint32_t word = 0;
+    for (int e = 0; e < cpw; ++e) word |= (uint32_t)c[e] << (e * bits);
+    reinterpret_cast<uint32_t*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
   }
 }
 
@@ -576,7 +602,7 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       e = cudaFuncSetAttribute(kivi_key_flush_kernel,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
       if (e != cudaSuccess) return e;
-      launch_pdl(kivi_key_flush_kernel, dim3(dim3(max_blocks, g.B * g.H)), dim3(128), sm, s, g, L, sk);
+      launch_pdl(kivi_key_flush_kernel, dim3(dim3(max_blocks, g.B * g.H)), dim3(256), sm, s, g, L, sk);
       const int64_t units = (int64_t)g.B * g.H * max_blocks * g.G * (g.D / g.G);
       const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
       launch_pdl(pack_pertoken_kernel, dim3(dim3(grid_for(threads, 256), 1)), dim3(256), 0, s, g, L, sk, sv, 0, 1, 0);

@@ -7,12 +7,13 @@
 //   * one CTA per SM; the RoPE pair-tiles (8 channels of one head and their
 //     partners D/2 further, 16 weight rows) are cut into contiguous ranges,
 //     one per CTA;
-//   * each tile streams through a ring of shared stages, 16 rows x 1024
-//     input channels per stage, one cp.async.bulk per row issued by its own
-//     lane, and the tile's 16 rows of B_p ride with its last stage; there is
-//     no producer warp: the last warp to finish with a stage (a shared
-//     counter) refills it at once with the stage ns further on;
-//   * the 16 warps hold the rows of X in registers, each warp the same two
+//   * each tile streams through a ring of shared stages as two stages of 8
+//     whole weight rows, each one contiguous cp.async.bulk of 16 d_in bytes
+//     (issuing many small copies costs the issuing warp microseconds), and
+//     the tile's 16 rows of B_p ride with its second stage; there is no
+//     producer warp: the last warp to finish with a stage (a shared counter)
+//     refills it at once with the stage ns further on;
+//   * the 16 warps hold the rows of X in registers, each warp the same
 //     32-channel chunks of every stage, so no shared memory goes to X;
 //     X is the MMA's A operand (tokens as rows), the weight rows are B
 //     operands (n = 8 rows), and within a 32-channel chunk the k index is
@@ -34,10 +35,8 @@ using pdec::rope_cos_sin;
 
 constexpr int kCW = 16;                    // warps (all consume; the last one out refills)
 constexpr int kPThreads = kCW * 32;
-constexpr int kKS = 1024;                  // input channels per stage
-constexpr int kRS = 2 * kKS + 64;          // bytes per staged row: two rows of a
-                                           // quarter-warp fall on different banks
-constexpr int kMaxS = 4;                   // stages per tile (d_in <= 4096)
+constexpr int kMaxK = 4096;                // input channels (X chunks held per warp: kMaxK / 512)
+constexpr int kXC = kMaxK / (32 * kCW);    // 32-channel chunks of X per warp
 constexpr int kMaxNS = 8;                  // ring stages
 constexpr int kSmemMax = 227 * 1024;
 
@@ -46,14 +45,14 @@ struct PSLayout {
   int red, fin, us, ring, total;
 };
 
-PSLayout ps_layout(int M16, int rmax) {
+PSLayout ps_layout(int M16, int K, int rmax) {
   PSLayout L;
   L.rmax = rmax;
   L.red = kMaxNS * 8 + kMaxNS * 4 + 16;                   // mbarriers, counters, flags
   L.fin = L.red + kCW * 2 * 32 * 4 * 4;                    // [warps][2][32 lanes][4]
   L.us = L.fin + 16 * 16 * 4;                              // [16 m][16 n]
   L.ring = (L.us + 3 * M16 * (rmax > 0 ? rmax : 1) * 4 + 127) & ~127;   // U [3][M16][rmax]
-  L.wb = 16 * kRS;                                         // B rows after the weight rows
+  L.wb = 16 * K;                                           // B rows after the 8 weight rows
   L.stage = (L.wb + 32 * rmax + 127) & ~127;
   L.ns = (kSmemMax - L.ring) / L.stage;
   if (L.ns > kMaxNS) L.ns = kMaxNS;
@@ -110,37 +109,35 @@ __device__ __forceinline__ void csync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kCW * 32) : "memory");
 }
 
-// Copies of stage s (tile s / S, input channels from (s % S) * kKS) into its
-// ring slot; called by a whole warp: lane l < 16 copies weight row l, lanes
-// 16 and 17 the two 8-row blocks of B_p with a pair-tile's last stage.
-__device__ void issue_stage(const ProjArgs& a, const PSLayout& L, int s, int S, int plo, int phi,
+// Copies of stage s (tile s / 2, rows 8 (s % 2) .. of it) into its ring slot:
+// lane 0 copies the 8 contiguous weight rows, lanes 1 and 2 the two 8-row
+// blocks of B_p with a pair-tile's second stage.  Called by a whole warp.
+__device__ void issue_stage(const ProjArgs& a, const PSLayout& L, int s, int plo, int phi,
                             int nut, int t0, int tph, uint64_t* full, unsigned char* ring,
                             int lane) {
   const int K = a.d_in, D = a.D, half = D / 2;
-  const int st = s % L.ns, ti = s / S, ch = s - ti * S;
+  const int st = s % L.ns, ti = s >> 1, hf = s & 1;
   const Tile t = tile_at(a, ti, plo, phi, nut, t0, tph);
-  const int k0 = ch * kKS, ks = min(kKS, K - k0);
   const int r = a.r[t.p];
-  const bool bcopy = !t.u && r > 0 && ch == S - 1;
+  const int rows = t.u ? max(0, min(8, r - t.j0 - 8 * hf)) : 8;
+  const bool bcopy = !t.u && r > 0 && hf == 1;
+  unsigned char* sp = ring + (size_t)st * L.stage;
   if (lane == 0) {
     // the slot was last read through the generic proxy; the copies write it
     // through the async proxy
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    dattn::mbar_expect_tx(&full[st], (uint32_t)(t.rows * ks * 2 + (bcopy ? 32 * r : 0)));
+    dattn::mbar_expect_tx(&full[st], (uint32_t)(rows * K * 2 + (bcopy ? 32 * r : 0)));
+    if (rows > 0) {
+      const __nv_bfloat16* src =
+          t.u ? reinterpret_cast<const __nv_bfloat16*>(a.a[t.p]) + (int64_t)(t.j0 + 8 * hf) * K
+              : reinterpret_cast<const __nv_bfloat16*>(a.w) +
+                    ((int64_t)t.hh * D + hf * half + t.c0) * K;
+      dattn::bulk_g2s(sp, src, (uint32_t)(rows * K * 2), &full[st]);
+    }
   }
   __syncwarp();
-  unsigned char* sp = ring + (size_t)st * L.stage;
-  if (lane < t.rows) {
-    const __nv_bfloat16* row;
-    if (t.u) {
-      row = reinterpret_cast<const __nv_bfloat16*>(a.a[t.p]) + (int64_t)(t.j0 + lane) * K;
-    } else {
-      const int c = lane < 8 ? t.c0 + lane : half + t.c0 + lane - 8;
-      row = reinterpret_cast<const __nv_bfloat16*>(a.w) + ((int64_t)t.hh * D + c) * K;
-    }
-    dattn::bulk_g2s(sp + lane * kRS, row + k0, (uint32_t)ks * 2, &full[st]);
-  } else if (bcopy && lane >= 16 && lane < 18) {
-    const int j = lane - 16;
+  if (bcopy && (lane == 1 || lane == 2)) {
+    const int j = lane - 1;
     const __nv_bfloat16* Bm = reinterpret_cast<const __nv_bfloat16*>(a.bm[t.p]);
     const int c = j == 0 ? t.c0 : half + t.c0;
     dattn::bulk_g2s(sp + L.wb + j * 16 * r, Bm + ((int64_t)t.head * D + c) * r,
@@ -171,8 +168,7 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
   int nut = 0;
   for (int q = plo; q <= phi; ++q) nut += (a.r[q] + 15) >> 4;
   const int ntl = nut + (t1 - t0);
-  const int S = (K + kKS - 1) / kKS;
-  const int nst = ntl * S;
+  const int nst = 2 * ntl;                                 // two 8-row stages per tile
   const int ns = L.ns;
 
   uint32_t* cnt = reinterpret_cast<uint32_t*>(full + kMaxNS);   // warps done per slot
@@ -189,7 +185,7 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
   __syncthreads();
   pdl_wait();
   pdl_trigger();
-  if (warp < min(ns, nst)) issue_stage(a, L, warp, S, plo, phi, nut, t0, tph, full, ring, lane);
+  if (warp < min(ns, nst)) issue_stage(a, L, warp, plo, phi, nut, t0, tph, full, ring, lane);
 
   // ---------------------------------------------------------------- consumers
   // a warp done with stage s counts itself out of the slot; the last one
@@ -208,24 +204,23 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
         cnt[s % ns] = 0;
         if (s + ns < nst) atomicMax(&flags[1], s + ns + 1);
       }
-      if (s + ns < nst) issue_stage(a, L, s + ns, S, plo, phi, nut, t0, tph, full, ring, lane);
+      if (s + ns < nst) issue_stage(a, L, s + ns, plo, phi, nut, t0, tph, full, ring, lane);
     }
   };
   const int gid = lane >> 2, tid = lane & 3, tc = threadIdx.x;
   const int M = a.B * a.L;
   const __nv_bfloat16* x = reinterpret_cast<const __nv_bfloat16*>(a.x);
-  // this warp's chunks of X: stage c, chunk warp + 16 h, channels 8 tid .. 8 tid + 7
-  uint4 xa[kMaxS][2], xb[kMaxS][2];
+  // this warp's chunks of X: chunk warp + 16 h, channels 8 tid .. 8 tid + 7
+  const int nch = K / 32;
+  uint4 xa[kXC], xb[kXC];
 #pragma unroll
-  for (int c = 0; c < kMaxS; ++c)
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int k = c * kKS + (warp + 16 * h) * 32 + 8 * tid;
-      xa[c][h] = xb[c][h] = make_uint4(0, 0, 0, 0);
-      if (k < K && gid < M) xa[c][h] = __ldg(reinterpret_cast<const uint4*>(x + (int64_t)gid * K + k));
-      if (M16 == 16 && k < K && gid + 8 < M)
-        xb[c][h] = __ldg(reinterpret_cast<const uint4*>(x + (int64_t)(gid + 8) * K + k));
-    }
+  for (int h = 0; h < kXC; ++h) {
+    const int k = (warp + 16 * h) * 32 + 8 * tid;
+    xa[h] = xb[h] = make_uint4(0, 0, 0, 0);
+    if (k < K && gid < M) xa[h] = __ldg(reinterpret_cast<const uint4*>(x + (int64_t)gid * K + k));
+    if (M16 == 16 && k < K && gid + 8 < M)
+      xb[h] = __ldg(reinterpret_cast<const uint4*>(x + (int64_t)(gid + 8) * K + k));
+  }
   const int pos_base = a.pos0 + (a.pos_dev ? *a.pos_dev : 0);
   float acc[2][4];
 #pragma unroll
@@ -236,9 +231,9 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
     const Tile t = tile_at(a, ti, plo, phi, nut, t0, tph);
     int st = 0;
 #pragma unroll
-    for (int c = 0; c < kMaxS; ++c) {
-      if (c < S) {
-        const int s = ti * S + c;
+    for (int hf = 0; hf < 2; ++hf) {        // weight rows 0..7, then 8..15
+      {
+        const int s = 2 * ti + hf;
         st = s % ns;
         if (!bad) {
           bool ok = true;
@@ -249,22 +244,20 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
           }
         }
         if (!bad) {
-          const unsigned char* sp = ring + (size_t)st * L.stage;
-          const int nch = min(kKS, K - c * kKS) / 32;
+          // rows are 2 K bytes apart: a quarter-warp's two rows share banks
+          // (two-way), which the idle consumers absorb
+          const unsigned char* sp = ring + (size_t)st * L.stage + gid * (2 * K) + 16 * tid;
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
+          for (int h = 0; h < kXC; ++h) {
             const int j = warp + 16 * h;
             if (j < nch) {
-              const uint4 w0 = lds128(sp + gid * kRS + j * 64 + 16 * tid);
-              const uint4 w1 = lds128(sp + (8 + gid) * kRS + j * 64 + 16 * tid);
-              const uint4 p = xa[c][h], q = xb[c][h];
-              pdec::mma16816_p(acc[0], p.x, q.x, p.y, q.y, w0.x, w0.y);
-              pdec::mma16816_p(acc[0], p.z, q.z, p.w, q.w, w0.z, w0.w);
-              pdec::mma16816_p(acc[1], p.x, q.x, p.y, q.y, w1.x, w1.y);
-              pdec::mma16816_p(acc[1], p.z, q.z, p.w, q.w, w1.z, w1.w);
+              const uint4 w = lds128(sp + j * 64);
+              const uint4 p = xa[h], q = xb[h];
+              pdec::mma16816_p(acc[hf], p.x, q.x, p.y, q.y, w.x, w.y);
+              pdec::mma16816_p(acc[hf], p.z, q.z, p.w, q.w, w.z, w.w);
             }
           }
-          if (c < S - 1) release(s);
+          if (hf == 0) release(s);
         }
       }
     }
@@ -331,7 +324,7 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
       }
     }
     // the tile's last stage (its B rows were read above) goes back to the ring
-    if (!bad) release(ti * S + S - 1);
+    if (!bad) release(2 * ti + 1);
   }
   // after a timeout, keep the CTA alive until the copies it started have landed
   if (bad && lane == 0) atomicOr(&flags[0], 1);
@@ -358,12 +351,12 @@ cudaError_t launch_ps(const ProjArgs& p, const PSLayout& L, int* err, cudaStream
 
 cudaError_t launch_project_decode_stream(const ProjArgs& p, int* err, cudaStream_t s) {
   const int M = p.B * p.L;
-  if (M < 1 || M > 16 || p.d_in % 64 || p.d_in > kMaxS * kKS) return cudaErrorNotSupported;
+  if (M < 1 || M > 16 || p.d_in % 64 || p.d_in > kMaxK) return cudaErrorNotSupported;
   int rmax = 0;
   for (int i = 0; i < 3; ++i) rmax = max(rmax, p.r[i]);
   if (rmax > 64) return cudaErrorNotSupported;
-  const PSLayout L = ps_layout(M <= 8 ? 8 : 16, rmax);
-  if (L.ns < 3) return cudaErrorNotSupported;
+  const PSLayout L = ps_layout(M <= 8 ? 8 : 16, p.d_in, rmax);
+  if (L.ns < 2) return cudaErrorNotSupported;
   return M <= 8 ? launch_ps<8>(p, L, err, s) : launch_ps<16>(p, L, err, s);
 }
 

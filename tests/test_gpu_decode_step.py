@@ -141,4 +141,5 @@ def test_decode_step_capacity_refused():
     after = c.planes()
     for k, v in before.items():
         if k != "workspace":
-            assert torch.equal(v, after[k]), k
+            assert torch.equal(v.contiguous().view(torch.uint8),
+                               after[k].contiguous().view(torch.uint8)), k

@@ -99,4 +99,7 @@ def test_captured_decode_step_replays(fmt_name):
     after = cache.planes()
     for n, t in before.items():
         if n != "workspace":
-            assert torch.equal(t, after[n]), n
+            # bit patterns: rows past the stored tokens hold whatever the
+            # allocator left there, NaN included
+            assert torch.equal(t.contiguous().view(torch.uint8),
+                               after[n].contiguous().view(torch.uint8)), n

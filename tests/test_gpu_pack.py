@@ -63,6 +63,12 @@ def test_pack_edge_values(name):
     k[:, :, 2, :32] = np.arange(32) * 0.5     # grid with ties
     k[:, :, 3] *= 3000.0                      # large values (fp16-safe scales)
     k[:, :, 4, :32] = 1e-30                   # tiny values: s floors at 1e-8
+    # quotients exactly on a half-integer (scale 1): ties to even, for 4-bit
+    # affine (0 .. 15), 2-bit affine (0 .. 3) and 4-bit symmetric (-7 .. 7)
+    k[:, :, 5, :32] = np.concatenate([[0.0, 15.0], np.arange(15) + 0.5, np.arange(15) + 0.25])
+    k[:, :, 6, :32] = np.concatenate([[0.0, 3.0], np.tile([0.5, 1.5, 2.5], 10)])
+    k[:, :, 7, :32] = np.concatenate([[-7.0, 7.0, 0.0, 0.0], np.arange(-7, 7) + 0.5,
+                                      np.arange(-7, 7) + 0.5])
     v = k[:, :, ::-1].copy()
     kt = torch.from_numpy(k).to(torch.bfloat16)
     vt = torch.from_numpy(v).to(torch.bfloat16)
