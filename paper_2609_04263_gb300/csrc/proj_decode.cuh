@@ -194,9 +194,4 @@ __host__ __device__ inline size_t proj_decode_smem_bytes(int M16, int NT, int d_
 }
 
 }  // namespace pdec
-
-// The weight-streaming decode projection (proj_stream.cu); cudaErrorNotSupported
-// when the shape is outside its range (M > 16, d_in > 4096, rank > 64).
-cudaError_t launch_project_decode_stream(const pdec::ProjArgs& p, int* err, cudaStream_t s);
-
 }  // namespace kvq

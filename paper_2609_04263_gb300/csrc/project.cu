@@ -6,6 +6,12 @@
 #include "proj_decode.cuh"
 
 namespace kvq {
+// The weight-streaming decode projection (proj_stream.cu); cudaErrorNotSupported
+// when the shape is outside its range (M > 16, d_in > 4096, rank > 64).
+cudaError_t launch_project_decode_stream(const pdec::ProjArgs& p, int* err, cudaStream_t s);
+}  // namespace kvq
+
+namespace kvq {
 namespace {
 using namespace pdec;
 
