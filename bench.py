@@ -578,6 +578,8 @@ def main():
     # smaller runs for profiler launch lists (not for reported numbers)
     ap.add_argument("--decode-steps", type=int, default=None,
                     help="decode steps per job (default: the workload's)")
+    ap.add_argument("--prefill", type=int, default=None,
+                    help="prefill tokens per sequence (default: the workload's)")
     ap.add_argument("--layers", type=int, default=None,
                     help="attention layers (default: the workload's)")
     ap.add_argument("--eager-decode", action="store_true",
@@ -605,6 +607,8 @@ def main():
         wl = dataclasses.replace(wl, decode=args.decode_steps)
     if args.layers is not None:
         wl = dataclasses.replace(wl, layers=args.layers)
+    if args.prefill is not None:
+        wl = dataclasses.replace(wl, prefill=args.prefill)
     peaks, peak_kind = load_peaks()
     run = Runner(wl, device)
     run.eager = args.eager_decode

@@ -353,6 +353,9 @@ kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L
   if ((int64_t)cache->T + L > cache->g.Tmax)
     return fail(KVQ_ERR_CAPACITY, "append of %d tokens to %d exceeds max_tokens %d", L,
                 cache->T, cache->g.Tmax);
+  if ((int64_t)cache->g.B * cache->g.H > 65535)
+    return fail(KVQ_ERR_SHAPE, "batch x kv heads = %d above 65535",
+                cache->g.B * cache->g.H);
   if ((int64_t)cache->g.B * cache->g.H * ((int64_t)L + cache->g.G) * (cache->g.D / 4) >=
       ((int64_t)1 << 31))
     return fail(KVQ_ERR_SHAPE, "append of %d tokens too large for one call: append it in chunks", L);

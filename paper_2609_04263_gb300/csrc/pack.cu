@@ -54,22 +54,23 @@ __device__ __forceinline__ float affine_scale(float mn, float mx, int bits) {
   return fmaxf(__fdiv_rn(__fsub_rn(mx, mn), (float)((1 << bits) - 1)), 1e-8f);
 }
 // rint(a / s) where the quotient is first rounded to fp32 (both roundings to
-// nearest even), which is how the cache format defines a code.  __fdividef is
-// within 2 ulp of a / s for s in the normal range; when its result q lies
+// nearest even), which is how the cache format defines a code.  inv is the
+// correctly rounded reciprocal of s (one per group), so q = RN(a inv) is
+// within 2^-23 |a / s| of a / s, below 2^-17 for |q| < 64.  When q lies
 // farther than 2^-14 from the half-integer between its two neighbouring
-// integers (and |q| < 64, where 2 ulp < 2^-17), the exact quotient and its
-// fp32 rounding lie on the same side of that representable half-integer
-// (rounding is monotone), so all three round to the same integer.  Otherwise
-// (near a tie, or NaN / out of range) the IEEE quotient is formed.
-__device__ __forceinline__ float rint_quot(float a, float s) {
-  const float q = __fdividef(a, s);
+// integers, the exact quotient and its fp32 rounding lie on the same side of
+// that representable half-integer (rounding is monotone), so all three round
+// to the same integer.  Otherwise (near a tie, or NaN / out of range) the IEEE
+// quotient is formed.
+__device__ __forceinline__ float rint_quot(float a, float s, float inv) {
+  const float q = __fmul_rn(a, inv);
   const float d = fabsf(q - (floorf(q) + 0.5f));
   if (d > 0x1p-14f && fabsf(q) < 64.f) return rintf(q);
   return rintf(__fdiv_rn(a, s));
 }
 
-__device__ __forceinline__ int affine_code(float x, float mn, float s, int bits) {
-  float c = rint_quot(__fsub_rn(x, mn), s);
+__device__ __forceinline__ int affine_code(float x, float mn, float s, float inv, int bits) {
+  float c = rint_quot(__fsub_rn(x, mn), s, inv);
   c = fminf(fmaxf(c, 0.f), (float)((1 << bits) - 1));
   return (int)c;
 }
@@ -78,11 +79,60 @@ __device__ __forceinline__ int affine_code(float x, float mn, float s, int bits)
 __device__ __forceinline__ float sym_scale(float amax, int bits) {
   return fmaxf(__fdiv_rn(amax, (float)((1 << (bits - 1)) - 1)), 1e-8f);
 }
-__device__ __forceinline__ int sym_code(float x, float s, int bits) {
+__device__ __forceinline__ int sym_code(float x, float s, float inv, int bits) {
   const float qmax = (float)((1 << (bits - 1)) - 1);
-  float q = rint_quot(x, s);
+  float q = rint_quot(x, s, inv);
   q = fminf(fmaxf(q, -qmax), qmax);
   return (int)q + (1 << (bits - 1));
+}
+
+// The 8 codes of one lane, LSB first (8 x BITS bits).
+template <int BITS, bool SYM>
+__device__ __forceinline__ uint64_t code8(const float v[8], float lo, float hi, float* s_out) {
+  const float s = SYM ? sym_scale(hi, BITS) : affine_scale(lo, hi, BITS);
+  const float inv = __frcp_rn(s);
+  *s_out = s;
+  if (BITS <= 4) {
+    uint32_t w = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      w |= (uint32_t)(SYM ? sym_code(v[i], s, inv, BITS) : affine_code(v[i], lo, s, inv, BITS))
+           << (i * BITS);
+    return w;
+  }
+  uint64_t w = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    w |= (uint64_t)(SYM ? sym_code(v[i], s, inv, BITS) : affine_code(v[i], lo, s, inv, BITS))
+         << (i * BITS);
+  return w;
+}
+
+// append_arrive with the arrivals spread over 32 counters (words 16..47 of
+// the state's padding): the CTAs of bucket id % 32 count themselves, the last
+// of each bucket counts the bucket, and the last bucket advances the token
+// count, so thousands of CTAs do not queue on one address.
+__device__ __forceinline__ void append_arrive_spread(CacheState* st, int T0, int L, bool ok) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    constexpr unsigned kBuckets = 32;
+    const unsigned total = gridDim.x * gridDim.y * gridDim.z;
+    const unsigned id = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
+    const unsigned nb = total < kBuckets ? total : kBuckets;
+    const unsigned b = id % nb;
+    const unsigned members = total / nb + (b < total % nb ? 1u : 0u);
+    unsigned* bucket = reinterpret_cast<unsigned*>(&st->pad[16 + b]);
+    if (atomicAdd(bucket, 1u) == members - 1) {
+      *bucket = 0;
+      __threadfence();
+      if (atomicAdd(&st->done, 1u) == nb - 1) {
+        if (ok) st->tokens = T0 + L;
+        st->done = 0;
+        __threadfence();
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -96,12 +146,12 @@ __device__ __forceinline__ int sym_code(float x, float s, int bits) {
 // 8-element chunks with 32-bit indices (the host bounds the chunk count).
 // ---------------------------------------------------------------------------
 __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
-                                     int final_kernel) {
+                                     int final_kernel, int lcpt, int llpg) {
   pdl_wait();
   pdl_trigger();
   bool ok;
   const int T0 = append_begin(g, L, &ok);
-  const int which = kivi ? 1 : blockIdx.y;
+  const int which = kivi ? 1 : blockIdx.z;
   int t_begin = T0, t_end = T0 + L;
   if (kivi) {
     t_begin = kivi_tq(T0, g.R, g.G);
@@ -111,27 +161,24 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
     TokSrc src = which ? sv : sk;
     src.T0 = T0;
     const int bits = which ? g.vb : g.kb;
-    const int lpg = g.G / 8;                 // lanes per group (a power of two)
     const int lane = threadIdx.x & 31;
-    const int cpt = g.D / 8;                 // 8-element chunks per token (a power of two)
+    const int cpt = 1 << lcpt;               // 8-element chunks per token (D / 8)
     const int ntok = t_end - t_begin;
-    const int cpr = ntok * cpt;              // chunks per (b, h) row
-    const int total = g.B * g.H * cpr;       // below 2^31 (checked by the host)
+    const int total = ntok << lcpt;          // chunks of this (b, h) row
+    const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
     const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
     const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
     const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
     const int stride = gridDim.x * blockDim.x;
-    // chunk i = ((b H + h) ntok + token) cpt + c8; a warp covers 32
-    // consecutive chunks, so a group's lanes are consecutive and aligned
+    // blockIdx.y is the (b, h) row; chunk i = token * cpt + c8 of it.  A warp
+    // covers 32 consecutive chunks, so a group's G/8 lanes are consecutive
+    // and aligned
     for (int i0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < total; i0 += stride) {
       const int i = i0 + lane;
       const bool live = i < total;
       const int ii = live ? i : total - 1;
-      const int row = ii / cpr, rem = ii - row * cpr;
-      const int tt = rem / cpt, c8 = rem & (cpt - 1);
-      const int b = row / g.H, h = row - b * g.H;
-      const int t = t_begin + tt;
-      const int grp = c8 / lpg, li = c8 & (lpg - 1);
+      const int t = t_begin + (ii >> lcpt), c8 = ii & (cpt - 1);
+      const int grp = c8 >> llpg, li = c8 & ((1 << llpg) - 1);
       const void* sb;
       const int64_t e = tok_elem(g, src, b, h, t, &sb) + c8 * 8;
       float v[8];
@@ -142,20 +189,18 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
         if (sym) hi = fmaxf(hi, fabsf(v[i]));
         else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
       }
-      for (int off = lpg / 2; off > 0; off >>= 1) {
+      for (int off = (1 << llpg) >> 1; off > 0; off >>= 1) {
         lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
         hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
       }
       float s;
-      uint64_t word = 0;
+      uint64_t word;
       if (sym) {
-        s = sym_scale(hi, bits);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) word |= (uint64_t)sym_code(v[i], s, bits) << (i * bits);
+        word = bits == 2 ? code8<2, true>(v, lo, hi, &s)
+             : bits == 4 ? code8<4, true>(v, lo, hi, &s) : code8<8, true>(v, lo, hi, &s);
       } else {
-        s = affine_scale(lo, hi, bits);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) word |= (uint64_t)affine_code(v[i], lo, s, bits) << (i * bits);
+        word = bits == 2 ? code8<2, false>(v, lo, hi, &s)
+             : bits == 4 ? code8<4, false>(v, lo, hi, &s) : code8<8, false>(v, lo, hi, &s);
       }
       if (!live) continue;
       uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
@@ -169,7 +214,7 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
       }
     }
   }
-  if (final_kernel) append_arrive(g.state, T0, L, ok);
+  if (final_kernel) append_arrive_spread(g.state, T0, L, ok);
 }
 
 // ---------------------------------------------------------------------------
@@ -228,7 +273,7 @@ __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
       dst[vi] = src[vi];
     }
   }
-  append_arrive(g.state, T0, L, ok);
+  append_arrive_spread(g.state, T0, L, ok);
 }
 
 // ---------------------------------------------------------------------------
@@ -272,8 +317,9 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
       mn = fminf(mn, xs[r * D + d]);
       mx = fmaxf(mx, xs[r * D + d]);
     }
-    const float s = affine_scale(mn, mx, bits);
-    for (int r = 0; r < G; ++r) cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, bits);
+    const float s = affine_scale(mn, mx, bits), inv = __frcp_rn(s);
+    for (int r = 0; r < G; ++r)
+      cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, inv, bits);
     *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
     *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
   }
@@ -391,8 +437,9 @@ __global__ void kvarn_block_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float in
     const float* row = y + r * D + gq * G;
     float mn = row[0], mx = row[0];
     for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
-    const float sc = affine_scale(mn, mx, bits);
-    for (int j = 0; j < G; ++j) cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, bits);
+    const float sc = affine_scale(mn, mx, bits), inv = __frcp_rn(sc);
+    for (int j = 0; j < G; ++j)
+      cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
     *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
     *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
   }
@@ -524,8 +571,9 @@ kvarn_block_fast_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
     const float* row = y + r * D + gq * G;
     float mn = row[0], mx = row[0];
     for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
-    const float sc = affine_scale(mn, mx, bits);
-    for (int j = 0; j < G; ++j) cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, bits);
+    const float sc = affine_scale(mn, mx, bits), inv = __frcp_rn(sc);
+    for (int j = 0; j < G; ++j)
+      cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
     *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
     *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
   }
@@ -568,6 +616,23 @@ cudaError_t launch_kvarn_blocks(const Geom& g, int max_blocks, int L, const TokS
   return cudaErrorNotSupported;
 }
 
+// Grid of the per-token coder: (chunk blocks of a row, B H rows, keys |
+// values), x capped so the whole grid stays within 8 CTAs per SM.
+dim3 pertoken_grid(const Geom& g, int ntok_max, int which_count) {
+  const int64_t chunks = (int64_t)ntok_max * (g.D / 8);
+  int64_t gx = (chunks + 255) / 256;
+  const int64_t cap = (int64_t)num_sms() * 8 / ((int64_t)g.B * g.H * which_count);
+  if (gx > cap) gx = cap;
+  if (gx < 1) gx = 1;
+  return dim3((unsigned)gx, (unsigned)(g.B * g.H), (unsigned)which_count);
+}
+
+int ilog2(int x) {
+  int l = 0;
+  while ((1 << (l + 1)) <= x) ++l;
+  return l;
+}
+
 int grid_for(int64_t threads_needed, int block) {
   int64_t n = (threads_needed + block - 1) / block;
   int64_t cap = (int64_t)num_sms() * 8;
@@ -590,9 +655,8 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
     case KVQ_FMT_AFFINE:
     case KVQ_FMT_SYMMETRIC: {
       const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
-      const int64_t units = (int64_t)g.B * g.H * L * (g.D / g.G);
-      const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
-      launch_pdl(pack_pertoken_kernel, dim3(dim3(grid_for(threads, 256), 2)), dim3(256), 0, s, g, L, sk, sv, sym, 0, 1);
+      launch_pdl(pack_pertoken_kernel, pertoken_grid(g, L, 2), dim3(256), 0, s, g, L, sk, sv, sym,
+                 0, 1, ilog2(g.D / 8), ilog2(g.G / 8));
       return cudaGetLastError();
     }
     case KVQ_FMT_KIVI: {
@@ -603,9 +667,8 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
       if (e != cudaSuccess) return e;
       launch_pdl(kivi_key_flush_kernel, dim3(dim3(max_blocks, g.B * g.H)), dim3(256), sm, s, g, L, sk);
-      const int64_t units = (int64_t)g.B * g.H * max_blocks * g.G * (g.D / g.G);
-      const int64_t threads = (units + (32 / (g.G / 8)) - 1) / (32 / (g.G / 8)) * 32;
-      launch_pdl(pack_pertoken_kernel, dim3(dim3(grid_for(threads, 256), 1)), dim3(256), 0, s, g, L, sk, sv, 0, 1, 0);
+      launch_pdl(pack_pertoken_kernel, pertoken_grid(g, max_blocks * g.G, 1), dim3(256), 0, s, g,
+                 L, sk, sv, 0, 1, 0, ilog2(g.D / 8), ilog2(g.G / 8));
       launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     }

@@ -19,6 +19,8 @@ FORMATS = {
     "affine4_g128": dict(fmt=O.FMT_AFFINE, key_bits=4, value_bits=2, group_size=128),
     "sym2": dict(fmt=O.FMT_SYMMETRIC, key_bits=2, value_bits=2, group_size=32),
     "sym4": dict(fmt=O.FMT_SYMMETRIC, key_bits=4, value_bits=4, group_size=32),
+    "sym4_g8": dict(fmt=O.FMT_SYMMETRIC, key_bits=4, value_bits=8, group_size=8),
+    "affine2_g16": dict(fmt=O.FMT_AFFINE, key_bits=2, value_bits=4, group_size=16),
     "kivi2": dict(fmt=O.FMT_KIVI, key_bits=2, value_bits=2, group_size=32,
                   residual_tokens=128),
     "kivi_r0": dict(fmt=O.FMT_KIVI, key_bits=2, value_bits=4, group_size=32,

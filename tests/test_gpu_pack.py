@@ -24,6 +24,9 @@ CASES = [
     ("affine4_g128", "bf16", 1, 2, 256, [150, 3]),
     ("sym2", "bf16", 2, 2, 64, [256, 3]),
     ("sym4", "f32", 1, 4, 64, [100, 1, 1]),
+    # the smallest groups: one and two lanes per group
+    ("sym4_g8", "bf16", 2, 3, 64, [90, 1, 17]),
+    ("affine2_g16", "bf16", 1, 2, 128, [65, 2]),
     ("float", "bf16", 2, 2, 64, [50, 13]),
     ("float", "f32", 1, 2, 128, [9, 1]),
     ("kivi2", "bf16", 2, 2, 128, [300, 1, 1, 40, 33]),
