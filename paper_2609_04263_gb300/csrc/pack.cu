@@ -68,6 +68,18 @@ __device__ __forceinline__ float rint_quot(float a, float s, float inv) {
   if (d > 0x1p-14f && fabsf(q) < 64.f) return rintf(q);
   return rintf(__fdiv_rn(a, s));
 }
+// The fast half of rint_quot without a branch: ok is cleared when the
+// caller must form the IEEE quotient instead (loops then redo their
+// elements once, exactly, when any was near a tie).
+__device__ __forceinline__ float rint_quot_fast(float a, float inv, bool& ok) {
+  const float q = __fmul_rn(a, inv);
+  const float d = fabsf(q - (floorf(q) + 0.5f));
+  ok = ok && d > 0x1p-14f && fabsf(q) < 64.f;
+  return rintf(q);
+}
+__device__ __forceinline__ int clamp_code(float c, int bits) {
+  return (int)fminf(fmaxf(c, 0.f), (float)((1 << bits) - 1));
+}
 
 __device__ __forceinline__ int affine_code(float x, float mn, float s, float inv, int bits) {
   float c = rint_quot(__fsub_rn(x, mn), s, inv);
@@ -79,12 +91,6 @@ __device__ __forceinline__ int affine_code(float x, float mn, float s, float inv
 __device__ __forceinline__ float sym_scale(float amax, int bits) {
   return fmaxf(__fdiv_rn(amax, (float)((1 << (bits - 1)) - 1)), 1e-8f);
 }
-__device__ __forceinline__ int sym_code(float x, float s, float inv, int bits) {
-  const float qmax = (float)((1 << (bits - 1)) - 1);
-  float q = rint_quot(x, s, inv);
-  q = fminf(fmaxf(q, -qmax), qmax);
-  return (int)q + (1 << (bits - 1));
-}
 
 // The 8 codes of one lane, LSB first (8 x BITS bits).
 template <int BITS, bool SYM>
@@ -92,19 +98,26 @@ __device__ __forceinline__ uint64_t code8(const float v[8], float lo, float hi, 
   const float s = SYM ? sym_scale(hi, BITS) : affine_scale(lo, hi, BITS);
   const float inv = __frcp_rn(s);
   *s_out = s;
-  if (BITS <= 4) {
-    uint32_t w = 0;
+  constexpr int half = 1 << (BITS - 1);
+  bool ok = true;
+  float c[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
-      w |= (uint32_t)(SYM ? sym_code(v[i], s, inv, BITS) : affine_code(v[i], lo, s, inv, BITS))
-           << (i * BITS);
-    return w;
+  for (int i = 0; i < 8; ++i) {
+    const float a = SYM ? v[i] : __fsub_rn(v[i], lo);
+    c[i] = rint_quot_fast(a, inv, ok);
+  }
+  if (!ok) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) c[i] = rintf(__fdiv_rn(SYM ? v[i] : __fsub_rn(v[i], lo), s));
   }
   uint64_t w = 0;
 #pragma unroll
-  for (int i = 0; i < 8; ++i)
-    w |= (uint64_t)(SYM ? sym_code(v[i], s, inv, BITS) : affine_code(v[i], lo, s, inv, BITS))
-         << (i * BITS);
+  for (int i = 0; i < 8; ++i) {
+    // the clamps of sym_code / affine_code
+    const int code = SYM ? (int)fminf(fmaxf(c[i], (float)(1 - half)), (float)(half - 1)) + half
+                         : clamp_code(c[i], BITS);
+    w |= (uint64_t)code << (i * BITS);
+  }
   return w;
 }
 
@@ -311,26 +324,160 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
     dst[1] = make_float4(v[4], v[5], v[6], v[7]);
   }
   __syncthreads();
-  for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    float mn = xs[d], mx = xs[d];
-    for (int r = 1; r < G; ++r) {
+  // parts threads per channel, each over G / parts tokens: partial min / max,
+  // then every part codes its tokens with the channel's scale
+  const int parts = (int)blockDim.x >= D ? (int)blockDim.x / D : 1;
+  float* pmn = reinterpret_cast<float*>(cs + G * D);     // [parts][D]
+  float* pmx = pmn + parts * D;
+  for (int t = threadIdx.x; t < D * parts; t += blockDim.x) {
+    const int d = t % D, part = t / D;
+    const int r0 = part * G / parts, r1 = (part + 1) * G / parts;
+    float mn = xs[r0 * D + d], mx = mn;
+    for (int r = r0 + 1; r < r1; ++r) {
       mn = fminf(mn, xs[r * D + d]);
       mx = fmaxf(mx, xs[r * D + d]);
     }
-    const float s = affine_scale(mn, mx, bits), inv = __frcp_rn(s);
-    for (int r = 0; r < G; ++r)
-      cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, inv, bits);
-    *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
-    *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+    pmn[t] = mn;
+    pmx[t] = mx;
   }
   __syncthreads();
-  // 32-bit words of packed codes, LSB first: 32 / bits channels per word
+  for (int t = threadIdx.x; t < D * parts; t += blockDim.x) {
+    const int d = t % D, part = t / D;
+    const int r0 = part * G / parts, r1 = (part + 1) * G / parts;
+    float mn = pmn[d], mx = pmx[d];
+    for (int p = 1; p < parts; ++p) {
+      mn = fminf(mn, pmn[p * D + d]);
+      mx = fmaxf(mx, pmx[p * D + d]);
+    }
+    const float s = affine_scale(mn, mx, bits), inv = __frcp_rn(s);
+    bool ok = true;
+    for (int r = r0; r < r1; ++r)
+      cs[r * D + d] = (uint8_t)clamp_code(rint_quot_fast(__fsub_rn(xs[r * D + d], mn), inv, ok), bits);
+    if (!ok)                                   // a quotient near a tie: all of them exactly
+      for (int r = r0; r < r1; ++r)
+        cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, inv, bits);
+    if (part == 0) {
+      *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
+      *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+    }
+  }
+  __syncthreads();
+  // 32-bit words of packed codes, LSB first: 32 / bits channels per word,
+  // gathered from the byte codes with word loads and shifts
   const int cpw = 32 / bits, wpr = D / cpw;
   for (int i = threadIdx.x; i < G * wpr; i += blockDim.x) {
     const int r = i / wpr, w = i - r * wpr;
     const uint8_t* c = cs + r * D + w * cpw;
-    uint32_t word = 0;
-    for (int e = 0; e < cpw; ++e) word |= (uint32_t)c[e] << (e * bits);
+    uint32_t word;
+    if (bits == 8) {
+      word = *reinterpret_cast<const uint32_t*>(c);
+    } else if (bits == 4) {                  // 4 bytes b0..b3 < 16 -> b0 | b1 << 4 | ...
+      const uint2 u = *reinterpret_cast<const uint2*>(c);
+      const uint32_t lo = u.x | (u.x >> 4), hi = u.y | (u.y >> 4);
+      word = (lo & 0xFFu) | ((lo >> 8) & 0xFF00u) | ((hi & 0xFFu) << 16) | ((hi >> 8) & 0xFF00u) << 16;
+    } else {                                 // 4 bytes b0..b3 < 4 -> b0 | b1 << 2 | ...
+      const uint4 u = *reinterpret_cast<const uint4*>(c);
+      auto crumbs = [](uint32_t q) {
+        uint32_t t = q | (q >> 6);
+        return (t | (t >> 12)) & 0xFFu;
+      };
+      word = crumbs(u.x) | crumbs(u.y) << 8 | crumbs(u.z) << 16 | crumbs(u.w) << 24;
+    }
+    reinterpret_cast<uint32_t*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
+  }
+}
+
+// The same flush for 32-token blocks with D and the bit width fixed at
+// compile time (the KIVI configuration): 256 threads, 256 / D of them per
+// channel over 32 D / 256 tokens each; codes go to shared memory as bytes and
+// leave as whole packed words.  Same arithmetic as kivi_key_flush_kernel.
+template <int D, int BITS>
+__global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, TokSrc src) {
+  constexpr int G = 32, NT = 256, CPT = D / 8, PARTS = NT / D, TPP = G / PARTS;
+  constexpr int CPW = 32 / BITS, WPR = D / CPW;
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ float smem[];
+  bool ok;
+  const int T0 = append_begin(g, L, &ok);
+  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + L, g.R, G);
+  const int blk = q0 / G + blockIdx.x;
+  if (!ok || blk >= q1 / G) return;
+  src.T0 = T0;
+  float* xs = smem;                                      // [G][D]
+  uint8_t* cs = reinterpret_cast<uint8_t*>(xs + G * D);  // [G][D]
+  float* pmn = reinterpret_cast<float*>(cs + G * D);     // [PARTS][D]
+  float* pmx = pmn + PARTS * D;
+  const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
+  const int t0 = blk * G;
+#pragma unroll
+  for (int k = 0; k < G * CPT / NT; ++k) {
+    const int i = threadIdx.x + k * NT;
+    const int r = i / CPT, c8 = i % CPT;
+    const void* sb;
+    const int64_t e = tok_elem(g, src, b, h, t0 + r, &sb) + c8 * 8;
+    float v[8];
+    load8(sb, e, g.act, v);
+    float4* dst = reinterpret_cast<float4*>(xs + r * D + c8 * 8);
+    dst[0] = make_float4(v[0], v[1], v[2], v[3]);
+    dst[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
+  __syncthreads();
+  const int d = threadIdx.x % D, part = threadIdx.x / D, r0 = part * TPP;
+  float x[TPP];
+  float mn, mx;
+#pragma unroll
+  for (int j = 0; j < TPP; ++j) x[j] = xs[(r0 + j) * D + d];
+  mn = mx = x[0];
+#pragma unroll
+  for (int j = 1; j < TPP; ++j) {
+    mn = fminf(mn, x[j]);
+    mx = fmaxf(mx, x[j]);
+  }
+  pmn[threadIdx.x] = mn;
+  pmx[threadIdx.x] = mx;
+  __syncthreads();
+  mn = pmn[d];
+  mx = pmx[d];
+#pragma unroll
+  for (int p = 1; p < PARTS; ++p) {
+    mn = fminf(mn, pmn[p * D + d]);
+    mx = fmaxf(mx, pmx[p * D + d]);
+  }
+  const float s = affine_scale(mn, mx, BITS), inv = __frcp_rn(s);
+  bool fast = true;
+  float c[TPP];
+#pragma unroll
+  for (int j = 0; j < TPP; ++j) c[j] = rint_quot_fast(__fsub_rn(x[j], mn), inv, fast);
+  if (!fast) {                                 // a quotient near a tie: all of them exactly
+#pragma unroll
+    for (int j = 0; j < TPP; ++j) c[j] = rintf(__fdiv_rn(__fsub_rn(x[j], mn), s));
+  }
+#pragma unroll
+  for (int j = 0; j < TPP; ++j) cs[(r0 + j) * D + d] = (uint8_t)clamp_code(c[j], BITS);
+  if (part == 0) {
+    *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
+    *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < G * WPR; i += NT) {
+    const int r = i / WPR, w = i % WPR;
+    const uint8_t* cp = cs + r * D + w * CPW;
+    uint32_t word;
+    if (BITS == 8) {
+      word = *reinterpret_cast<const uint32_t*>(cp);
+    } else if (BITS == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(cp);
+      const uint32_t lo = u.x | (u.x >> 4), hi = u.y | (u.y >> 4);
+      word = (lo & 0xFFu) | ((lo >> 8) & 0xFF00u) | ((hi & 0xFFu) << 16) | ((hi >> 8) & 0xFF00u) << 16;
+    } else {
+      const uint4 u = *reinterpret_cast<const uint4*>(cp);
+      auto crumbs = [](uint32_t q) {
+        uint32_t t = q | (q >> 6);
+        return (t | (t >> 12)) & 0xFFu;
+      };
+      word = crumbs(u.x) | crumbs(u.y) << 8 | crumbs(u.z) << 16 | crumbs(u.w) << 24;
+    }
     reinterpret_cast<uint32_t*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
   }
 }
@@ -438,8 +585,12 @@ __global__ void kvarn_block_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float in
     float mn = row[0], mx = row[0];
     for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
     const float sc = affine_scale(mn, mx, bits), inv = __frcp_rn(sc);
+    bool ok = true;
     for (int j = 0; j < G; ++j)
-      cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
+      cs[r * D + gq * G + j] = (uint8_t)clamp_code(rint_quot_fast(__fsub_rn(row[j], mn), inv, ok), bits);
+    if (!ok)                                   // a quotient near a tie: all of them exactly
+      for (int j = 0; j < G; ++j)
+        cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
     *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
     *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
   }
@@ -572,8 +723,12 @@ kvarn_block_fast_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
     float mn = row[0], mx = row[0];
     for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
     const float sc = affine_scale(mn, mx, bits), inv = __frcp_rn(sc);
+    bool ok = true;
     for (int j = 0; j < G; ++j)
-      cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
+      cs[r * D + gq * G + j] = (uint8_t)clamp_code(rint_quot_fast(__fsub_rn(row[j], mn), inv, ok), bits);
+    if (!ok)                                   // a quotient near a tie: all of them exactly
+      for (int j = 0; j < G; ++j)
+        cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
     *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
     *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
   }
@@ -662,11 +817,23 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
     case KVQ_FMT_KIVI: {
       sk.ring_plane = KVQ_PLANE_K_FULL; sk.ring_rows = g.ring;
       sv.ring_plane = KVQ_PLANE_V_FULL; sv.ring_rows = g.ring;
-      const size_t sm = (size_t)g.G * g.D * 5;
+      const size_t sm = (size_t)g.G * g.D * 5 + 2 * 256 * sizeof(float);
       e = cudaFuncSetAttribute(kivi_key_flush_kernel,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
       if (e != cudaSuccess) return e;
-      launch_pdl(kivi_key_flush_kernel, dim3(dim3(max_blocks, g.B * g.H)), dim3(256), sm, s, g, L, sk);
+      const dim3 fgrid(max_blocks, g.B * g.H);
+      auto fk = kivi_key_flush_kernel;
+      if (g.G == 32) {
+        const int b = g.kb;
+        if (g.D == 64) fk = b == 2 ? kivi_key_flush32_kernel<64, 2> : b == 4 ? kivi_key_flush32_kernel<64, 4> : kivi_key_flush32_kernel<64, 8>;
+        if (g.D == 128) fk = b == 2 ? kivi_key_flush32_kernel<128, 2> : b == 4 ? kivi_key_flush32_kernel<128, 4> : kivi_key_flush32_kernel<128, 8>;
+        if (g.D == 256) fk = b == 2 ? kivi_key_flush32_kernel<256, 2> : b == 4 ? kivi_key_flush32_kernel<256, 4> : kivi_key_flush32_kernel<256, 8>;
+      }
+      if (fk != kivi_key_flush_kernel) {
+        e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        if (e != cudaSuccess) return e;
+      }
+      launch_pdl(fk, fgrid, dim3(256), sm, s, g, L, sk);
       launch_pdl(pack_pertoken_kernel, pertoken_grid(g, max_blocks * g.G, 1), dim3(256), 0, s, g,
                  L, sk, sv, 0, 1, 0, ilog2(g.D / 8), ilog2(g.G / 8));
       launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);

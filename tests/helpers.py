@@ -25,6 +25,8 @@ FORMATS = {
                   residual_tokens=128),
     "kivi_r0": dict(fmt=O.FMT_KIVI, key_bits=2, value_bits=4, group_size=32,
                     residual_tokens=0),
+    "kivi_g64": dict(fmt=O.FMT_KIVI, key_bits=4, value_bits=2, group_size=64,
+                     residual_tokens=64),
     "kvarn": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=64,
                   sink_tokens=128, norm_iters=8),
     "kvarn_small": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=32,

@@ -31,6 +31,9 @@ CASES = [
     ("float", "f32", 1, 2, 128, [9, 1]),
     ("kivi2", "bf16", 2, 2, 128, [300, 1, 1, 40, 33]),
     ("kivi_r0", "bf16", 1, 2, 64, [31, 1, 64, 5]),
+    # KIVI blocks of 64 tokens: the flush kernel for other group sizes
+    ("kivi_g64", "bf16", 2, 2, 128, [200, 1, 70]),
+    ("kivi2", "bf16", 1, 2, 256, [170, 2]),
     ("kvarn_small", "bf16", 1, 2, 64, [70, 1, 1, 100]),
     ("kvarn", "bf16", 1, 2, 256, [330, 60]),
     ("kvarn_small", "f32", 1, 1, 128, [45, 64]),
