@@ -9,7 +9,8 @@
 //     one per CTA;
 //   * each tile streams through a ring of shared stages as two stages of 8
 //     whole weight rows, each one contiguous cp.async.bulk of 16 d_in bytes
-//     (issuing many small copies costs the issuing warp microseconds), and
+//     (with 18 row copies per stage the refilling warp held the other warps
+//     at the tile-end barrier), and
 //     the tile's 16 rows of B_p ride with its second stage; there is no
 //     producer warp: the last warp to finish with a stage (a shared counter)
 //     refills it at once with the stage ns further on;
