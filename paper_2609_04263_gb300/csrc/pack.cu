@@ -717,18 +717,28 @@ kvarn_block_fast_kernel(Geom g, int L, TokSrc sk, TokSrc sv, float inv_sqrt_d) {
   const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
   const int row_plane = which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW;
   const int col_plane = which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL;
+  // a thread per (row, group); each lane walks its group from its own lane
+  // offset, so the lanes of a warp read (and write) different banks (min, max
+  // and the codes do not depend on the order)
+  const int rot = threadIdx.x & 31;
   for (int p = threadIdx.x; p < G * NG; p += blockDim.x) {
     const int r = p / NG, gq = p % NG;
     const float* row = y + r * D + gq * G;
-    float mn = row[0], mx = row[0];
-    for (int j = 1; j < G; ++j) { mn = fminf(mn, row[j]); mx = fmaxf(mx, row[j]); }
+    uint8_t* crow = cs + r * D + gq * G;
+    float mn = row[rot & (G - 1)], mx = mn;
+    for (int jj = 1; jj < G; ++jj) {
+      const float x = row[(jj + rot) & (G - 1)];
+      mn = fminf(mn, x);
+      mx = fmaxf(mx, x);
+    }
     const float sc = affine_scale(mn, mx, bits), inv = __frcp_rn(sc);
     bool ok = true;
-    for (int j = 0; j < G; ++j)
-      cs[r * D + gq * G + j] = (uint8_t)clamp_code(rint_quot_fast(__fsub_rn(row[j], mn), inv, ok), bits);
+    for (int jj = 0; jj < G; ++jj) {
+      const int j = (jj + rot) & (G - 1);
+      crow[j] = (uint8_t)clamp_code(rint_quot_fast(__fsub_rn(row[j], mn), inv, ok), bits);
+    }
     if (!ok)                                   // a quotient near a tie: all of them exactly
-      for (int j = 0; j < G; ++j)
-        cs[r * D + gq * G + j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
+      for (int j = 0; j < G; ++j) crow[j] = (uint8_t)affine_code(row[j], mn, sc, inv, bits);
     *plane_ptr<__half>(g, scale_plane, b, h, q0 + r, gq) = __float2half_rn(sc);
     *plane_ptr<__half>(g, zero_plane, b, h, q0 + r, gq) = __float2half_rn(mn + 0.0f);
   }
