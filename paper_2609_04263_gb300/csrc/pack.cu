@@ -293,9 +293,10 @@ __global__ void store_full_kernel(Geom g, int L, const void* k, const void* v) {
 // KIVI keys: one group per (G-token block, channel).  One CTA per block that
 // this append completes (grid sized for the most an append of L can flush):
 // the block's G x D keys come in as 8-element vectors (residual ring or
-// input) into shared memory, a thread per channel finds its min / max and
-// codes its G values, and each output word of a token's packed row is
-// gathered from the byte codes and stored whole.
+// input) into shared memory, 256 / D threads per channel find partial min /
+// max over their share of the G tokens, combine them and code their share,
+// and each output word of a token's packed row is gathered from the byte
+// codes and stored whole.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokSrc src) {
   pdl_wait();
