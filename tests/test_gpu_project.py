@@ -59,6 +59,8 @@ CASES = [
     ("bf16", 4, 1, 3840, 16, 8, 256, (32, 32, 32), 8700, 10000.0),
     ("bf16", 1, 1, 2112, 4, 1, 64, (8, 0, 64), 3, 10000.0),
     ("bf16", 2, 4, 1024, 6, 2, 64, (24, 8, 40), 0, 10000.0),
+    # d_in above the streaming kernel's range: the per-tile decode kernel
+    ("bf16", 3, 1, 4160, 4, 2, 64, (16, 0, 8), 11, 10000.0),
     ("bf16", 1, 64, 256, 4, 4, 64, (0, 0, 0), 0, 0.0),
     ("f32", 1, 96, 256, 4, 4, 64, (8, 8, 8), 0, 10000.0),
     ("f32", 1, 1, 256, 4, 4, 64, (8, 8, 8), 511, 10000.0),
