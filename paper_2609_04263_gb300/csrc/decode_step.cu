@@ -12,7 +12,7 @@
 // launch, so all CTAs are resident while some poll others' results):
 //
 //   entry    each warp issues TMA bulk copies of its projection units (8
-//            stacked weight rows x 256 or 512 input channels) into a ring of
+//            stacked weight rows x 1024, 512 or 256 input channels) into a ring of
 //            shared slots; one thread issues the first chunks of this CTA's
 //            attention split (codes of the tokens already stored); the LoRA
 //            up-projections are prefetched into L2; x goes to shared memory.
@@ -41,8 +41,9 @@ namespace {
 constexpr int kWarpsF = 8;                   // warps per CTA
 constexpr int kMaxSlots = 32;
 constexpr size_t kSmemBudget = 227 * 1024 - 8192;   // dynamic shared memory (static kept aside)
-// A projection unit is 8 stacked rows x ks input channels (ks = 512 when
-// d_in allows, else 256); its rows sit in shared memory at a stride of
+// A projection unit is 8 stacked rows x ks input channels (ks = 1024 when
+// d_in allows, else 512 or 256: fewer K slices mean fewer partials to hand
+// over per output); its rows sit in shared memory at a stride of
 // 2 ks + 64 bytes, so that the 16-byte operand loads of two rows in one
 // quarter-warp fall on different banks.
 __host__ __device__ constexpr int unit_bytes(int ks) { return 8 * (2 * ks + 64); }
@@ -571,7 +572,7 @@ bool plan_step(const Geom& g, int d_in, const int r[3], size_t att_bytes, StepAr
                size_t* smem) {
   const int n_out = (g.Hq + 2 * g.H) * g.D;
   const int rows = n_out + r[0] + r[1] + r[2];
-  const int ks = d_in % 512 == 0 ? 512 : 256;
+  const int ks = d_in % 1024 == 0 ? 1024 : d_in % 512 == 0 ? 512 : 256;
   const int S = d_in / ks;
   const int units = rows / 8 * S;
   const int grid = num_sms();
