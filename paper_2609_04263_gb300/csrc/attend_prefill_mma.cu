@@ -213,6 +213,71 @@ __device__ void kvarn_tile(const Geom& g, int which, int b, int h, int t0, int T
   }
 }
 
+// KVarN tile with full-precision rows (sinks, staged tokens) among its NT
+// tokens: a warp per token builds the key and value rows in the layout
+// x[i] = row[lane + 32 i]; coded tokens are reconstructed as stored (rotated),
+// full-precision ones are rotated forward in registers by fwht_warp (the same
+// butterflies, in the same order, as the rotation of the queries), so the tile
+// needs no scratch and no CTA barrier.
+template <int D, int NT, int THREADS>
+__device__ __noinline__ void kvarn_tile_rows(const Geom& g, int b, int h, int t0, int T,
+                                __nv_bfloat16* khi, __nv_bfloat16* klo, __half* vdst, int lds,
+                                float inv_sqrt_d) {
+  constexpr int NS = D / 32, NW = THREADS / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = g.G, S = g.S;
+  const int nbq = kvarn_nblocks(T, S, G) * G;
+  for (int r = warp; r < NT; r += NW) {
+    const int t = t0 + r;
+    float kx[NS], vx[NS];
+    if (t >= T) {
+#pragma unroll
+      for (int i = 0; i < NS; ++i) kx[i] = vx[i] = 0.f;
+    } else if (t < S || t - S >= nbq) {
+      const __nv_bfloat16* ks = t < S ? plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, h, t, 0)
+                                      : plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_PEND, b, h, (t - S) % G, 0);
+      const __nv_bfloat16* vs = t < S ? plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, h, t, 0)
+                                      : plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_PEND, b, h, (t - S) % G, 0);
+#pragma unroll
+      for (int i = 0; i < NS; ++i) {
+        kx[i] = __bfloat162float(ks[lane + 32 * i]);
+        vx[i] = __bfloat162float(vs[lane + 32 * i]);
+      }
+      fwht_warp<D>(kx, lane, inv_sqrt_d);
+      fwht_warp<D>(vx, lane, inv_sqrt_d);
+    } else {
+      const int qi = t - S;
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        const int bits = which ? g.vb : g.kb;
+        const unsigned mask = (1u << bits) - 1;
+        const uint8_t* row = plane_ptr<uint8_t>(g, which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES, b, h, qi);
+        const float rr = __half2float(*plane_ptr<__half>(g, which ? KVQ_PLANE_V_ROW : KVQ_PLANE_K_ROW, b, h, 0, qi));
+        const __half* col = plane_ptr<__half>(g, which ? KVQ_PLANE_V_COL : KVQ_PLANE_K_COL, b, h, qi / G, 0);
+        const __half* scp = plane_ptr<__half>(g, which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE, b, h, qi, 0);
+        const __half* zp = plane_ptr<__half>(g, which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO, b, h, qi, 0);
+#pragma unroll
+        for (int i = 0; i < NS; ++i) {
+          const int j = lane + 32 * i, bit = j * bits;
+          const unsigned code = ((unsigned)row[bit >> 3] >> (bit & 7)) & mask;
+          const float sc = __half2float(scp[j / G]), mz = __half2float(zp[j / G]);
+          const float v = rr * __half2float(col[j]) * ((float)code * sc + mz);
+          if (which) vx[i] = v;
+          else kx[i] = v;
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const int j = lane + 32 * i;
+      const __nv_bfloat16 hb = __float2bfloat16_rn(kx[i]);
+      khi[r * lds + j] = hb;
+      klo[r * lds + j] = __float2bfloat16_rn(kx[i] - __bfloat162float(hb));
+      vdst[r * lds + j] = __float2half_rn(vx[i]);
+    }
+  }
+}
+
 // KVarN tile whose tokens are all coded (stored rotated: r_t c_j (s code + m)),
 // keys and values in one pass.  A thread keeps one 8-channel chunk for all
 // of its tokens; the tile lies inside one column-scale block (NT divides the
@@ -413,6 +478,8 @@ attend_prefill_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, fl
     } else if (D != 128 && g.fmt == KVQ_FMT_KVARN && t0 >= g.S && t0 + NT <= T &&
                t0 + NT <= g.S + kvarn_nblocks(T, g.S, g.G) * g.G && g.G % NT == 0 && g.S % NT == 0) {
       kvarn_tile_coded<D, NT, C::THREADS>(g, b, hkv, t0, Ks, Kl, Vs, LDS);
+    } else if (g.fmt == KVQ_FMT_KVARN && D != 128) {
+      kvarn_tile_rows<D, NT, C::THREADS>(g, b, hkv, t0, T, Ks, Kl, Vs, LDS, inv_sqrt_d);
     } else if (g.fmt == KVQ_FMT_KVARN) {
       float* scr = reinterpret_cast<float*>(smem + C::SCR_OFF);
       kvarn_tile<D, NT, C::THREADS>(g, 0, b, hkv, t0, T, Ks, Kl, Vs, LDS, scr, inv_sqrt_d);
