@@ -34,6 +34,9 @@ CASES = [
     # KIVI blocks of 64 tokens: the flush kernel for other group sizes
     ("kivi_g64", "bf16", 2, 2, 128, [200, 1, 70]),
     ("kivi2", "bf16", 1, 2, 256, [170, 2]),
+    # 4- and 8-bit KIVI keys in 32-token blocks (the compile-time flush)
+    ("kivi_k4", "bf16", 2, 2, 128, [150, 1, 40]),
+    ("kivi_k8", "bf16", 1, 2, 64, [100, 3]),
     ("kvarn_small", "bf16", 1, 2, 64, [70, 1, 1, 100]),
     ("kvarn", "bf16", 1, 2, 256, [330, 60]),
     ("kvarn_small", "f32", 1, 1, 128, [45, 64]),
