@@ -190,9 +190,9 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
  * cache after T tokens is the same whether they arrive in one call or in
  * chunks.  KVQ_ERR_CAPACITY if T + L > max_tokens (host mirror); the kernels
  * check the device count again and refuse an overflowing replayed append.
- * KVQ_ERR_SHAPE if B * Hkv * (L + group_size) * D / 4 reaches 2^31 (the
- * kernels index one call's elements in 32 bits): append such a span in
- * chunks instead.
+ * KVQ_ERR_SHAPE if B * Hkv exceeds 65535, or if B * Hkv * (L + group_size) *
+ * D / 4 reaches 2^31 (the kernels index one call's elements in 32 bits):
+ * append such a span in chunks instead.
  */
 kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L,
                            void* stream);
