@@ -124,3 +124,29 @@ def test_project_validation(kvq):
             kvq.kvq_project_lora(P, 1, 4, c.get("d_in", 2048), P, P, P, c.get("r_q", 16), P, P,
                                  16, P, P, 16, 2.0, hq, hkv, c.get("head_dim", 64), 0, None, 1e4,
                                  c.get("dtype", kvq.KVQ_BF16), P, P, P, 0)
+
+
+def test_append_index_range_is_checked_on_the_host(kvq):
+    """Appends whose elements a kernel could not index in 32 bits, or whose
+    batch x kv heads exceed the grid's y range, are refused before any launch."""
+    fake = 1 << 32
+    # batch x kv heads above 65535
+    d = _desc(kvq, batch=65536, kv_heads=1, q_heads=1, max_tokens=64)
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_append_pack(h, 1 << 33, 1 << 33, 1, 0)
+        assert ei.value.status == kvq.KVQ_ERR_SHAPE
+        assert kvq.kvq_cache_tokens(h) == 0
+    finally:
+        kvq.kvq_destroy_cache(h)
+    # B Hkv (L + G) D / 4 at 2^31: 64 x 8 x (2^17 + 32) x 256 / 4 > 2^31
+    d = _desc(kvq, batch=64, kv_heads=8, q_heads=8, head_dim=256, max_tokens=1 << 17)
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_append_pack(h, 1 << 33, 1 << 33, 1 << 17, 0)
+        assert ei.value.status == kvq.KVQ_ERR_SHAPE
+        assert kvq.kvq_cache_tokens(h) == 0
+    finally:
+        kvq.kvq_destroy_cache(h)
