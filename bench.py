@@ -375,8 +375,8 @@ class ClockSampler:
         self.index, self.proc, self.path = index, None, None
 
     def start(self):
-        out_dir = os.path.join(ROOT, "gpurun_out")
-        os.makedirs(out_dir, exist_ok=True)
+        import tempfile
+        out_dir = tempfile.mkdtemp(prefix="kvq_clocks_")
         self.path = os.path.join(out_dir, f"clocks_rank{self.index}.csv")
         try:
             self.proc = subprocess.Popen(
@@ -406,6 +406,8 @@ class ClockSampler:
                 for n, v in zip(names, parts[5:9]):
                     if v.lower().startswith("active"):
                         reasons.add(n)
+        import shutil
+        shutil.rmtree(os.path.dirname(self.path), ignore_errors=True)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
                 "samples": len(sm), "reasons": sorted(reasons)}
 
