@@ -1,14 +1,18 @@
 """Benchmark of the packed-cache attention step on GB300.
 
-One step is one pass of the whole path over one batch of the TinyLlama-shaped
-workload (22 layers, batch 4, hidden 2048, 32 query / 4 KV heads, head_dim 64,
-4-bit affine cache with groups of 32, rank-16 LoRA on Q, K and V): reset the
-caches, prefill 2048 tokens per sequence (LoRA Q/K/V projection with RoPE,
-quantize-and-pack append, causal prefill attention, per layer), then 256 decode
-steps (projection, append, split-K decode attention: one fused kvq_decode_step
-kernel per layer; one captured CUDA graph per decode step).  `value` is tokens processed per second
-(batch x (prefill + decode) tokens per step); the decode phase alone, pack
-bandwidth and projection TFLOP/s are reported beside it.
+One step is one pass of the whole path over one batch of the default workload,
+the Llama-3.1-8B-shaped attention stack (32 layers, batch 16, hidden 4096, 32
+query / 8 KV heads, head_dim 128, RoPE base 500000, KIVI K2V2 cache with groups
+of 32 and a 128-token full-precision residual, rank-16 LoRA on Q, K and V):
+reset the caches, prefill 8192 tokens per sequence (LoRA Q/K/V projection with
+RoPE, quantize-and-pack append, causal prefill attention, per layer), then 64
+decode steps (projection, append, split-K decode attention through
+kvq_decode_step; one captured CUDA graph per decode step).  `value` is tokens
+processed per second (batch x (prefill + decode) tokens per step); the decode
+phase alone, the packed-cache decode attention against HBM, pack bandwidth and
+projection TFLOP/s are reported beside it.  --workload selects another shape
+(the TinyLlama-shaped affine/symmetric stacks, the 12B-class KVarN stack, the
+single fp32 layer).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl kvq|reference]
 
@@ -37,7 +41,7 @@ from paper_2609_04263_gb300 import synth  # noqa: E402
 
 METRIC = ("packed-KV decode attention tokens/s and % HBM roofline; pack GB/s; "
           "QKV TFLOP/s")
-WORKLOAD = "tinyllama_affine4"
+WORKLOAD = "llama8b_kivi"
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -467,12 +471,18 @@ def cold_graph_time_ms(fn, reps, flush):
 # ---------------------------------------------------------------------------
 # CPU oracle (the reported baseline and the reference arm)
 # ---------------------------------------------------------------------------
-def oracle_sample(wl, decode_steps=8, prefill=None):
+def oracle_sample(wl, decode_steps=8, prefill=None, max_queries=64):
     """Time the CPU oracle on one layer of one sequence: a full-length prefill
     (projection, pack, attention) and `decode_steps` decode steps.  Returns
-    (seconds, job-equivalent tokens/s) where the per-layer-per-sequence cost
-    is scaled to all layers and sequences and the decode steps to the full
-    count (decode steps cost the same to within the cache growth)."""
+    (seconds, job-equivalent tokens/s, description): the per-layer-per-sequence
+    cost is scaled to all layers and sequences and the decode steps to the
+    full count (decode steps cost the same to within the cache growth).
+
+    When the prefill has more than `max_queries` tokens, the prefill attention
+    runs the oracle's plain attention for `max_queries` evenly spaced queries
+    over every key they see (a full [Hq, P, P] fp64 score tensor would not fit
+    in host memory at P = 8192), and its time is scaled by the ratio of
+    visible (query, key) pairs of all P queries to those of the sample."""
     from oracle import kvq_oracle as O
     P = wl.prefill if prefill is None else prefill
     w, lora = synth.layer_weights(wl, 0)
@@ -487,22 +497,35 @@ def oracle_sample(wl, decode_steps=8, prefill=None):
                           residual_tokens=wl.residual_tokens, sink_tokens=wl.sink_tokens,
                           norm_iters=wl.norm_iters)
     args = (wl.alpha_over_r, wl.n_q_heads, wl.n_kv_heads, wl.head_dim)
+    nq = min(P, max_queries)
+    ls = np.unique(np.linspace(0, P - 1, nq).round().astype(np.int64))
     t0 = time.perf_counter()
     q, k, v = O.project_lora(x_pre, w, lora, *args, pos0=0, rope_base=wl.rope_base)
     cache.append(O.round_to(k, act), O.round_to(v, act))
-    O.attend(cache, O.round_to(q, act))
     t1 = time.perf_counter()
+    if len(ls) == P:
+        O.attend(cache, O.round_to(q, act))
+        attn_scale = 1.0
+    else:
+        kh, vh = cache.reconstruct()
+        O.attention(O.round_to(q[:, :, ls], act), kh, vh, ls, 1.0 / math.sqrt(wl.head_dim))
+        attn_scale = (P * (P + 1) / 2) / float((ls + 1).sum())
+    t2 = time.perf_counter()
     for s in range(decode_steps):
         q, k, v = O.project_lora(x_dec[:, s:s + 1], w, lora, *args, pos0=P + s,
                                  rope_base=wl.rope_base)
         cache.append(O.round_to(k, act), O.round_to(v, act))
         O.attend(cache, O.round_to(q, act))
-    t2 = time.perf_counter()
-    job_s = ((t1 - t0) + (t2 - t1) * wl.decode / decode_steps) * wl.layers * wl.batch
+    t3 = time.perf_counter()
+    prefill_s = (t1 - t0) + (t2 - t1) * attn_scale
+    job_s = (prefill_s + (t3 - t2) * wl.decode / decode_steps) * wl.layers * wl.batch
     tokens = wl.batch * (wl.prefill + wl.decode)
-    return t2 - t0, tokens / job_s, (f"1 of {wl.layers} layers x 1 of {wl.batch} sequences: "
-                                     f"{P}-token prefill + {decode_steps} of {wl.decode} decode "
-                                     f"steps, scaled to the full job")
+    attn = ("" if len(ls) == P else
+            f" (prefill attention of {len(ls)} evenly spaced queries over all their keys, "
+            f"scaled by visible pairs x{attn_scale:.1f})")
+    return t3 - t0, tokens / job_s, (f"1 of {wl.layers} layers x 1 of {wl.batch} sequences: "
+                                     f"{P}-token prefill{attn} + {decode_steps} of {wl.decode} "
+                                     f"decode steps, scaled to the full job")
 
 
 def cpu_cores():
@@ -542,13 +565,27 @@ def max_over_ranks(world, x):
     return float(t.item())
 
 
+def workload_config(wl, world):
+    """The `config` object of the JSON line (both arms)."""
+    return {
+        "workload": wl.name, "layers": wl.layers, "batch": wl.batch,
+        "prefill": wl.prefill, "decode": wl.decode, "d_in": wl.d_in,
+        "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+        "cache": f"{synth.FMT_NAMES[wl.fmt]} K{wl.key_bits}V{wl.value_bits} G{wl.group_size}",
+        "lora_rank": wl.rank, "tokens_per_step": wl.batch * (wl.prefill + wl.decode),
+        "l2": "flushed between timed steps (256 MiB written, then 256 MiB read so no dirty "
+              "line is left); job working set > L2",
+        "parallelism": f"replicas x{world}",
+    }
+
+
 def run_reference(args, world, rank):
     if rank != 0:
         return
     wl = synth.WORKLOADS[args.workload]
     vals, secs = [], []
     for _ in range(args.warmup):
-        oracle_sample(wl, decode_steps=2)
+        oracle_sample(wl, decode_steps=2, prefill=min(wl.prefill, 1024))
     sample = None
     for _ in range(args.steps):
         s, v, sample = oracle_sample(wl, decode_steps=4)
@@ -560,8 +597,7 @@ def run_reference(args, world, rank):
             "ms_per_step": 1000.0 * wl.batch * (wl.prefill + wl.decode) / value,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch,
-                       "prefill": wl.prefill, "decode": wl.decode},
+            "config": dict(workload_config(wl, world), decode_path="CPU oracle"),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -637,6 +673,18 @@ def main():
     t_wall = time.perf_counter() - t_wall
     barrier(world)
     clk = clocks.stop()
+    # a bounded wait that gave up inside a kernel returns early with wrong
+    # output and would time as a fast step: no value is reported then
+    from paper_2609_04263_gb300 import kvq
+    status = kvq.kvq_device_status(torch.cuda.current_stream().cuda_stream)
+    status = int(max_over_ranks(world, float(status)))
+    if status:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": None, "unit": "tokens/s",
+                              "n_gpus": world, "device_status": status,
+                              "error": "a bounded device-side wait gave up during the timed "
+                                       "region: the timed output is not valid"}), flush=True)
+        raise SystemExit(1)
     step_ms = [e[0].elapsed_time(e[2]) for e in ev]
     pre_ms = [e[0].elapsed_time(e[1]) for e in ev]
     dec_ms = [e[1].elapsed_time(e[2]) for e in ev]
@@ -736,6 +784,8 @@ def main():
         torch.cuda.synchronize()
         e2e_vals.append(time.perf_counter() - t0)
     e2e_s = max_over_ranks(world, statistics.mean(e2e_vals))
+    status = int(max_over_ranks(world, float(
+        kvq.kvq_device_status(torch.cuda.current_stream().cuda_stream))))
     e2e_value = world * tokens_per_step / e2e_s
 
     cpu = None
@@ -750,16 +800,7 @@ def main():
             "steps": args.steps, "warmup": max(args.warmup, 3),
             "ms_per_step": statistics.mean(step_ms), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-            "config": {
-                "workload": wl.name, "layers": wl.layers, "batch": wl.batch,
-                "prefill": wl.prefill, "decode": wl.decode, "d_in": wl.d_in,
-                "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
-                "cache": f"{synth.FMT_NAMES[wl.fmt]} K{wl.key_bits}V{wl.value_bits} G{wl.group_size}",
-                "lora_rank": wl.rank, "tokens_per_step": tokens_per_step,
-                "l2": "flushed between timed steps (256 MiB written, then 256 MiB read so no dirty line is left); job working set > L2",
-                "parallelism": f"replicas x{world}",
-                "decode_path": run.decode_path(),
-            },
+            "config": dict(workload_config(wl, world), decode_path=run.decode_path()),
             "phases": {"prefill_ms": statistics.mean(pre_ms), "decode_ms": statistics.mean(dec_ms),
                        "decode_tokens_per_s": decode_tps,
                        "pack_gbs": kernels["append"]["achieved"],
@@ -778,6 +819,7 @@ def main():
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": run.launches_per_step() * args.steps,
+            "device_status": status,
             "clocks": clk,
             "wall_s_timed": t_wall,
         }

@@ -263,7 +263,9 @@ int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, in
  * KVQ_ERR_CAPACITY, launching nothing, if batch * q_heads * 32 * (head_dim + 2)
  * floats exceed the array (1,048,576 floats).  The first call on each device
  * looks up the array's device address with that device current; make that
- * first call before any stream capture.  Every call uses the same array and
+ * first call before any stream capture.  The address is kept for the life of
+ * the process: do not use the library on a device after cudaDeviceReset().
+ * Every call uses the same array and
  * leaves its contents behind (the kernels write every partial they later
  * read, so nothing needs clearing), so calls that overlap on the GPU (other
  * streams, other threads) race: serialise them.
@@ -272,7 +274,11 @@ kvq_status kvq_attend_decode_noalloc(kvq_cache* cache, const void* q, int n_q_he
                                      float softmax_scale, void* out, void* stream);
 
 /* Read and clear the device-side error word of the library (synchronises
- * `stream`).  *out = 0 when no bounded wait has timed out. */
+ * `stream`).  *out = 0 when no bounded wait has timed out; otherwise a kernel
+ * gave up waiting (a TMA ring, a handoff between CTAs, a merge), returned
+ * early and left its output incomplete, and KVQ_ERR_TIMEOUT is returned.  The
+ * word's address is looked up once per device: do not use the library on a
+ * device after cudaDeviceReset(). */
 kvq_status kvq_device_status(void* stream, int* out);
 
 /* Description of the last failure on this thread ("" if none). */

@@ -119,3 +119,16 @@ def compare_planes(gc, oc):
             diff = np.argwhere(a.view(np.uint8) != b.view(np.uint8)) if a.dtype != np.float32 \
                 else np.argwhere(a != b)
             raise AssertionError(f"plane {name}: {len(diff)} mismatches, first at {diff[:3].tolist()}")
+
+
+def check_projection(got, ref, act, what=""):
+    """Projection parity per (sequence, head): the max-abs difference from the
+    oracle's fp64 result rounded to the activation dtype, over that head's
+    largest oracle value, within 1e-2 (bf16) or 1e-5 (fp32).
+    got (numpy, the GPU output as fp32) and ref (fp64): [B, H, L, D]."""
+    tol = 1e-5 if act == "f32" else 1e-2
+    r = O.round_to(ref, act).astype(np.float64)
+    err = np.abs(np.asarray(got, dtype=np.float64) - r).max(axis=(2, 3))
+    rel = err / np.maximum(np.abs(ref).max(axis=(2, 3)), 1e-30)
+    worst = tuple(int(i) for i in np.unravel_index(int(rel.argmax()), rel.shape))
+    assert rel.max() <= tol, f"{what}: (sequence, head) {worst} relative error {rel.max():.2e}"

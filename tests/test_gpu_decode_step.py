@@ -14,7 +14,7 @@ import torch
 from oracle import kvq_oracle as O
 from paper_2609_04263_gb300 import synth
 from tests.gpu_common import require_gpu
-from tests.helpers import FORMATS, compare_planes, oracle_cache
+from tests.helpers import FORMATS, check_projection, compare_planes, oracle_cache
 
 pytestmark = pytest.mark.gpu
 
@@ -27,6 +27,9 @@ def _gpu():
 # fmt, B, d_in, Hq, Hkv, D, rank, prefill, fused expected
 CASES = [
     ("affine4", 4, 512, 32, 4, 64, 16, 100, True),
+    ("affine4", 4, 2048, 32, 4, 64, 16, 300, True),   # 1024-channel projection units
+    ("sym2", 8, 2048, 32, 4, 64, 64, 130, True),      # the same at rank 64
+    ("affine2", 2, 1536, 8, 2, 128, 16, 100, True),   # 512-channel units (1536 % 1024 != 0)
     ("sym2", 8, 256, 16, 2, 64, 64, 100, True),      # rank 64
     ("affine2", 3, 256, 8, 2, 128, 8, 100, True),    # D = 128
     ("sym4", 12, 256, 8, 2, 64, 8, 70, True),        # B > 8: second MMA row block
@@ -61,6 +64,8 @@ def test_decode_step_matches_separate_calls(fmt_name, B, d_in, Hq, Hkv, D, r, pr
     tl = {p: tuple(torch.from_numpy(t).to(bf).cuda() for t in lora[p]) for p in "qkv"}
     x = torch.from_numpy(synth.hidden_states((B, prefill + steps, d_in), outlier_frac=0.01,
                                              seed=7)).to(bf).cuda()
+    nw = tw.float().cpu().numpy()
+    nl = {p: tuple(t.float().cpu().numpy() for t in tl[p]) for p in "qkv"}
     kw = dict(spec)
     fmt = kw.pop("fmt")
 
@@ -104,6 +109,11 @@ def test_decode_step_matches_separate_calls(fmt_name, B, d_in, Hq, Hkv, D, r, pr
         torch.cuda.synchronize()
         for a_, b_, name in zip(qkv, (q2, k2, v2), "qkv"):
             assert _bf16_close(a_, b_), f"step {s}: {name} differs beyond one bf16 rounding"
+        # the fused step's own q, k, v against the oracle projection
+        ref_p = O.project_lora(xs.float().cpu().numpy(), nw, nl, 2.0, Hq, Hkv, D,
+                               pos0=prefill + s, rope_base=10000.0)
+        for a_, r_, name in zip(qkv, ref_p, "qkv"):
+            check_projection(a_.float().cpu().numpy(), r_, "bf16", f"step {s} fused {name}")
         oc_f.append(qkv[1].float().cpu().numpy(), qkv[2].float().cpu().numpy())
         oc_r.append(k2.float().cpu().numpy(), v2.float().cpu().numpy())
         ref_f = O.attend(oc_f, qkv[0].float().cpu().numpy())

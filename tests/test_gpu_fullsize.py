@@ -7,10 +7,15 @@ For every workload (single layer of each model shape, layer 0 weights):
   * prefill append: the packed planes of sampled (sequence, kv head) pairs bit
     for bit, against oracle caches fed the same projected k, v;
   * prefill attention: sampled queries of every query head of those kv heads;
-  * decode: all decode steps of the workload; the planes at the end bit for
-    bit and the attention output of the first and last step.
-Outputs are bf16 (fp32 for the single-layer workload); the attention bound is
-max-abs 2e-2 beyond the output's own rounding (bf16 holds |o| ~ 8 to 0.03).
+  * decode: all decode steps of the workload through kvq_decode_step (the
+    fused single-kernel step where the library takes it, as the bench does),
+    replayed from one captured graph; the step's q, k, v and attention output
+    at the first and last step against the oracle, and at the end the planes
+    bit for bit against oracle caches fed the steps' own keys and values.
+Projections are checked per (sequence, head) against the oracle rounded to
+the activation dtype (relative 1e-2 for bf16, 1e-5 for fp32).  Attention
+outputs must be a rounding of a value within max-abs 2e-2 (bf16) or 1e-4
+(fp32) of the fp64 oracle.
 """
 import math
 
@@ -21,6 +26,7 @@ import torch
 from oracle import kvq_oracle as O
 from paper_2609_04263_gb300 import synth
 from tests.gpu_common import require_gpu
+from tests.helpers import check_projection
 
 pytestmark = pytest.mark.gpu
 
@@ -30,16 +36,36 @@ def _gpu():
     require_gpu()
 
 
-def _act_tol(act):
-    return (1e-4, 2.0 ** -23) if act == "f32" else (2e-2, 2.0 ** -8)
+def _floor_act(x, act):
+    """Largest value of the activation dtype that is <= x (x in fp64)."""
+    x = np.asarray(x, dtype=np.float64)
+    f = x.astype(np.float32)
+    f = np.where(f.astype(np.float64) > x, np.nextafter(f, np.float32(-np.inf)), f)
+    f = np.asarray(f, dtype=np.float32)
+    if act == "f32":
+        return f.astype(np.float64)
+    bits = f.view(np.uint32)
+    t = bits & np.uint32(0xFFFF0000)             # bf16 truncation (toward zero)
+    t = np.where((f < 0) & (t != bits), t + np.uint32(0x10000), t).astype(np.uint32)
+    return t.view(np.float32).astype(np.float64)
+
+
+def _ceil_act(x, act):
+    return -_floor_act(-np.asarray(x, dtype=np.float64), act)
 
 
 def _check_attention(got, ref, act, what):
-    atol, rtol = _act_tol(act)
-    err = np.abs(got - ref)
-    bound = atol + rtol * np.abs(ref)
-    worst = float((err - bound).max())
-    assert worst <= 0, f"{what}: max-abs {err.max():.3e} exceeds the bound by {worst:.3e}"
+    """The literal bound on the unrounded result: `got` (in the activation
+    dtype) must be a rounding, up or down, of some value within atol of the
+    fp64 oracle, i.e. lie between the dtype's neighbours of ref - atol and
+    ref + atol.  atol is 2e-2 for bf16 and 1e-4 for fp32 outputs."""
+    atol = 1e-4 if act == "f32" else 2e-2
+    lo, hi = _floor_act(ref - atol, act), _ceil_act(ref + atol, act)
+    bad = (got < lo) | (got > hi)
+    if bad.any():
+        i = np.unravel_index(int(np.argmax(np.abs(got - ref))), got.shape)
+        raise AssertionError(f"{what}: {int(bad.sum())} outputs outside the bound; worst "
+                             f"{got[i]:.6g} vs oracle {ref[i]:.6g} at {tuple(int(j) for j in i)}")
 
 
 def _planes_subset(cache, b, h):
@@ -74,6 +100,11 @@ def _compare_subset(cache, b, h, oc):
         assert same, f"plane {name} of (b={b}, h={h}) differs from the oracle"
 
 
+# which decode path bench.py's kvq_decode_step takes on each workload
+FUSED = {"single_layer_f32": False, "tinyllama_affine4": True, "tinyllama_sym2": True,
+         "llama8b_kivi": False, "gemma12b_kvarn": False}
+
+
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))
 def test_full_size_layer(name):
     from paper_2609_04263_gb300 import api
@@ -97,19 +128,18 @@ def test_full_size_layer(name):
                          sink_tokens=wl.sink_tokens, norm_iters=wl.norm_iters)
     cache = api.Cache(desc)
     args = (wl.alpha_over_r, Hq, Hkv, D)
+    assert cache.decode_step_fused(wl.d_in, dl) == FUSED[name]
 
-    # ---- prefill projection (sampled row segments) ----
+    # ---- prefill projection (sampled row segments, every head) ----
     q, k, v = api.project_lora(x_pre.to(dev), dw, dl, *args, rope_base=wl.rope_base,
                                pos_cache=cache)
     torch.cuda.synchronize()
-    ptol = 1e-5 if act == "f32" else 1e-2
     for b, lo in ((0, 0), (B - 1, P - 64)):
         seg = x_pre[b:b + 1, lo:lo + 64].float().numpy()
         ref = O.project_lora(seg, nw, nl, *args, pos0=lo, rope_base=wl.rope_base)
-        for got_t, ref_t in zip((q, k, v), ref):
+        for got_t, ref_t, pn in zip((q, k, v), ref, "qkv"):
             got = got_t[b:b + 1, :, lo:lo + 64].float().cpu().numpy()
-            rel = np.abs(got - ref_t).max() / np.abs(ref_t).max()
-            assert rel <= ptol, f"projection rows {lo}..{lo + 63} of sequence {b}: {rel:.2e}"
+            check_projection(got, ref_t, act, f"prefill {pn} rows {lo}..{lo + 63} of sequence {b}")
 
     # ---- prefill append and attention ----
     cache.append(k, v)
@@ -135,17 +165,16 @@ def test_full_size_layer(name):
         got = o[b:b + 1, heads][:, :, ls].float().cpu().numpy()
         _check_attention(got, ref, act, f"prefill attention (b={b}, kv head {h})")
 
-    # ---- decode: the bench's captured step, replayed Dn times ----
+    # ---- decode: bench.py's captured kvq_decode_step, replayed Dn times ----
     xs = torch.empty(B, 1, wl.d_in, dtype=dt, device=dev)
     outs = tuple(torch.empty(B, hh, 1, D, dtype=dt, device=dev) for hh in (Hq, Hkv, Hkv))
     od = torch.empty(B, Hq, 1, D, dtype=dt, device=dev)
+    torch.cuda.synchronize()
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=side):
-        api.project_lora(xs, dw, dl, *args, rope_base=wl.rope_base, out=outs, pos_cache=cache)
-        cache.append(outs[1], outs[2])
-        cache.attend_decode(outs[0], out=od)
+        cache.decode_step(xs, dw, dl, wl.alpha_over_r, wl.rope_base, qkv=outs, out=od)
     x_dec_dev = x_dec.to(dev)
     for s in range(Dn):
         xs.copy_(x_dec_dev[:, s:s + 1])
@@ -156,12 +185,12 @@ def test_full_size_layer(name):
         for (b, h), oc in ocs.items():
             oc.append(kk[b:b + 1, h:h + 1], vv[b:b + 1, h:h + 1])
         if s in (0, Dn - 1):
-            if s == 0:     # decode projection rows against the oracle
-                ref = O.project_lora(x_dec[:, 0:1].float().numpy(), nw, nl, *args, pos0=P,
-                                     rope_base=wl.rope_base)
-                for got_t, ref_t in zip(outs, ref):
-                    rel = np.abs(got_t.float().cpu().numpy() - ref_t).max() / np.abs(ref_t).max()
-                    assert rel <= ptol, f"decode projection: {rel:.2e}"
+            # the step's own q, k, v against the oracle projection, per head
+            ref = O.project_lora(x_dec[:, s:s + 1].float().numpy(), nw, nl, *args, pos0=P + s,
+                                 rope_base=wl.rope_base)
+            for got_t, ref_t, pn in zip(outs, ref, "qkv"):
+                check_projection(got_t.float().cpu().numpy(), ref_t, act,
+                                  f"decode step {s} projection {pn}")
             for (b, h), oc in ocs.items():
                 heads = list(range(h * g, (h + 1) * g))
                 qd = outs[0][b:b + 1, heads].float().cpu().numpy()
@@ -169,5 +198,6 @@ def test_full_size_layer(name):
                 got = od[b:b + 1, heads].float().cpu().numpy()
                 _check_attention(got, ref, act, f"decode step {s} (b={b}, kv head {h})")
     assert cache.sync() == wl.max_tokens
+    # the planes the decode steps wrote, against oracle caches fed the steps' own k, v
     for (b, h), oc in ocs.items():
         _compare_subset(cache, b, h, oc)

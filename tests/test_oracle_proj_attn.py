@@ -116,6 +116,48 @@ def test_rope_quarter_turn():
     assert np.allclose(z[..., 0], 0.0, atol=1e-15) and np.allclose(z[..., 1], 1.0)
 
 
+@pytest.mark.parametrize("base,thetas", [
+    # base^(-2i/D) for D = 8, i = 0..3, written out by hand
+    (10000.0, (1.0, 0.1, 0.01, 0.001)),
+    (100.0, (1.0, 0.31622776601683794, 0.1, 0.031622776601683794)),   # 100^(-1/4) = 1/sqrt(10)
+])
+def test_rope_frequency_schedule_hand_worked(base, thetas):
+    """The frequency of channel pair i at D = 8 and its pairing partner.
+
+    Rotate-half pairs channel i with channel i + D/2 = i + 4; at position 3 the
+    pair turns by 3 theta_i.  A unit vector on channel i must land on
+    (cos 3 theta_i) e_i + (sin 3 theta_i) e_(i+4), and one on channel i + 4 on
+    -(sin 3 theta_i) e_i + (cos 3 theta_i) e_(i+4).  A schedule of base^(-i/D),
+    an interleaved pairing (2i, 2i + 1) or a flipped sign fails here, which the
+    invariants (identity at 0, norm, relative position) cannot see."""
+    for i, th in enumerate(thetas):
+        c, s = math.cos(3 * th), math.sin(3 * th)
+        e = np.zeros((1, 1, 1, 8))
+        e[..., i] = 1.0
+        want = np.zeros(8)
+        want[i], want[i + 4] = c, s
+        got = O.rope_rotate_half(e, np.array([3]), base)[0, 0, 0]
+        assert np.allclose(got, want, rtol=0, atol=1e-15), (i, got, want)
+        e = np.zeros((1, 1, 1, 8))
+        e[..., i + 4] = 1.0
+        want = np.zeros(8)
+        want[i], want[i + 4] = -s, c
+        got = O.rope_rotate_half(e, np.array([3]), base)[0, 0, 0]
+        assert np.allclose(got, want, rtol=0, atol=1e-15), (i + 4, got, want)
+
+
+def test_rope_second_pair_at_position_one():
+    """D = 4, base 10000, position 1: pair (1, 3) turns by 10000^(-1/2) = 0.01 rad
+    and pair (0, 2) by 1 rad."""
+    y = np.array([[[[0.0, 2.0, 0.0, 0.0]]]])
+    z = O.rope_rotate_half(y, np.array([1]), 10000.0)[0, 0, 0]
+    assert np.allclose(z, [0.0, 2.0 * math.cos(0.01), 0.0, 2.0 * math.sin(0.01)],
+                       rtol=0, atol=1e-15)
+    y = np.array([[[[1.0, 0.0, 0.0, 0.0]]]])
+    z = O.rope_rotate_half(y, np.array([1]), 10000.0)[0, 0, 0]
+    assert np.allclose(z, [math.cos(1.0), 0.0, math.sin(1.0), 0.0], rtol=0, atol=1e-15)
+
+
 def _sdpa_ref(q, k, v, q_pos, scale):
     """torch's scaled_dot_product_attention in fp64 (library routine)."""
     g = q.shape[1] // k.shape[1]
