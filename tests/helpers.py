@@ -132,3 +132,35 @@ def check_projection(got, ref, act, what=""):
     rel = err / np.maximum(np.abs(ref).max(axis=(2, 3)), 1e-30)
     worst = tuple(int(i) for i in np.unravel_index(int(rel.argmax()), rel.shape))
     assert rel.max() <= tol, f"{what}: (sequence, head) {worst} relative error {rel.max():.2e}"
+
+
+def floor_act(x, act):
+    """Largest value of the activation dtype that is <= x (x in fp64)."""
+    x = np.asarray(x, dtype=np.float64)
+    f = x.astype(np.float32)
+    f = np.where(f.astype(np.float64) > x, np.nextafter(f, np.float32(-np.inf)), f)
+    f = np.asarray(f, dtype=np.float32)
+    if act == "f32":
+        return f.astype(np.float64)
+    bits = f.view(np.uint32)
+    t = bits & np.uint32(0xFFFF0000)             # bf16 truncation (toward zero)
+    t = np.where((f < 0) & (t != bits), t + np.uint32(0x10000), t).astype(np.uint32)
+    return t.view(np.float32).astype(np.float64)
+
+
+def ceil_act(x, act):
+    return -floor_act(-np.asarray(x, dtype=np.float64), act)
+
+
+def check_attention(got, ref, act, what=""):
+    """The literal bound on the unrounded result: `got` (in the activation
+    dtype) must be a rounding, up or down, of some value within atol of the
+    fp64 oracle, i.e. lie between the dtype's neighbours of ref - atol and
+    ref + atol.  atol is 2e-2 for bf16 and 1e-4 for fp32 outputs."""
+    atol = 1e-4 if act == "f32" else 2e-2
+    lo, hi = floor_act(ref - atol, act), ceil_act(ref + atol, act)
+    bad = (got < lo) | (got > hi)
+    if bad.any():
+        i = np.unravel_index(int(np.argmax(np.abs(got - ref))), got.shape)
+        raise AssertionError(f"{what}: {int(bad.sum())} outputs outside the bound; worst "
+                             f"{got[i]:.6g} vs oracle {ref[i]:.6g} at {tuple(int(j) for j in i)}")

@@ -6,7 +6,10 @@ against the oracle.
 The fused kernel sums the projection in its own order, so its q/k/v may
 differ from the separate calls' by a bf16 rounding step; each path's packed
 planes are checked bit for bit against an oracle cache fed that path's own
-keys and values, and each path's attention against the oracle."""
+keys and values, and each path's attention against the oracle: the bf16
+output must be a rounding of a value within max-abs 2e-2 of the fp64 oracle
+(the d_in 2048 cases give outputs of magnitude 4-8, where one bf16 step is
+0.03)."""
 import numpy as np
 import pytest
 import torch
@@ -14,7 +17,7 @@ import torch
 from oracle import kvq_oracle as O
 from paper_2609_04263_gb300 import synth
 from tests.gpu_common import require_gpu
-from tests.helpers import FORMATS, check_projection, compare_planes, oracle_cache
+from tests.helpers import FORMATS, check_attention, check_projection, compare_planes, oracle_cache
 
 pytestmark = pytest.mark.gpu
 
@@ -118,10 +121,8 @@ def test_decode_step_matches_separate_calls(fmt_name, B, d_in, Hq, Hkv, D, r, pr
         oc_r.append(k2.float().cpu().numpy(), v2.float().cpu().numpy())
         ref_f = O.attend(oc_f, qkv[0].float().cpu().numpy())
         ref_r = O.attend(oc_r, q2.float().cpu().numpy())
-        err_f = np.abs(out.float().cpu().numpy() - ref_f).max()
-        err_r = np.abs(o2.float().cpu().numpy() - ref_r).max()
-        assert err_f <= 2e-2, f"step {s}: fused attention {err_f:.3e}"
-        assert err_r <= 2e-2, f"step {s}: separate attention {err_r:.3e}"
+        check_attention(out.float().cpu().numpy(), ref_f, "bf16", f"step {s}: fused attention")
+        check_attention(o2.float().cpu().numpy(), ref_r, "bf16", f"step {s}: separate attention")
     assert fused.sync() == Tmax
     compare_planes(fused, oc_f)
     compare_planes(ref, oc_r)

@@ -26,7 +26,7 @@ import torch
 from oracle import kvq_oracle as O
 from paper_2609_04263_gb300 import synth
 from tests.gpu_common import require_gpu
-from tests.helpers import check_projection
+from tests.helpers import check_attention, check_projection
 
 pytestmark = pytest.mark.gpu
 
@@ -34,38 +34,6 @@ pytestmark = pytest.mark.gpu
 @pytest.fixture(scope="module", autouse=True)
 def _gpu():
     require_gpu()
-
-
-def _floor_act(x, act):
-    """Largest value of the activation dtype that is <= x (x in fp64)."""
-    x = np.asarray(x, dtype=np.float64)
-    f = x.astype(np.float32)
-    f = np.where(f.astype(np.float64) > x, np.nextafter(f, np.float32(-np.inf)), f)
-    f = np.asarray(f, dtype=np.float32)
-    if act == "f32":
-        return f.astype(np.float64)
-    bits = f.view(np.uint32)
-    t = bits & np.uint32(0xFFFF0000)             # bf16 truncation (toward zero)
-    t = np.where((f < 0) & (t != bits), t + np.uint32(0x10000), t).astype(np.uint32)
-    return t.view(np.float32).astype(np.float64)
-
-
-def _ceil_act(x, act):
-    return -_floor_act(-np.asarray(x, dtype=np.float64), act)
-
-
-def _check_attention(got, ref, act, what):
-    """The literal bound on the unrounded result: `got` (in the activation
-    dtype) must be a rounding, up or down, of some value within atol of the
-    fp64 oracle, i.e. lie between the dtype's neighbours of ref - atol and
-    ref + atol.  atol is 2e-2 for bf16 and 1e-4 for fp32 outputs."""
-    atol = 1e-4 if act == "f32" else 2e-2
-    lo, hi = _floor_act(ref - atol, act), _ceil_act(ref + atol, act)
-    bad = (got < lo) | (got > hi)
-    if bad.any():
-        i = np.unravel_index(int(np.argmax(np.abs(got - ref))), got.shape)
-        raise AssertionError(f"{what}: {int(bad.sum())} outputs outside the bound; worst "
-                             f"{got[i]:.6g} vs oracle {ref[i]:.6g} at {tuple(int(j) for j in i)}")
 
 
 def _planes_subset(cache, b, h):
@@ -163,7 +131,7 @@ def test_full_size_layer(name):
         qs = q[b:b + 1, heads][:, :, ls].float().cpu().numpy()
         ref = O.attention(qs, kh, vh, np.array(ls), 1.0 / math.sqrt(D))
         got = o[b:b + 1, heads][:, :, ls].float().cpu().numpy()
-        _check_attention(got, ref, act, f"prefill attention (b={b}, kv head {h})")
+        check_attention(got, ref, act, f"prefill attention (b={b}, kv head {h})")
 
     # ---- decode: bench.py's captured kvq_decode_step, replayed Dn times ----
     xs = torch.empty(B, 1, wl.d_in, dtype=dt, device=dev)
@@ -196,7 +164,7 @@ def test_full_size_layer(name):
                 qd = outs[0][b:b + 1, heads].float().cpu().numpy()
                 ref = O.attend(oc, qd)
                 got = od[b:b + 1, heads].float().cpu().numpy()
-                _check_attention(got, ref, act, f"decode step {s} (b={b}, kv head {h})")
+                check_attention(got, ref, act, f"decode step {s} (b={b}, kv head {h})")
     assert cache.sync() == wl.max_tokens
     # the planes the decode steps wrote, against oracle caches fed the steps' own k, v
     for (b, h), oc in ocs.items():
