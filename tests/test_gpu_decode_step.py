@@ -3,8 +3,10 @@ cooperative kernel for bf16 affine/symmetric caches) against the three
 separate calls, step after step and replayed from a captured graph, and both
 against the oracle.
 
-The fused kernel sums the projection in its own order, so its q/k/v may
-differ from the separate calls' by a bf16 rounding step; each path's packed
+The fused kernel sums the projection (and its rank-r branch) in its own
+order and precision, so its q/k/v may differ from the separate calls' in the
+last bits; each path's q/k/v is checked against the oracle projection per
+(sequence, head), each path's packed
 planes are checked bit for bit against an oracle cache fed that path's own
 keys and values, and each path's attention against the oracle: the bf16
 output must be a rounding of a value within max-abs 2e-2 of the fp64 oracle
@@ -41,12 +43,6 @@ CASES = [
     ("kivi2", 2, 256, 8, 2, 128, 16, 100, False),    # three calls
     ("affine4_g128", 2, 256, 4, 2, 256, 16, 100, False),
 ]
-
-
-def _bf16_close(a, b):
-    """Equal up to one bf16 rounding of the fp32 result."""
-    a, b = a.float(), b.float()
-    return bool(((a - b).abs() <= 2.0 ** -7 * torch.maximum(a.abs(), b.abs()) + 1e-6).all())
 
 
 @pytest.mark.parametrize("fmt_name,B,d_in,Hq,Hkv,D,r,prefill,fused_expected", CASES)
@@ -110,13 +106,12 @@ def test_decode_step_matches_separate_calls(fmt_name, B, d_in, Hq, Hkv, D, r, pr
         ref.append(k2, v2)
         o2 = ref.attend_decode(q2)
         torch.cuda.synchronize()
-        for a_, b_, name in zip(qkv, (q2, k2, v2), "qkv"):
-            assert _bf16_close(a_, b_), f"step {s}: {name} differs beyond one bf16 rounding"
-        # the fused step's own q, k, v against the oracle projection
+        # each path's q, k, v against the oracle projection, per head
         ref_p = O.project_lora(xs.float().cpu().numpy(), nw, nl, 2.0, Hq, Hkv, D,
                                pos0=prefill + s, rope_base=10000.0)
-        for a_, r_, name in zip(qkv, ref_p, "qkv"):
+        for a_, b_, r_, name in zip(qkv, (q2, k2, v2), ref_p, "qkv"):
             check_projection(a_.float().cpu().numpy(), r_, "bf16", f"step {s} fused {name}")
+            check_projection(b_.float().cpu().numpy(), r_, "bf16", f"step {s} separate {name}")
         oc_f.append(qkv[1].float().cpu().numpy(), qkv[2].float().cpu().numpy())
         oc_r.append(k2.float().cpu().numpy(), v2.float().cpu().numpy())
         ref_f = O.attend(oc_f, qkv[0].float().cpu().numpy())
