@@ -522,6 +522,11 @@ int decode_splits(const Geom& g) {
 
 cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
                           bool decode, int t_hint, cudaStream_t s) {
+  if (!decode && prefill_m256_supported(g)) {
+    int* err = device_error_word();
+    if (!err) return cudaErrorInvalidDevice;
+    return launch_prefill_m256(g, q, L, scale, out, err, s);
+  }
   if (!decode && prefill_tc_supported(g)) {
     int* err = device_error_word();
     if (!err) return cudaErrorInvalidDevice;

@@ -153,6 +153,10 @@ bool decode_mma_supported(const Geom& g);
 bool prefill_tc_supported(const Geom& g);
 cudaError_t launch_prefill_tc(const Geom& g, const void* q, int L, float scale, void* out,
                               int* err, cudaStream_t s);
+// tcgen05 causal prefill with 256 query rows per CTA (attend_prefill_m256.cu).
+bool prefill_m256_supported(const Geom& g);
+cudaError_t launch_prefill_m256(const Geom& g, const void* q, int L, float scale, void* out,
+                                int* err, cudaStream_t s);
 bool prefill_mma_supported(const Geom& g);
 cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale, void* out,
                                cudaStream_t s);
