@@ -99,13 +99,13 @@ PREFILL = [
     ("sym4", "bf16", 2, 1, 6, 128, [37], 90),        # group 6 does not divide the rows
     ("affine4", "bf16", 1, 1, 2, 256, [50], 333),
     # head_dim 128 on the 256-row tensor-core kernel: several 64-token KV
-    # tiles, GQA 1 (the two query tiles at different positions), 4 and 32
-    # (8 queries per CTA), a KIVI residual window inside the last tiles, a
+    # tiles, GQA 1 (the two query tiles at different positions), 4 and 16
+    # (16 queries per CTA), a KIVI residual window inside the last tiles, a
     # prefill shorter than one tile
     ("affine4", "bf16", 2, 2, 8, 128, [300], 700),
     ("kivi2", "bf16", 1, 2, 8, 128, [0], 1000),
     ("kivi2", "bf16", 2, 1, 1, 128, [64], 333),
-    ("sym2", "bf16", 1, 1, 32, 128, [0], 200),
+    ("sym2", "bf16", 1, 1, 16, 128, [0], 200),
     ("affine2", "bf16", 1, 2, 4, 128, [0], 40),
     ("sym4", "bf16", 1, 2, 8, 128, [500], 129),
 ]
