@@ -16,10 +16,12 @@
 //     (code x scale + offset, one rounding), into double-buffered shared
 //     tiles in the 128-byte-swizzled K-major layout of the MMA descriptors
 //     (V transposed: D rows, tokens along K);
-//   issuer (warp 12, one thread): S_X = Q_X K_hi^T + Q_X K_lo^T for X = A, B
-//     into double-buffered TMEM tiles (128 x 64 fp32), then, one KV tile
-//     behind, O_X += P_X V into a TMEM accumulator (128 x D fp32) per query
-//     tile; completions are signalled by tcgen05.commit on mbarriers;
+//   issuer (warp 12, one thread): per KV tile j, first O_X += P_X V of tile
+//     j - 1 into a TMEM accumulator (128 x D fp32) per query tile X = A, B
+//     (this frees tile j - 1's K/V buffer, so the producers run a tile
+//     ahead), then S_X = Q_X K_hi^T + Q_X K_lo^T of tile j into
+//     double-buffered TMEM tiles (128 x 64 fp32); completions are signalled
+//     by tcgen05.commit on mbarriers;
 //   softmax A (warps 0-3) and B (warps 4-7): thread r owns row r of its
 //     query tile (TMEM lane r): reads the 64 scores, masks causally, keeps
 //     the running maximum m and sum l in log2 units, writes P as fp16 into
@@ -40,11 +42,13 @@ using namespace tc;
 constexpr int kM = 128;              // rows per query tile (MMA M)
 constexpr int kTok = 64;             // tokens per KV tile
 constexpr int kRowsCta = 2 * kM;     // query rows per CTA
-constexpr int kThreads = 13 * 32;    // 8 softmax warps, 4 producer warps, 1 issuer warp
+constexpr int kThreads = 14 * 32;    // 8 softmax, 4 producer, 1 issuer, 1 loader warp
+constexpr int kKvBufs = 2;           // reconstructed K/V tile buffers
+constexpr int kRaw = 3;              // packed-tile stages (bulk copies run up to 3 tiles ahead)
 constexpr float kRescale = 8.f;      // log2 growth of a row maximum that forces a rescale
 
 // Shared memory (bytes from a 1024-aligned base).
-template <int D>
+template <int D, int BITS>
 struct M256Layout {
   static constexpr int QT = kM * D * 2;             // one query tile: D/64 atoms of 16 KB
   static constexpr int Q_OFF = 0;
@@ -53,11 +57,17 @@ struct M256Layout {
   static constexpr int KL = kTok * D * 2;           // K lo: the same
   static constexpr int VT = 2 * kTok * D * 2;       // V^T: D rows x 128 B (64 tokens)
   static constexpr int KV_B = VT + D * 128;
-  static constexpr int P_OFF = KV_OFF + 2 * KV_B;   // P of tile A, then of tile B
-  static constexpr int P_B = kM * kTok * 2;         // 128 rows x 128 B (fp16)
-  static constexpr int SC_OFF = P_OFF + 2 * P_B;    // KIVI key block scales, 2 buffers
-  static constexpr int SC_B = 2 * 2 * D * 2;        // 2 blocks x (scale, zero) x D fp16
-  static constexpr int TOTAL = SC_OFF + 2 * SC_B;
+  // packed tile as stored in the cache planes: 64 code rows of K and of V,
+  // then four metadata pieces of 4 D bytes each (per-token group scales and
+  // offsets of 64 tokens, or KIVI's per-channel scales and offsets of the
+  // tile's two 32-token key blocks)
+  static constexpr int CROW = D * BITS / 8;         // code bytes per token
+  static constexpr int RKC = 0, RVC = kTok * CROW;
+  static constexpr int RKS = 2 * kTok * CROW, RKZ = RKS + 4 * D, RVS = RKZ + 4 * D,
+                       RVZ = RVS + 4 * D;
+  static constexpr int RAW_B = RVZ + 4 * D;
+  static constexpr int RAW_OFF = KV_OFF + kKvBufs * KV_B;
+  static constexpr int TOTAL = RAW_OFF + kRaw * RAW_B;
   static constexpr int ALLOC = TOTAL + 1024;        // alignment slack
 };
 
@@ -71,6 +81,30 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// Packed fp32 pairs (two lanes of one 64-bit register).
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
 }
 
 __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
@@ -89,6 +123,42 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t r[16]) 
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// D (+)= A B with A (M x 16, 16-bit elements packed two per 32-bit column)
+// read from tensor memory and B from shared memory.
+__device__ __forceinline__ void umma_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n"
+      ::"r"(tmem_d), "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+// True in exactly one lane of the (fully active) warp.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t p;
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n selp.u32 %0, 1, 0, e;\n}\n"
+      : "=r"(p));
+  return p != 0;
+}
+
+// Non-blocking probe of an mbarrier phase.
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ void bulk_copy(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
 
 // Bounded mbarrier wait whose result is the same in every lane of the warp
@@ -110,169 +180,136 @@ __device__ __forceinline__ bool producers_all(bool ok) {
   return r != 0;
 }
 
-// What one producer thread loads for one KV tile ahead of its use.
-//   K: token tk of the tile, channel half hf (D/2 channels): its code words,
-//      and (affine/symmetric) the token's fp16 group scales and offsets of
-//      that half; (KIVI) one 16-byte piece of the tile's per-channel block
-//      scales, staged in shared memory for all producers.
-//   V: tokens 8 tb .. 8 tb + 7 of the tile, channels CV vq .. CV vq + CV - 1
-//      (CV = D/16): each token's code word of those channels and its group
-//      scale and offset, paired by token for half2 arithmetic.
-template <int D, int BITS>
-struct TileCodes {
-  static constexpr int NKW = D / 2 * BITS / 32;      // K code words per thread
-  uint32_t kw[NKW];
-  uint32_t ks, kz;                                   // fp16 pairs (groups of the half)
-  uint4 stage;                                       // KIVI block scales piece
-  uint32_t vw[8];                                    // V code word per token
-  uint32_t vs[4], vz[4];                             // half2 (token 2i, 2i + 1)
-};
-
-// Where a tile's tokens come from: codes (t < tq), the KIVI residual ring
-// (tq <= t < T) or nothing (t >= T: zeros).
+// Bytes of one packed tile the loader copies (codes of K and V, metadata).
 template <int D, int BITS, int FMT>
-__device__ __forceinline__ void load_tile(const Geom& g, int b, int h, int t0, int T, int tq,
-                                          int tid, TileCodes<D, BITS>& r) {
-  constexpr bool KIVI = FMT == KVQ_FMT_KIVI;
-  constexpr bool SYM = FMT == KVQ_FMT_SYMMETRIC;
-  constexpr int CV = D / 16;
-  const int tk = tid & 63, hf = tid >> 6;
-  const int t = t0 + tk;
-  // ---- K ----
-  if (t < tq) {
-    const uint8_t* row = plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t) + hf * (D / 2 * BITS / 8);
-    if constexpr (TileCodes<D, BITS>::NKW >= 4) {
-#pragma unroll
-      for (int i = 0; i < TileCodes<D, BITS>::NKW / 4; ++i) {
-        const uint4 u = __ldg(reinterpret_cast<const uint4*>(row) + i);
-        r.kw[4 * i] = u.x; r.kw[4 * i + 1] = u.y; r.kw[4 * i + 2] = u.z; r.kw[4 * i + 3] = u.w;
-      }
-    } else {
-      const uint2 u = __ldg(reinterpret_cast<const uint2*>(row));
-      r.kw[0] = u.x; r.kw[1] = u.y;
-    }
-    if constexpr (!KIVI) {
-      // groups of 32 channels: D/64 groups in this half
-      const __half* sp = plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t, hf * (D / 64));
-      if constexpr (D == 128) {
-        r.ks = __ldg(reinterpret_cast<const uint32_t*>(sp));
-        r.kz = SYM ? 0u : __ldg(reinterpret_cast<const uint32_t*>(
-                              plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t, hf * 2)));
-      } else {
-        r.ks = __half_as_ushort(__ldg(sp));
-        r.kz = SYM ? 0u : __half_as_ushort(__ldg(plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t, hf)));
-      }
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < TileCodes<D, BITS>::NKW; ++i) r.kw[i] = 0;
-    r.ks = r.kz = 0;
-  }
-  if constexpr (KIVI) {
-    // staged block scales: [block 0, 1][scale, zero][D] fp16 = 4 D / 8 pieces
-    r.stage = make_uint4(0, 0, 0, 0);
-    if (tid < 4 * D / 8) {
-      const int blk = tid / (2 * D / 8), rem = tid % (2 * D / 8);
-      const int sz = rem / (D / 8), ch = rem % (D / 8);
-      const int tb0 = t0 + 32 * blk;
-      if (tb0 < tq)
-        r.stage = __ldg(reinterpret_cast<const uint4*>(
-            plane_ptr<__half>(g, sz ? KVQ_PLANE_K_ZERO : KVQ_PLANE_K_SCALE, b, h, tb0 / 32, 8 * ch)));
-    }
-  }
-  // ---- V ----
-  const int tb = tid & 7, vq = tid >> 3;
-  const int grp_v = vq * CV / 32;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int tv = t0 + 8 * tb + i;
-    uint32_t w = 0;
-    __half s = __ushort_as_half(0), z = __ushort_as_half(0);
-    if (tv < tq) {
-      const uint8_t* row = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, tv) + vq * (CV * BITS / 8);
-      if constexpr (CV * BITS == 32) w = __ldg(reinterpret_cast<const uint32_t*>(row));
-      else if constexpr (CV * BITS == 16) w = __ldg(reinterpret_cast<const unsigned short*>(row));
-      else w = __ldg(row);
-      s = __ldg(plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, tv, grp_v));
-      z = SYM ? __hmul(s, __float2half_rn(-(float)(1 << (BITS - 1))))
-              : __ldg(plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, tv, grp_v));
-    }
-    r.vw[i] = w;
-    if (i & 1) {
-      r.vs[i >> 1] |= (uint32_t)__half_as_ushort(s) << 16;
-      r.vz[i >> 1] |= (uint32_t)__half_as_ushort(z) << 16;
-    } else {
-      r.vs[i >> 1] = __half_as_ushort(s);
-      r.vz[i >> 1] = __half_as_ushort(z);
-    }
-  }
+__host__ __device__ constexpr int raw_bytes() {
+  return 2 * kTok * (D * BITS / 8) + (FMT == KVQ_FMT_SYMMETRIC ? 2 : 4) * 4 * D;
 }
 
-// K: 8 channels (chunk c of this thread's half) reconstructed in fp32 and
-// split into bf16 high (truncation) and low (rounded remainder) parts.
-__device__ __forceinline__ void split_store(float (&k)[8], unsigned char* hi_dst,
+// Loader: the packed rows of tile t0 .. t0 + 63 of every plane the tile
+// reads, one bulk copy per plane.  Planes hold whole 64-row tiles (their
+// row counts are padded to multiples of 64), so a tile reaching past the
+// stored tokens copies rows that are never used.
+template <int D, int BITS, int FMT>
+__device__ __forceinline__ void load_raw(const Geom& g, int b, int h, int t0, unsigned char* raw,
+                                         uint64_t* bar) {
+  using S = M256Layout<D, BITS>;
+  constexpr uint32_t CB = kTok * S::CROW;
+  mbar_expect_tx(bar, raw_bytes<D, BITS, FMT>());
+  bulk_copy(raw + S::RKC, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0), CB, bar);
+  bulk_copy(raw + S::RVC, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t0), CB, bar);
+  const int krow = FMT == KVQ_FMT_KIVI ? t0 / 32 : t0;   // KIVI: two key blocks of D channels
+  bulk_copy(raw + S::RKS, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, krow), 4 * D, bar);
+  if (FMT != KVQ_FMT_SYMMETRIC)
+    bulk_copy(raw + S::RKZ, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, krow), 4 * D, bar);
+  bulk_copy(raw + S::RVS, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, t0), 4 * D, bar);
+  if (FMT != KVQ_FMT_SYMMETRIC)
+    bulk_copy(raw + S::RVZ, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, t0), 4 * D, bar);
+}
+
+// K: 8 channels reconstructed in fp32 and split into a bf16 high part (the
+// value truncated) and the bf16 of the remainder.
+__device__ __forceinline__ void split_store(const uint64_t (&k2)[4], unsigned char* hi_dst,
                                             unsigned char* lo_dst) {
   uint32_t h[4], l[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint32_t a = __float_as_uint(k[2 * i]), c = __float_as_uint(k[2 * i + 1]);
-    h[i] = __byte_perm(a, c, 0x7632);
-    const float ra = k[2 * i] - __uint_as_float(a & 0xFFFF0000u);
-    const float rc = k[2 * i + 1] - __uint_as_float(c & 0xFFFF0000u);
+    float a, c;
+    f2unpack(k2[i], a, c);
+    const uint32_t ab = __float_as_uint(a) & 0xFFFF0000u, cb = __float_as_uint(c) & 0xFFFF0000u;
+    h[i] = __byte_perm(ab, cb, 0x7632);
+    float ra, rc;
+    f2unpack(fadd2(k2[i], f2pack(-__uint_as_float(ab), -__uint_as_float(cb))), ra, rc);
     l[i] = pack_bf16(ra, rc);
   }
   *reinterpret_cast<uint4*>(hi_dst) = make_uint4(h[0], h[1], h[2], h[3]);
   *reinterpret_cast<uint4*>(lo_dst) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
+// Code e of a word of BITS-bit codes as an exact float plus 2^23.
 template <int BITS>
-__device__ __forceinline__ float code_f(uint32_t w, int e) {
+__device__ __forceinline__ float code_biased(uint32_t w, int e) {
   constexpr uint32_t mask = (1u << BITS) - 1;
-  return __uint_as_float(0x4B000000u | ((w >> (e * BITS)) & mask)) - 8388608.f;
+  return __uint_as_float(0x4B000000u | ((w >> (e * BITS)) & mask));
 }
 
+// Producers: reconstruct the K and V operand tiles of KV tile t0 from the
+// packed tile in `raw` (tokens below tq), the KIVI residual ring (tq <= t <
+// T) or zeros (t >= T).
+//   K: thread (tk = tid % 64, hf = tid / 64): token tk, channels of half hf.
+//   V: thread (tb = tid % 8, vq = tid / 8): tokens 8 tb .. 8 tb + 7 and
+//      channels CV vq .. CV vq + CV - 1 (CV = D / 16), in half2 arithmetic,
+//      stored as D rows of the transposed tile (one 16-byte chunk per row).
 template <int D, int BITS, int FMT>
 __device__ __forceinline__ void build_tile(const Geom& g, int b, int h, int t0, int T, int tq,
-                                           int tid, const TileCodes<D, BITS>& r,
-                                           const unsigned char* stage, unsigned char* kv) {
-  using S = M256Layout<D>;
+                                           int tid, const unsigned char* raw, unsigned char* kv) {
+  using S = M256Layout<D, BITS>;
   constexpr bool KIVI = FMT == KVQ_FMT_KIVI;
   constexpr bool SYM = FMT == KVQ_FMT_SYMMETRIC;
   constexpr int CV = D / 16;
   constexpr int NCH = D / 16;                     // K chunks of 8 channels per thread
+  constexpr int NKW = D / 2 * BITS / 32;          // K code words per thread
   const int tk = tid & 63, hf = tid >> 6;
   const int t = t0 + tk;
   // ---- K tile ----
-  if (!KIVI || t < tq) {
+  if (t < tq) {
+    uint32_t kw[NKW];
+    const unsigned char* cp = raw + S::RKC + tk * S::CROW + hf * (S::CROW / 2);
+    if constexpr (NKW >= 4) {
+#pragma unroll
+      for (int i = 0; i < NKW / 4; ++i) {
+        const uint4 u = *reinterpret_cast<const uint4*>(cp + 16 * i);
+        kw[4 * i] = u.x; kw[4 * i + 1] = u.y; kw[4 * i + 2] = u.z; kw[4 * i + 3] = u.w;
+      }
+    } else {
+      const uint2 u = *reinterpret_cast<const uint2*>(cp);
+      kw[0] = u.x; kw[1] = u.y;
+    }
+    uint32_t ks = 0, kz = 0;                      // affine/symmetric: the half's group metadata
+    if constexpr (!KIVI) {
+      const unsigned char* sp = raw + S::RKS + tk * (D / 16) + hf * (D / 32);
+      if constexpr (D == 128) {
+        ks = *reinterpret_cast<const uint32_t*>(sp);
+        if (!SYM) kz = *reinterpret_cast<const uint32_t*>(sp + (S::RKZ - S::RKS));
+      } else {
+        ks = *reinterpret_cast<const unsigned short*>(sp);
+        if (!SYM) kz = *reinterpret_cast<const unsigned short*>(sp + (S::RKZ - S::RKS));
+      }
+    }
+    const uint64_t bias2 = f2pack(-8388608.f, -8388608.f);
 #pragma unroll
     for (int c = 0; c < NCH; ++c) {
       const int cc = hf * NCH + c;                // chunk along D
       constexpr int CB = 8 * BITS;                // code bits per chunk
-      const uint32_t w = (r.kw[(c * CB) / 32] >> ((c * CB) % 32));
-      float k[8];
+      const uint32_t w = kw[(c * CB) / 32] >> ((c * CB) % 32);
+      uint64_t k2[4];
       if constexpr (KIVI) {
-        const unsigned char* st = stage + (tk >> 5) * (4 * D) + cc * 16;
+        const unsigned char* st = raw + S::RKS + (tk >> 5) * (2 * D) + cc * 16;
         const uint4 su = *reinterpret_cast<const uint4*>(st);
-        const uint4 zu = *reinterpret_cast<const uint4*>(st + 2 * D);
+        const uint4 zu = *reinterpret_cast<const uint4*>(st + (S::RKZ - S::RKS));
         const __half2* s2 = reinterpret_cast<const __half2*>(&su);
         const __half2* z2 = reinterpret_cast<const __half2*>(&zu);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const float2 sf = __half22float2(s2[i]), zf = __half22float2(z2[i]);
-          k[2 * i] = fmaf(code_f<BITS>(w, 2 * i), sf.x, zf.x);
-          k[2 * i + 1] = fmaf(code_f<BITS>(w, 2 * i + 1), sf.y, zf.y);
+          const uint64_t c2 = fadd2(f2pack(code_biased<BITS>(w, 2 * i), code_biased<BITS>(w, 2 * i + 1)), bias2);
+          k2[i] = ffma2(c2, f2pack(sf.x, sf.y), f2pack(zf.x, zf.y));
         }
       } else {
         const int gi = (c * 8) / 32;              // group within the half
-        const __half2 s2 = *reinterpret_cast<const __half2*>(&r.ks);
-        const __half2 z2 = *reinterpret_cast<const __half2*>(&r.kz);
+        const __half2 s2 = *reinterpret_cast<const __half2*>(&ks);
+        const __half2 z2 = *reinterpret_cast<const __half2*>(&kz);
         const float s = gi ? __high2float(s2) : __low2float(s2);
         const float m = SYM ? -(float)(1 << (BITS - 1)) * s : (gi ? __high2float(z2) : __low2float(z2));
+        const uint64_t ss = f2pack(s, s), mm = f2pack(m, m);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) k[e] = fmaf(code_f<BITS>(w, e), s, m);
+        for (int i = 0; i < 4; ++i) {
+          const uint64_t c2 = fadd2(f2pack(code_biased<BITS>(w, 2 * i), code_biased<BITS>(w, 2 * i + 1)), bias2);
+          k2[i] = ffma2(c2, ss, mm);
+        }
       }
       unsigned char* base = kv + (cc >> 3) * (kTok * 128);
-      split_store(k, base + S::KH + sw128(tk, cc & 7), base + S::KL + sw128(tk, cc & 7));
+      split_store(k2, base + S::KH + sw128(tk, cc & 7), base + S::KL + sw128(tk, cc & 7));
     }
   } else {
     // KIVI residual window (full precision) or beyond the cache (zeros)
@@ -280,7 +317,7 @@ __device__ __forceinline__ void build_tile(const Geom& g, int b, int h, int t0, 
     for (int c = 0; c < NCH; ++c) {
       const int cc = hf * NCH + c;
       uint4 u = make_uint4(0, 0, 0, 0);
-      if (t < T)
+      if (KIVI && t < T)
         u = *reinterpret_cast<const uint4*>(
             plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_K_FULL, b, h, t % g.ring, 8 * cc));
       unsigned char* base = kv + (cc >> 3) * (kTok * 128);
@@ -290,21 +327,43 @@ __device__ __forceinline__ void build_tile(const Geom& g, int b, int h, int t0, 
   }
   // ---- V^T tile: rows d = CV vq + e, 16-byte chunk tb (tokens 8 tb ..) ----
   const int tb = tid & 7, vq = tid >> 3;
+  const int grp_v = vq * CV / 32;
   uint32_t out[CV][4];
   const __half2 bias = __float2half2_rn(1024.f);
 #pragma unroll
   for (int p = 0; p < 4; ++p) {                   // token pair (2p, 2p + 1)
-    const uint32_t w0 = r.vw[2 * p], w1 = r.vw[2 * p + 1];
+    uint32_t w2[2], s2u, z2u;
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int tv = 8 * tb + 2 * p + u;          // token within the tile
+      const unsigned char* cp = raw + S::RVC + tv * S::CROW + vq * (CV * BITS / 8);
+      if constexpr (CV * BITS == 32) w2[u] = *reinterpret_cast<const uint32_t*>(cp);
+      else if constexpr (CV * BITS == 16) w2[u] = *reinterpret_cast<const unsigned short*>(cp);
+      else w2[u] = *cp;
+    }
+    {
+      const int tv = 8 * tb + 2 * p;
+      const unsigned short* sp = reinterpret_cast<const unsigned short*>(raw + S::RVS) + tv * (D / 32) + grp_v;
+      s2u = (uint32_t)sp[0] | ((uint32_t)sp[D / 32] << 16);
+      if constexpr (SYM) {
+        const __half2 z = __hmul2(*reinterpret_cast<const __half2*>(&s2u),
+                                  __float2half2_rn(-(float)(1 << (BITS - 1))));
+        z2u = *reinterpret_cast<const uint32_t*>(&z);
+      } else {
+        const unsigned short* zp = reinterpret_cast<const unsigned short*>(raw + S::RVZ) + tv * (D / 32) + grp_v;
+        z2u = (uint32_t)zp[0] | ((uint32_t)zp[D / 32] << 16);
+      }
+    }
     uint32_t pw[2];
     if constexpr (CV * BITS == 32) {
-      pw[0] = __byte_perm(w0, w1, 0x5410);        // low halves: channels 0 .. 16/BITS - 1
-      pw[1] = __byte_perm(w0, w1, 0x7632);
+      pw[0] = __byte_perm(w2[0], w2[1], 0x5410);  // low halves of both tokens
+      pw[1] = __byte_perm(w2[0], w2[1], 0x7632);
     } else {
-      pw[0] = (w0 & 0xFFFFu) | (w1 << 16);
+      pw[0] = (w2[0] & 0xFFFFu) | (w2[1] << 16);
       pw[1] = 0;
     }
-    const __half2 s2 = *reinterpret_cast<const __half2*>(&r.vs[p]);
-    const __half2 z2 = *reinterpret_cast<const __half2*>(&r.vz[p]);
+    const __half2 s2 = *reinterpret_cast<const __half2*>(&s2u);
+    const __half2 z2 = *reinterpret_cast<const __half2*>(&z2u);
 #pragma unroll
     for (int e = 0; e < CV; ++e) {
       constexpr uint32_t m2 = ((1u << BITS) - 1) * 0x00010001u;
@@ -314,35 +373,32 @@ __device__ __forceinline__ void build_tile(const Geom& g, int b, int h, int t0, 
       out[e][p] = *reinterpret_cast<const uint32_t*>(&v2);
     }
   }
-  if constexpr (KIVI) {
-    // tokens of the residual window (or beyond the cache) replace their pair halves
-    const int tv0 = t0 + 8 * tb;
-    if (tv0 + 7 >= tq) {
+  // tokens of the KIVI residual window, or beyond the cache, replace theirs
+  const int tv0 = t0 + 8 * tb;
+  if (tv0 + 7 >= tq) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int tv = tv0 + i;
-        if (tv < tq) continue;
-        uint4 raw[CV / 8 > 0 ? CV / 8 : 1];
-        __nv_bfloat16 vals[CV];
-        if (tv < T) {
-          const __nv_bfloat16* src = plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, h, tv % g.ring, vq * CV);
-          if constexpr (CV == 8) {
-            raw[0] = *reinterpret_cast<const uint4*>(src);
-            memcpy(vals, raw, sizeof(vals));
-          } else {
-            const uint2 u = *reinterpret_cast<const uint2*>(src);
-            memcpy(vals, &u, sizeof(vals));
-          }
+    for (int i = 0; i < 8; ++i) {
+      const int tv = tv0 + i;
+      if (tv < tq) continue;
+      __nv_bfloat16 vals[CV];
+      if (KIVI && tv < T) {
+        const __nv_bfloat16* src = plane_ptr<__nv_bfloat16>(g, KVQ_PLANE_V_FULL, b, h, tv % g.ring, vq * CV);
+        if constexpr (CV == 8) {
+          const uint4 u = *reinterpret_cast<const uint4*>(src);
+          memcpy(vals, &u, sizeof(vals));
         } else {
-#pragma unroll
-          for (int e = 0; e < CV; ++e) vals[e] = __float2bfloat16_rn(0.f);
+          const uint2 u = *reinterpret_cast<const uint2*>(src);
+          memcpy(vals, &u, sizeof(vals));
         }
+      } else {
 #pragma unroll
-        for (int e = 0; e < CV; ++e) {
-          const uint32_t hv = __half_as_ushort(__float2half_rn(__bfloat162float(vals[e])));
-          out[e][i >> 1] = (i & 1) ? ((out[e][i >> 1] & 0xFFFFu) | (hv << 16))
-                                   : ((out[e][i >> 1] & 0xFFFF0000u) | hv);
-        }
+        for (int e = 0; e < CV; ++e) vals[e] = __float2bfloat16_rn(0.f);
+      }
+#pragma unroll
+      for (int e = 0; e < CV; ++e) {
+        const uint32_t hv = __half_as_ushort(__float2half_rn(__bfloat162float(vals[e])));
+        out[e][i >> 1] = (i & 1) ? ((out[e][i >> 1] & 0xFFFFu) | (hv << 16))
+                                 : ((out[e][i >> 1] & 0xFFFF0000u) | hv);
       }
     }
   }
@@ -358,12 +414,12 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
                            __nv_bfloat16* __restrict__ out, int nq, int* err) {
   pdl_wait();
   pdl_trigger();
-  using S = M256Layout<D>;
+  using S = M256Layout<D, BITS>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ uint64_t kv_full[2], kv_free[2], s_full[2][2], s_free[2][2], p_full[2], pv_done[2],
-      done_bar;
+  __shared__ uint64_t raw_full[kRaw], raw_free[kRaw], kv_full[kKvBufs], kv_free[kKvBufs],
+      s_full[2][2], p_full[2][2], s_free[2][2], done_bar;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
 
@@ -382,16 +438,20 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
   volatile int* abort = &abort_flag;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kRaw; ++i) {
+      mbar_init(&raw_full[i], 1);
+      mbar_init(&raw_free[i], 128);
+    }
+    for (int i = 0; i < kKvBufs; ++i) {
       mbar_init(&kv_full[i], 128);
       mbar_init(&kv_free[i], 1);
-      mbar_init(&p_full[i], 128);
-      mbar_init(&pv_done[i], 1);
-      for (int x = 0; x < 2; ++x) {
-        mbar_init(&s_full[x][i], 1);
-        mbar_init(&s_free[x][i], 128);
-      }
     }
+    for (int x = 0; x < 2; ++x)
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&s_full[x][i], 1);
+        mbar_init(&p_full[x][i], 128);
+        mbar_init(&s_free[x][i], 1);
+      }
     mbar_init(&done_bar, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -424,84 +484,132 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
   tc_fence_after();
   const uint32_t tmem = tmem_base;
 
-  if (warp >= 8 && warp < 12) {
+  if (warp == 13) {
+    // ---------------- loader: packed tiles into the raw ring ----------------
+    if (lane == 0) {
+      int issued = 0;
+      for (int j = 0; j < ntiles; ++j) {
+        const int st = j % kRaw;
+        if (j >= kRaw && !mbar_wait_or_abort(&raw_free[st], ((j - kRaw) / kRaw) & 1, abort)) break;
+        load_raw<D, BITS, FMT>(g, b, hkv, j * kTok, smem + S::RAW_OFF + st * S::RAW_B,
+                               &raw_full[st]);
+        issued = j + 1;
+      }
+      // no copy may still be landing in shared memory when the CTA exits
+      // (after a timeout the producers stop consuming): wait, bounded, for
+      // the last tile issued on each stage
+      for (int t = issued > kRaw ? issued - kRaw : 0; t < issued; ++t)
+        if (!mbar_wait(&raw_full[t % kRaw], (t / kRaw) & 1)) *abort = 1;
+    }
+  } else if (warp >= 8 && warp < 12) {
     // ---------------- producers: reconstruct K and V tiles ----------------
     const int tid = threadIdx.x - 256;
-    TileCodes<D, BITS> cur, nxt;
-    load_tile<D, BITS, FMT>(g, b, hkv, 0, T, tq, tid, cur);
     for (int j = 0; j < ntiles; ++j) {
-      const int bf = j & 1;
-      unsigned char* stage = smem + S::SC_OFF + bf * S::SC_B;
-      if (FMT == KVQ_FMT_KIVI && tid < 4 * D / 8)
-        *reinterpret_cast<uint4*>(stage + 16 * tid) = cur.stage;
-      const bool ok = j < 2 || mbar_wait_or_abort(&kv_free[bf], ((j - 2) >> 1) & 1, abort);
-      if (!producers_all(ok)) break;                  // also publishes the staged scales
-      if (j + 1 < ntiles) load_tile<D, BITS, FMT>(g, b, hkv, (j + 1) * kTok, T, tq, tid, nxt);
-      unsigned char* kv = smem + S::KV_OFF + bf * S::KV_B;
-      build_tile<D, BITS, FMT>(g, b, hkv, j * kTok, T, tq, tid, cur, stage, kv);
+      const int st = j % kRaw, kb = j % kKvBufs;
+      bool ok = mbar_wait_or_abort(&raw_full[st], (j / kRaw) & 1, abort);
+      ok = ok && (j < kKvBufs ||
+                  mbar_wait_or_abort(&kv_free[kb], ((j - kKvBufs) / kKvBufs) & 1, abort));
+      if (!producers_all(ok)) break;
+      unsigned char* kv = smem + S::KV_OFF + kb * S::KV_B;
+      build_tile<D, BITS, FMT>(g, b, hkv, j * kTok, T, tq, tid, smem + S::RAW_OFF + st * S::RAW_B, kv);
+      mbar_arrive(&raw_free[st]);
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_arrive(&kv_full[bf]);
-      cur = nxt;
+      mbar_arrive(&kv_full[kb]);
     }
-  } else if (warp == 12 && lane == 0) {
+  } else if (warp == 12) {
     // ---------------- MMA issuer ----------------
+    // Issues, as soon as each is ready: Q K^T of the next tile for both
+    // query tiles (its K/V tile built, the S buffer's previous P V done),
+    // and P V of each query tile's next tile (its P written).  S runs one
+    // tile ahead of the softmax threads; the tensor pipe executes in issue
+    // order.  The whole warp runs the loop (its values stay warp-uniform)
+    // and one elected lane issues the MMAs and their commits.  Descriptors
+    // are formed once: a K step of 16 elements advances the start address by
+    // 32 bytes (2 in the descriptor's 16-byte units).
     constexpr uint32_t id_qk = idesc_bf16(kM, kTok);
     constexpr uint32_t id_pv = idesc_f16(kM, D);
-    bool ok = true;
-    for (int j = 0; j <= ntiles && ok; ++j) {
-      if (j < ntiles) {
-        const int bf = j & 1;
-        if (!mbar_wait_or_abort(&kv_full[bf], (j >> 1) & 1, abort)) break;
-        const unsigned char* kv = smem + S::KV_OFF + bf * S::KV_B;
-        for (int x = 0; x < 2 && ok; ++x) {
-          if (j >= 2 && !mbar_wait_or_abort(&s_free[x][bf], ((j - 2) >> 1) & 1, abort)) {
-            ok = false;
-            break;
-          }
+    const uint64_t qdesc0 = sw128_desc(smem + S::Q_OFF);
+    const uint64_t kvdesc0 = sw128_desc(smem + S::KV_OFF);   // K/V buffer b: + b KV_B / 16
+    const bool leader = elect_one();
+    int nqk = 0, npv[2] = {0, 0};
+    long idle = 0;
+    uint64_t idle_since = 0;
+    while (npv[0] < ntiles || npv[1] < ntiles) {
+      bool progressed = false;
+      if (nqk < ntiles && nqk <= min(npv[0], npv[1]) + 1) {
+        const int kb = nqk % kKvBufs, bf = nqk & 1;
+        const uint32_t fpar = (nqk >= 2) ? ((nqk - 2) >> 1) & 1 : 0;
+        bool ready = false;
+        if (lane == 0)
+          ready = mbar_test(&kv_full[kb], (nqk / kKvBufs) & 1) &&
+                  (nqk < 2 || (mbar_test(&s_free[0][bf], fpar) && mbar_test(&s_free[1][bf], fpar)));
+        if (__shfl_sync(0xffffffffu, ready, 0)) {
           tc_fence_after();
-          const uint32_t ts = tmem + x * 128 + bf * kTok;
-          const unsigned char* qt = smem + S::Q_OFF + x * S::QT;
+          if (leader) {
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const int a = kk >> 2, k4 = (kk & 3) * 32;
-            const uint64_t qd = sw128_desc(qt + a * (kM * 128) + k4);
-            umma(ts, qd, sw128_desc(kv + S::KH + a * (kTok * 128) + k4), id_qk, kk > 0);
-            umma(ts, qd, sw128_desc(kv + S::KL + a * (kTok * 128) + k4), id_qk, 1);
+            for (int x = 0; x < 2; ++x) {
+              const uint32_t ts = tmem + x * 128 + bf * kTok;
+#pragma unroll
+              for (int kk = 0; kk < D / 16; ++kk) {
+                // Q atom: 128 rows x 128 B (1024 units); K atom: 64 rows x 128 B (512 units)
+                const uint64_t qd = qdesc0 + (uint64_t)(x * (S::QT >> 4) + (kk >> 2) * 1024 + (kk & 3) * 2);
+                const uint64_t kd = kvdesc0 + (uint64_t)(kb * (S::KV_B >> 4) + (kk >> 2) * 512 + (kk & 3) * 2);
+                umma(ts, qd, kd + (S::KH >> 4), id_qk, kk > 0);
+                umma(ts, qd, kd + (S::KL >> 4), id_qk, 1);
+              }
+              umma_commit(&s_full[x][bf]);
+            }
           }
-          umma_commit(&s_full[x][bf]);
+          __syncwarp();
+          ++nqk;
+          progressed = true;
         }
       }
-      if (j >= 1 && ok) {
-        const int jj = j - 1, bf = jj & 1;
-        const unsigned char* kv = smem + S::KV_OFF + bf * S::KV_B;
-        for (int x = 0; x < 2; ++x) {
-          if (!mbar_wait_or_abort(&p_full[x], jj & 1, abort)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const unsigned char* p = smem + S::P_OFF + x * S::P_B;
+#pragma unroll
+      for (int x = 0; x < 2; ++x) {
+        const int j = npv[x];
+        if (j >= nqk) continue;
+        const int bf = j & 1;
+        bool ready = false;
+        if (lane == 0) ready = mbar_test(&p_full[x][bf], (j >> 1) & 1);
+        if (!__shfl_sync(0xffffffffu, ready, 0)) continue;
+        tc_fence_after();
+        const int kb = j % kKvBufs;
+        if (leader) {
+          const uint32_t tp = tmem + x * 128 + bf * kTok;   // P (fp16 pairs) over S's columns
           const uint32_t to = tmem + 256 + x * D;
 #pragma unroll
           for (int kk = 0; kk < kTok / 16; ++kk)
-            umma(to, sw128_desc(p + kk * 32), sw128_desc(kv + S::VT + kk * 32), id_pv,
-                 (jj > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(&pv_done[x]);
+            umma_ts(to, tp + kk * 8, kvdesc0 + (uint64_t)(kb * (S::KV_B >> 4) + (S::VT >> 4) + kk * 2),
+                    id_pv, (j > 0 || kk > 0) ? 1u : 0u);
+          umma_commit(&s_free[x][bf]);           // S/P buffer free, and O holds tile j
+          if (npv[x ^ 1] > j) umma_commit(&kv_free[kb]);   // both query tiles done with it
         }
-        if (ok) umma_commit(&kv_free[bf]);
+        __syncwarp();
+        ++npv[x];
+        progressed = true;
+      }
+      if (progressed) {
+        idle = 0;
+      } else {
+        if (idle == 0) idle_since = global_ns();
+        __nanosleep(20);
+        const bool stop = (++idle & 63) == 0 && (*abort || global_ns() - idle_since > kWaitNs);
+        if (__shfl_sync(0xffffffffu, stop, 0)) break;   // the whole warp leaves together
       }
     }
-    umma_commit(&done_bar);                    // every MMA issued above has completed
-    if (!mbar_wait(&done_bar, 0)) *abort = 1;
+    if (lane == 0 && (npv[0] < ntiles || npv[1] < ntiles)) *abort = 1;
+    if (leader) umma_commit(&done_bar);        // every MMA issued above has completed
+    if (lane == 0 && !mbar_wait(&done_bar, 0)) *abort = 1;
+    __syncwarp();
   } else if (warp < 8) {
     // ---------------- softmax: one row per thread ----------------
     const int x = warp >> 2;                   // query tile
-    const int r = row & 127;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t s_col = tmem + lane_base + x * 128;
     const uint32_t o_col = tmem + lane_base + 256 + x * D;
-    unsigned char* prow = smem + S::P_OFF + x * S::P_B;
     const float c2 = scale * 1.4426950408889634f;   // scores in log2 units
+    const uint64_t c22 = f2pack(c2, c2);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
@@ -515,70 +623,79 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
 #pragma unroll
       for (int c = 0; c < kTok; c += 16) tmem_ld16_nowait(s_col + bf * kTok + c, sr + c);
       tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&s_free[x][bf]);             // the scores are in registers
       const bool full = t0 + kTok - 1 <= pos;  // no key of the tile is masked
-      float mx = -INFINITY;
-      if (full) {
-#pragma unroll
-        for (int i = 0; i < kTok; ++i) mx = fmaxf(mx, __uint_as_float(sr[i]));
-      } else {
+      if (!full) {
 #pragma unroll
         for (int i = 0; i < kTok; ++i)
-          if (t0 + i <= pos) mx = fmaxf(mx, __uint_as_float(sr[i]));
+          if (t0 + i > pos) sr[i] = __float_as_uint(-INFINITY);
       }
+      // row maximum: four independent chains of three-input maxima over
+      // 16 scores each
+      float mx4[4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        const uint32_t* v = sr + 16 * a;
+        float mv = fmax3(__uint_as_float(v[0]), __uint_as_float(v[1]), __uint_as_float(v[2]));
+#pragma unroll
+        for (int k = 3; k < 15; k += 2)
+          mv = fmax3(mv, __uint_as_float(v[k]), __uint_as_float(v[k + 1]));
+        mx4[a] = fmaxf(mv, __uint_as_float(v[15]));
+      }
+      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
       const float m_new = fmaxf(m, mx * c2);   // (c2 > 0: the maximum commutes)
       if (j == 0) {
         m = m_new;
-      } else {
-        // P(j) overwrites P(j - 1) and a rescale rewrites O: both wait for
-        // the MMAs of tile j - 1
-        if (!warp_wait(&pv_done[x], (j - 1) & 1, abort)) {
+      } else if (__any_sync(0xffffffffu, m_new > m + kRescale)) {
+        // O is rewritten: the P V of tile j - 1 must have completed
+        if (!warp_wait(&s_free[x][(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) {
           ok = false;
           break;
         }
-        const bool need = m_new > m + kRescale;
-        if (__any_sync(0xffffffffu, need)) {
-          tc_fence_after();
-          const float alpha = m_new > m ? ex2_approx(m - m_new) : 1.f;
-          if (m_new > m) {
-            l *= alpha;
-            m = m_new;
-          }
+        tc_fence_after();
+        const float alpha = m_new > m ? ex2_approx(m - m_new) : 1.f;
+        if (m_new > m) {
+          l *= alpha;
+          m = m_new;
+        }
 #pragma unroll 1
-          for (int c = 0; c < D; c += 16) {
-            uint32_t o[16];
-            tmem_ld16_nowait(o_col + c, o);
-            tmem_wait_ld();
+        for (int c = 0; c < D; c += 16) {
+          uint32_t o[16];
+          tmem_ld16_nowait(o_col + c, o);
+          tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            tmem_st16(o_col + c, o);
-          }
-          tmem_wait_st();
+          for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st16(o_col + c, o);
         }
       }
-      float sum = 0.f;
+      // P = 2^(s c2 - m) as fp16 pairs over the first 32 columns of this S
+      // buffer (masked keys hold -inf: 2^-inf = 0; a row without any visible
+      // key so far has m = -inf and keeps P = 0)
+      const bool live = m != -INFINITY;
+      const uint64_t negm = f2pack(-m, -m);
+      uint64_t sum2 = f2pack(0.f, 0.f);
+      uint32_t pk[kTok / 2];
 #pragma unroll
-      for (int c = 0; c < kTok / 8; ++c) {     // 8 tokens = one 16-byte chunk of P
-        float p[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int i = 8 * c + e;
-          const float v = ex2_approx(fmaf(__uint_as_float(sr[i]), c2, -m));
-          p[e] = full || t0 + i <= pos ? v : 0.f;
-          sum += p[e];
-        }
-        *reinterpret_cast<uint4*>(prow + sw128(r, c)) =
-            make_uint4(pack_h2(p[0], p[1]), pack_h2(p[2], p[3]), pack_h2(p[4], p[5]),
-                       pack_h2(p[6], p[7]));
+      for (int i = 0; i < kTok; i += 2) {
+        float a0, a1;
+        f2unpack(ffma2(f2pack(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c22, negm), a0, a1);
+        float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
+        if (!live) p0 = p1 = 0.f;
+        sum2 = fadd2(sum2, f2pack(p0, p1));
+        pk[i / 2] = pack_h2(p0, p1);
       }
-      l += sum;
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tmem_st16(s_col + bf * kTok, pk);
+      tmem_st16(s_col + bf * kTok + 16, pk + 16);
+      float s0, s1;
+      f2unpack(sum2, s0, s1);
+      l += s0 + s1;
+      tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&p_full[x]);
+      mbar_arrive(&p_full[x][bf]);
     }
     // ---------------- epilogue ----------------
-    if (ok && ntiles > 0 && !warp_wait(&pv_done[x], (ntiles - 1) & 1, abort)) ok = false;
+    if (ok && ntiles > 0 &&
+        !warp_wait(&s_free[x][(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, abort))
+      ok = false;
     if (__all_sync(0xffffffffu, ok && !*abort)) {
       tc_fence_after();
       const float inv = l > 0.f ? 1.f / l : 0.f;
@@ -614,11 +731,11 @@ cudaError_t launch_m256(const Geom& g, const void* q, int L, float scale, void* 
                         cudaStream_t s) {
   auto kern = attend_prefill_m256_kernel<D, BITS, FMT>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       M256Layout<D>::ALLOC);
+                                       M256Layout<D, BITS>::ALLOC);
   if (e != cudaSuccess) return e;
   const int nq = kRowsCta / (g.Hq / g.H);
   dim3 grid((L + nq - 1) / nq, g.H, g.B);
-  launch_pdl(kern, dim3(grid), dim3(kThreads), (size_t)M256Layout<D>::ALLOC, s, g,
+  launch_pdl(kern, dim3(grid), dim3(kThreads), (size_t)M256Layout<D, BITS>::ALLOC, s, g,
              reinterpret_cast<const __nv_bfloat16*>(q), L, scale,
              reinterpret_cast<__nv_bfloat16*>(out), nq, err);
   return cudaGetLastError();

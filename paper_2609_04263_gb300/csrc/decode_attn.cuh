@@ -37,7 +37,7 @@ constexpr int kCT = 64;          // tokens per chunk (4 tiles of 16)
 constexpr int kStages = 4;
 constexpr int kWarps = 4;
 constexpr uint32_t kMagic = 0x43004300u;
-constexpr long kWaitLimit = 1L << 24;   // bounded mbarrier polling
+constexpr long kWaitLimit = 1L << 24;   // polls of an mbarrier before a wait gives up at the latest
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -60,11 +60,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
   return ok != 0;
 }
-// Bounded wait; returns false (and the caller flags an error) on timeout.
+// Wait bounded in time (try_wait may suspend the thread between polls, so a
+// count of polls alone does not bound it); returns false (and the caller
+// flags an error) after about a second.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (long i = 0; i < kWaitLimit; ++i)
+  if (mbar_try_wait(bar, parity)) return true;
+  uint64_t t0;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  for (long i = 0;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-  return false;
+    if ((i & 7) == 7) {
+      uint64_t t;
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+      if (t - t0 > 1000000000ull || i > kWaitLimit) return false;
+    }
+  }
 }
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
                                          uint64_t* bar) {

@@ -9,10 +9,16 @@
 namespace kvq {
 namespace tc {
 
-constexpr long kWaitLimit = 1L << 26;   // bounded mbarrier polling
+constexpr long kWaitLimit = 1L << 26;            // bounded polling loops without a barrier
+constexpr uint64_t kWaitNs = 1000000000ull;      // a bounded wait gives up after 1 s
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
 }
 __device__ __forceinline__ void mbar_init(uint64_t* bar, int count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
@@ -29,18 +35,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
   return ok != 0;
 }
+// Wait bounded in time (try_wait may suspend the thread between polls, so a
+// count of polls alone does not bound the wait): false after kWaitNs.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (long i = 0; i < kWaitLimit; ++i)
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (long i = 0;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-  return false;
+    if ((i & 7) == 7 && global_ns() - t0 > kWaitNs) return false;
+  }
 }
 // Bounded wait that also gives up once *abort is set (another role of the
 // CTA timed out); sets *abort itself on a timeout.
 __device__ __forceinline__ bool mbar_wait_or_abort(uint64_t* bar, uint32_t parity,
                                                    volatile int* abort) {
-  for (long i = 0; i < kWaitLimit; ++i) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (long i = 0;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255) == 255 && *abort) return false;
+    if ((i & 7) == 7) {
+      if (*abort) return false;
+      if (global_ns() - t0 > kWaitNs) break;
+    }
   }
   *abort = 1;
   return false;
