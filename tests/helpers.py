@@ -16,6 +16,8 @@ FORMATS = {
     "affine4": dict(fmt=O.FMT_AFFINE, key_bits=4, value_bits=4, group_size=32),
     "affine2": dict(fmt=O.FMT_AFFINE, key_bits=2, value_bits=2, group_size=32),
     "affine8_g64": dict(fmt=O.FMT_AFFINE, key_bits=8, value_bits=8, group_size=64),
+    "affine8": dict(fmt=O.FMT_AFFINE, key_bits=8, value_bits=8, group_size=32),
+    "sym8": dict(fmt=O.FMT_SYMMETRIC, key_bits=8, value_bits=8, group_size=32),
     "affine4_g128": dict(fmt=O.FMT_AFFINE, key_bits=4, value_bits=2, group_size=128),
     "sym2": dict(fmt=O.FMT_SYMMETRIC, key_bits=2, value_bits=2, group_size=32),
     "sym4": dict(fmt=O.FMT_SYMMETRIC, key_bits=4, value_bits=4, group_size=32),

@@ -70,6 +70,12 @@ DECODE = [
     # sinks and staged tokens go through the split kernel, then one combine)
     ("kvarn", "bf16", 8, 8, 16, 256, [1500]),
     ("kvarn_small", "bf16", 16, 8, 32, 64, [700, 1]),
+    # 8-bit caches (the paper's 2/4/8-bit operating points)
+    ("affine8", "bf16", 2, 2, 8, 64, [300, 1]),
+    ("affine8", "f32", 1, 2, 2, 64, [129]),
+    ("sym8", "bf16", 1, 2, 8, 128, [517]),
+    ("affine8_g64", "bf16", 2, 1, 4, 128, [1000, 3]),
+    ("kivi_k8", "bf16", 1, 2, 8, 128, [400, 1]),
 ]
 
 
@@ -108,6 +114,12 @@ PREFILL = [
     ("sym2", "bf16", 1, 1, 16, 128, [0], 200),
     ("affine2", "bf16", 1, 2, 4, 128, [0], 40),
     ("sym4", "bf16", 1, 2, 8, 128, [500], 129),
+    # 8-bit caches
+    ("affine8", "bf16", 1, 2, 8, 64, [100], 300),
+    ("affine8", "f32", 1, 1, 2, 64, [0], 97),
+    ("sym8", "bf16", 2, 1, 4, 128, [64], 200),
+    ("affine8_g64", "bf16", 1, 2, 4, 256, [0], 130),
+    ("kivi_k8", "bf16", 1, 2, 8, 128, [200], 180),
 ]
 
 
