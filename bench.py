@@ -198,6 +198,8 @@ class Runner:
         # where the cache format allows) unless separate calls are asked for
         self.separate = False
         self.fused = self.caches[0].decode_step_fused(wl.d_in, self.layers[0][1])
+        # prefill: projection fused with the append where the cache format allows
+        self.fused_append = self.caches[0].project_append_supported(P, wl.d_in, self.layers[0][1])
 
     # one layer's calls ----------------------------------------------------
     def _project(self, l, x, out):
@@ -213,6 +215,20 @@ class Runner:
 
     def prefill(self, timer=None):
         for l, c in enumerate(self.caches):
+            if self.fused_append:
+                # one kernel projects and codes the new keys and values into the cache
+                w, lora = self.layers[l]
+                if timer:
+                    timer("project", 0)
+                q = c.project_append(self.x_pre, w, lora, self.wl.alpha_over_r, self.wl.rope_base,
+                                     q=self.pre[0])
+                if timer:
+                    timer("project", 1)
+                    timer("attend_prefill", 0)
+                c.attend_prefill(q, out=self.o_pre)
+                if timer:
+                    timer("attend_prefill", 1)
+                continue
             if timer:
                 timer("project", 0)
             q, k, v = self._project(l, self.x_pre, self.pre)
@@ -341,7 +357,7 @@ class Runner:
                        and wl.head_dim in (64, 128)) else 2
         if self.kvarn_streamed():
             attend = 3          # coded tokens, sinks and staged tokens, combine
-        prefill = wl.layers * (1 + append + 1)
+        prefill = wl.layers * (2 if self.fused_append else 1 + append + 1)
         per_layer = 1 if (self.fused and not self.separate) else 1 + append + attend
         return prefill + wl.decode * wl.layers * per_layer
 
@@ -719,6 +735,9 @@ def main():
         "attend_prefill": ("tensor", prefill_attn_flops(wl, wl.prefill, wl.prefill), wl.layers),
         "append": ("hbm", pack_bytes(wl, wl.prefill), wl.layers),
     }
+    if run.fused_append:
+        # the projection kernel also codes the keys and values: no separate append
+        del work["append"]
     if run.separate:
         for name, fn in (("project_decode", run.decode_project_layers),
                          ("append_decode", run.decode_append_layers),
@@ -803,7 +822,9 @@ def main():
             "config": dict(workload_config(wl, world), decode_path=run.decode_path()),
             "phases": {"prefill_ms": statistics.mean(pre_ms), "decode_ms": statistics.mean(dec_ms),
                        "decode_tokens_per_s": decode_tps,
-                       "pack_gbs": kernels["append"]["achieved"],
+                       "pack_gbs": kernels["append"]["achieved"] if "append" in kernels else None,
+                       "prefill_append": ("fused into the projection (kvq_project_append)"
+                                          if run.fused_append else "separate kvq_append_pack"),
                        "qkv_tflops": kernels["project"]["achieved"]},
             "roofline": {"bound": bound, "kernel": dominant, "achieved": round(achieved, 3),
                          "peak": peak, "unit": unit, "frac": round(achieved / peak, 4),

@@ -185,6 +185,40 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
                             int dtype, void* q, void* k, void* v, void* stream);
 
 /*
+ * Projection of L new tokens per sequence fused with their append (Section 3,
+ * Eq. (1) and Eq. (lora), then Section 3.1: the new keys and values are coded
+ * into the packed cache straight from the projection, without an unquantized
+ * copy in device memory).
+ *
+ *   x      [B][L][d_in] hidden states, B the cache's batch
+ *   w_qkv, a_p, b_p, r_p, alpha_over_r, rope_base  as in kvq_project_lora; the
+ *          projection dimensions are the cache's (Hq, Hkv, head_dim)
+ *   q      [B][Hq][L][D] receives the rotated queries
+ *
+ * Keys (after RoPE) and values are rounded to bf16, exactly the values
+ * kvq_project_lora would store, and coded per token into the cache at
+ * positions T .. T + L - 1 (T = the cache's device token count, which the call
+ * then advances by L): the cache after the call is bit for bit the cache
+ * kvq_project_lora + kvq_append_pack would leave.  Covered shapes
+ * (kvq_project_append_supported tells): bf16 affine or symmetric caches with
+ * group size 32 and 2/4/8-bit codes, B * L > 16 rows, d_in a multiple of 64,
+ * head counts that tile the tensor-core projection, ranks multiples of 8 up to
+ * 64.  Otherwise KVQ_ERR_UNSUPPORTED and nothing is launched: use the two calls.
+ * KVQ_ERR_CAPACITY if T + L > max_tokens (host mirror; a replayed call that
+ * would overflow is refused on the device like an append).
+ */
+kvq_status kvq_project_append(kvq_cache* cache, const void* x, int L, int d_in,
+                              const void* w_qkv, const void* a_q, const void* b_q, int r_q,
+                              const void* a_k, const void* b_k, int r_k,
+                              const void* a_v, const void* b_v, int r_v,
+                              float alpha_over_r, float rope_base, void* q, void* stream);
+
+/* 1 when kvq_project_append covers this cache, L, d_in and ranks, 0 when it
+ * does not, -1 for a NULL cache.  Launches nothing. */
+int kvq_project_append_supported(const kvq_cache* cache, int L, int d_in, int r_q, int r_k,
+                                 int r_v);
+
+/*
  * Append L new tokens per sequence: k, v [B][Hkv][L][D] (activation dtype).
  * Codes them per the cache format (Section 3.1) into the packed planes.  The
  * cache after T tokens is the same whether they arrive in one call or in

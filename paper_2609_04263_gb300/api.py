@@ -101,6 +101,24 @@ class Cache:
                             _stream())
         return qkv, out
 
+    def project_append(self, x, w_qkv, lora, alpha_over_r, rope_base, q=None):
+        """Project x [B,L,d_in] and code the new keys and values straight into
+        the cache (positions continue it); returns q [B,Hq,L,D]."""
+        d = self.desc
+        B, L, d_in = x.shape
+        q = torch.empty(B, d.q_heads, L, d.head_dim, dtype=x.dtype, device=x.device) if q is None else q
+        args = []
+        for p in "qkv":
+            ab = lora.get(p)
+            args += [None, None, 0] if ab is None else [_ptr(ab[0]), _ptr(ab[1]), ab[0].shape[0]]
+        kvq.kvq_project_append(self.handle, _ptr(x), L, d_in, _ptr(w_qkv), *args, alpha_over_r,
+                               rope_base, _ptr(q), _stream())
+        return q
+
+    def project_append_supported(self, L, d_in, lora) -> bool:
+        r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
+        return kvq.kvq_project_append_supported(self.handle, L, d_in, *r)
+
     def decode_step_fused(self, d_in, lora) -> bool:
         """Whether decode_step with this d_in and these LoRA factors runs as
         one fused kernel."""

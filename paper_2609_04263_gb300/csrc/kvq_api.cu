@@ -443,6 +443,68 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
   return KVQ_OK;
 }
 
+// The shapes the fused projection-and-append covers (no launch).
+static const char* project_append_gap(const kvq_cache* c, int L, int d_in, const int r[3]) {
+  const Geom& g = c->g;
+  if (g.act != KVQ_BF16) return "the activation dtype is not bf16";
+  if (g.fmt != KVQ_FMT_AFFINE && g.fmt != KVQ_FMT_SYMMETRIC) return "the cache is not affine or symmetric";
+  if (g.G != 32) return "the group size is not 32";
+  for (int b : {g.kb, g.vb})
+    if (b != 2 && b != 4 && b != 8) return "code widths must be 2, 4 or 8 bits";
+  if ((int64_t)g.B * L <= 16) return "16 rows or fewer (decode rows take the weight-streaming kernel)";
+  if (d_in <= 0 || d_in % 64) return "d_in is not a positive multiple of 64";
+  if (!project_tc_tile(g.Hq, g.H, g.D, d_in)) return "the head shapes do not tile the tensor-core kernel";
+  for (int p = 0; p < 3; ++p)
+    if (r[p] < 0 || r[p] > 64 || r[p] % 8) return "LoRA ranks must be multiples of 8 up to 64";
+  return nullptr;
+}
+
+int kvq_project_append_supported(const kvq_cache* cache, int L, int d_in, int r_q, int r_k,
+                                 int r_v) {
+  if (!cache) return -1;
+  const int r[3] = {r_q, r_k, r_v};
+  return project_append_gap(cache, L, d_in, r) == nullptr ? 1 : 0;
+}
+
+kvq_status kvq_project_append(kvq_cache* cache, const void* x, int L, int d_in,
+                              const void* w_qkv, const void* a_q, const void* b_q, int r_q,
+                              const void* a_k, const void* b_k, int r_k,
+                              const void* a_v, const void* b_v, int r_v,
+                              float alpha_over_r, float rope_base, void* q, void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (L < 0) return fail(KVQ_ERR_ARG, "L = %d < 0", L);
+  if (!(rope_base >= 0.f)) return fail(KVQ_ERR_ARG, "rope_base < 0");
+  if (L == 0) return KVQ_OK;
+  const Geom& g = cache->g;
+  const int r[3] = {r_q, r_k, r_v};
+  if (const char* why = project_append_gap(cache, L, d_in, r))
+    return fail(KVQ_ERR_UNSUPPORTED, "kvq_project_append: %s", why);
+  if (!x || !w_qkv || !q) return fail(KVQ_ERR_ARG, "NULL tensor pointer");
+  if (misaligned(x) || misaligned(w_qkv) || misaligned(q))
+    return fail(KVQ_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  const void* a[3] = {a_q, a_k, a_v};
+  const void* bm[3] = {b_q, b_k, b_v};
+  for (int p = 0; p < 3; ++p) {
+    if (r[p] > 0 && (!a[p] || !bm[p])) return fail(KVQ_ERR_ARG, "rank %d but NULL factor", r[p]);
+    if (r[p] == 0) { a[p] = nullptr; bm[p] = nullptr; }
+    if (misaligned(a[p]) || misaligned(bm[p]))
+      return fail(KVQ_ERR_ARG, "LoRA factors must be 16-byte aligned");
+  }
+  if ((int64_t)cache->T + L > g.Tmax)
+    return fail(KVQ_ERR_CAPACITY, "append of %d tokens to %d exceeds max_tokens %d", L, cache->T,
+                g.Tmax);
+  int* err = device_error_word();
+  if (!err) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
+  cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_project_append");
+  void* out[3] = {q, nullptr, nullptr};
+  e = launch_project_tc(x, g.B, L, d_in, w_qkv, a, bm, r, alpha_over_r, g.Hq, g.H, g.D, 0,
+                        &cache->g.state->tokens, rope_base, out, err, (cudaStream_t)stream, &g);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_project_append launch");
+  cache->T += L;
+  return KVQ_OK;
+}
+
 kvq_status kvq_decode_step(kvq_cache* cache, const void* x, int d_in, const void* w_qkv,
                            const void* a_q, const void* b_q, int r_q,
                            const void* a_k, const void* b_k, int r_k,

@@ -128,11 +128,15 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
 
 // tcgen05 projection (project_tc.cu) for bf16 and more than 16 rows;
 // cudaErrorNotSupported if the head shapes do not tile.
+// append_to: if non-NULL, k and v are not stored but coded into that cache
+// (affine or symmetric, G = 32) at its device token count, which the last CTA
+// then advances by B's L tokens (the fused projection-and-append).
 cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void* w,
                               const void* const a[3], const void* const bm[3], const int r[3],
                               float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
-                              cudaStream_t s);
+                              cudaStream_t s, const Geom* append_to = nullptr);
+int project_tc_tile(int Hq, int Hkv, int D, int d_in);
 void rope_theta_table(float rope_base, int D, float* hi, float* lo);
 
 // Fused decode step (decode_step.cu): projection of the new token, append,

@@ -17,10 +17,12 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <math.h>
+#include <string.h>
 
 #include <mutex>
 
 #include "kvq_internal.cuh"
+#include "quant_common.cuh"
 #include "tc_common.cuh"
 
 namespace kvq {
@@ -47,6 +49,8 @@ struct TcArgs {
   int rope;
   int k_blocks;
   int* err;
+  int pack;                     // 1: code k and v into the cache g instead of storing them
+  Geom g;
   float theta_hi[128], theta_lo[128];
 };
 
@@ -60,6 +64,57 @@ __device__ __forceinline__ void rope_cs(int pos, float th_hi, float th_lo, float
   r = fmaf(-k, 1.0253132e-11f, r);
   r += e;
   sincosf(r, s, c);
+}
+
+// Rotate-half pair (a, b) by the angle with cosine c and sine s.  Products
+// are rounded before the fused add, so both epilogues (bf16 store, or coding
+// into the cache) produce the same values bit for bit.
+__device__ __forceinline__ void rope_rot(float& a, float& b, float c, float s) {
+  const float a0 = a, b0 = b;
+  a = fmaf(a0, c, -__fmul_rn(b0, s));
+  b = fmaf(b0, c, __fmul_rn(a0, s));
+}
+
+// One token's group of 32 channels (values already rounded to bf16, as the
+// unfused path stores them) coded into the cache planes: 4 x 8 codes LSB
+// first, fp16 scale (and offset).
+template <int BITS, bool SYM>
+__device__ __forceinline__ void code_group32(const Geom& g, int cplane, int splane, int zplane,
+                                             int b, int h, int t, int gi, const float v[32]) {
+  float lo = v[0], hi = SYM ? fabsf(v[0]) : v[0];
+#pragma unroll
+  for (int i = 1; i < 32; ++i) {
+    if (SYM) hi = fmaxf(hi, fabsf(v[i]));
+    else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
+  }
+  uint64_t w[4];
+  float s = 0.f;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) w[q] = quant::code8<BITS, SYM>(v + 8 * q, lo, hi, &s);
+  uint8_t* crow = plane_ptr<uint8_t>(g, cplane, b, h, t) + gi * (32 * BITS / 8);
+  if (BITS == 2) {
+    *reinterpret_cast<uint2*>(crow) = make_uint2((uint32_t)w[0] | ((uint32_t)w[1] << 16),
+                                                 (uint32_t)w[2] | ((uint32_t)w[3] << 16));
+  } else if (BITS == 4) {
+    *reinterpret_cast<uint4*>(crow) =
+        make_uint4((uint32_t)w[0], (uint32_t)w[1], (uint32_t)w[2], (uint32_t)w[3]);
+  } else {
+    uint4* d = reinterpret_cast<uint4*>(crow);
+    d[0] = make_uint4((uint32_t)w[0], (uint32_t)(w[0] >> 32), (uint32_t)w[1], (uint32_t)(w[1] >> 32));
+    d[1] = make_uint4((uint32_t)w[2], (uint32_t)(w[2] >> 32), (uint32_t)w[3], (uint32_t)(w[3] >> 32));
+  }
+  *plane_ptr<__half>(g, splane, b, h, t, gi) = __float2half_rn(s);
+  if (!SYM) *plane_ptr<__half>(g, zplane, b, h, t, gi) = __float2half_rn(lo + 0.0f);
+}
+
+template <int BITS, bool SYM>
+__device__ __forceinline__ void code_pair(const Geom& g, int which, int b, int h, int t, int g1,
+                                          int g2, const float* x1, const float* x2) {
+  const int cp = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int sp = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int zp = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  code_group32<BITS, SYM>(g, cp, sp, zp, b, h, t, g1, x1);
+  code_group32<BITS, SYM>(g, cp, sp, zp, b, h, t, g2, x2);
 }
 
 template <int BN>
@@ -91,6 +146,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
   __shared__ uint32_t tmem_base;
   __shared__ int fail;
 
+  bool app_ok = true;                    // appending: the cache has room for the L tokens
+  const int T0 = args.pack ? append_begin(args.g, args.L, &app_ok) : 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
   const int proj = n0 < args.n_off[1] ? 0 : n0 < args.n_off[2] ? 1 : 2;
@@ -221,6 +278,49 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(args.out[proj]);
     const bool rope = args.rope && proj < 2;
     const int pos = args.pos0 + (args.pos_dev ? *args.pos_dev : 0) + l;
+    if (args.pack && proj > 0) {
+      // append: k (after RoPE) and v rounded to bf16, then coded per token
+      // in groups of 32 channels straight into the cache planes
+      const Geom& gg = args.g;
+      const int bits = proj == 1 ? gg.kb : gg.vb;
+      const bool sym = gg.fmt == KVQ_FMT_SYMMETRIC;
+      const int t = T0 + l;
+      for (int hc = 0; hc < BN; hc += D) {
+        const int head = (col0 + hc) / D;
+        for (int j = 0; j < half; j += 32) {
+          float x1[32], x2[32];
+#pragma unroll
+          for (int u = 0; u < 32; u += 16) {
+            tmem_ld16(tmem + lane_base + hc + j + u, x1 + u);
+            tmem_ld16(tmem + lane_base + hc + half + j + u, x2 + u);
+            if (rope) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                float c, sn;
+                rope_cs(pos, args.theta_hi[j + u + i], args.theta_lo[j + u + i], &c, &sn);
+                rope_rot(x1[u + i], x2[u + i], c, sn);
+              }
+            }
+          }
+          if (!active || !app_ok) continue;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            x1[i] = __bfloat162float(__float2bfloat16_rn(x1[i]));
+            x2[i] = __bfloat162float(__float2bfloat16_rn(x2[i]));
+          }
+          const int g1 = j / 32, g2 = (half + j) / 32, which = proj - 1;
+          if (sym) {
+            if (bits == 2) code_pair<2, true>(gg, which, b, head, t, g1, g2, x1, x2);
+            else if (bits == 4) code_pair<4, true>(gg, which, b, head, t, g1, g2, x1, x2);
+            else code_pair<8, true>(gg, which, b, head, t, g1, g2, x1, x2);
+          } else {
+            if (bits == 2) code_pair<2, false>(gg, which, b, head, t, g1, g2, x1, x2);
+            else if (bits == 4) code_pair<4, false>(gg, which, b, head, t, g1, g2, x1, x2);
+            else code_pair<8, false>(gg, which, b, head, t, g1, g2, x1, x2);
+          }
+        }
+      }
+    } else
     for (int j = 0; j < half; j += 16) {              // 16 frequencies at a time
       float cs[16], sn[16];
       if (rope) {
@@ -236,11 +336,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
         tmem_ld16(tmem + lane_base + hc + half + j, x2);
         if (rope) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const float a = x1[i], bb = x2[i];
-            x1[i] = a * cs[i] - bb * sn[i];
-            x2[i] = bb * cs[i] + a * sn[i];
-          }
+          for (int i = 0; i < 16; ++i) rope_rot(x1[i], x2[i], cs[i], sn[i]);
         }
         if (!active) continue;
         uint32_t w1[8], w2[8];
@@ -265,6 +361,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
   }
+  // appending: the last CTA to arrive advances the cache's token count
+  if (args.pack) quant::append_arrive_spread(args.g.state, T0, args.L, app_ok);
 }
 
 // ---------------------------------------------------------------------------
@@ -329,10 +427,13 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const void* const a[3], const void* const bm[3], const int r[3],
                               float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
-                              cudaStream_t s) {
+                              cudaStream_t s, const Geom* append_to) {
   const int bn = project_tc_tile(Hq, Hkv, D, d_in);
   if (!bn) return cudaErrorNotSupported;
   TcArgs t;
+  t.pack = append_to != nullptr;
+  if (append_to) t.g = *append_to;
+  else memset(&t.g, 0, sizeof t.g);
   const int M = B * L;
   for (int i = 0; i < 3; ++i) {
     t.out[i] = out[i];

@@ -72,6 +72,10 @@ _SIGS = {
                                 c_float, c_float, c_void_p, c_void_p, c_void_p, c_void_p,
                                 c_void_p]),
     "kvq_decode_step_fused": (c_int, [c_void_p, c_int, c_int, c_int, c_int]),
+    "kvq_project_append": (c_int, [c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p, c_void_p,
+                                   c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
+                                   c_float, c_float, c_void_p, c_void_p]),
+    "kvq_project_append_supported": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int]),
 }
 
 _lib = None
@@ -192,3 +196,15 @@ def kvq_device_status(stream=0) -> int:
     if st not in (KVQ_OK, KVQ_ERR_TIMEOUT):
         _check(st)
     return out.value
+
+
+def kvq_project_append(handle, x, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,
+                       alpha_over_r, rope_base, q, stream=0) -> None:
+    _check(lib().kvq_project_append(c_void_p(handle), c_void_p(x), L, d_in, c_void_p(w_qkv),
+                                    c_void_p(a_q), c_void_p(b_q), r_q, c_void_p(a_k),
+                                    c_void_p(b_k), r_k, c_void_p(a_v), c_void_p(b_v), r_v,
+                                    alpha_over_r, rope_base, c_void_p(q), c_void_p(stream or 0)))
+
+
+def kvq_project_append_supported(handle, L, d_in, r_q, r_k, r_v) -> bool:
+    return lib().kvq_project_append_supported(c_void_p(handle), L, d_in, r_q, r_k, r_v) == 1

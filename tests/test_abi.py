@@ -150,3 +150,35 @@ def test_append_index_range_is_checked_on_the_host(kvq):
         assert kvq.kvq_cache_tokens(h) == 0
     finally:
         kvq.kvq_destroy_cache(h)
+
+
+def test_project_append_shape_rules_on_the_host(kvq):
+    """The fused projection-and-append states which caches it covers and
+    refuses the others (and capacity overflows) before any launch."""
+    fake = 1 << 32
+    P = 1 << 33
+    d = _desc(kvq, max_tokens=64)                       # affine 4-bit, G 32, bf16
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        assert kvq.kvq_project_append_supported(h, 32, 2048, 16, 16, 16)
+        assert not kvq.kvq_project_append_supported(h, 2, 2048, 16, 16, 16)   # decode rows
+        assert not kvq.kvq_project_append_supported(h, 32, 100, 16, 16, 16)   # d_in
+        assert not kvq.kvq_project_append_supported(h, 32, 2048, 12, 16, 16)  # rank
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_project_append(h, P, 65, 2048, P, P, P, 16, P, P, 16, P, P, 16, 2.0, 1e4, P, 0)
+        assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_project_append(h, P, 2, 2048, P, P, P, 16, P, P, 16, P, P, 16, 2.0, 1e4, P, 0)
+        assert ei.value.status == kvq.KVQ_ERR_UNSUPPORTED
+        assert kvq.kvq_cache_tokens(h) == 0
+    finally:
+        kvq.kvq_destroy_cache(h)
+    for kw in (dict(fmt=kvq.KVQ_FMT_KIVI, residual_tokens=32), dict(group_size=64),
+               dict(dtype=kvq.KVQ_F32)):
+        d = _desc(kvq, max_tokens=64, **kw)
+        h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+        try:
+            assert not kvq.kvq_project_append_supported(h, 32, 2048, 16, 16, 16)
+        finally:
+            kvq.kvq_destroy_cache(h)
+    assert kvq.kvq_project_append_supported(None, 32, 2048, 16, 16, 16) is False

@@ -5,7 +5,9 @@ For every workload (single layer of each model shape, layer 0 weights):
   * projection: contiguous segments of rows at the start of the first
     sequence and the end of the last, against the oracle's fp64 projection;
   * prefill append: the packed planes of sampled (sequence, kv head) pairs bit
-    for bit, against oracle caches fed the same projected k, v;
+    for bit, against oracle caches fed the same projected k, v; where the
+    fused projection-and-append covers the cache (the bench's prefill path),
+    its whole cache and queries bit for bit against the separate calls';
   * prefill attention: sampled queries of every query head of those kv heads;
   * decode: all decode steps of the workload through kvq_decode_step (the
     fused single-kernel step where the library takes it, as the bench does),
@@ -111,6 +113,20 @@ def test_full_size_layer(name):
 
     # ---- prefill append and attention ----
     cache.append(k, v)
+    if cache.project_append_supported(P, wl.d_in, dl):
+        # bench.py's prefill takes the fused projection-and-append here: its
+        # cache and queries must be the separate calls', bit for bit
+        fused = api.Cache(desc)
+        q_f = fused.project_append(x_pre.to(dev), dw, dl, wl.alpha_over_r, wl.rope_base)
+        torch.cuda.synchronize()
+        assert torch.equal(q_f.view(torch.int16), q.view(torch.int16))
+        assert fused.sync() == P
+        gp, fp = cache.planes(), fused.planes()
+        for name, t in gp.items():
+            if isinstance(t, torch.Tensor) and name != "workspace":
+                assert torch.equal(t.contiguous().view(torch.uint8),
+                                   fp[name].contiguous().view(torch.uint8)), name
+        del fused, q_f
     o = cache.attend_prefill(q)
     torch.cuda.synchronize()
     samples = [(0, 0), (B - 1, Hkv - 1)]
