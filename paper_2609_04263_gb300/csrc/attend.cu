@@ -527,11 +527,6 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
     if (!err) return cudaErrorInvalidDevice;
     return launch_prefill_m256(g, q, L, scale, out, err, s);
   }
-  if (!decode && prefill_tc_supported(g)) {
-    int* err = device_error_word();
-    if (!err) return cudaErrorInvalidDevice;
-    return launch_prefill_tc(g, q, L, scale, out, err, s);
-  }
   if (!decode && prefill_mma_supported(g)) return launch_prefill_mma(g, q, L, scale, out, s);
   // the streaming decode pays off once every CTA streams a few stages; short
   // caches keep the split kernel (both read T on the device and are exact

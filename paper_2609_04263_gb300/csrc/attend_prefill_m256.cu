@@ -757,10 +757,10 @@ cudaError_t launch_m256_d(const Geom& g, const void* q, int L, float scale, void
 }  // namespace
 
 // bf16 affine/symmetric/KIVI caches with equal 2- or 4-bit key and value
-// codes, G = 32 (KIVI: 32-token key blocks), head_dim 128, GQA group <= 256.
+// codes, G = 32 (KIVI: 32-token key blocks), head_dim 64 or 128, GQA group <= 256.
 bool prefill_m256_supported(const Geom& g) {
   const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC || g.fmt == KVQ_FMT_KIVI;
-  return fmt_ok && g.act == KVQ_BF16 && g.D == 128 && g.G == 32 && g.kb == g.vb &&
+  return fmt_ok && g.act == KVQ_BF16 && (g.D == 64 || g.D == 128) && g.G == 32 && g.kb == g.vb &&
          (g.kb == 2 || g.kb == 4) && g.Hq / g.H <= kRowsCta;
 }
 

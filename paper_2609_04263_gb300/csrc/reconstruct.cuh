@@ -1,5 +1,5 @@
 // Reconstruction of stored keys/values for the prefill attention kernels
-// (attend_prefill_mma.cu, attend_prefill_tc.cu): the value the cache stores
+// (attend_prefill_mma.cu): the value the cache stores
 // for a token and channel, per format (Section 3.1): codes x scale + offset
 // for the quantized formats, the full-precision copy for FLOAT caches and
 // the KIVI residual window.

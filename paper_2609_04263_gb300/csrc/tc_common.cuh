@@ -1,5 +1,5 @@
 // tcgen05 / TMA / mbarrier helpers shared by the tensor-core kernels
-// (project_tc.cu, attend_prefill_tc.cu).  Inline PTX for sm_100-family GPUs.
+// (project_tc.cu, attend_prefill_m256.cu).  Inline PTX for sm_100-family GPUs.
 #pragma once
 
 #include <cuda.h>
