@@ -153,11 +153,12 @@ int decode_splits(const Geom& g);
 // Tensor-core split decode (attend_mma.cu): the formats it covers, and the
 // launch (partials to the workspace plane; the caller merges them).
 bool decode_mma_supported(const Geom& g);
-// Tensor-core causal prefill (attend_prefill_mma.cu).
 // tcgen05 causal prefill with 256 query rows per CTA (attend_prefill_m256.cu).
 bool prefill_m256_supported(const Geom& g);
 cudaError_t launch_prefill_m256(const Geom& g, const void* q, int L, float scale, void* out,
                                 int* err, cudaStream_t s);
+// mma.sync causal prefill for the other formats and head dimensions
+// (attend_prefill_mma.cu).
 bool prefill_mma_supported(const Geom& g);
 cudaError_t launch_prefill_mma(const Geom& g, const void* q, int L, float scale, void* out,
                                cudaStream_t s);
