@@ -15,6 +15,9 @@ What each function follows (paper sections and equations):
   * projections            Section 3, Eq. (1)  Q = H W_Q^T, K = H W_K^T, V = H W_V^T
   * LoRA update            Section 3, Eq. (lora)  W' = W + (alpha/r) B A
   * adapter cost           Section 3.4: r (d_in + d_out) parameters / MACs per token
+  * NF4 base weights       Section 2 (QLoRA's 4-bit NormalFloat), Sections 3.4 and
+                           4 (NF4 bases with explicit adapters): levels, blocks of 64
+                           inputs with one absmax each
   * affine quantizer       Section 3.1, Eq. (affine) + clipping to [0, 2^b - 1],
                            FP16 scale and FP16 offset
   * symmetric quantizer    Section 3.1: maximum-magnitude scale, no offset
@@ -118,6 +121,49 @@ def project_lora(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim,
             y = rope_rotate_half(y, pos, rope_base)
         out.append(y)
     return tuple(out)
+
+
+# ----------------------------------------------------------------------------
+# NF4 base weights (Section 2 cites QLoRA's 4-bit NormalFloat for frozen bases;
+# Sections 3.4 and 4 report NF4 Gemma and Llama-3.1 bases with explicit
+# adapters).  A row of W is stored as 4-bit codes, one absmax scale per block
+# of 64 consecutive inputs; a weight is level[code] * absmax.
+# ----------------------------------------------------------------------------
+NF4_BLOCK = 64
+
+
+def nf4_levels() -> np.ndarray:
+    """The 16 NF4 levels in fp64, built as QLoRA defines the data type:
+    quantiles of the standard normal distribution, 8 for the positive half and
+    7 for the negative half (so that zero is represented exactly), taken at
+    evenly spaced probabilities from 1 - delta to 1/2 with
+    delta = (1/30 + 1/32) / 2, then scaled so that the largest magnitude is 1."""
+    from scipy.stats import norm     # the inverse normal CDF (library routine)
+    delta = 0.5 * (1.0 / 30.0 + 1.0 / 32.0)
+    pos = norm.ppf(np.linspace(1.0 - delta, 0.5, 9)[:-1])
+    neg = -norm.ppf(np.linspace(1.0 - delta, 0.5, 8)[:-1])
+    v = np.sort(np.concatenate([pos, [0.0], neg]))
+    return v / np.abs(v).max()
+
+
+def nf4_dequant(codes, absmax) -> np.ndarray:
+    """W [N, d_in] in fp64 from codes [N, d_in / 2] (uint8; input k in byte
+    k // 2, the low nibble for even k) and absmax [N, d_in / 64]."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    idx = np.empty((codes.shape[0], codes.shape[1] * 2), dtype=np.int64)
+    idx[:, 0::2] = codes & 0xF
+    idx[:, 1::2] = codes >> 4
+    w = nf4_levels()[idx]
+    scale = np.repeat(np.asarray(absmax, dtype=np.float64), NF4_BLOCK, axis=1)
+    return w * scale
+
+
+def project_lora_nf4(x, codes, absmax, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim,
+                     pos0=0, rope_base=0.0):
+    """project_lora with the frozen base W_qkv given in NF4: the base weights
+    are the dequantized ones, the rank-r branches stay explicit."""
+    return project_lora(x, nf4_dequant(codes, absmax), lora, alpha_over_r, n_q_heads,
+                        n_kv_heads, head_dim, pos0=pos0, rope_base=rope_base)
 
 
 def adapter_params(d_in: int, d_out: int, r: int) -> int:
