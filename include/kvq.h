@@ -185,6 +185,31 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
                             int dtype, void* q, void* k, void* v, void* stream);
 
 /*
+ * kvq_project_lora over a frozen NF4 base (Sections 3.4 and 4: the reported
+ * Gemma and Llama-3.1 runs keep NF4 bases with explicit rank-r branches;
+ * Section 2 cites QLoRA's 4-bit NormalFloat data type for them).  bf16 only.
+ *
+ *   w_codes   uint8 [(Hq + 2 Hkv) * D][d_in / 2]: 4-bit NF4 codes, input k of a
+ *             row in byte k / 2 (even k in the low nibble)
+ *   w_absmax  float [(Hq + 2 Hkv) * D][d_in / 64]: one scale per block of 64
+ *             consecutive inputs (4-byte aligned)
+ *   a base weight is level[code] * absmax, with the 16 NF4 levels of QLoRA;
+ *   every other argument as in kvq_project_lora.
+ *
+ * The base is dequantized inside the GEMM (per 64-input tile, into shared
+ * memory as bf16) and never materialised in device memory.  KVQ_ERR_UNSUPPORTED
+ * unless d_in % 64 == 0, head_dim is 64 or 128, Hq * D and Hkv * D are
+ * multiples of 128, and the ranks are multiples of 8 up to 64.
+ */
+kvq_status kvq_project_lora_nf4(const void* x, int B, int L, int d_in, const void* w_codes,
+                                const void* w_absmax, const void* a_q, const void* b_q, int r_q,
+                                const void* a_k, const void* b_k, int r_k,
+                                const void* a_v, const void* b_v, int r_v,
+                                float alpha_over_r, int n_q_heads, int n_kv_heads, int head_dim,
+                                int pos0, kvq_cache* pos_cache, float rope_base, void* q, void* k,
+                                void* v, void* stream);
+
+/*
  * Projection of L new tokens per sequence fused with their append (Section 3,
  * Eq. (1) and Eq. (lora), then Section 3.1: the new keys and values are coded
  * into the packed cache straight from the projection, without an unquantized

@@ -174,3 +174,24 @@ def project_lora(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, 
                          _DT[x.dtype], _ptr(out[0]),
                          _ptr(out[1]), _ptr(out[2]), _stream())
     return out
+
+
+def project_lora_nf4(x, w_codes, w_absmax, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim,
+                     pos0=0, rope_base=0.0, out=None, pos_cache: "Cache | None" = None):
+    """project_lora over an NF4 base: w_codes uint8 [N, d_in/2], w_absmax
+    float32 [N, d_in/64]; the LoRA branches stay explicit bf16."""
+    B, L, d_in = x.shape
+    D = head_dim
+    if out is None:
+        out = (torch.empty(B, n_q_heads, L, D, dtype=x.dtype, device=x.device),
+               torch.empty(B, n_kv_heads, L, D, dtype=x.dtype, device=x.device),
+               torch.empty(B, n_kv_heads, L, D, dtype=x.dtype, device=x.device))
+    args = []
+    for p in "qkv":
+        ab = lora.get(p)
+        args += [None, None, 0] if ab is None else [_ptr(ab[0]), _ptr(ab[1]), ab[0].shape[0]]
+    kvq.kvq_project_lora_nf4(_ptr(x), B, L, d_in, _ptr(w_codes), _ptr(w_absmax), *args,
+                             alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0,
+                             pos_cache.handle if pos_cache is not None else None, rope_base,
+                             _ptr(out[0]), _ptr(out[1]), _ptr(out[2]), _stream())
+    return out

@@ -443,6 +443,50 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
   return KVQ_OK;
 }
 
+kvq_status kvq_project_lora_nf4(const void* x, int B, int L, int d_in, const void* w_codes,
+                                const void* w_absmax, const void* a_q, const void* b_q, int r_q,
+                                const void* a_k, const void* b_k, int r_k,
+                                const void* a_v, const void* b_v, int r_v,
+                                float alpha_over_r, int n_q_heads, int n_kv_heads, int head_dim,
+                                int pos0, kvq_cache* pos_cache, float rope_base, void* q, void* k,
+                                void* v, void* stream) {
+  if (B < 0 || L < 0 || d_in <= 0) return fail(KVQ_ERR_SHAPE, "bad B/L/d_in");
+  if (n_q_heads <= 0 || n_kv_heads <= 0 || n_q_heads % n_kv_heads)
+    return fail(KVQ_ERR_SHAPE, "heads %d/%d", n_q_heads, n_kv_heads);
+  if (pos0 < 0) return fail(KVQ_ERR_ARG, "pos0 < 0");
+  if (!(rope_base >= 0.f)) return fail(KVQ_ERR_ARG, "rope_base < 0");
+  const int r[3] = {r_q, r_k, r_v};
+  if (!project_nf4_supported(d_in, n_q_heads, n_kv_heads, head_dim, r))
+    return fail(KVQ_ERR_UNSUPPORTED,
+                "NF4 projection: needs d_in %% 64 == 0, head_dim 64 or 128, Hq*D and Hkv*D "
+                "multiples of 128, ranks multiples of 8 up to 64");
+  if (B == 0 || L == 0) return KVQ_OK;
+  if (!x || !w_codes || !w_absmax || !q || !k || !v) return fail(KVQ_ERR_ARG, "NULL tensor pointer");
+  if (misaligned(x) || misaligned(w_codes) || misaligned(q) || misaligned(k) || misaligned(v) ||
+      (reinterpret_cast<uintptr_t>(w_absmax) & 3))
+    return fail(KVQ_ERR_ARG, "tensor pointers must be 16-byte aligned (absmax: 4-byte)");
+  const void* a[3] = {a_q, a_k, a_v};
+  const void* bm[3] = {b_q, b_k, b_v};
+  for (int p = 0; p < 3; ++p) {
+    if (r[p] > 0 && (!a[p] || !bm[p])) return fail(KVQ_ERR_ARG, "rank %d but NULL factor", r[p]);
+    if (r[p] == 0) { a[p] = nullptr; bm[p] = nullptr; }
+    if (misaligned(a[p]) || misaligned(bm[p]))
+      return fail(KVQ_ERR_ARG, "LoRA factors must be 16-byte aligned");
+  }
+  const int* pos_dev = nullptr;
+  if (pos_cache) {
+    cudaError_t e0 = ensure_init(pos_cache, (cudaStream_t)stream);
+    if (e0 != cudaSuccess) return cuda_fail(e0, "kvq_project_lora_nf4");
+    pos_dev = &pos_cache->g.state->tokens;
+  }
+  void* out[3] = {q, k, v};
+  cudaError_t e = launch_project_nf4(x, B, L, d_in, w_codes, w_absmax, a, bm, r, alpha_over_r,
+                                     n_q_heads, n_kv_heads, head_dim, pos0, pos_dev, rope_base,
+                                     out, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora_nf4 launch");
+  return KVQ_OK;
+}
+
 // The shapes the fused projection-and-append covers (no launch).
 static const char* project_append_gap(const kvq_cache* c, int L, int d_in, const int r[3]) {
   const Geom& g = c->g;

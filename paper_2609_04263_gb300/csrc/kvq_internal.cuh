@@ -137,6 +137,15 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
                               cudaStream_t s, const Geom* append_to = nullptr);
 int project_tc_tile(int Hq, int Hkv, int D, int d_in);
+
+// Projection over an NF4 base (project_nf4.cu): codes [N][d_in/2], fp32 absmax
+// [N][d_in/64]; bf16 activations.
+bool project_nf4_supported(int d_in, int Hq, int Hkv, int D, const int r[3]);
+cudaError_t launch_project_nf4(const void* x, int B, int L, int d_in, const void* codes,
+                               const void* absmax, const void* const a[3],
+                               const void* const bm[3], const int r[3], float alpha_over_r,
+                               int Hq, int Hkv, int D, int pos0, const int* pos_dev,
+                               float rope_base, void* const out[3], cudaStream_t s);
 void rope_theta_table(float rope_base, int D, float* hi, float* lo);
 
 // Fused decode step (decode_step.cu): projection of the new token, append,

@@ -76,6 +76,11 @@ _SIGS = {
                                    c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
                                    c_float, c_float, c_void_p, c_void_p]),
     "kvq_project_append_supported": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_int]),
+    "kvq_project_lora_nf4": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
+                                     c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
+                                     c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
+                                     c_int, c_void_p, c_float, c_void_p, c_void_p, c_void_p,
+                                     c_void_p]),
 }
 
 _lib = None
@@ -208,3 +213,13 @@ def kvq_project_append(handle, x, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, 
 
 def kvq_project_append_supported(handle, L, d_in, r_q, r_k, r_v) -> bool:
     return lib().kvq_project_append_supported(c_void_p(handle), L, d_in, r_q, r_k, r_v) == 1
+
+
+def kvq_project_lora_nf4(x, B, L, d_in, w_codes, w_absmax, a_q, b_q, r_q, a_k, b_k, r_k, a_v,
+                         b_v, r_v, alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0,
+                         pos_cache, rope_base, q, k, v, stream=0) -> None:
+    _check(lib().kvq_project_lora_nf4(
+        c_void_p(x), B, L, d_in, c_void_p(w_codes), c_void_p(w_absmax), c_void_p(a_q),
+        c_void_p(b_q), r_q, c_void_p(a_k), c_void_p(b_k), r_k, c_void_p(a_v), c_void_p(b_v), r_v,
+        alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, c_void_p(pos_cache), rope_base,
+        c_void_p(q), c_void_p(k), c_void_p(v), c_void_p(stream or 0)))

@@ -141,6 +141,23 @@ def layer_weights(wl: Workload, layer: int, seed: int = 0, rank=None):
     return w, lora
 
 
+def nf4_base(wl: Workload, layer: int, seed: int = 0):
+    """A frozen NF4 base for one layer: codes [(Hq + 2 Hkv) D, d_in / 2]
+    (uint8, two 4-bit codes per byte, the even input in the low nibble) and
+    absmax [(Hq + 2 Hkv) D, d_in / 64] (float32).
+
+    NF4 levels are normal quantiles of equal probability, so the codes of
+    normally distributed weights are uniform over the 16 levels: the codes
+    are drawn uniformly; each block's absmax is the largest magnitude of 64
+    draws of N(0, 0.02), the scale of the bf16 bases above.
+    """
+    rng = np.random.default_rng([seed, 6, layer])
+    n, d_in = wl.n_out, wl.d_in
+    codes = rng.integers(0, 256, size=(n, d_in // 2), dtype=np.uint8)
+    absmax = np.abs(0.02 * rng.standard_normal((n, d_in // 64, 64))).max(axis=-1)
+    return codes, absmax.astype(np.float32)
+
+
 def kv_states(shape, seed: int = 0, stream: int = 0,
               channel_spread: float = 2.0) -> np.ndarray:
     """Key/value-like tensors [B, H, L, D] for exercising the cache alone.
