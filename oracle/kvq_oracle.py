@@ -30,6 +30,8 @@ What each function follows (paper sections and equations):
                            normalised Hadamard, dual-axis variance normalisation
   * reconstruction R_phi   Section 3.2: attention sees the stored reconstruction
   * attention              Section 3.3: forward attention over the reconstruction
+  * STE backward           Section 3.3: x_hat + x - stopgrad(x) for appended states;
+                           attention and adapter gradients by fp64 autograd
 
 Readings where the paper is silent are listed in the design notes (group
 arithmetic order, code range of the symmetric quantizer, bit order, KIVI flush
@@ -579,3 +581,92 @@ def attend(cache: OracleCache, q, scale=None):
     if scale is None:
         scale = 1.0 / math.sqrt(cache.D)
     return attention(q, k_hat, v_hat, np.arange(cache.T - L, cache.T), scale)
+
+
+# ----------------------------------------------------------------------------
+# Section 3.3: straight-through backward of the packed path.  Newly appended
+# states are replaced by x_hat + x - stopgrad(x): the forward attention sees
+# the stored reconstruction and the K and V adapters receive an identity
+# backward path.  The gradients are taken by PyTorch autograd in fp64 (a
+# library routine) through a torch restatement of attention() and
+# project_lora() above; the tests pin both restatements to those functions.
+# ----------------------------------------------------------------------------
+def _attention_torch(q, k_hat, v_hat, q_pos, scale):
+    B, Hq, L, D = q.shape
+    Hkv, T = k_hat.shape[1], k_hat.shape[2]
+    g = Hq // Hkv
+    kk = k_hat.repeat_interleave(g, dim=1)
+    vv = v_hat.repeat_interleave(g, dim=1)
+    s = torch.einsum("bhld,bhtd->bhlt", q, kk) * scale
+    visible = torch.arange(T)[None, :] <= torch.as_tensor(np.asarray(q_pos))[:, None]
+    s = s.masked_fill(~visible[None, None], float("-inf"))
+    p = torch.softmax(s, dim=-1)
+    return torch.einsum("bhlt,bhtd->bhld", p, vv)
+
+
+def attention_backward(q, k_hat, v_hat, q_pos, scale, d_out):
+    """Gradients (dq, dk_hat, dv_hat) of sum(attention(q, k_hat, v_hat) * d_out)
+    in fp64.  dk_hat, dv_hat [B, Hkv, T, D] collect every query head of the kv
+    head's group.  By the straight-through estimator these are also the
+    gradients of the keys and values that were coded into the cache."""
+    t = lambda a: torch.tensor(np.asarray(a, dtype=np.float64), requires_grad=True)
+    tq, tk, tv = t(q), t(k_hat), t(v_hat)
+    o = _attention_torch(tq, tk, tv, q_pos, scale)
+    (o * torch.as_tensor(np.asarray(d_out, dtype=np.float64))).sum().backward()
+    return tq.grad.numpy(), tk.grad.numpy(), tv.grad.numpy()
+
+
+def _rope_torch(y, pos, base):
+    D = y.shape[-1]
+    half = D // 2
+    theta = base ** (-2.0 * torch.arange(half, dtype=torch.float64) / D)
+    ang = torch.as_tensor(np.asarray(pos, dtype=np.float64))[:, None] * theta[None, :]
+    c, s = torch.cos(ang), torch.sin(ang)
+    x1, x2 = y[..., :half], y[..., half:]
+    return torch.cat([x1 * c - x2 * s, x2 * c + x1 * s], dim=-1)
+
+
+def _project_torch(x, w_qkv, lora_t, alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0,
+                   rope_base):
+    B, L, _ = x.shape
+    D = head_dim
+    bounds = {"q": (0, n_q_heads * D),
+              "k": (n_q_heads * D, (n_q_heads + n_kv_heads) * D),
+              "v": ((n_q_heads + n_kv_heads) * D, (n_q_heads + 2 * n_kv_heads) * D)}
+    heads = {"q": n_q_heads, "k": n_kv_heads, "v": n_kv_heads}
+    pos = pos0 + np.arange(L)
+    out = []
+    for p in "qkv":
+        lo, hi = bounds[p]
+        y = x @ w_qkv[lo:hi].T
+        if lora_t.get(p) is not None:
+            a, b = lora_t[p]
+            y = y + alpha_over_r * ((x @ a.T) @ b.T)
+        y = y.reshape(B, L, heads[p], D).transpose(1, 2)
+        if p in "qk" and rope_base > 0:
+            y = _rope_torch(y, pos, rope_base)
+        out.append(y)
+    return out
+
+
+def lora_backward(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, d_q, d_k,
+                  d_v, pos0=0, rope_base=0.0):
+    """Gradients of the rank-r factors, {p: (dA_p, dB_p)} in fp64, given the
+    gradients d_q [B, Hq, L, D], d_k, d_v [B, Hkv, L, D] of the projection's
+    outputs (q and k after RoPE) for the L tokens of x."""
+    f64 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.float64))
+    lora_t = {}
+    for p in "qkv":
+        if lora.get(p) is None:
+            lora_t[p] = None
+        else:
+            a, b = (f64(m).clone().requires_grad_(True) for m in lora[p])
+            lora_t[p] = (a, b)
+    q, k, v = _project_torch(f64(x), f64(w_qkv), lora_t, alpha_over_r, n_q_heads, n_kv_heads,
+                             head_dim, pos0, rope_base)
+    loss = (q * f64(d_q)).sum() + (k * f64(d_k)).sum() + (v * f64(d_v)).sum()
+    leaves = [t for p in "qkv" if lora_t[p] is not None for t in lora_t[p]]
+    if leaves:
+        loss.backward()
+    return {p: None if lora_t[p] is None else tuple(t.grad.numpy() for t in lora_t[p])
+            for p in "qkv"}
