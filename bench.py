@@ -484,6 +484,113 @@ def cold_graph_time_ms(fn, reps, flush):
     return statistics.mean(ms)
 
 
+def nf4_projection_rates(run, peaks, flush):
+    """The projection of layer 0 over an NF4 base (kvq_project_lora_nf4) at the
+    workload's prefill rows (tensor bound) and decode rows (HBM bound: codes,
+    absmax, LoRA factors, x and outputs), beside the bf16-base rows above.
+    None when the head shapes are outside the NF4 kernel's range."""
+    wl = run.wl
+    D = wl.head_dim
+    if D not in (64, 128) or (wl.n_q_heads * D) % 128 or (wl.n_kv_heads * D) % 128:
+        return None
+    codes, absmax = synth.nf4_base(wl, 0)
+    tc = torch.from_numpy(codes).to(run.dev)
+    ta = torch.from_numpy(absmax).to(run.dev)
+    lora = run.layers[0][1]
+    args = (wl.alpha_over_r, wl.n_q_heads, wl.n_kv_heads, D)
+
+    def pre():
+        run.api.project_lora_nf4(run.x_pre, tc, ta, lora, *args, rope_base=wl.rope_base,
+                                 out=run.pre)
+
+    def dec():
+        run.api.project_lora_nf4(run.xs, tc, ta, lora, *args, pos0=wl.prefill,
+                                 rope_base=wl.rope_base, out=run.dec)
+    pre_ms = cold_graph_time_ms(pre, 3, flush)
+    dec_ms = cold_graph_time_ms(dec, 10, flush)
+    flops = proj_flops(wl, wl.batch * wl.prefill)
+    r = wl.rank
+    dec_bytes = (codes.nbytes + absmax.nbytes + 2 * (3 * r * wl.d_in + r * wl.n_out)
+                 + 2 * wl.batch * (wl.d_in + wl.n_out))
+    return {"prefill": {"mean_ms": round(pre_ms, 4), "rows": wl.batch * wl.prefill,
+                        "achieved": round(flops / pre_ms / 1e9, 3), "unit": "TFLOP/s",
+                        "frac": round(flops / pre_ms / 1e9 / peaks["bf16_tflops_sustained"], 4)},
+            "decode": {"mean_ms": round(dec_ms, 5), "rows": wl.batch,
+                       "algorithmic_bytes": dec_bytes,
+                       "achieved": round(dec_bytes / dec_ms / 1e6, 3), "unit": "GB/s",
+                       "frac": round(dec_bytes / dec_ms / 1e6 / peaks["hbm_gbs"], 4)},
+            "l2": "flushed before each timed launch"}
+
+
+# fp32 FMA rate of the GB300: 152 SMs x 128 fp32 lanes x 2 flops x 2070 MHz
+FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
+
+
+def ste_backward_rates(run, flush, max_len=2048):
+    """The straight-through backward of one layer (kvq_attend_backward, then
+    kvq_lora_backward with d_x) for one sequence of min(prefill, 2048) tokens
+    of the workload's shape and cache format: the adapter-training step.  Its
+    products run on fp32 SIMT GEMMs, so the rates are against the fp32 FMA
+    rate.  None for KVarN caches (no backward)."""
+    from paper_2609_04263_gb300 import kvq
+    wl, api = run.wl, run.api
+    if wl.fmt == synth.FMT_KVARN:
+        return None
+    L, D, Hq, Hkv, d_in, r = min(wl.prefill, max_len), wl.head_dim, wl.n_q_heads, \
+        wl.n_kv_heads, wl.d_in, wl.rank
+    dev, dt = run.dev, run.dt
+    desc = api.make_desc(wl.fmt, wl.key_bits, wl.value_bits, wl.group_size, 1, Hkv, Hq, D, L,
+                         dt, residual_tokens=wl.residual_tokens)
+    cache = api.Cache(desc, device=dev)
+    x = run.x_pre[:1, :L].contiguous()
+    w, lora = run.layers[0]
+    q, k, v = api.project_lora(x, w, lora, wl.alpha_over_r, Hq, Hkv, D, rope_base=wl.rope_base)
+    cache.append(k, v)
+    g = torch.Generator(device="cpu").manual_seed(7)
+    d_out = torch.randn(q.shape, generator=g).to(dt).to(dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty(1, Hq, L, D, **f32), torch.empty(1, Hkv, L, D, **f32), \
+        torch.empty(1, Hkv, L, D, **f32)
+    ws_bytes = kvq.kvq_attend_backward_workspace(cache.handle, L, Hq) * Hkv
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    lws_bytes = kvq.kvq_lora_backward_workspace(1, L, Hq, Hkv, D, r, r, r)
+    lws = torch.empty(lws_bytes, dtype=torch.uint8, device=dev)
+    grads = [torch.empty(lora[p][i].shape, **f32) for p in "qkv" for i in (0, 1)]
+    dx = torch.empty(1, L, d_in, **f32)
+    scale = 1.0 / math.sqrt(D)
+    ptr = lambda t: t.data_ptr()
+
+    def attn():
+        kvq.kvq_attend_backward(cache.handle, ptr(q), ptr(d_out), L, Hq, scale, ptr(dq),
+                                ptr(dk), ptr(dv), ptr(ws), ws_bytes,
+                                torch.cuda.current_stream().cuda_stream)
+
+    def adapters():
+        fac = [a for p in "qkv" for a in (ptr(lora[p][0]), ptr(lora[p][1]), r)]
+        kvq.kvq_lora_backward(ptr(x), 1, L, d_in, ptr(w), *fac, wl.alpha_over_r, Hq, Hkv, D, 0,
+                              wl.rope_base, 1 if dt == torch.bfloat16 else 0, ptr(dq), ptr(dk),
+                              ptr(dv), L, *[ptr(t) for t in grads], ptr(dx), ptr(lws),
+                              lws_bytes, torch.cuda.current_stream().cuda_stream)
+    att_ms = cold_graph_time_ms(attn, 3, flush)
+    lora_ms = cold_graph_time_ms(adapters, 3, flush)
+    visible = L * (L + 1) // 2
+    att_flops = 10 * D * Hq * visible             # S, dP, dQ, dK, dV: 2 D per visible pair
+    n_out = (Hq + 2 * Hkv) * D
+    lora_flops = (2 * L * d_in * 3 * r + 2 * 2 * L * r * n_out + 2 * L * r * 3 * d_in
+                  + 2 * L * n_out * d_in + 2 * L * 3 * r * d_in)
+    rate = lambda f, ms: round(f / ms / 1e9, 3)
+    return {"tokens": L, "sequences": 1,
+            "attention": {"mean_ms": round(att_ms, 4), "flops": att_flops,
+                          "achieved": rate(att_flops, att_ms), "unit": "TFLOP/s",
+                          "frac": round(att_flops / att_ms / 1e9 / FP32_FMA_TFLOPS, 4)},
+            "adapters": {"mean_ms": round(lora_ms, 4), "flops": lora_flops,
+                         "achieved": rate(lora_flops, lora_ms), "unit": "TFLOP/s",
+                         "frac": round(lora_flops / lora_ms / 1e9 / FP32_FMA_TFLOPS, 4)},
+            "peak": {"bound": "alu", "value": round(FP32_FMA_TFLOPS, 2), "unit": "TFLOP/s",
+                     "what": "fp32 FMA: 152 SMs x 128 lanes x 2 flops x 2070 MHz"},
+            "l2": "flushed before each timed launch"}
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle (the reported baseline and the reference arm)
 # ---------------------------------------------------------------------------
@@ -762,6 +869,8 @@ def main():
                         "unit": "GB/s", "frac": round(att_rate / peaks["hbm_gbs"], 4),
                         "l2": "flushed before each replay of all layers' calls",
                         "traffic": measured_traffic(wl.name, "decode_attention")}
+    nf4 = nf4_projection_rates(run, peaks, flush) if wl.dtype == "bf16" else None
+    ste = ste_backward_rates(run, flush)
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)
     bound, amount, _ = work[dominant]
@@ -836,6 +945,8 @@ def main():
                          "algorithmic_bytes" if bound == "hbm" else "algorithmic_flops": amount},
             "kernels": kernels,
             "decode_attention": decode_attention,
+            "nf4_projection": nf4,
+            "ste_backward": ste,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},

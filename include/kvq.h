@@ -14,6 +14,8 @@
  *   kvq_attend_prefill  Sections 3.1-3.3: causal attention of the newly
  *   kvq_attend_decode   appended tokens over the stored reconstruction
  *                       R_phi(K, V) of every cached token.
+ *   kvq_attend_backward Section 3.3: straight-through backward (x_hat + x -
+ *   kvq_lora_backward   stopgrad(x)) through attention into the adapters.
  *
  * Conventions for every call:
  *   - Tensor arguments are DEVICE pointers owned by the caller, row-major and
@@ -331,6 +333,58 @@ int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, in
  */
 kvq_status kvq_attend_decode_noalloc(kvq_cache* cache, const void* q, int n_q_heads,
                                      float softmax_scale, void* out, void* stream);
+
+/*
+ * Backward of attention over the stored reconstruction (Section 3.3): the
+ * gradients of sum(out * d_out) for out = kvq_attend_prefill(q) of the L
+ * newest queries over all T cached tokens.  Appended states enter attention
+ * as x_hat + x - stopgrad(x) (the straight-through estimator), so d_k and d_v,
+ * the gradients at the reconstruction x_hat, are also the gradients of the
+ * keys and values that were coded into the cache, and feed the K and V
+ * adapters unchanged (kvq_lora_backward).
+ *   q, d_out  [B][Hq][L][D] in the cache's dtype (d_out: gradient of out)
+ *   d_q       [B][Hq][L][D] fp32
+ *   d_k, d_v  [B][Hkv][T][D] fp32 (every query head of a kv head's group
+ *             summed; tokens no query sees get 0)
+ * workspace: caller-owned device memory, at least
+ * kvq_attend_backward_workspace() bytes (one (sequence, kv head) pair's fp32
+ * reconstruction, scores and score gradients); a larger workspace processes
+ * that many pairs per pass.  Formats FLOAT, AFFINE, SYMMETRIC and KIVI;
+ * KVarN returns KVQ_ERR_UNSUPPORTED.  Too small a workspace returns
+ * KVQ_ERR_CAPACITY.  The cache is not modified.
+ */
+size_t kvq_attend_backward_workspace(const kvq_cache* cache, int L, int n_q_heads);
+kvq_status kvq_attend_backward(kvq_cache* cache, const void* q, const void* d_out, int L,
+                               int n_q_heads, float softmax_scale, float* d_q, float* d_k,
+                               float* d_v, void* workspace, size_t workspace_bytes,
+                               void* stream);
+
+/*
+ * Backward of kvq_project_lora into its rank-r factors (Eq. (1), Eq. (lora),
+ * Section 3.4: the base W stays frozen).  d_q [B][Hq][L][D], d_k and d_v
+ * [B][Hkv][kv_rows][D] (fp32) are gradients of the projection's outputs after
+ * RoPE; the last L of each head's kv_rows rows belong to the L tokens of x
+ * (kv_rows = T passes kvq_attend_backward's d_k, d_v directly when the cache
+ * holds x's tokens last).  Writes, in fp32:
+ *   da_p [r_p][d_in] = (alpha/r) (g_p B_p)^T x,  db_p [n_p][r_p] = (alpha/r) g_p^T (x A_p^T)
+ * where g_p is the gradient before RoPE, and, if d_x is not NULL,
+ *   d_x [B][L][d_in] = g W + sum_p (alpha/r) (g_p B_p) A_p   (needs w_qkv).
+ * x, w_qkv and the factors are in `dtype`, laid out as for kvq_project_lora;
+ * a projection with r_p = 0 has no factors and its gradients are not written.
+ * workspace: at least kvq_lora_backward_workspace() bytes.
+ */
+size_t kvq_lora_backward_workspace(int B, int L, int n_q_heads, int n_kv_heads, int head_dim,
+                                   int r_q, int r_k, int r_v);
+kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* w_qkv,
+                             const void* a_q, const void* b_q, int r_q,
+                             const void* a_k, const void* b_k, int r_k,
+                             const void* a_v, const void* b_v, int r_v,
+                             float alpha_over_r, int n_q_heads, int n_kv_heads, int head_dim,
+                             int pos0, float rope_base, int dtype,
+                             const float* d_q, const float* d_k, const float* d_v, int kv_rows,
+                             float* da_q, float* db_q, float* da_k, float* db_k,
+                             float* da_v, float* db_v, float* d_x,
+                             void* workspace, size_t workspace_bytes, void* stream);
 
 /* Read and clear the device-side error word of the library (synchronises
  * `stream`).  *out = 0 when no bounded wait has timed out; otherwise a kernel

@@ -125,6 +125,27 @@ class Cache:
         r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
         return kvq.kvq_decode_step_fused(self.handle, d_in, *r)
 
+    def attend_backward(self, q, d_out, scale=None, workspace=None):
+        """Straight-through backward of attend_prefill(q): returns fp32
+        (d_q [B,Hq,L,D], d_k, d_v [B,Hkv,T,D]), the gradients at the stored
+        reconstruction, which by the estimator are those of the coded keys
+        and values.  workspace: a uint8 device tensor (default: all pairs in
+        one pass)."""
+        d = self.desc
+        B, Hq, L, D = q.shape
+        T = self.tokens
+        per = kvq.kvq_attend_backward_workspace(self.handle, L, Hq)
+        if workspace is None:
+            workspace = torch.empty(per * B * d.kv_heads, dtype=torch.uint8, device=q.device)
+        scale = 1.0 / math.sqrt(D) if scale is None else scale
+        f32 = dict(dtype=torch.float32, device=q.device)
+        dq = torch.empty(B, Hq, L, D, **f32)
+        dk = torch.empty(B, d.kv_heads, T, D, **f32)
+        dv = torch.empty(B, d.kv_heads, T, D, **f32)
+        kvq.kvq_attend_backward(self.handle, _ptr(q), _ptr(d_out), L, Hq, scale, _ptr(dq),
+                                _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(), _stream())
+        return dq, dk, dv
+
     def planes(self) -> dict:
         """name -> tensor view [B, H, rows, cols] of each present plane."""
         v = kvq.kvq_cache_view(self.handle)
@@ -195,3 +216,35 @@ def project_lora_nf4(x, w_codes, w_absmax, lora, alpha_over_r, n_q_heads, n_kv_h
                              pos_cache.handle if pos_cache is not None else None, rope_base,
                              _ptr(out[0]), _ptr(out[1]), _ptr(out[2]), _stream())
     return out
+
+
+def lora_backward(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim, d_q, d_k, d_v,
+                  pos0=0, rope_base=0.0, want_dx=False, workspace=None):
+    """Gradients of the rank-r factors of project_lora given fp32 gradients of
+    its outputs (d_q [B,Hq,L,D]; d_k, d_v [B,Hkv,kv_rows,D], the last L rows
+    belonging to x's tokens).  Returns ({p: (dA_p, dB_p) or None}, d_x or None),
+    fp32; the base weight stays frozen (w_qkv is read only for d_x)."""
+    B, L, d_in = x.shape
+    D = head_dim
+    r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
+    if workspace is None:
+        nb = kvq.kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, D, *r)
+        workspace = torch.empty(nb, dtype=torch.uint8, device=x.device)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    grads, args = {}, []
+    for i, p in enumerate("qkv"):
+        ab = lora.get(p)
+        if ab is None:
+            grads[p] = None
+            args += [None, None, 0]
+        else:
+            grads[p] = (torch.empty(ab[0].shape, **f32), torch.empty(ab[1].shape, **f32))
+            args += [_ptr(ab[0]), _ptr(ab[1]), r[i]]
+    gp = [None if grads[p] is None else _ptr(t) for p in "qkv" for t in (grads[p] or (None, None))]
+    dx = torch.empty(B, L, d_in, **f32) if want_dx else None
+    kvq.kvq_lora_backward(_ptr(x), B, L, d_in, _ptr(w_qkv), *args, alpha_over_r, n_q_heads,
+                          n_kv_heads, D, pos0, rope_base, _DT[x.dtype], _ptr(d_q), _ptr(d_k),
+                          _ptr(d_v), d_k.shape[2], *gp, _ptr(dx), _ptr(workspace),
+                          workspace.numel(), _stream())
+    return grads, dx
+

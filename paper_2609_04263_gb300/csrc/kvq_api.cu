@@ -612,6 +612,95 @@ int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, in
   return cache->g.act == KVQ_BF16 && decode_step_supported(cache->g, d_in, r) ? 1 : 0;
 }
 
+static const char* attend_backward_gap(const kvq_cache* c, int L, int n_q_heads) {
+  if (c->g.fmt == KVQ_FMT_KVARN) return "KVarN caches have no backward";
+  if (L <= 0) return "L must be positive";
+  if (n_q_heads != c->g.Hq) return "n_q_heads differs from the cache's q_heads";
+  if (L > c->T) return "more queries than cached tokens (append first)";
+  return nullptr;
+}
+
+size_t kvq_attend_backward_workspace(const kvq_cache* cache, int L, int n_q_heads) {
+  if (!cache || attend_backward_gap(cache, L, n_q_heads)) return 0;
+  return attend_backward_pair_bytes(cache->g, cache->T, L);
+}
+
+kvq_status kvq_attend_backward(kvq_cache* cache, const void* q, const void* d_out, int L,
+                               int n_q_heads, float softmax_scale, float* d_q, float* d_k,
+                               float* d_v, void* workspace, size_t workspace_bytes,
+                               void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (const char* gap = attend_backward_gap(cache, L, n_q_heads))
+    return fail(cache->g.fmt == KVQ_FMT_KVARN ? KVQ_ERR_UNSUPPORTED : KVQ_ERR_SHAPE,
+                "kvq_attend_backward: %s", gap);
+  if (!q || !d_out || !d_q || !d_k || !d_v || !workspace)
+    return fail(KVQ_ERR_ARG, "NULL tensor pointer");
+  if (misaligned(q) || misaligned(d_out) || misaligned(d_q) || misaligned(d_k) ||
+      misaligned(d_v) || misaligned(workspace))
+    return fail(KVQ_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  if (!(softmax_scale > 0.f)) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
+  const size_t per = attend_backward_pair_bytes(cache->g, cache->T, L);
+  if (workspace_bytes < per)
+    return fail(KVQ_ERR_CAPACITY, "workspace of %zu bytes < %zu (one sequence and kv head)",
+                workspace_bytes, per);
+  cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
+  if (e == cudaSuccess)
+    e = launch_attend_backward(cache->g, cache->T, q, d_out, L, softmax_scale, d_q, d_k, d_v,
+                               workspace, workspace_bytes, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_attend_backward launch");
+  return KVQ_OK;
+}
+
+size_t kvq_lora_backward_workspace(int B, int L, int n_q_heads, int n_kv_heads, int head_dim,
+                                   int r_q, int r_k, int r_v) {
+  if (B <= 0 || L <= 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0 || r_q < 0 ||
+      r_k < 0 || r_v < 0)
+    return 0;
+  const int r[3] = {r_q, r_k, r_v};
+  return lora_backward_bytes(B, L, n_q_heads, n_kv_heads, head_dim, r);
+}
+
+kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* w_qkv,
+                             const void* a_q, const void* b_q, int r_q,
+                             const void* a_k, const void* b_k, int r_k,
+                             const void* a_v, const void* b_v, int r_v,
+                             float alpha_over_r, int n_q_heads, int n_kv_heads, int head_dim,
+                             int pos0, float rope_base, int dtype,
+                             const float* d_q, const float* d_k, const float* d_v, int kv_rows,
+                             float* da_q, float* db_q, float* da_k, float* db_k,
+                             float* da_v, float* db_v, float* d_x,
+                             void* workspace, size_t workspace_bytes, void* stream) {
+  if (dtype != KVQ_F32 && dtype != KVQ_BF16) return fail(KVQ_ERR_ARG, "unknown dtype %d", dtype);
+  if (B <= 0 || L <= 0 || d_in <= 0) return fail(KVQ_ERR_SHAPE, "bad B/L/d_in");
+  if (n_q_heads <= 0 || n_kv_heads <= 0 || n_q_heads % n_kv_heads)
+    return fail(KVQ_ERR_SHAPE, "heads %d/%d", n_q_heads, n_kv_heads);
+  if (head_dim != 64 && head_dim != 128 && head_dim != 256)
+    return fail(KVQ_ERR_UNSUPPORTED, "head_dim %d (supported: 64, 128, 256)", head_dim);
+  if (pos0 < 0 || !(rope_base >= 0.f)) return fail(KVQ_ERR_ARG, "pos0 < 0 or rope_base < 0");
+  if (kv_rows < L) return fail(KVQ_ERR_SHAPE, "kv_rows %d < L %d", kv_rows, L);
+  if (!x || !d_q || !d_k || !d_v || !workspace) return fail(KVQ_ERR_ARG, "NULL tensor pointer");
+  if (d_x && !w_qkv) return fail(KVQ_ERR_ARG, "d_x needs w_qkv");
+  const void* a[3] = {a_q, a_k, a_v};
+  const void* bm[3] = {b_q, b_k, b_v};
+  float* da[3] = {da_q, da_k, da_v};
+  float* db[3] = {db_q, db_k, db_v};
+  const int r[3] = {r_q, r_k, r_v};
+  for (int p = 0; p < 3; ++p) {
+    if (r[p] < 0 || r[p] > 64) return fail(KVQ_ERR_SHAPE, "rank %d outside [0, 64]", r[p]);
+    if (r[p] > 0 && (!a[p] || !bm[p] || !da[p] || !db[p]))
+      return fail(KVQ_ERR_ARG, "rank %d but a NULL factor or gradient", r[p]);
+  }
+  const size_t need = lora_backward_bytes(B, L, n_q_heads, n_kv_heads, head_dim, r);
+  if (workspace_bytes < need)
+    return fail(KVQ_ERR_CAPACITY, "workspace of %zu bytes < %zu", workspace_bytes, need);
+  if (misaligned(workspace)) return fail(KVQ_ERR_ARG, "workspace must be 16-byte aligned");
+  cudaError_t e = launch_lora_backward(x, B, L, d_in, w_qkv, a, bm, r, alpha_over_r, n_q_heads,
+                                       n_kv_heads, head_dim, pos0, rope_base, dtype, d_q, d_k,
+                                       d_v, kv_rows, da, db, d_x, workspace, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_lora_backward launch");
+  return KVQ_OK;
+}
+
 kvq_status kvq_device_status(void* stream, int* out) {
   if (!out) return fail(KVQ_ERR_ARG, "out is NULL");
   int* p = device_error_word();

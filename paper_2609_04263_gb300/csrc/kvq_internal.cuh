@@ -148,6 +148,22 @@ cudaError_t launch_project_nf4(const void* x, int B, int L, int d_in, const void
                                float rope_base, void* const out[3], cudaStream_t s);
 void rope_theta_table(float rope_base, int D, float* hi, float* lo);
 
+// Straight-through backward (backward.cu): attention over a cache's
+// reconstruction, then the adapters.  Workspace bytes per (sequence, kv head)
+// pair of the attention backward, and of the adapter backward.
+size_t attend_backward_pair_bytes(const Geom& g, int T, int L);
+cudaError_t launch_attend_backward(const Geom& g, int T, const void* q, const void* d_out,
+                                   int L, float scale, float* dq, float* dk, float* dv,
+                                   void* ws, size_t ws_bytes, cudaStream_t s);
+size_t lora_backward_bytes(int B, int L, int Hq, int Hkv, int D, const int r[3]);
+cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const void* w,
+                                 const void* const a[3], const void* const bm[3],
+                                 const int r[3], float alpha_over_r, int Hq, int Hkv, int D,
+                                 int pos0, float rope_base, int act, const float* dq,
+                                 const float* dk, const float* dv, int kv_rows,
+                                 float* const da[3], float* const db[3], float* dx, void* ws,
+                                 cudaStream_t s);
+
 // Fused decode step (decode_step.cu): projection of the new token, append,
 // decode attention in one cooperative kernel.
 bool decode_step_supported(const Geom& g, int d_in, const int r[3]);

@@ -81,6 +81,18 @@ _SIGS = {
                                      c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
                                      c_int, c_void_p, c_float, c_void_p, c_void_p, c_void_p,
                                      c_void_p]),
+    "kvq_attend_backward_workspace": (c_size_t, [c_void_p, c_int, c_int]),
+    "kvq_attend_backward": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_float,
+                                    c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
+                                    c_void_p]),
+    "kvq_lora_backward_workspace": (c_size_t, [c_int, c_int, c_int, c_int, c_int, c_int, c_int,
+                                               c_int]),
+    "kvq_lora_backward": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p,
+                                  c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
+                                  c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
+                                  c_int, c_float, c_int, c_void_p, c_void_p, c_void_p, c_int,
+                                  c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                  c_void_p, c_void_p, c_size_t, c_void_p]),
 }
 
 _lib = None
@@ -223,3 +235,34 @@ def kvq_project_lora_nf4(x, B, L, d_in, w_codes, w_absmax, a_q, b_q, r_q, a_k, b
         c_void_p(b_q), r_q, c_void_p(a_k), c_void_p(b_k), r_k, c_void_p(a_v), c_void_p(b_v), r_v,
         alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, c_void_p(pos_cache), rope_base,
         c_void_p(q), c_void_p(k), c_void_p(v), c_void_p(stream or 0)))
+
+
+def kvq_attend_backward_workspace(handle, L, n_q_heads) -> int:
+    return lib().kvq_attend_backward_workspace(c_void_p(handle), L, n_q_heads)
+
+
+def kvq_attend_backward(handle, q, d_out, L, n_q_heads, softmax_scale, d_q, d_k, d_v,
+                        workspace, workspace_bytes, stream=0) -> None:
+    _check(lib().kvq_attend_backward(c_void_p(handle), c_void_p(q), c_void_p(d_out), L,
+                                     n_q_heads, softmax_scale, c_void_p(d_q), c_void_p(d_k),
+                                     c_void_p(d_v), c_void_p(workspace), workspace_bytes,
+                                     c_void_p(stream or 0)))
+
+
+def kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, head_dim, r_q, r_k, r_v) -> int:
+    return lib().kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, head_dim, r_q, r_k,
+                                             r_v)
+
+
+def kvq_lora_backward(x, B, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,
+                      alpha_over_r, n_q_heads, n_kv_heads, head_dim, pos0, rope_base, dtype,
+                      d_q, d_k, d_v, kv_rows, da_q, db_q, da_k, db_k, da_v, db_v, d_x,
+                      workspace, workspace_bytes, stream=0) -> None:
+    _check(lib().kvq_lora_backward(
+        c_void_p(x), B, L, d_in, c_void_p(w_qkv), c_void_p(a_q), c_void_p(b_q), r_q,
+        c_void_p(a_k), c_void_p(b_k), r_k, c_void_p(a_v), c_void_p(b_v), r_v, alpha_over_r,
+        n_q_heads, n_kv_heads, head_dim, pos0, rope_base, dtype, c_void_p(d_q), c_void_p(d_k),
+        c_void_p(d_v), kv_rows, c_void_p(da_q), c_void_p(db_q), c_void_p(da_k), c_void_p(db_k),
+        c_void_p(da_v), c_void_p(db_v), c_void_p(d_x), c_void_p(workspace), workspace_bytes,
+        c_void_p(stream or 0)))
+

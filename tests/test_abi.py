@@ -182,3 +182,45 @@ def test_project_append_shape_rules_on_the_host(kvq):
         finally:
             kvq.kvq_destroy_cache(h)
     assert kvq.kvq_project_append_supported(None, 32, 2048, 16, 16, 16) is False
+
+
+def test_backward_host_rules(kvq):
+    """The straight-through backward refuses, before any launch: queries
+    beyond the cached tokens, KVarN caches, too small a workspace; the
+    adapter backward's workspace is the pre-RoPE gradient plus two rank-wide
+    buffers per adapter."""
+    fake = 1 << 32
+    P = 1 << 33
+    d = _desc(kvq, max_tokens=64)
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        assert kvq.kvq_attend_backward_workspace(h, 1, d.q_heads) == 0     # nothing cached
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_attend_backward(h, P, P, 1, d.q_heads, 0.125, P, P, P, P, 1 << 30, 0)
+        assert ei.value.status == kvq.KVQ_ERR_SHAPE
+    finally:
+        kvq.kvq_destroy_cache(h)
+    d = _desc(kvq, max_tokens=256, fmt=kvq.KVQ_FMT_KVARN, group_size=64, sink_tokens=16)
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        with pytest.raises(kvq.KvqError) as ei:
+            kvq.kvq_attend_backward(h, P, P, 1, d.q_heads, 0.125, P, P, P, P, 1 << 30, 0)
+        assert ei.value.status == kvq.KVQ_ERR_UNSUPPORTED
+    finally:
+        kvq.kvq_destroy_cache(h)
+    B, L, Hq, Hkv, D, r = 2, 100, 8, 2, 64, (16, 0, 8)
+
+    def a256(n):
+        return (n + 255) // 256 * 256
+    want = a256(B * L * (Hq + 2 * Hkv) * D * 4) + sum(2 * a256(B * L * x * 4) for x in r)
+    assert kvq.kvq_lora_backward_workspace(B, L, Hq, Hkv, D, *r) == want
+    with pytest.raises(kvq.KvqError) as ei:
+        kvq.kvq_lora_backward(P, B, L, 256, P, P, P, 16, None, None, 0, P, P, 8, 2.0, Hq, Hkv, D,
+                              0, 1e4, kvq.KVQ_BF16, P, P, P, L, P, P, None, None, P, P, None,
+                              P, want - 1, 0)
+    assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+    with pytest.raises(kvq.KvqError) as ei:                 # kv_rows < L
+        kvq.kvq_lora_backward(P, B, L, 256, P, P, P, 16, None, None, 0, P, P, 8, 2.0, Hq, Hkv, D,
+                              0, 1e4, kvq.KVQ_BF16, P, P, P, L - 1, P, P, None, None, P, P, None,
+                              P, want, 0)
+    assert ei.value.status == kvq.KVQ_ERR_SHAPE
