@@ -67,6 +67,38 @@ __device__ __forceinline__ uint32_t pair_group(uint32_t wa, uint32_t wb, int gq)
   return __byte_perm(wa, wb, (gq & 1) ? 0x7632 : 0x5410);
 }
 
+// KIVI keys, read in place.  A 32-bit word of a token's codes holds CPW
+// channels, the first CPW / 2 in its low half and the rest in its high half,
+// each at bit KB p of its half.  (w >> sh) & (mask << KB j) | 0x64006400 is
+// the pair (channel p, channel CPW / 2 + p) as fp16 1024 + c 2^(KB j) for
+// p = PER sh / (KB PER) + j, j < PER: a LOP3 per pair (and a shift per PER
+// pairs).  PER keeps 2^(KB j) <= 16, so the weights 2^-(KB j) folded into the
+// query operand and 2^(KB j) into the zero points stay far from fp16's range.
+// Register i of a thread is position i % RPW of its code word i / RPW; the
+// thread reads words tid NWT .. tid NWT + NWT - 1 of a token.
+template <int D, int KB>
+struct KPos {
+  static constexpr int CPW = 32 / KB;                 // channels per code word
+  static constexpr int RPW = CPW / 2;                 // register pairs per word
+  static constexpr int NWT = D * KB / 128;            // code words per thread and token
+  static constexpr int NR = NWT * RPW;                // = D / 8 registers per token
+  static constexpr int PER = KB == 2 ? 3 : 2;         // positions per shift
+  static constexpr uint32_t MASK = KB == 2 ? 0x00030003u : 0x000F000Fu;
+  __host__ __device__ static constexpr int e(int p) { return KB * (p % PER); }
+  // channels (within the thread's D / 4) of register i's low and high halves
+  __host__ __device__ static constexpr int lo(int i) { return (i / RPW) * CPW + i % RPW; }
+  __host__ __device__ static constexpr int hi(int i) { return lo(i) + CPW / 2; }
+  // register i from its code word w
+  __device__ static __forceinline__ uint32_t get(int i, uint32_t w) {
+    const int p = i % RPW;
+    return magic2h(w >> (KB * PER * (p / PER)), MASK << e(p));
+  }
+};
+// fp16 pair (2^e, 2^e), 0 <= e <= 15
+__host__ __device__ constexpr uint32_t pow2_h2(int e) {
+  return ((uint32_t)(15 + e) << 10) | ((uint32_t)(15 + e) << 26);
+}
+
 template <int D, int KB, int VB, int FMT>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err,
@@ -208,21 +240,53 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   const uint32_t vmask = VB == 4 ? 0x000F000Fu : 0x00030003u;
   const int zb = C::SYM ? (1 << (KB - 1)) : 0;       // symmetric key code bias
   const int zbv = C::SYM ? (1 << (VB - 1)) : 0;
-  const __half kbias = __float2half_rn(1024.f + (float)zbv);
-  const uint32_t kbias2 = h2u(kbias, kbias);
+  // values: bits between a thread's consecutive channels, and the bit of the
+  // channel of row gid in m-tile u (see the P V step)
+  constexpr int SH = VB == 4 ? 4 : 2;
+  auto vsh = [](int u) { return VB == 4 ? 0 : 2 * SH * u; };
   const int tc = threadIdx.x;                        // 0 .. kNW * 32 - 1
   float* wsb = reinterpret_cast<float*>(g.pl[KVQ_PLANE_WORKSPACE].p);
 
   int b = 0, hkv = 0;
   bool bad = false;                                  // a wait timed out: stop computing
-  uint32_t qb[KSS][2];                               // B fragments of q (head gid)
-  float qs[NG][2];                                   // per-group sum of q, heads 2tid, 2tid+1
+  using KP = KPos<D, KB>;
+  // per-token keys: B fragments of q (head gid) and per-group sums of q;
+  // KIVI keys: q of head gid in the positional layout, q_d 2^-e as fp16
+  uint32_t qb[C::KIVI ? 1 : KSS][2];
+  float qs[C::KIVI ? 1 : NG][2];
+  uint32_t qw[C::KIVI ? KP::NR : 1];
   float m_run[2], l_run[2];
   float o[MT][4], bias[NG][4], offa[4];
+  bool folded = false;          // the coded blocks' terms are folded into o
 
-  // q of the head: thread (gid, tid) holds head gid, channels 32 gq + 8 tid + e
+  // bf16 B fragments of q in the qk_chan layout (head gid, channels 32 gq + 8 tid + e)
+  auto q_frags = [&](uint32_t (&f)[KSS][2]) {
+    const __nv_bfloat16* qh = q + ((int64_t)b * g.Hq + hkv * grp) * D;
+#pragma unroll
+    for (int gq = 0; gq < NG; ++gq) {
+      uint4 u = make_uint4(0, 0, 0, 0);
+      if (gid < grp) u = *reinterpret_cast<const uint4*>(qh + gid * D + 32 * gq + 8 * tid);
+      const uint16_t* e = reinterpret_cast<const uint16_t*>(&u);
+#pragma unroll
+      for (int sub = 0; sub < 2; ++sub) {
+        f[2 * gq + sub][0] = pack_raw(e[qk_chan<KB>(sub, 0, 0)], e[qk_chan<KB>(sub, 0, 1)]);
+        f[2 * gq + sub][1] = pack_raw(e[qk_chan<KB>(sub, 1, 0)], e[qk_chan<KB>(sub, 1, 1)]);
+      }
+    }
+  };
+
   auto load_q = [&]() {
     const __nv_bfloat16* qh = q + ((int64_t)b * g.Hq + hkv * grp) * D;
+    if constexpr (C::KIVI) {
+      const __nv_bfloat16* qr = qh + gid * D + tid * (D / 4);
+#pragma unroll
+      for (int i = 0; i < KP::NR; ++i) {
+        const float sc = 1.f / (float)(1 << KP::e(i % KP::RPW));
+        qw[i] = gid < grp ? pack_f16(__bfloat162float(qr[KP::lo(i)]) * sc,
+                                     __bfloat162float(qr[KP::hi(i)]) * sc)
+                          : 0u;
+      }
+    } else {
 #pragma unroll
     for (int gq = 0; gq < NG; ++gq) {
       uint4 u = make_uint4(0, 0, 0, 0);
@@ -245,6 +309,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
       qs[gq][0] = __shfl_sync(0xffffffffu, s, 4 * (2 * tid));
       qs[gq][1] = __shfl_sync(0xffffffffu, s, 4 * (2 * tid + 1));
     }
+    }
     m_run[0] = m_run[1] = -INFINITY;
     l_run[0] = l_run[1] = 0.f;
 #pragma unroll
@@ -252,6 +317,29 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
 #pragma unroll
     for (int i = 0; i < NG; ++i) bias[i][0] = bias[i][1] = bias[i][2] = bias[i][3] = 0.f;
     offa[0] = offa[1] = offa[2] = offa[3] = 0.f;
+    folded = false;
+  };
+
+  // Fold the coded blocks' code bias (bias[gq] = 1024 sum_t p s_tg), channel
+  // weights and offset terms into o.  Done once per head: before the first
+  // full-precision block (KIVI's newest tokens, whose values enter o as they
+  // are), else after the last block.
+  auto fold_o = [&]() {
+#pragma unroll
+    for (int gq = 0; gq < NG; ++gq) {
+      const float b0 = bias[gq][0], b1 = bias[gq][1];
+      const float f0 = __shfl_sync(0xffffffffu, offa[0], 4 * gq + tid) - (zbv / 1024.f) * b0;
+      const float f1 = __shfl_sync(0xffffffffu, offa[1], 4 * gq + tid) - (zbv / 1024.f) * b1;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const float w0 = 1.f / (float)(1 << vsh(u)), w1 = 1.f / (float)(1 << (vsh(u) + SH));
+        o[2 * gq + u][0] = fmaf(o[2 * gq + u][0] - b0, w0, f0);
+        o[2 * gq + u][1] = fmaf(o[2 * gq + u][1] - b1, w0, f1);
+        o[2 * gq + u][2] = fmaf(o[2 * gq + u][2] - b0, w1, f0);
+        o[2 * gq + u][3] = fmaf(o[2 * gq + u][3] - b1, w1, f1);
+      }
+    }
+    folded = true;
   };
 
   // one 32-token block: scores, online softmax, P V
@@ -263,7 +351,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
     const unsigned char* vsp = sp + C::VS + sub_blk * C::VMETA;
     const unsigned char* vzp = sp + C::VZ + sub_blk * C::VMETA;
     float S[2][4];
-    if (coded && !C::KIVI) {
+    if constexpr (!C::KIVI) {
       float acc[NG][2][4];
 #pragma unroll
       for (int gq = 0; gq < NG; ++gq)
@@ -320,86 +408,72 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
           S[mt][2 * r] = valid ? s0 * c2 : -INFINITY;
           S[mt][2 * r + 1] = valid ? s1 * c2 : -INFINITY;
         }
-    } else if (coded) {  // KIVI keys: B = q * s_blk (scaled) as bf16 high + low parts
-      const __half* ksc = reinterpret_cast<const __half*>(ksp);
-      const __half* kze = reinterpret_cast<const __half*>(kzp);
-      uint32_t qh[KSS][2], ql[KSS][2];
-      float qm = 0.f;                                // sum_d q_d m_d over this thread's channels
+    } else if (coded) {
+      // KIVI keys (one scale s_d and zero z_d per block and channel):
+      //   S_h = sum_d (q_hd s_d) c_d + sum_d q_hd z_d
+      // A = codes in place (1024 + c 2^e), B = q 2^-e s as fp16 hi + lo.
+      // the block's scales and zeros of the thread's D / 4 channels, as pairs
+      const uint32_t* sw = reinterpret_cast<const uint32_t*>(ksp) + tid * (D / 8);
+      const uint32_t* zw = reinterpret_cast<const uint32_t*>(kzp) + tid * (D / 8);
+      // code words of rows gid, gid + 8 of both 16-token halves
+      uint32_t cw[2][2][KP::NWT];
 #pragma unroll
-      for (int gq = 0; gq < NG; ++gq) {
-        const uint4 su = *reinterpret_cast<const uint4*>(ksc + 32 * gq + 8 * tid);
-        const uint4 zu = *reinterpret_cast<const uint4*>(kze + 32 * gq + 8 * tid);
-        const __half* sv = reinterpret_cast<const __half*>(&su);
-        const __half* zv = reinterpret_cast<const __half*>(&zu);
+      for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-        for (int sub = 0; sub < 2; ++sub)
+        for (int rr = 0; rr < 2; ++rr) {
+          const uint32_t* row = reinterpret_cast<const uint32_t*>(
+              kcp + (16 * mt + gid + 8 * rr) * C::KCB) + tid * KP::NWT;
 #pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            const int e0 = qk_chan<KB>(sub, hf, 0), e1 = qk_chan<KB>(sub, hf, 1);
-            const uint32_t qw = qb[2 * gq + sub][hf];
-            const float2 qq = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw));
-            const float x0 = qq.x * __half2float(sv[e0]);
-            const float x1 = qq.y * __half2float(sv[e1]);
-            const uint32_t hw = pack_bf16(x0, x1);
-            const float2 hv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hw));
-            qh[2 * gq + sub][hf] = hw;
-            ql[2 * gq + sub][hf] = pack_bf16(x0 - hv.x, x1 - hv.y);
-            qm += qq.x * __half2float(zv[e0]) + qq.y * __half2float(zv[e1]);
-          }
-      }
-      qm += __shfl_xor_sync(0xffffffffu, qm, 1);
-      qm += __shfl_xor_sync(0xffffffffu, qm, 2);     // head gid
-      // the codes enter as 128 + c: the same MMA over a constant 128 operand
-      // gives the 128 sum(hi + lo) to remove, per head, as the tensor core sums it
-      float bh[4] = {0.f, 0.f, 0.f, 0.f}, bl[4] = {0.f, 0.f, 0.f, 0.f};
-      const uint32_t a128[4] = {kMagic, kMagic, kMagic, kMagic};
+          for (int m = 0; m < KP::NWT; ++m) cw[mt][rr][m] = row[m];
+        }
+      float acc[2][4] = {}, sacc[4] = {0.f, 0.f, 0.f, 0.f}, qacc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int ks = 0; ks < KSS; ++ks) {
-        mma16816(bh, a128, qh[ks][0], qh[ks][1]);
-        mma16816(bl, a128, ql[ks][0], ql[ks][1]);
-      }
-      const float cs0 = __shfl_sync(0xffffffffu, qm, 4 * (2 * tid)) - (bh[0] + bl[0]);
-      const float cs1 = __shfl_sync(0xffffffffu, qm, 4 * (2 * tid + 1)) - (bh[1] + bl[1]);
+        // B = q 2^-e s split exactly into fp16 hi + lo (an FMA gives the
+        // product's rounding error); the scales and the weighted zeros as A
+        // rows against B = q 2^-e give sum_d q s 2^-e and sum_d q z exactly
+        uint32_t bh[2], bl[2], as[2], az[2];
 #pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        float acc[2][4];                             // [high, low]
-#pragma unroll
-        for (int k = 0; k < 2; ++k) acc[k][0] = acc[k][1] = acc[k][2] = acc[k][3] = 0.f;
-        const unsigned char* r0 = kcp + (16 * mt + gid) * C::KCB;
-        const unsigned char* r1 = r0 + 8 * C::KCB;
-#pragma unroll
-        for (int gq = 0; gq < NG; ++gq) {
-          uint32_t w0, w1;
-          if (KB == 4) {
-            w0 = *reinterpret_cast<const uint32_t*>(r0 + 16 * gq + 4 * tid);
-            w1 = *reinterpret_cast<const uint32_t*>(r1 + 16 * gq + 4 * tid);
-          } else {
-            const uint32_t v0 = *reinterpret_cast<const uint16_t*>(r0 + 8 * gq + 2 * tid);
-            const uint32_t v1 = *reinterpret_cast<const uint16_t*>(r1 + 8 * gq + 2 * tid);
-            w0 = v0 | (v0 << 14);
-            w1 = v1 | (v1 << 14);
-          }
-#pragma unroll
-          for (int sub = 0; sub < 2; ++sub) {
-            uint32_t a[4];
-            a[0] = magic2(w0 >> (8 * sub), kmask);
-            a[1] = magic2(w1 >> (8 * sub), kmask);
-            a[2] = magic2(w0 >> (8 * sub + 4), kmask);
-            a[3] = magic2(w1 >> (8 * sub + 4), kmask);
-            mma16816(acc[0], a, qh[2 * gq + sub][0], qh[2 * gq + sub][1]);
-            mma16816(acc[1], a, ql[2 * gq + sub][0], ql[2 * gq + sub][1]);
-          }
+        for (int hf = 0; hf < 2; ++hf) {
+          const int i = 2 * ks + hf;
+          const int sel = (KP::lo(i) & 1) ? 0x7632 : 0x5410;
+          as[hf] = __byte_perm(sw[KP::lo(i) >> 1], sw[KP::hi(i) >> 1], sel);
+          az[hf] = hmul2u(__byte_perm(zw[KP::lo(i) >> 1], zw[KP::hi(i) >> 1], sel),
+                          pow2_h2(KP::e(i % KP::RPW)));
+          bh[hf] = hmul2u(qw[i], as[hf]);
+          bl[hf] = hfma2u_neg(qw[i], as[hf], bh[hf]);
         }
+        const uint32_t aS[4] = {as[0], as[0], as[1], as[1]};
+        mma16816_f16(sacc, aS, qw[2 * ks], qw[2 * ks + 1]);
+        const uint32_t aZ[4] = {az[0], az[0], az[1], az[1]};
+        mma16816_f16(qacc, aZ, qw[2 * ks], qw[2 * ks + 1]);
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          const int i0 = 2 * ks, i1 = 2 * ks + 1;
+          const int m0 = i0 / KP::RPW, m1 = i1 / KP::RPW;
+          uint32_t a[4];
+          a[0] = KP::get(i0, cw[mt][0][m0]);
+          a[1] = KP::get(i0, cw[mt][1][m0]);
+          a[2] = KP::get(i1, cw[mt][0][m1]);
+          a[3] = KP::get(i1, cw[mt][1][m1]);
+          mma16816_f16(acc[mt], a, bh[0], bh[1]);
+          mma16816_f16(acc[mt], a, bl[0], bl[1]);
+        }
+      }
+      // per head (columns 2 tid, 2 tid + 1): sum_d q z less the 1024 terms
+      const float cs0 = qacc[0] - 1024.f * sacc[0];
+      const float cs1 = qacc[1] - 1024.f * sacc[1];
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
           const bool valid = 16 * mt + gid + 8 * r < nv;
-          const float v0 = acc[0][2 * r] + acc[1][2 * r];
-          const float v1 = acc[0][2 * r + 1] + acc[1][2 * r + 1];
-          S[mt][2 * r] = valid ? (v0 + cs0) * c2 : -INFINITY;
-          S[mt][2 * r + 1] = valid ? (v1 + cs1) * c2 : -INFINITY;
+          S[mt][2 * r] = valid ? (acc[mt][2 * r] + cs0) * c2 : -INFINITY;
+          S[mt][2 * r + 1] = valid ? (acc[mt][2 * r + 1] + cs1) * c2 : -INFINITY;
         }
-      }
     } else {  // full-precision keys (KIVI residual ring), read from global memory
+      uint32_t qb[KSS][2];
+      q_frags(qb);
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt) {
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -517,21 +591,27 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
             x01 = (uint32_t)vc[tk[0] * C::VCB + 8 * gq + gid] | ((uint32_t)vc[tk[1] * C::VCB + 8 * gq + gid] << 16);
             x89 = (uint32_t)vc[tk[2] * C::VCB + 8 * gq + gid] | ((uint32_t)vc[tk[3] * C::VCB + 8 * gq + gid] << 16);
           }
-          constexpr int SH = VB == 4 ? 4 : 2;        // bits between consecutive channels
+          // rows gid and gid + 8 of m-tile u are the channels at bits vsh(u)
+          // and vsh(u) + SH of each half, read in place as 1024 + c 2^bit
+          // (4-bit: the upper pair after a shift by 8); the weights come
+          // off when the head's output is folded
 #pragma unroll
           for (int u = 0; u < 2; ++u) {
+            const uint32_t y01 = (VB == 4 && u) ? x01 >> 8 : x01;
+            const uint32_t y89 = (VB == 4 && u) ? x89 >> 8 : x89;
             uint32_t a[4];
-            a[0] = magic2h(x01 >> (2 * SH * u), vmask);
-            a[1] = magic2h(x01 >> (2 * SH * u + SH), vmask);
-            a[2] = magic2h(x89 >> (2 * SH * u), vmask);
-            a[3] = magic2h(x89 >> (2 * SH * u + SH), vmask);
+            a[0] = magic2h(y01, vmask << vsh(u));
+            a[1] = magic2h(y01, vmask << (vsh(u) + SH));
+            a[2] = magic2h(y89, vmask << vsh(u));
+            a[3] = magic2h(y89, vmask << (vsh(u) + SH));
             mma16816_f16(o[2 * gq + u], a, b0, b1);
           }
-          const uint32_t ab[4] = {kbias2, kbias2, kbias2, kbias2};
+          const uint32_t ab[4] = {kMagicH, kMagicH, kMagicH, kMagicH};
           mma16816_f16(bias[gq], ab, b0, b1);
         }
       }
     } else {  // full-precision values
+      if (!folded) fold_o();
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt) {
         const __nv_bfloat16* vr[4];
@@ -592,19 +672,8 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
       if (lane == 0) mbar_arrive1(&empty[st]);
     }
     if (mine) {
-      // fold the bias and offset terms into O; reduce l over the rows
-#pragma unroll
-      for (int gq = 0; gq < NG; ++gq) {
-        const float f0 = __shfl_sync(0xffffffffu, offa[0], 4 * gq + tid) - bias[gq][0];
-        const float f1 = __shfl_sync(0xffffffffu, offa[1], 4 * gq + tid) - bias[gq][1];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          o[2 * gq + u][0] += f0;
-          o[2 * gq + u][1] += f1;
-          o[2 * gq + u][2] += f0;
-          o[2 * gq + u][3] += f1;
-        }
-      }
+      if (!folded) fold_o();
+      // reduce l over the rows
 #pragma unroll
       for (int jh = 0; jh < 2; ++jh) {
         l_run[jh] += __shfl_xor_sync(0xffffffffu, l_run[jh], 4);

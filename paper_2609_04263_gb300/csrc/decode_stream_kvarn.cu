@@ -460,8 +460,9 @@ decode_stream_kvarn_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float sc
     const int64_t hs = (int64_t)hd * nb;
     const int a = (int)(max(k0, hs) - k0), e = (int)(min(k1, hs + nb) - k0);
     const int b = hd / g.H, hkv = hd % g.H;
-    // rotated queries of the head (times the softmax scale, log2 units)
-    {
+    // rotated queries of the head (times the softmax scale, log2 units):
+    // rows 0-7 of qr, zero for the MMA columns beyond the group
+    if (warp < 8) {
       float x[D / 32];
       const bool live = warp < grp;
       const __nv_bfloat16* src = q + ((int64_t)b * g.Hq + hkv * grp + (live ? warp : 0)) * D;

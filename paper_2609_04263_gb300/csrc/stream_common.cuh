@@ -11,7 +11,7 @@ namespace stream {
 
 constexpr int kBT = 32;            // tokens per block (one KIVI key block)
 constexpr int kSB = 8;             // blocks per ring stage (copied together)
-constexpr int kNW = 8;             // consumer warps
+constexpr int kNW = 11;            // consumer warps (12 warps: the register file holds 168 a thread)
 constexpr int kThreads = (kNW + 1) * 32;
 constexpr int kMaxStages = 64;
 constexpr int kSmemMax = 227 * 1024;
@@ -27,6 +27,13 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
 }
 __device__ __forceinline__ uint32_t hmul2u(uint32_t a, uint32_t b) {
   __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&a), *reinterpret_cast<const __half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+// a * b - c as one fused fp16x2 operation: with c = a * b rounded, the
+// exact rounding error of the product
+__device__ __forceinline__ uint32_t hfma2u_neg(uint32_t a, uint32_t b, uint32_t c) {
+  __half2 r = __hfma2(*reinterpret_cast<const __half2*>(&a), *reinterpret_cast<const __half2*>(&b),
+                      __hneg2(*reinterpret_cast<const __half2*>(&c)));
   return *reinterpret_cast<uint32_t*>(&r);
 }
 __device__ __forceinline__ uint32_t h2u(__half lo, __half hi) {
