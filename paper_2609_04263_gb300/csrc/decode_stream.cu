@@ -426,12 +426,14 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
 #pragma unroll
           for (int m = 0; m < KP::NWT; ++m) cw[mt][rr][m] = row[m];
         }
-      float acc[2][4] = {}, sacc[4] = {0.f, 0.f, 0.f, 0.f}, qacc[4] = {0.f, 0.f, 0.f, 0.f};
+      // sz rows 0-7: sum_d q s 2^-e, rows 8-15: sum_d q z (heads in the columns)
+      float acc[2][4] = {}, sz[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int ks = 0; ks < KSS; ++ks) {
         // B = q 2^-e s split exactly into fp16 hi + lo (an FMA gives the
-        // product's rounding error); the scales and the weighted zeros as A
-        // rows against B = q 2^-e give sum_d q s 2^-e and sum_d q z exactly
+        // product's rounding error); the scales (A rows 0-7) and the weighted
+        // zeros (rows 8-15) against B = q 2^-e give sum_d q s 2^-e and
+        // sum_d q z exactly
         uint32_t bh[2], bl[2], as[2], az[2];
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
@@ -443,10 +445,8 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
           bh[hf] = hmul2u(qw[i], as[hf]);
           bl[hf] = hfma2u_neg(qw[i], as[hf], bh[hf]);
         }
-        const uint32_t aS[4] = {as[0], as[0], as[1], as[1]};
-        mma16816_f16(sacc, aS, qw[2 * ks], qw[2 * ks + 1]);
-        const uint32_t aZ[4] = {az[0], az[0], az[1], az[1]};
-        mma16816_f16(qacc, aZ, qw[2 * ks], qw[2 * ks + 1]);
+        const uint32_t aSZ[4] = {as[0], az[0], as[1], az[1]};
+        mma16816_f16(sz, aSZ, qw[2 * ks], qw[2 * ks + 1]);
 #pragma unroll
         for (int mt = 0; mt < 2; ++mt) {
           const int i0 = 2 * ks, i1 = 2 * ks + 1;
@@ -461,8 +461,8 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         }
       }
       // per head (columns 2 tid, 2 tid + 1): sum_d q z less the 1024 terms
-      const float cs0 = qacc[0] - 1024.f * sacc[0];
-      const float cs1 = qacc[1] - 1024.f * sacc[1];
+      const float cs0 = sz[2] - 1024.f * sz[0];
+      const float cs1 = sz[3] - 1024.f * sz[1];
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
