@@ -554,8 +554,8 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
                 // Q atom: 128 rows x 128 B (1024 units); K atom: 64 rows x 128 B (512 units)
                 const uint64_t qd = qdesc0 + (uint64_t)(x * (S::QT >> 4) + (kk >> 2) * 1024 + (kk & 3) * 2);
                 const uint64_t kd = kvdesc0 + (uint64_t)(kb * (S::KV_B >> 4) + (kk >> 2) * 512 + (kk & 3) * 2);
-                umma(ts, qd, kd + (S::KH >> 4), id_qk, kk > 0);
-                umma(ts, qd, kd + (S::KL >> 4), id_qk, 1);
+                umma_a_fill(ts, qd, kd + (S::KH >> 4), id_qk, kk > 0);   // Q read once
+                umma_a_lastuse(ts, qd, kd + (S::KL >> 4), id_qk, 1);     // for K hi and lo
               }
               umma_commit(&s_full[x][bf]);
             }
