@@ -84,13 +84,34 @@ typedef struct {
   int32_t residual_tokens;  /* KIVI: R (>= 0)                                    */
   int32_t sink_tokens;      /* KVarN: S (>= 0)                                   */
   int32_t norm_iters;       /* KVarN: normalisation iterations (paper: 8)        */
-  int32_t batch;            /* B sequences, all holding the same token count    */
+  int32_t batch;            /* B sequences (layout UNIFORM: all holding the same
+                               token count)                                      */
   int32_t kv_heads;         /* Hkv                                               */
   int32_t q_heads;          /* Hq (multiple of Hkv); sizes the decode workspace */
   int32_t head_dim;         /* D: 64, 128 or 256                                 */
   int32_t max_tokens;       /* capacity per sequence                             */
   int32_t dtype;            /* kvq_dtype of the full-precision windows           */
+  int32_t layout;           /* kvq_layout (0 = UNIFORM)                          */
+  int32_t num_pages;        /* layout PAGED: pages of KVQ_PAGE_TOKENS tokens in
+                               the pool shared by all sequences                 */
 } kvq_cache_desc;
+
+/* Token layout of a cache.
+ *   UNIFORM  every sequence holds the same number of tokens T (appends add L
+ *            tokens to all of them).
+ *   RAGGED   every sequence b has its own count T_b <= max_tokens, in its own
+ *            rows (continuous batching: sequences start, grow and are
+ *            released independently).
+ *   PAGED    RAGGED, with each sequence's tokens in pages of KVQ_PAGE_TOKENS
+ *            tokens taken from one pool of num_pages pages by the library's
+ *            allocator as the sequence grows, and returned by
+ *            kvq_seq_release; a sequence holds ceil(T_b / 64) pages.
+ * RAGGED and PAGED caches are built for bf16 AFFINE and SYMMETRIC caches with
+ * group_size 32, key_bits == value_bits in {2, 4}, head_dim 64 or 128, at most
+ * 16 query heads per kv head and at most KVQ_MAX_SEQS sequences. */
+typedef enum { KVQ_LAYOUT_UNIFORM = 0, KVQ_LAYOUT_RAGGED = 1, KVQ_LAYOUT_PAGED = 2 } kvq_layout;
+#define KVQ_PAGE_TOKENS 64
+#define KVQ_MAX_SEQS 512
 
 typedef struct kvq_cache kvq_cache;   /* opaque, host-side bookkeeping only */
 
@@ -385,6 +406,38 @@ kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* 
                              float* da_q, float* db_q, float* da_k, float* db_k,
                              float* da_v, float* db_v, float* d_x,
                              void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Ragged appends (layouts RAGGED and PAGED): sequence b appends the first
+ * n[b] (0 <= n[b] <= L) of its L rows of k, v [B][Hkv][L][D] at its own
+ * positions T_b .. T_b + n[b] - 1.  n is a HOST array of B counts; NULL means
+ * n[b] = L for every b (kvq_append_pack on a ragged cache does the same).
+ * A PAGED cache first takes the pages the new tokens need from its pool;
+ * KVQ_ERR_CAPACITY (nothing appended, no page taken) if some T_b + n[b]
+ * exceeds max_tokens or the pool runs out.  kvq_attend_prefill and
+ * kvq_attend_decode then attend, per sequence, the n[b] rows of the last
+ * append (prefill: rows l < n[b] of q and out; the rest of out is not
+ * written) or its newest token (decode; a sequence holding no token gets a
+ * zero output) over that sequence's T_b tokens.
+ */
+kvq_status kvq_append_pack_ragged(kvq_cache* cache, const void* k, const void* v, int L,
+                                  const int* n, void* stream);
+
+/* Tokens held by sequence b (any layout; -1 for a bad argument). */
+int kvq_seq_tokens(const kvq_cache* cache, int b);
+
+/* Layouts RAGGED and PAGED: sequence b becomes empty (T_b = 0) and a PAGED
+ * cache returns its pages to the pool.  Stream-ordered like an append. */
+kvq_status kvq_seq_release(kvq_cache* cache, int b, void* stream);
+
+/* Pages of a PAGED cache's pool not held by any sequence (-1 otherwise). */
+int kvq_free_pages(const kvq_cache* cache);
+
+/* PAGED: the pool pages of sequence b in token order (page i holds its tokens
+ * 64 i .. 64 i + 63; in kvq_cache_view's planes a page is rows 64 p .. 64 p +
+ * 63 of batch index 0).  Writes at most max_pages ids to pages and returns
+ * the sequence's page count, or -1. */
+int kvq_seq_pages(const kvq_cache* cache, int b, int* pages, int max_pages);
 
 /* Read and clear the device-side error word of the library (synchronises
  * `stream`).  *out = 0 when no bounded wait has timed out; otherwise a kernel

@@ -26,12 +26,14 @@ def _ptr(t):
 
 
 def make_desc(fmt, key_bits, value_bits, group_size, batch, kv_heads, q_heads, head_dim,
-              max_tokens, dtype, residual_tokens=0, sink_tokens=0, norm_iters=8):
+              max_tokens, dtype, residual_tokens=0, sink_tokens=0, norm_iters=8,
+              layout=kvq.KVQ_LAYOUT_UNIFORM, num_pages=0):
     return kvq.kvq_cache_desc(fmt=fmt, key_bits=key_bits, value_bits=value_bits,
                               group_size=group_size, residual_tokens=residual_tokens,
                               sink_tokens=sink_tokens, norm_iters=norm_iters, batch=batch,
                               kv_heads=kv_heads, q_heads=q_heads, head_dim=head_dim,
-                              max_tokens=max_tokens, dtype=_DT.get(dtype, dtype))
+                              max_tokens=max_tokens, dtype=_DT.get(dtype, dtype),
+                              layout=layout, num_pages=num_pages)
 
 
 class Cache:
@@ -124,6 +126,23 @@ class Cache:
         one fused kernel."""
         r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
         return kvq.kvq_decode_step_fused(self.handle, d_in, *r)
+
+    def append_ragged(self, k, v, n=None) -> None:
+        """Ragged / paged caches: sequence b appends the first n[b] of its
+        rows of k, v [B, H, L, D] (all L when n is None)."""
+        kvq.kvq_append_pack_ragged(self.handle, _ptr(k), _ptr(v), k.shape[2], n, _stream())
+
+    def seq_tokens(self, b) -> int:
+        return kvq.kvq_seq_tokens(self.handle, b)
+
+    def seq_release(self, b) -> None:
+        kvq.kvq_seq_release(self.handle, b, _stream())
+
+    def free_pages(self) -> int:
+        return kvq.kvq_free_pages(self.handle)
+
+    def seq_pages(self, b) -> list:
+        return kvq.kvq_seq_pages(self.handle, b)
 
     def attend_backward(self, q, d_out, scale=None, workspace=None):
         """Straight-through backward of attend_prefill(q): returns fp32

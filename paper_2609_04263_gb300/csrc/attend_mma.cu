@@ -17,7 +17,7 @@ attend_decode_mma_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scal
   const int grp = g.Hq / g.H;
   decode_split<D, BITS, FMT, kStages, kWarps>(
       g, q + ((int64_t)blockIdx.z * g.Hq + blockIdx.y * grp) * D, scale, err, out, blockIdx.x,
-      g.splits, kMaxSplits, blockIdx.y, blockIdx.z, cache_tokens(g), smem, bars, false);
+      g.splits, kMaxSplits, blockIdx.y, blockIdx.z, seq_tokens(g, blockIdx.z), smem, bars, false);
 }
 
 template <int D, int BITS, int FMT>

@@ -196,15 +196,22 @@ __device__ __forceinline__ void load_raw(const Geom& g, int b, int h, int t0, un
   using S = M256Layout<D, BITS>;
   constexpr uint32_t CB = kTok * S::CROW;
   mbar_expect_tx(bar, raw_bytes<D, BITS, FMT>());
-  bulk_copy(raw + S::RKC, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0), CB, bar);
-  bulk_copy(raw + S::RVC, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t0), CB, bar);
-  const int krow = FMT == KVQ_FMT_KIVI ? t0 / 32 : t0;   // KIVI: two key blocks of D channels
-  bulk_copy(raw + S::RKS, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, krow), 4 * D, bar);
+  // a tile is one 64-token page of a paged cache: tok_ptr finds its rows
+  bulk_copy(raw + S::RKC, tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0), CB, bar);
+  bulk_copy(raw + S::RVC, tok_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t0), CB, bar);
+  // KIVI: two key blocks of D channels (uniform layout only)
+  const __half* ks = FMT == KVQ_FMT_KIVI ? plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t0 / 32)
+                                         : tok_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t0);
+  bulk_copy(raw + S::RKS, ks, 4 * D, bar);
+  if (FMT != KVQ_FMT_SYMMETRIC) {
+    const __half* kz = FMT == KVQ_FMT_KIVI
+                           ? plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t0 / 32)
+                           : tok_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t0);
+    bulk_copy(raw + S::RKZ, kz, 4 * D, bar);
+  }
+  bulk_copy(raw + S::RVS, tok_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, t0), 4 * D, bar);
   if (FMT != KVQ_FMT_SYMMETRIC)
-    bulk_copy(raw + S::RKZ, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, krow), 4 * D, bar);
-  bulk_copy(raw + S::RVS, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, h, t0), 4 * D, bar);
-  if (FMT != KVQ_FMT_SYMMETRIC)
-    bulk_copy(raw + S::RVZ, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, t0), 4 * D, bar);
+    bulk_copy(raw + S::RVZ, tok_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, h, t0), 4 * D, bar);
 }
 
 // K: 8 channels reconstructed in fp32 and split into a bf16 high part (the
@@ -428,11 +435,14 @@ attend_prefill_m256_kernel(Geom g, const __nv_bfloat16* __restrict__ q, int L, f
   const int qtile = nqt - 1 - blockIdx.x;              // longest first
   const int hkv = blockIdx.y, b = blockIdx.z;
   const int grp = g.Hq / g.H;
-  const int T = cache_tokens(g);
+  const int T = seq_tokens(g, b);
   const int tq = FMT == KVQ_FMT_KIVI ? kivi_tq(T, g.R, g.G) : T;
+  // a ragged cache's sequence b attends the rows of its last append
+  const int Lb = g.layout == KVQ_LAYOUT_UNIFORM ? L : g.seq_new[b];
   const int q0 = qtile * nq;
-  const int nql = min(nq, L - q0);
-  const int pos_first = T - L + q0;
+  if (q0 >= Lb) return;                                // no query of this sequence here
+  const int nql = min(nq, Lb - q0);
+  const int pos_first = T - Lb + q0;
   const int t_end = pos_first + nql;                   // keys [0, t_end)
   const int ntiles = (t_end + kTok - 1) / kTok;
   volatile int* abort = &abort_flag;

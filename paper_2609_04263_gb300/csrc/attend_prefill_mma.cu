@@ -658,7 +658,7 @@ bool prefill_mma_supported(const Geom& g) {
                       g.fmt == KVQ_FMT_KIVI || g.fmt == KVQ_FMT_FLOAT || g.fmt == KVQ_FMT_KVARN;
   const int grp = g.Hq / g.H;
   const int rows = g.D == 256 ? 64 : 128;
-  return fmt_ok && g.act == KVQ_BF16 && grp <= rows &&
+  return fmt_ok && g.layout == KVQ_LAYOUT_UNIFORM && g.act == KVQ_BF16 && grp <= rows &&
          (g.D == 64 || g.D == 128 || g.D == 256);
 }
 

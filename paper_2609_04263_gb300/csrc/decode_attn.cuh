@@ -201,9 +201,10 @@ __device__ void split_issue(const Geom& g, int b, int hkv, const SplitPlan& sp, 
   uint32_t total = 2 * code_bytes + kmeta + vmeta;
   if (zero_planes) total += kmeta + vmeta;
   mbar_expect_tx(&bars[stage], total);
-  bulk_g2s(st + C::KC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, c0), code_bytes,
+  // a chunk is one 64-token page of a paged cache: tok_ptr finds its rows
+  bulk_g2s(st + C::KC_OFF, tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, hkv, c0), code_bytes,
            &bars[stage]);
-  bulk_g2s(st + C::VC_OFF, plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
+  bulk_g2s(st + C::VC_OFF, tok_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
            &bars[stage]);
   if (FMT == KVQ_FMT_KIVI) {
     bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
@@ -211,16 +212,16 @@ __device__ void split_issue(const Geom& g, int b, int hkv, const SplitPlan& sp, 
     bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
              &bars[stage]);
   } else {
-    bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,
+    bulk_g2s(st + C::KS_OFF, tok_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,
              &bars[stage]);
     if (zero_planes)
-      bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0), kmeta,
+      bulk_g2s(st + C::KZ_OFF, tok_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0), kmeta,
                &bars[stage]);
   }
-  bulk_g2s(st + C::VS_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, c0), vmeta,
+  bulk_g2s(st + C::VS_OFF, tok_ptr<__half>(g, KVQ_PLANE_V_SCALE, b, hkv, c0), vmeta,
            &bars[stage]);
   if (zero_planes)
-    bulk_g2s(st + C::VZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, c0), vmeta,
+    bulk_g2s(st + C::VZ_OFF, tok_ptr<__half>(g, KVQ_PLANE_V_ZERO, b, hkv, c0), vmeta,
              &bars[stage]);
 }
 

@@ -679,7 +679,9 @@ bool decode_step_supported(const Geom& g, int d_in, const int r[3]) {
   const bool fmt_ok = (g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC) &&
                       g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb &&
                       (g.kb == 2 || g.kb == 4) && (g.D == 64 || g.D == 128);
-  if (!fmt_ok || g.Hq / g.H > 16 || g.B > 16 || d_in <= 0 || d_in % 256) return false;
+  if (!fmt_ok || g.layout != KVQ_LAYOUT_UNIFORM || g.Hq / g.H > 16 || g.B > 16 || d_in <= 0 ||
+      d_in % 256)
+    return false;
   for (int p = 0; p < 3; ++p)
     if (r[p] < 0 || r[p] > 64 || r[p] % 8) return false;
   StepArgs a;

@@ -833,8 +833,8 @@ int decode_stream_ctas(const Geom& g) {
 
 bool decode_stream_supported(const Geom& g) {
   const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC || g.fmt == KVQ_FMT_KIVI;
-  return fmt_ok && g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb && (g.kb == 2 || g.kb == 4) &&
-         (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
+  return fmt_ok && g.layout == KVQ_LAYOUT_UNIFORM && g.act == KVQ_BF16 && g.G == 32 &&
+         g.kb == g.vb && (g.kb == 2 || g.kb == 4) && (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
 }
 
 cudaError_t launch_decode_stream(const Geom& g, const void* q, float scale, int* err, void* out,

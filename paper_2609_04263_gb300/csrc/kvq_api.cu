@@ -3,8 +3,10 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <algorithm>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "kvq_internal.cuh"
 
@@ -94,16 +96,42 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
       *st = KVQ_ERR_UNSUPPORTED; return 0;
     }
   }
+  if (d->layout < KVQ_LAYOUT_UNIFORM || d->layout > KVQ_LAYOUT_PAGED) {
+    fail(KVQ_ERR_ARG, "unknown layout %d", d->layout); *st = KVQ_ERR_ARG; return 0;
+  }
+  if (d->layout != KVQ_LAYOUT_UNIFORM) {
+    const bool ok = (d->fmt == KVQ_FMT_AFFINE || d->fmt == KVQ_FMT_SYMMETRIC) &&
+                    d->dtype == KVQ_BF16 && G == 32 && d->key_bits == d->value_bits &&
+                    (d->key_bits == 2 || d->key_bits == 4) && (D == 64 || D == 128) &&
+                    d->q_heads / d->kv_heads <= 16;
+    if (!ok) {
+      fail(KVQ_ERR_UNSUPPORTED, "ragged and paged layouts need a bf16 affine or symmetric cache "
+           "with group_size 32, key_bits == value_bits in {2, 4} and head_dim 64 or 128");
+      *st = KVQ_ERR_UNSUPPORTED; return 0;
+    }
+    if (d->batch > KVQ_MAX_SEQS) {
+      fail(KVQ_ERR_UNSUPPORTED, "%d sequences > %d", d->batch, KVQ_MAX_SEQS);
+      *st = KVQ_ERR_UNSUPPORTED; return 0;
+    }
+    if (d->layout == KVQ_LAYOUT_PAGED && d->num_pages <= 0) {
+      fail(KVQ_ERR_SHAPE, "a paged cache needs num_pages > 0"); return 0;
+    }
+  }
   const int B = d->batch, H = d->kv_heads, Tm = d->max_tokens;
+  const bool paged = d->layout == KVQ_LAYOUT_PAGED;
   // per-token planes hold whole 64-token chunks (the decode kernel copies
-  // whole chunks), so their rows are padded to a multiple of 64
-  const int Tp = (Tm + 63) / 64 * 64;
+  // whole chunks), so their rows are padded to a multiple of 64; a paged
+  // cache's planes hold the page pool of all sequences (batch index 0)
+  const int Tp = paged ? d->num_pages * kPageTok : (Tm + 63) / 64 * 64;
+  const int pb = paged ? 1 : B;               // batch extent of the cache planes
   const int act = d->dtype == KVQ_BF16 ? 2 : 4;
   memset(g, 0, sizeof *g);
   g->fmt = d->fmt; g->kb = d->key_bits; g->vb = d->value_bits; g->G = G;
   g->R = d->residual_tokens; g->S = d->sink_tokens; g->iters = d->norm_iters;
   g->B = B; g->H = H; g->Hq = d->q_heads; g->D = D; g->Tmax = Tm; g->act = d->dtype;
   g->ring = d->residual_tokens + G;
+  g->layout = d->layout;
+  g->max_pages = paged ? (Tm + kPageTok - 1) / kPageTok : 0;
   auto set = [&](int which, int64_t rows, int64_t cols, int elem) {
     g->pl[which].rows = rows; g->pl[which].cols = cols; g->pl[which].elem = elem;
   };
@@ -160,7 +188,7 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     }
   }
   g->splits = decode_splits(*g);
-  size_t total = state_region_bytes(B, H);   // device state + split counters at offset 0
+  size_t total = state_region_bytes(*g);     // device state, split counters, ragged arrays
   static_assert(sizeof(CacheState) == 256, "state block is 256 bytes");
   for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
     off[i] = 0;
@@ -168,7 +196,7 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     Plane& p = g->pl[i];
     if (p.rows == 0) continue;
     off[i] = total;
-    total = align256(total + (size_t)B * H * p.rows * p.cols * p.elem);
+    total = align256(total + (size_t)pb * H * p.rows * p.cols * p.elem);
   }
   // decode workspace: [B][Hq][kMaxSplits][D + 2] fp32, indexed by q head
   off[KVQ_PLANE_WORKSPACE] = total;
@@ -219,7 +247,7 @@ cudaError_t ensure_cache_init(kvq_cache* c, cudaStream_t s) {
     e = cudaMemsetAsync(ws, 0, reinterpret_cast<char*>(c->g.epoch) + 256 - ws, s);
     if (e == cudaSuccess) c->need_clear = false;
   }
-  if (e == cudaSuccess) e = cudaMemsetAsync(c->g.state, 0, state_region_bytes(c->g.B, c->g.H), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->g.state, 0, state_region_bytes(c->g), s);
   if (e == cudaSuccess) c->need_init = false;
   return e;
 }
@@ -283,6 +311,19 @@ kvq_status kvq_create_cache(const kvq_cache_desc* desc, void* dev_buf, size_t by
   c->g.epoch = reinterpret_cast<uint32_t*>(c->base + need - 256);
   for (int i = 0; i < KVQ_NUM_PLANES; ++i)
     c->g.pl[i].p = c->g.pl[i].rows ? c->base + off[i] : nullptr;
+  c->g.seq_len = c->g.seq_new = c->g.page_table = nullptr;
+  if (g.layout != KVQ_LAYOUT_UNIFORM) {
+    char* p = c->base + state_region_bytes(g.B, g.H);
+    c->g.seq_len = reinterpret_cast<int32_t*>(p);
+    c->g.seq_new = c->g.seq_len + g.B;
+    if (g.layout == KVQ_LAYOUT_PAGED)
+      c->g.page_table = reinterpret_cast<int32_t*>(p + align256((size_t)2 * g.B * 4));
+    c->seq_T.assign(g.B, 0);
+    c->seq_n.assign(g.B, 0);
+    c->seq_pages.assign(g.B, std::vector<int>());
+    if (g.layout == KVQ_LAYOUT_PAGED)
+      for (int i = desc->num_pages - 1; i >= 0; --i) c->free_pages.push_back(i);
+  }
   *out = c;
   g_last_error.clear();
   return KVQ_OK;
@@ -298,6 +339,13 @@ kvq_status kvq_reset_cache(kvq_cache* cache) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
   cache->T = 0;
   cache->need_init = true;
+  if (cache->g.layout != KVQ_LAYOUT_UNIFORM) {
+    for (int b = 0; b < cache->g.B; ++b) {
+      cache->seq_T[b] = cache->seq_n[b] = 0;
+      for (int p : cache->seq_pages[b]) cache->free_pages.push_back(p);
+      cache->seq_pages[b].clear();
+    }
+  }
   return KVQ_OK;
 }
 
@@ -313,6 +361,18 @@ kvq_status kvq_cache_sync(kvq_cache* cache, void* stream) {
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e == cudaSuccess && st.error)
     e = cudaMemsetAsync(&cache->g.state->error, 0, sizeof(int32_t), s);
+  if (e == cudaSuccess && cache->g.layout != KVQ_LAYOUT_UNIFORM) {
+    // per-sequence counts (replayed ragged appends advance them on the device)
+    e = cudaMemcpyAsync(cache->seq_T.data(), cache->g.seq_len, cache->g.B * sizeof(int32_t),
+                        cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(cache->seq_n.data(), cache->g.seq_new, cache->g.B * sizeof(int32_t),
+                          cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    int tmax = 0;
+    for (int x : cache->seq_T) tmax = std::max(tmax, x);
+    st.tokens = tmax;
+  }
   if (e != cudaSuccess) return cuda_fail(e, "kvq_cache_sync");
   cache->T = st.tokens;
   if (st.error & kErrCapacity)
@@ -327,7 +387,7 @@ kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out) {
   const Geom& g = cache->g;
   for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
     out->ptr[i] = g.pl[i].p;
-    out->dims[i][0] = g.pl[i].rows ? g.B : 0;
+    out->dims[i][0] = g.pl[i].rows ? (g.layout == KVQ_LAYOUT_PAGED && i != KVQ_PLANE_WORKSPACE ? 1 : g.B) : 0;
     out->dims[i][1] = g.pl[i].rows ? (i == KVQ_PLANE_WORKSPACE ? g.Hq : g.H) : 0;
     out->dims[i][2] = g.pl[i].rows;
     out->dims[i][3] = g.pl[i].cols;
@@ -346,6 +406,8 @@ kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out) {
 kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L,
                            void* stream) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (cache->g.layout != KVQ_LAYOUT_UNIFORM)
+    return kvq_append_pack_ragged(cache, k, v, L, nullptr, stream);
   if (L < 0) return fail(KVQ_ERR_ARG, "L = %d < 0", L);
   if (L == 0) return KVQ_OK;
   if (!k || !v) return fail(KVQ_ERR_ARG, "k or v is NULL");
@@ -366,6 +428,109 @@ kvq_status kvq_append_pack(kvq_cache* cache, const void* k, const void* v, int L
   return KVQ_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Ragged and paged layouts: per-sequence counts on the host and the device,
+// and the page pool's allocator (host side; the device reads the table)
+// ---------------------------------------------------------------------------
+kvq_status kvq_append_pack_ragged(kvq_cache* cache, const void* k, const void* v, int L,
+                                  const int* n, void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  const Geom& g = cache->g;
+  if (g.layout == KVQ_LAYOUT_UNIFORM)
+    return fail(KVQ_ERR_UNSUPPORTED, "kvq_append_pack_ragged needs a ragged or paged cache");
+  if (L < 0) return fail(KVQ_ERR_ARG, "L = %d < 0", L);
+  std::vector<int> cnt(g.B, L);
+  if (n)
+    for (int b = 0; b < g.B; ++b) {
+      if (n[b] < 0 || n[b] > L) return fail(KVQ_ERR_ARG, "n[%d] = %d outside [0, %d]", b, n[b], L);
+      cnt[b] = n[b];
+    }
+  int total = 0;
+  for (int b = 0; b < g.B; ++b) total += cnt[b];
+  if (total > 0 && (!k || !v)) return fail(KVQ_ERR_ARG, "k or v is NULL");
+  if (misaligned(k) || misaligned(v)) return fail(KVQ_ERR_ARG, "k and v must be 16-byte aligned");
+  if ((int64_t)g.B * g.H * (int64_t)L * (g.D / 4) >= ((int64_t)1 << 31))
+    return fail(KVQ_ERR_SHAPE, "append of %d tokens too large for one call: append it in chunks", L);
+  // capacity, and the pages the new tokens need (taken only if all fit)
+  int need_pages = 0;
+  for (int b = 0; b < g.B; ++b) {
+    const int64_t t1 = (int64_t)cache->seq_T[b] + cnt[b];
+    if (t1 > g.Tmax)
+      return fail(KVQ_ERR_CAPACITY, "sequence %d: %d + %d tokens exceed max_tokens %d", b,
+                  cache->seq_T[b], cnt[b], g.Tmax);
+    if (g.layout == KVQ_LAYOUT_PAGED)
+      need_pages += (int)((t1 + kPageTok - 1) / kPageTok) - (int)cache->seq_pages[b].size();
+  }
+  if (need_pages > (int)cache->free_pages.size())
+    return fail(KVQ_ERR_CAPACITY, "the append needs %d pages, %d are free", need_pages,
+                (int)cache->free_pages.size());
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = ensure_init(cache, s);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_append_pack_ragged");
+  if (g.layout == KVQ_LAYOUT_PAGED) {
+    for (int b = 0; b < g.B; ++b) {
+      std::vector<int>& pg = cache->seq_pages[b];
+      const int have = (int)pg.size();
+      const int want = (cache->seq_T[b] + cnt[b] + kPageTok - 1) / kPageTok;
+      if (want <= have) continue;
+      for (int i = have; i < want; ++i) {
+        pg.push_back(cache->free_pages.back());
+        cache->free_pages.pop_back();
+      }
+      // the table entries travel with the stream (a pageable copy is staged
+      // before the call returns, so pg may change afterwards)
+      e = cudaMemcpyAsync(g.page_table + (size_t)b * g.max_pages + have, pg.data() + have,
+                          (size_t)(want - have) * sizeof(int32_t), cudaMemcpyHostToDevice, s);
+      if (e != cudaSuccess) return cuda_fail(e, "kvq_append_pack_ragged page table");
+    }
+  }
+  e = launch_append_ragged(g, L, k, v, cnt.data(), s);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_append_pack_ragged launch");
+  int tmax = 0;
+  for (int b = 0; b < g.B; ++b) {
+    cache->seq_T[b] += cnt[b];
+    cache->seq_n[b] = cnt[b];
+    tmax = std::max(tmax, cache->seq_T[b]);
+  }
+  cache->T = tmax;
+  return KVQ_OK;
+}
+
+int kvq_seq_tokens(const kvq_cache* cache, int b) {
+  if (!cache || b < 0 || b >= cache->g.B) return -1;
+  return cache->g.layout == KVQ_LAYOUT_UNIFORM ? cache->T : cache->seq_T[b];
+}
+
+kvq_status kvq_seq_release(kvq_cache* cache, int b, void* stream) {
+  if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
+  if (cache->g.layout == KVQ_LAYOUT_UNIFORM)
+    return fail(KVQ_ERR_UNSUPPORTED, "kvq_seq_release needs a ragged or paged cache");
+  if (b < 0 || b >= cache->g.B) return fail(KVQ_ERR_ARG, "sequence %d outside [0, %d)", b, cache->g.B);
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = ensure_init(cache, s);
+  if (e == cudaSuccess) e = launch_seq_reset(cache->g, b, s);
+  if (e != cudaSuccess) return cuda_fail(e, "kvq_seq_release");
+  for (int p : cache->seq_pages[b]) cache->free_pages.push_back(p);
+  cache->seq_pages[b].clear();
+  cache->seq_T[b] = cache->seq_n[b] = 0;
+  int tmax = 0;
+  for (int x : cache->seq_T) tmax = std::max(tmax, x);
+  cache->T = tmax;
+  return KVQ_OK;
+}
+
+int kvq_free_pages(const kvq_cache* cache) {
+  if (!cache || cache->g.layout != KVQ_LAYOUT_PAGED) return -1;
+  return (int)cache->free_pages.size();
+}
+
+int kvq_seq_pages(const kvq_cache* cache, int b, int* pages, int max_pages) {
+  if (!cache || cache->g.layout != KVQ_LAYOUT_PAGED || b < 0 || b >= cache->g.B) return -1;
+  const std::vector<int>& pg = cache->seq_pages[b];
+  for (int i = 0; i < (int)pg.size() && i < max_pages && pages; ++i) pages[i] = pg[i];
+  return (int)pg.size();
+}
+
 static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_heads,
                                 float scale, void* out, void* stream, bool decode) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
@@ -374,9 +539,14 @@ static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_
   if (L <= 0) return fail(KVQ_ERR_ARG, "L = %d must be positive", L);
   if (n_q_heads != cache->g.Hq)
     return fail(KVQ_ERR_SHAPE, "n_q_heads %d != cache q_heads %d", n_q_heads, cache->g.Hq);
-  if (L > cache->T)
+  if (cache->g.layout == KVQ_LAYOUT_UNIFORM && L > cache->T)
     return fail(KVQ_ERR_SHAPE, "%d queries but only %d cached tokens (append first)", L,
                 cache->T);
+  if (cache->g.layout != KVQ_LAYOUT_UNIFORM && !decode)
+    for (int b = 0; b < cache->g.B; ++b)
+      if (cache->seq_n[b] > L)
+        return fail(KVQ_ERR_SHAPE, "sequence %d appended %d tokens, more than L = %d query rows",
+                    b, cache->seq_n[b], L);
   if (!(scale > 0.f) || scale != scale) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
   cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
   if (e == cudaSuccess) e = launch_attend(cache->g, q, L, scale, out, decode, cache->T,
@@ -431,14 +601,21 @@ kvq_status kvq_project_lora(const void* x, int B, int L, int d_in, const void* w
   int* err = device_error_word();
   if (!err) return fail(KVQ_ERR_CUDA, "cannot resolve the device error word");
   const int* pos_dev = nullptr;
+  int pos_stride = 0;
   if (pos_cache) {
     cudaError_t e0 = ensure_init(pos_cache, (cudaStream_t)stream);
     if (e0 != cudaSuccess) return cuda_fail(e0, "kvq_project_lora");
-    pos_dev = &pos_cache->g.state->tokens;
+    if (pos_cache->g.layout != KVQ_LAYOUT_UNIFORM) {   // each sequence at its own count
+      if (B > pos_cache->g.B) return fail(KVQ_ERR_SHAPE, "B %d > the cache's %d sequences", B, pos_cache->g.B);
+      pos_dev = pos_cache->g.seq_len;
+      pos_stride = 1;
+    } else {
+      pos_dev = &pos_cache->g.state->tokens;
+    }
   }
   cudaError_t e = launch_project(x, B, L, d_in, w_qkv, a, bm, r, alpha_over_r, n_q_heads,
                                  n_kv_heads, head_dim, pos0, pos_dev, rope_base, dtype, out,
-                                 err, (cudaStream_t)stream);
+                                 err, (cudaStream_t)stream, pos_stride);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora launch");
   return KVQ_OK;
 }
@@ -474,15 +651,22 @@ kvq_status kvq_project_lora_nf4(const void* x, int B, int L, int d_in, const voi
       return fail(KVQ_ERR_ARG, "LoRA factors must be 16-byte aligned");
   }
   const int* pos_dev = nullptr;
+  int pos_stride = 0;
   if (pos_cache) {
     cudaError_t e0 = ensure_init(pos_cache, (cudaStream_t)stream);
     if (e0 != cudaSuccess) return cuda_fail(e0, "kvq_project_lora_nf4");
-    pos_dev = &pos_cache->g.state->tokens;
+    if (pos_cache->g.layout != KVQ_LAYOUT_UNIFORM) {   // each sequence at its own count
+      if (B > pos_cache->g.B) return fail(KVQ_ERR_SHAPE, "B %d > the cache's %d sequences", B, pos_cache->g.B);
+      pos_dev = pos_cache->g.seq_len;
+      pos_stride = 1;
+    } else {
+      pos_dev = &pos_cache->g.state->tokens;
+    }
   }
   void* out[3] = {q, k, v};
   cudaError_t e = launch_project_nf4(x, B, L, d_in, w_codes, w_absmax, a, bm, r, alpha_over_r,
                                      n_q_heads, n_kv_heads, head_dim, pos0, pos_dev, rope_base,
-                                     out, (cudaStream_t)stream);
+                                     out, (cudaStream_t)stream, pos_stride);
   if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora_nf4 launch");
   return KVQ_OK;
 }
@@ -490,6 +674,7 @@ kvq_status kvq_project_lora_nf4(const void* x, int B, int L, int d_in, const voi
 // The shapes the fused projection-and-append covers (no launch).
 static const char* project_append_gap(const kvq_cache* c, int L, int d_in, const int r[3]) {
   const Geom& g = c->g;
+  if (g.layout != KVQ_LAYOUT_UNIFORM) return "the cache is ragged or paged";
   if (g.act != KVQ_BF16) return "the activation dtype is not bf16";
   if (g.fmt != KVQ_FMT_AFFINE && g.fmt != KVQ_FMT_SYMMETRIC) return "the cache is not affine or symmetric";
   if (g.G != 32) return "the group size is not 32";
@@ -614,6 +799,7 @@ int kvq_decode_step_fused(const kvq_cache* cache, int d_in, int r_q, int r_k, in
 
 static const char* attend_backward_gap(const kvq_cache* c, int L, int n_q_heads) {
   if (c->g.fmt == KVQ_FMT_KVARN) return "KVarN caches have no backward";
+  if (c->g.layout != KVQ_LAYOUT_UNIFORM) return "ragged and paged caches have no backward";
   if (L <= 0) return "L must be positive";
   if (n_q_heads != c->g.Hq) return "n_q_heads differs from the cache's q_heads";
   if (L > c->T) return "more queries than cached tokens (append first)";
@@ -631,7 +817,8 @@ kvq_status kvq_attend_backward(kvq_cache* cache, const void* q, const void* d_ou
                                void* stream) {
   if (!cache) return fail(KVQ_ERR_ARG, "cache is NULL");
   if (const char* gap = attend_backward_gap(cache, L, n_q_heads))
-    return fail(cache->g.fmt == KVQ_FMT_KVARN ? KVQ_ERR_UNSUPPORTED : KVQ_ERR_SHAPE,
+    return fail(cache->g.fmt == KVQ_FMT_KVARN || cache->g.layout != KVQ_LAYOUT_UNIFORM
+                    ? KVQ_ERR_UNSUPPORTED : KVQ_ERR_SHAPE,
                 "kvq_attend_backward: %s", gap);
   if (!q || !d_out || !d_q || !d_k || !d_v || !workspace)
     return fail(KVQ_ERR_ARG, "NULL tensor pointer");

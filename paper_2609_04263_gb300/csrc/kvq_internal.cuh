@@ -9,6 +9,7 @@
 #include <stdint.h>
 
 #include <utility>
+#include <vector>
 
 #include "../../include/kvq.h"
 
@@ -48,7 +49,16 @@ struct Geom {
   uint32_t* counters;    // [B][Hkv] split arrival counters (zeroed with the state)
   uint32_t* epoch;       // launch counter of the fused decode step; kept across resets
   Plane pl[KVQ_NUM_PLANES];
+  // token layout (kvq_layout).  RAGGED / PAGED: seq_len[b] tokens of sequence
+  // b, seq_new[b] of them appended by the last append; PAGED: token t of
+  // sequence b in pool page page_table[b max_pages + t / 64], and the planes
+  // hold the pool ([1][H][num_pages 64][cols]) instead of [B][H][Tmax][cols]
+  int32_t layout, max_pages;
+  int32_t* seq_len;
+  int32_t* seq_new;
+  int32_t* page_table;
 };
+constexpr int kPageTok = KVQ_PAGE_TOKENS;
 
 __host__ __device__ inline int64_t plane_index(const Plane& pl, int b, int h, int H,
                                                int64_t row, int64_t col) {
@@ -114,6 +124,11 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 // They return cudaGetLastError() of their launches.
 // All launchers read the token count from g.state on the device.
 cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cudaStream_t s);
+// RAGGED / PAGED: sequence b appends its first n[b] (host array) of L tokens;
+// then its device count advances.  seq_reset: sequence b becomes empty.
+cudaError_t launch_append_ragged(const Geom& g, int L, const void* k, const void* v,
+                                 const int* n, cudaStream_t s);
+cudaError_t launch_seq_reset(const Geom& g, int b, cudaStream_t s);
 // t_hint: the host's count of stored tokens, used only to choose between
 // decode kernels (the kernels read the count from the device).
 cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void* out,
@@ -124,7 +139,7 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const void* const a[3], const void* const bm[3], const int r[3],
                            float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                            const int* pos_dev, float rope_base, int act,
-                           void* const out[3], int* err, cudaStream_t s);
+                           void* const out[3], int* err, cudaStream_t s, int pos_stride = 0);
 
 // tcgen05 projection (project_tc.cu) for bf16 and more than 16 rows;
 // cudaErrorNotSupported if the head shapes do not tile.
@@ -135,7 +150,7 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const void* const a[3], const void* const bm[3], const int r[3],
                               float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
-                              cudaStream_t s, const Geom* append_to = nullptr);
+                              cudaStream_t s, const Geom* append_to = nullptr, int pos_stride = 0);
 int project_tc_tile(int Hq, int Hkv, int D, int d_in);
 
 // Projection over an NF4 base (project_nf4.cu): codes [N][d_in/2], fp32 absmax
@@ -145,7 +160,8 @@ cudaError_t launch_project_nf4(const void* x, int B, int L, int d_in, const void
                                const void* absmax, const void* const a[3],
                                const void* const bm[3], const int r[3], float alpha_over_r,
                                int Hq, int Hkv, int D, int pos0, const int* pos_dev,
-                               float rope_base, void* const out[3], cudaStream_t s);
+                               float rope_base, void* const out[3], cudaStream_t s,
+                               int pos_stride = 0);
 void rope_theta_table(float rope_base, int D, float* hi, float* lo);
 
 // Straight-through backward (backward.cu): attention over a cache's
@@ -241,14 +257,54 @@ __device__ __forceinline__ void append_arrive(CacheState* st, int T0, int L, boo
 __device__ __forceinline__ int cache_tokens(const Geom& g) {
   return *reinterpret_cast<volatile int32_t*>(&g.state->tokens);
 }
+// RoPE position offset of sequence b: *pos_dev for every sequence
+// (stride 0), or pos_dev[b] (stride 1: a ragged cache's counts), or 0.
+__device__ __forceinline__ int pos_of(const int* pos_dev, int stride, int b) {
+  return pos_dev ? pos_dev[b * stride] : 0;
+}
+// Tokens of sequence b (every layout).
+__device__ __forceinline__ int seq_tokens(const Geom& g, int b) {
+  return g.layout == KVQ_LAYOUT_UNIFORM ? cache_tokens(g)
+                                        : *reinterpret_cast<volatile int32_t*>(&g.seq_len[b]);
+}
+// Where token t of sequence b sits in a per-token plane: its batch index and
+// row (PAGED: the pool page's row).  Runs of tokens inside one 64-token page
+// are contiguous rows in every layout.
+__device__ __forceinline__ void tok_loc(const Geom& g, int b, int t, int* pb, int64_t* row) {
+  if (g.layout == KVQ_LAYOUT_PAGED) {
+    *pb = 0;
+    *row = (int64_t)g.page_table[b * g.max_pages + (t >> 6)] * kPageTok + (t & (kPageTok - 1));
+  } else {
+    *pb = b;
+    *row = t;
+  }
+}
+template <typename T>
+__device__ __forceinline__ T* tok_ptr(const Geom& g, int which, int b, int h, int t,
+                                      int64_t col = 0) {
+  int pb;
+  int64_t row;
+  tok_loc(g, b, t, &pb, &row);
+  return plane_ptr<T>(g, which, pb, h, row, col);
+}
 
 // Device address of the library's error word (set up once per device).
 int* device_error_word();
 
-// Bytes of the device state region at the start of a cache buffer: the
-// CacheState block, then one split arrival counter per (sequence, kv head).
-inline size_t state_region_bytes(int B, int H) {
-  return sizeof(CacheState) + (((size_t)B * H * 4 + 255) & ~size_t(255));
+// Bytes of the device state region at the start of a cache buffer (zeroed
+// on the first launch after create/reset): the CacheState block, one split
+// arrival counter per (sequence, kv head), then for RAGGED / PAGED layouts
+// seq_len[B], seq_new[B] and the page table [B][max_pages].
+inline size_t state_region_bytes(int B, int H, int layout = KVQ_LAYOUT_UNIFORM,
+                                 int max_pages = 0) {
+  auto a256 = [](size_t x) { return (x + 255) & ~size_t(255); };
+  size_t n = sizeof(CacheState) + a256((size_t)B * H * 4);
+  if (layout != KVQ_LAYOUT_UNIFORM) n += a256((size_t)2 * B * 4);
+  if (layout == KVQ_LAYOUT_PAGED) n += a256((size_t)B * max_pages * 4);
+  return n;
+}
+inline size_t state_region_bytes(const Geom& g) {
+  return state_region_bytes(g.B, g.H, g.layout, g.max_pages);
 }
 
 // Floats of split-K partials a decode over this geometry addresses:
@@ -270,9 +326,14 @@ struct kvq_cache {
   kvq::Geom g;
   char* base;
   size_t bytes;
-  int T;            // host mirror of the device token count
+  int T;            // host mirror of the device token count (RAGGED / PAGED: max T_b)
   bool need_init;   // device state not yet zeroed since create/reset
   bool need_clear;  // workspace and epoch not yet zeroed since create
+  // RAGGED / PAGED: host mirrors of the per-sequence counts; PAGED: each
+  // sequence's pool pages in token order and the pool's free list
+  std::vector<int> seq_T, seq_n;
+  std::vector<std::vector<int>> seq_pages;
+  std::vector<int> free_pages;
 };
 
 namespace kvq {

@@ -61,6 +61,64 @@ __device__ __forceinline__ void load8(const void* base, int64_t e, int act, floa
 // input); else code the new tokens [T0, T0 + L).  A grid-stride loop over
 // 8-element chunks with 32-bit indices (the host bounds the chunk count).
 // ---------------------------------------------------------------------------
+// Code tokens [t_begin, t_begin + ntok) of the (b, h) row of keys (which = 0)
+// or values; src.T0 is the row's first new token.  Stores go through
+// tok_ptr, so the same code serves every token layout.
+__device__ __forceinline__ void pack_rows(const Geom& g, const TokSrc& src, int b, int h,
+                                          int t_begin, int ntok, int which, int sym, int lcpt,
+                                          int llpg) {
+  const int bits = which ? g.vb : g.kb;
+  const int lane = threadIdx.x & 31;
+  const int cpt = 1 << lcpt;               // 8-element chunks per token (D / 8)
+  const int total = ntok << lcpt;          // chunks of this (b, h) row
+  const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
+  const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
+  const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
+  const int stride = gridDim.x * blockDim.x;
+  // chunk i = token * cpt + c8 of the row.  A warp covers 32 consecutive
+  // chunks, so a group's G/8 lanes are consecutive and aligned
+  for (int i0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < total; i0 += stride) {
+    const int i = i0 + lane;
+    const bool live = i < total;
+    const int ii = live ? i : total - 1;
+    const int t = t_begin + (ii >> lcpt), c8 = ii & (cpt - 1);
+    const int grp = c8 >> llpg, li = c8 & ((1 << llpg) - 1);
+    const void* sb;
+    const int64_t e = tok_elem(g, src, b, h, t, &sb) + c8 * 8;
+    float v[8];
+    load8(sb, e, g.act, v);
+    float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) {
+      if (sym) hi = fmaxf(hi, fabsf(v[i]));
+      else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
+    }
+    for (int off = (1 << llpg) >> 1; off > 0; off >>= 1) {
+      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
+      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
+    }
+    float s;
+    uint64_t word;
+    if (sym) {
+      word = bits == 2 ? code8<2, true>(v, lo, hi, &s)
+           : bits == 4 ? code8<4, true>(v, lo, hi, &s) : code8<8, true>(v, lo, hi, &s);
+    } else {
+      word = bits == 2 ? code8<2, false>(v, lo, hi, &s)
+           : bits == 4 ? code8<4, false>(v, lo, hi, &s) : code8<8, false>(v, lo, hi, &s);
+    }
+    if (!live) continue;
+    uint8_t* crow = tok_ptr<uint8_t>(g, codes_plane, b, h, t);
+    const int byte0 = c8 * bits;
+    if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
+    else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
+    else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
+    if (li == 0) {
+      *tok_ptr<__half>(g, scale_plane, b, h, t, grp) = __float2half_rn(s);
+      if (!sym) *tok_ptr<__half>(g, zero_plane, b, h, t, grp) = __float2half_rn(lo + 0.0f);
+    }
+  }
+}
+
 __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
                                      int final_kernel, int lcpt, int llpg) {
   pdl_wait();
@@ -76,61 +134,39 @@ __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sy
   if (ok && t_end > t_begin) {
     TokSrc src = which ? sv : sk;
     src.T0 = T0;
-    const int bits = which ? g.vb : g.kb;
-    const int lane = threadIdx.x & 31;
-    const int cpt = 1 << lcpt;               // 8-element chunks per token (D / 8)
-    const int ntok = t_end - t_begin;
-    const int total = ntok << lcpt;          // chunks of this (b, h) row
     const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
-    const int codes_plane = which ? KVQ_PLANE_V_CODES : KVQ_PLANE_K_CODES;
-    const int scale_plane = which ? KVQ_PLANE_V_SCALE : KVQ_PLANE_K_SCALE;
-    const int zero_plane = which ? KVQ_PLANE_V_ZERO : KVQ_PLANE_K_ZERO;
-    const int stride = gridDim.x * blockDim.x;
-    // blockIdx.y is the (b, h) row; chunk i = token * cpt + c8 of it.  A warp
-    // covers 32 consecutive chunks, so a group's G/8 lanes are consecutive
-    // and aligned
-    for (int i0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < total; i0 += stride) {
-      const int i = i0 + lane;
-      const bool live = i < total;
-      const int ii = live ? i : total - 1;
-      const int t = t_begin + (ii >> lcpt), c8 = ii & (cpt - 1);
-      const int grp = c8 >> llpg, li = c8 & ((1 << llpg) - 1);
-      const void* sb;
-      const int64_t e = tok_elem(g, src, b, h, t, &sb) + c8 * 8;
-      float v[8];
-      load8(sb, e, g.act, v);
-      float lo = v[0], hi = sym ? fabsf(v[0]) : v[0];
-#pragma unroll
-      for (int i = 1; i < 8; ++i) {
-        if (sym) hi = fmaxf(hi, fabsf(v[i]));
-        else { lo = fminf(lo, v[i]); hi = fmaxf(hi, v[i]); }
-      }
-      for (int off = (1 << llpg) >> 1; off > 0; off >>= 1) {
-        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, off));
-        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, off));
-      }
-      float s;
-      uint64_t word;
-      if (sym) {
-        word = bits == 2 ? code8<2, true>(v, lo, hi, &s)
-             : bits == 4 ? code8<4, true>(v, lo, hi, &s) : code8<8, true>(v, lo, hi, &s);
-      } else {
-        word = bits == 2 ? code8<2, false>(v, lo, hi, &s)
-             : bits == 4 ? code8<4, false>(v, lo, hi, &s) : code8<8, false>(v, lo, hi, &s);
-      }
-      if (!live) continue;
-      uint8_t* crow = plane_ptr<uint8_t>(g, codes_plane, b, h, t);
-      const int byte0 = c8 * bits;
-      if (bits == 2) *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)word;
-      else if (bits == 4) *reinterpret_cast<uint32_t*>(crow + byte0) = (uint32_t)word;
-      else *reinterpret_cast<uint64_t*>(crow + byte0) = word;
-      if (li == 0) {
-        *plane_ptr<__half>(g, scale_plane, b, h, t, grp) = __float2half_rn(s);
-        if (!sym) *plane_ptr<__half>(g, zero_plane, b, h, t, grp) = __float2half_rn(lo + 0.0f);
-      }
-    }
+    pack_rows(g, src, b, h, t_begin, t_end - t_begin, which, sym, lcpt, llpg);
   }
   if (final_kernel) append_arrive_spread(g.state, T0, L, ok);
+}
+
+// Ragged append (layouts RAGGED and PAGED, affine or symmetric): sequence b
+// codes the first n.n[b] of its L new tokens at its own positions
+// seq_len[b] ..; the host has checked capacity and assigned the pages.
+struct SeqCounts {
+  int32_t n[KVQ_MAX_SEQS];
+};
+
+__global__ void pack_ragged_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int lcpt,
+                                   int llpg, SeqCounts n) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
+  const int nb = n.n[b];
+  if (nb <= 0) return;
+  TokSrc src = blockIdx.z ? sv : sk;
+  src.T0 = seq_tokens(g, b);
+  pack_rows(g, src, b, h, src.T0, nb, blockIdx.z, sym, lcpt, llpg);
+}
+
+// After a ragged append: the sequences' counts.
+__global__ void seq_advance_kernel(Geom g, SeqCounts n) {
+  pdl_wait();
+  pdl_trigger();
+  for (int b = threadIdx.x; b < g.B; b += blockDim.x) {
+    g.seq_len[b] += n.n[b];
+    g.seq_new[b] = n.n[b];
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -710,6 +746,35 @@ int grid_for(int64_t threads_needed, int block) {
 }
 
 }  // namespace
+
+cudaError_t launch_append_ragged(const Geom& g, int L, const void* k, const void* v,
+                                 const int* n, cudaStream_t s) {
+  TokSrc sk{k, 0, L, -1, 0, 1}, sv{v, 0, L, -1, 0, 1};
+  SeqCounts c = {};
+  for (int b = 0; b < g.B; ++b) c.n[b] = n[b];
+  const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
+  launch_pdl(pack_ragged_kernel, pertoken_grid(g, L, 2), dim3(256), 0, s, g, L, sk, sv, sym,
+             ilog2(g.D / 8), ilog2(g.G / 8), c);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  launch_pdl(seq_advance_kernel, dim3(1), dim3(256), 0, s, g, c);
+  return cudaGetLastError();
+}
+
+// A sequence of a ragged cache becomes empty.
+__global__ void seq_reset_kernel(Geom g, int b) {
+  pdl_wait();
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    g.seq_len[b] = 0;
+    g.seq_new[b] = 0;
+  }
+}
+
+cudaError_t launch_seq_reset(const Geom& g, int b, cudaStream_t s) {
+  launch_pdl(seq_reset_kernel, dim3(1), dim3(32), 0, s, g, b);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cudaStream_t s) {
   TokSrc sk{k, 0, L, -1, 0, 1}, sv{v, 0, L, -1, 0, 1};

@@ -17,7 +17,8 @@ struct ProjArgs {
   int r[3];
   void* out[3];
   int B, L, d_in, Hq, Hkv, D, pos0, act;
-  const int* pos_dev;   // if set, positions start at *pos_dev + pos0
+  const int* pos_dev;   // if set, positions start at pos_of(pos_dev, pos_stride, b) + pos0
+  int pos_stride;
   float alpha_over_r, rope_base;
   // RoPE frequencies base^(-2i/D), i < D/2, computed in fp64 on the host and
   // split into hi + lo floats
@@ -173,7 +174,7 @@ __device__ void proj_decode_tile(const ProjArgs& p, int tile, unsigned char* dsm
     const int b = m / p.L, l = m % p.L;
     const int c = c0 + i;
     if (proj < 2 && p.rope_base > 0.f) {
-      const int pos = p.pos0 + (p.pos_dev ? *p.pos_dev : 0) + l;
+      const int pos = p.pos0 + pos_of(p.pos_dev, p.pos_stride, b) + l;
       float cs, sn;
       rope_cos_sin(pos, p.theta_hi[c], p.theta_lo[c], &cs, &sn);
       const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;

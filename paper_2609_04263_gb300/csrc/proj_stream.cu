@@ -222,7 +222,6 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
     if (M16 == 16 && k < K && gid + 8 < M)
       xb[h] = __ldg(reinterpret_cast<const uint4*>(x + (int64_t)(gid + 8) * K + k));
   }
-  const int pos_base = a.pos0 + (a.pos_dev ? *a.pos_dev : 0);
   float acc[2][4];
 #pragma unroll
   for (int n = 0; n < 2; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
@@ -311,7 +310,8 @@ project_decode_stream_kernel(const ProjArgs a, const PSLayout L, int* err) {
       const int c = t.c0 + i;
       if (t.p < 2 && a.rope_base > 0.f) {
         float cs, sn;
-        rope_cos_sin(pos_base + l, a.theta_hi[c], a.theta_lo[c], &cs, &sn);
+        rope_cos_sin(a.pos0 + pos_of(a.pos_dev, a.pos_stride, b) + l, a.theta_hi[c],
+                     a.theta_lo[c], &cs, &sn);
         const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
         y1 = o1;
         y2 = o2;

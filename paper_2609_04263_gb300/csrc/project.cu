@@ -110,7 +110,6 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
   __syncthreads();
   // RoPE (rotate-half) on q and k; angle in fp64 for accuracy
   const bool rope = proj < 2 && p.rope_base > 0.f;
-  const int pos_base = p.pos0 + (p.pos_dev ? *p.pos_dev : 0);
   const int H = proj == 0 ? p.Hq : p.Hkv;
   for (int i = threadIdx.x; i < kMT * D; i += kThreads) {
     const int m = i / D, d = i % D;
@@ -121,7 +120,8 @@ __global__ void __launch_bounds__(kThreads) project_simt_kernel(ProjArgs p) {
     if (rope) {
       const int half = D / 2, fi = d % half;
       float c, s;
-      rope_cos_sin(pos_base + l, p.theta_hi[fi], p.theta_lo[fi], &c, &s);
+      rope_cos_sin(p.pos0 + pos_of(p.pos_dev, p.pos_stride, b) + l, p.theta_hi[fi],
+                   p.theta_lo[fi], &c, &s);
       if (d < half) v = Y[m * D + d] * c - Y[m * D + d + half] * s;
       else v = Y[m * D + d] * c + Y[m * D + d - half] * s;
     }
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(kSkinnyWarps * 32, 3) project_skinny_kernel(Pr
     }
     const int b = lane / p.L, l = lane % p.L;
     if (proj < 2 && p.rope_base > 0.f) {
-      const int pos = p.pos0 + (p.pos_dev ? *p.pos_dev : 0) + l;
+      const int pos = p.pos0 + pos_of(p.pos_dev, p.pos_stride, b) + l;
       float cs, sn;
       rope_cos_sin(pos, p.theta_hi[c], p.theta_lo[c], &cs, &sn);
       const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
@@ -418,18 +418,19 @@ cudaError_t launch_project(const void* x, int B, int L, int d_in, const void* w,
                            const void* const a[3], const void* const bm[3], const int r[3],
                            float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                            const int* pos_dev, float rope_base, int act,
-                           void* const out[3], int* err, cudaStream_t s) {
+                           void* const out[3], int* err, cudaStream_t s, int pos_stride) {
   ProjArgs p;
   p.x = x; p.w = w;
   for (int i = 0; i < 3; ++i) { p.a[i] = a[i]; p.bm[i] = bm[i]; p.r[i] = r[i]; p.out[i] = out[i]; }
   p.B = B; p.L = L; p.d_in = d_in; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.pos0 = pos0; p.act = act;
   p.pos_dev = pos_dev;
+  p.pos_stride = pos_stride;
   p.alpha_over_r = alpha_over_r; p.rope_base = rope_base;
   rope_theta_table(rope_base, D, p.theta_hi, p.theta_lo);
   const int M = B * L;
   if (act == KVQ_BF16 && M > kSkinnyMaxM) {
     cudaError_t e = launch_project_tc(x, B, L, d_in, w, a, bm, r, alpha_over_r, Hq, Hkv, D, pos0,
-                                      pos_dev, rope_base, out, err, s);
+                                      pos_dev, rope_base, out, err, s, nullptr, pos_stride);
     if (e != cudaErrorNotSupported) return e;
     (void)cudaGetLastError();
   }

@@ -48,6 +48,7 @@ struct Nf4Args {
   int n_off[4];
   int pos0;
   const int* pos_dev;
+  int pos_stride;
   float alpha_over_r;
   int rope;
   float theta_hi[128], theta_lo[128];
@@ -279,7 +280,6 @@ project_nf4_kernel(const Nf4Args args) {
   const int H = proj == 0 ? args.Hq : args.Hkv;
   const int col0 = n0 - args.n_off[proj];
   const bool rope = args.rope && proj < 2;
-  const int pos_base = args.pos0 + (args.pos_dev ? *args.pos_dev : 0);
   // work items: (row, head of the tile, 8 frequencies)
   const int per_row = (NBN / D) * (half / 8);
   for (int it = tid; it < BM * per_row; it += kNThreads) {
@@ -299,7 +299,8 @@ project_nf4_kernel(const Nf4Args args) {
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         float cs, sn;
-        pdec::rope_cos_sin(pos_base + l, args.theta_hi[f0 + i], args.theta_lo[f0 + i], &cs, &sn);
+        pdec::rope_cos_sin(args.pos0 + pos_of(args.pos_dev, args.pos_stride, b) + l,
+                           args.theta_hi[f0 + i], args.theta_lo[f0 + i], &cs, &sn);
         const float a = x1[i], bb = x2[i];
         x1[i] = a * cs - bb * sn;
         x2[i] = bb * cs + a * sn;
@@ -344,7 +345,8 @@ cudaError_t launch_project_nf4(const void* x, int B, int L, int d_in, const void
                                const void* absmax, const void* const a[3],
                                const void* const bm[3], const int r[3], float alpha_over_r,
                                int Hq, int Hkv, int D, int pos0, const int* pos_dev,
-                               float rope_base, void* const out[3], cudaStream_t s) {
+                               float rope_base, void* const out[3], cudaStream_t s,
+                               int pos_stride) {
   Nf4Args t;
   t.x = static_cast<const __nv_bfloat16*>(x);
   t.codes = static_cast<const uint8_t*>(codes);
@@ -357,7 +359,7 @@ cudaError_t launch_project_nf4(const void* x, int B, int L, int d_in, const void
   }
   t.B = B; t.L = L; t.M = B * L; t.d_in = d_in; t.Hq = Hq; t.Hkv = Hkv; t.D = D;
   t.n_off[0] = 0; t.n_off[1] = Hq * D; t.n_off[2] = (Hq + Hkv) * D; t.n_off[3] = (Hq + 2 * Hkv) * D;
-  t.pos0 = pos0; t.pos_dev = pos_dev; t.alpha_over_r = alpha_over_r;
+  t.pos0 = pos0; t.pos_dev = pos_dev; t.pos_stride = pos_stride; t.alpha_over_r = alpha_over_r;
   t.rope = rope_base > 0.f;
   rope_theta_table(rope_base, D, t.theta_hi, t.theta_lo);
   return t.M <= 16 ? launch_nf4_bm<16>(t, s) : launch_nf4_bm<64>(t, s);

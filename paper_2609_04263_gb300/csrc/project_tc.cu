@@ -45,6 +45,7 @@ struct TcArgs {
   int r[3], rp[3];              // ranks and ranks padded to 16
   int pos0;
   const int* pos_dev;
+  int pos_stride;
   float alpha_over_r;
   int rope;
   int k_blocks;
@@ -277,7 +278,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     const int col0 = n0 - args.n_off[proj];           // first column within projection
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(args.out[proj]);
     const bool rope = args.rope && proj < 2;
-    const int pos = args.pos0 + (args.pos_dev ? *args.pos_dev : 0) + l;
+    const int pos = args.pos0 + pos_of(args.pos_dev, args.pos_stride, b) + l;
     if (args.pack && proj > 0) {
       // append: k (after RoPE) and v rounded to bf16, then coded per token
       // in groups of 32 channels straight into the cache planes
@@ -427,7 +428,7 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const void* const a[3], const void* const bm[3], const int r[3],
                               float alpha_over_r, int Hq, int Hkv, int D, int pos0,
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
-                              cudaStream_t s, const Geom* append_to) {
+                              cudaStream_t s, const Geom* append_to, int pos_stride) {
   const int bn = project_tc_tile(Hq, Hkv, D, d_in);
   if (!bn) return cudaErrorNotSupported;
   TcArgs t;
@@ -442,7 +443,7 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
   }
   t.B = B; t.L = L; t.M = M; t.D = D; t.Hq = Hq; t.Hkv = Hkv;
   t.n_off[0] = 0; t.n_off[1] = Hq * D; t.n_off[2] = (Hq + Hkv) * D; t.n_off[3] = (Hq + 2 * Hkv) * D;
-  t.pos0 = pos0; t.pos_dev = pos_dev; t.alpha_over_r = alpha_over_r;
+  t.pos0 = pos0; t.pos_dev = pos_dev; t.pos_stride = pos_stride; t.alpha_over_r = alpha_over_r;
   t.rope = rope_base > 0.f; t.k_blocks = d_in / 64; t.err = err;
   rope_theta_table(rope_base, D, t.theta_hi, t.theta_lo);
   CUtensorMap maps[8];

@@ -16,6 +16,9 @@ KVQ_OK, KVQ_ERR_ARG, KVQ_ERR_SHAPE, KVQ_ERR_CAPACITY, KVQ_ERR_UNSUPPORTED, \
     KVQ_ERR_CUDA, KVQ_ERR_TIMEOUT = range(7)
 KVQ_FMT_FLOAT, KVQ_FMT_AFFINE, KVQ_FMT_SYMMETRIC, KVQ_FMT_KIVI, KVQ_FMT_KVARN = range(5)
 KVQ_F32, KVQ_BF16 = 0, 1
+KVQ_LAYOUT_UNIFORM, KVQ_LAYOUT_RAGGED, KVQ_LAYOUT_PAGED = range(3)
+KVQ_PAGE_TOKENS = 64
+KVQ_MAX_SEQS = 512
 
 PLANES = ["k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "k_full",
           "v_full", "k_pend", "v_pend", "k_row", "k_col", "v_row", "v_col", "workspace"]
@@ -33,7 +36,8 @@ class KvqError(RuntimeError):
 class kvq_cache_desc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "fmt", "key_bits", "value_bits", "group_size", "residual_tokens", "sink_tokens",
-        "norm_iters", "batch", "kv_heads", "q_heads", "head_dim", "max_tokens", "dtype")]
+        "norm_iters", "batch", "kv_heads", "q_heads", "head_dim", "max_tokens", "dtype",
+        "layout", "num_pages")]
 
 
 class kvq_cache_planes(ctypes.Structure):
@@ -81,6 +85,12 @@ _SIGS = {
                                      c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
                                      c_int, c_void_p, c_float, c_void_p, c_void_p, c_void_p,
                                      c_void_p]),
+    "kvq_append_pack_ragged": (c_int, [c_void_p, c_void_p, c_void_p, c_int,
+                                       ctypes.POINTER(c_int), c_void_p]),
+    "kvq_seq_tokens": (c_int, [c_void_p, c_int]),
+    "kvq_seq_release": (c_int, [c_void_p, c_int, c_void_p]),
+    "kvq_free_pages": (c_int, [c_void_p]),
+    "kvq_seq_pages": (c_int, [c_void_p, c_int, ctypes.POINTER(c_int), c_int]),
     "kvq_attend_backward_workspace": (c_size_t, [c_void_p, c_int, c_int]),
     "kvq_attend_backward": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_float,
                                     c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
@@ -265,4 +275,31 @@ def kvq_lora_backward(x, B, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b
         c_void_p(d_v), kv_rows, c_void_p(da_q), c_void_p(db_q), c_void_p(da_k), c_void_p(db_k),
         c_void_p(da_v), c_void_p(db_v), c_void_p(d_x), c_void_p(workspace), workspace_bytes,
         c_void_p(stream or 0)))
+
+
+def kvq_append_pack_ragged(handle, k, v, L, n=None, stream=0) -> None:
+    arr = None if n is None else (c_int * len(n))(*[int(x) for x in n])
+    _check(lib().kvq_append_pack_ragged(c_void_p(handle), c_void_p(k), c_void_p(v), L, arr,
+                                        c_void_p(stream or 0)))
+
+
+def kvq_seq_tokens(handle, b) -> int:
+    return lib().kvq_seq_tokens(c_void_p(handle), b)
+
+
+def kvq_seq_release(handle, b, stream=0) -> None:
+    _check(lib().kvq_seq_release(c_void_p(handle), b, c_void_p(stream or 0)))
+
+
+def kvq_free_pages(handle) -> int:
+    return lib().kvq_free_pages(c_void_p(handle))
+
+
+def kvq_seq_pages(handle, b) -> list:
+    n = lib().kvq_seq_pages(c_void_p(handle), b, None, 0)
+    if n < 0:
+        return []
+    buf = (c_int * max(n, 1))()
+    lib().kvq_seq_pages(c_void_p(handle), b, buf, n)
+    return [buf[i] for i in range(n)]
 

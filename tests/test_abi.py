@@ -224,3 +224,51 @@ def test_backward_host_rules(kvq):
                               0, 1e4, kvq.KVQ_BF16, P, P, P, L - 1, P, P, None, None, P, P, None,
                               P, want, 0)
     assert ei.value.status == kvq.KVQ_ERR_SHAPE
+
+
+def test_ragged_and_paged_layout_rules(kvq):
+    """Ragged and paged layouts are built for bf16 affine / symmetric caches
+    (G 32, equal 2- or 4-bit keys and values, head_dim 64 or 128); a paged
+    cache sizes its planes by the pool, starts with every page free, and
+    refuses appends beyond max_tokens before any launch."""
+    fake = 1 << 32
+    P = 1 << 33
+    base = dict(batch=3, kv_heads=2, q_heads=8, head_dim=64, max_tokens=500)
+    for kw in (dict(fmt=kvq.KVQ_FMT_KIVI, residual_tokens=32), dict(dtype=kvq.KVQ_F32),
+               dict(key_bits=2), dict(group_size=64), dict(head_dim=256)):
+        d = _desc(kvq, **{**base, **kw, "layout": kvq.KVQ_LAYOUT_RAGGED})
+        with pytest.raises(kvq.KvqError):
+            kvq.kvq_cache_bytes(d)
+    d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_PAGED, num_pages=0)
+    with pytest.raises(kvq.KvqError):                       # a pool needs pages
+        kvq.kvq_cache_bytes(d)
+    d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_PAGED, num_pages=10)
+    n = kvq.kvq_cache_bytes(d)
+    h = kvq.kvq_create_cache(d, fake, n)
+    try:
+        assert kvq.kvq_free_pages(h) == 10
+        assert kvq.kvq_seq_pages(h, 0) == []
+        assert kvq.kvq_seq_tokens(h, 2) == 0 and kvq.kvq_seq_tokens(h, 3) == -1
+        v = kvq.kvq_cache_view(h)
+        assert v.dims[0][0] == 1 and v.dims[0][2] == 10 * 64       # codes: the pool
+        with pytest.raises(kvq.KvqError) as ei:                    # beyond max_tokens
+            kvq.kvq_append_pack_ragged(h, P, P, 600, [600, 0, 0], 0)
+        assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+        with pytest.raises(kvq.KvqError) as ei:                    # more pages than the pool
+            kvq.kvq_append_pack_ragged(h, P, P, 400, [400, 400, 0], 0)
+        assert ei.value.status == kvq.KVQ_ERR_CAPACITY
+        with pytest.raises(kvq.KvqError) as ei:                    # a count above L
+            kvq.kvq_append_pack_ragged(h, P, P, 4, [5, 0, 0], 0)
+        assert ei.value.status == kvq.KVQ_ERR_ARG
+        assert kvq.kvq_free_pages(h) == 10                          # nothing was taken
+    finally:
+        kvq.kvq_destroy_cache(h)
+    # a ragged cache of the same shape holds B x max_tokens rows and no pool
+    d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_RAGGED)
+    h = kvq.kvq_create_cache(d, fake, kvq.kvq_cache_bytes(d))
+    try:
+        assert kvq.kvq_free_pages(h) == -1
+        v = kvq.kvq_cache_view(h)
+        assert v.dims[0][0] == 3 and v.dims[0][2] == 512
+    finally:
+        kvq.kvq_destroy_cache(h)
