@@ -522,6 +522,48 @@ def nf4_projection_rates(run, peaks, flush):
             "l2": "flushed before each timed launch"}
 
 
+def paged_decode_rates(run, peaks, flush):
+    """Decode attention over a PAGED cache (64-token pages from one pool, each
+    sequence at its own length: continuous batching) with the workload's head
+    shape, batch and bit width, lengths spread evenly over [P/2, P] for a
+    P-token prefill.  The workload's own format when a paged cache supports it
+    (affine, symmetric), otherwise an affine cache of the same bit width (KIVI
+    and KVarN caches are uniform only).  Against HBM: the coded tokens' bytes
+    of every sequence plus q and out."""
+    from paper_2609_04263_gb300 import kvq
+    wl, api = run.wl, run.api
+    if wl.dtype != "bf16" or wl.head_dim not in (64, 128) or wl.key_bits not in (2, 4):
+        return None
+    fmt = wl.fmt if wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC) else synth.FMT_AFFINE
+    B, H, Hq, D, P = wl.batch, wl.n_kv_heads, wl.n_q_heads, wl.head_dim, wl.prefill
+    lens = [P // 2 + (P - P // 2) * b // max(B - 1, 1) for b in range(B)]
+    pages = sum((t + 64) // 64 for t in lens)
+    desc = api.make_desc(fmt, wl.key_bits, wl.key_bits, 32, B, H, Hq, D, P + 64, torch.bfloat16,
+                         layout=kvq.KVQ_LAYOUT_PAGED, num_pages=pages)
+    cache = api.Cache(desc, device=run.dev)
+    g = torch.Generator(device="cpu").manual_seed(3)
+    for lo in range(0, P, 1024):               # ragged prefill in chunks
+        n = [max(0, min(1024, t - lo)) for t in lens]
+        L = max(n)
+        if L == 0:
+            break
+        k = torch.randn(B, H, L, D, generator=g).to(torch.bfloat16).to(run.dev)
+        v = torch.randn(B, H, L, D, generator=g).to(torch.bfloat16).to(run.dev)
+        cache.append_ragged(k, v, n)
+    q = torch.randn(B, Hq, 1, D, generator=g).to(torch.bfloat16).to(run.dev)
+    out = torch.empty_like(q)
+    ms = cold_graph_time_ms(lambda: cache.attend_decode(q, out=out), 10, flush)
+    per_tok = D * wl.key_bits // 8 * 2 + 2 * (D // 32) * (2 if fmt == synth.FMT_SYMMETRIC else 4)
+    nbytes = H * per_tok * sum(lens) + 2 * B * Hq * D * 2
+    return {"format": {synth.FMT_AFFINE: "affine", synth.FMT_SYMMETRIC: "symmetric"}[fmt],
+            "bits": wl.key_bits, "sequences": B, "tokens_min": min(lens), "tokens_max": max(lens),
+            "pages": pages, "mean_ms": round(ms, 5), "algorithmic_bytes": nbytes,
+            "achieved": round(nbytes / ms / 1e6, 3), "unit": "GB/s",
+            "frac": round(nbytes / ms / 1e6 / peaks["hbm_gbs"], 4),
+            "kernel": "attend_decode_mma_kernel (split-K, chunks through the page table)",
+            "l2": "flushed before each timed launch"}
+
+
 # fp32 FMA rate of the GB300: 152 SMs x 128 fp32 lanes x 2 flops x 2070 MHz
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
 
@@ -871,6 +913,7 @@ def main():
                         "traffic": measured_traffic(wl.name, "decode_attention")}
     nf4 = nf4_projection_rates(run, peaks, flush) if wl.dtype == "bf16" else None
     ste = ste_backward_rates(run, flush)
+    paged = paged_decode_rates(run, peaks, flush)
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)
     bound, amount, _ = work[dominant]
@@ -947,6 +990,7 @@ def main():
             "decode_attention": decode_attention,
             "nf4_projection": nf4,
             "ste_backward": ste,
+            "paged_decode": paged,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},

@@ -418,7 +418,10 @@ kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* 
  * kvq_attend_decode then attend, per sequence, the n[b] rows of the last
  * append (prefill: rows l < n[b] of q and out; the rest of out is not
  * written) or its newest token (decode; a sequence holding no token gets a
- * zero output) over that sequence's T_b tokens.
+ * zero output) over that sequence's T_b tokens.  A PAGED append that takes
+ * new pages copies their table entries from host memory on `stream`, so it
+ * must not be captured in a CUDA graph; RAGGED appends and the attention
+ * calls can be (kvq_cache_sync then refreshes the host's per-sequence counts).
  */
 kvq_status kvq_append_pack_ragged(kvq_cache* cache, const void* k, const void* v, int L,
                                   const int* n, void* stream);
