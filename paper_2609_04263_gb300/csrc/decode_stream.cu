@@ -32,6 +32,8 @@
 //     the bias and the per-token offsets m are two small MMAs (rows = groups).
 // KIVI's newest tokens (its full-precision residual ring) are read from
 // global memory as bf16 rows in the same layout.
+#include <type_traits>
+
 #include "decode_attn.cuh"
 #include "stream_common.cuh"
 
@@ -343,7 +345,11 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   };
 
   // one 32-token block: scores, online softmax, P V
-  auto process = [&](const unsigned char* sp, int sub_blk, int t0, int nv, bool coded) {
+  // full: all kBT tokens of the block are stored (every block but a head's
+  // last), so the per-token validity checks fold away
+  auto process = [&](auto full, const unsigned char* sp, int sub_blk, int t0, int nv_in,
+                     bool coded) {
+    const int nv = decltype(full)::value ? kBT : nv_in;
     const unsigned char* kcp = sp + C::KC + sub_blk * kBT * C::KCB;
     const unsigned char* vcp = sp + C::VC + sub_blk * kBT * C::VCB;
     const unsigned char* ksp = sp + C::KS + sub_blk * C::KMETA;
@@ -667,7 +673,11 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         break;
       }
       const int t0 = (int)(k0 + j - hs) * kBT;
-      process(smem + (size_t)st * C::STAGE, j % kSB, t0, min(kBT, T - t0), t0 < tq);
+      const int nv = min(kBT, T - t0);
+      if (nv == kBT)
+        process(std::true_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tq);
+      else
+        process(std::false_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tq);
       __syncwarp();
       if (lane == 0) mbar_arrive1(&empty[st]);
     }
