@@ -523,7 +523,7 @@ def nf4_projection_rates(run, peaks, flush):
 
 
 def paged_decode_rates(run, peaks, flush):
-    """Decode attention over a PAGED cache (64-token pages from one pool, each
+    """Decode attention over a PAGED cache (256-token pages from one pool, each
     sequence at its own length: continuous batching) with the workload's head
     shape, batch and bit width, lengths spread evenly over [P/2, P] for a
     P-token prefill.  The workload's own format when a paged cache supports it
@@ -537,7 +537,7 @@ def paged_decode_rates(run, peaks, flush):
     fmt = wl.fmt if wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC) else synth.FMT_AFFINE
     B, H, Hq, D, P = wl.batch, wl.n_kv_heads, wl.n_q_heads, wl.head_dim, wl.prefill
     lens = [P // 2 + (P - P // 2) * b // max(B - 1, 1) for b in range(B)]
-    pages = sum((t + 64) // 64 for t in lens)
+    pages = sum((t + 256) // 256 for t in lens)
     desc = api.make_desc(fmt, wl.key_bits, wl.key_bits, 32, B, H, Hq, D, P + 64, torch.bfloat16,
                          layout=kvq.KVQ_LAYOUT_PAGED, num_pages=pages)
     cache = api.Cache(desc, device=run.dev)
@@ -560,7 +560,7 @@ def paged_decode_rates(run, peaks, flush):
             "pages": pages, "mean_ms": round(ms, 5), "algorithmic_bytes": nbytes,
             "achieved": round(nbytes / ms / 1e6, 3), "unit": "GB/s",
             "frac": round(nbytes / ms / 1e6 / peaks["hbm_gbs"], 4),
-            "kernel": "attend_decode_mma_kernel (split-K, chunks through the page table)",
+            "kernel": "the decode of a uniform cache of this shape, runs of blocks inside one page",
             "l2": "flushed before each timed launch"}
 
 

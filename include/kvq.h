@@ -105,12 +105,12 @@ typedef struct {
  *   PAGED    RAGGED, with each sequence's tokens in pages of KVQ_PAGE_TOKENS
  *            tokens taken from one pool of num_pages pages by the library's
  *            allocator as the sequence grows, and returned by
- *            kvq_seq_release; a sequence holds ceil(T_b / 64) pages.
+ *            kvq_seq_release; a sequence holds ceil(T_b / 256) pages.
  * RAGGED and PAGED caches are built for bf16 AFFINE and SYMMETRIC caches with
  * group_size 32, key_bits == value_bits in {2, 4}, head_dim 64 or 128, at most
  * 16 query heads per kv head and at most KVQ_MAX_SEQS sequences. */
 typedef enum { KVQ_LAYOUT_UNIFORM = 0, KVQ_LAYOUT_RAGGED = 1, KVQ_LAYOUT_PAGED = 2 } kvq_layout;
-#define KVQ_PAGE_TOKENS 64
+#define KVQ_PAGE_TOKENS 256
 #define KVQ_MAX_SEQS 512
 
 typedef struct kvq_cache kvq_cache;   /* opaque, host-side bookkeeping only */

@@ -119,21 +119,91 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   Merge* mg = reinterpret_cast<Merge*>(slot + kNW * PW);
   uint64_t* full = reinterpret_cast<uint64_t*>(mg + 1);
   uint64_t* empty = full + ns;
+  // ragged / paged caches: each sequence's tokens and first flattened block
+  int* s_T = reinterpret_cast<int*>(empty + ns);     // [B]
+  int64_t* s_pre = reinterpret_cast<int64_t*>(s_T + ((g.B + 1) & ~1));   // [B + 1]
 
-  const int T = cache_tokens(g);
+  // (KIVI caches are uniform only)
+  const bool rag = !C::KIVI && g.layout != KVQ_LAYOUT_UNIFORM;
+  const bool paged = !C::KIVI && g.layout == KVQ_LAYOUT_PAGED;
+  const int T = rag ? 0 : cache_tokens(g);
   const int BH = g.B * g.H;
-  const int nb = (T + kBT - 1) / kBT;                // blocks per head
-  const int64_t N = (int64_t)BH * nb;
-  if (N == 0) {                                      // nothing stored: zero output
+  const int nb = (T + kBT - 1) / kBT;                // blocks per head (uniform layout)
+  if (rag) {
+    // s_pre[b] = blocks of the sequences before b (H heads each): one warp,
+    // 32 sequences per step, a shuffle scan within the step
+    if (warp == 0) {
+      int64_t run = 0;
+      for (int b0 = 0; b0 < g.B; b0 += 32) {
+        const int b = b0 + lane;
+        const int tb = b < g.B ? *reinterpret_cast<volatile int32_t*>(&g.seq_len[b]) : 0;
+        if (b < g.B) s_T[b] = tb;
+        int64_t x = (int64_t)g.H * ((tb + kBT - 1) / kBT), incl = x;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int64_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (b < g.B) s_pre[b] = run + incl - x;
+        run += __shfl_sync(0xffffffffu, incl, 31);
+      }
+      if (lane == 0) s_pre[g.B] = run;
+    }
+    __syncthreads();
+    // a sequence holding no token attends to nothing: zero output (no block
+    // of the flattened space belongs to it, so no CTA writes it otherwise)
     if (blockIdx.x == 0)
+      for (int i = threadIdx.x; i < g.B * g.Hq * D; i += blockDim.x)
+        if (s_T[i / (g.Hq * D)] == 0) out[i] = __float2bfloat16(0.f);
+  }
+  const int64_t N = rag ? s_pre[g.B] : (int64_t)BH * nb;
+  if (N == 0) {                                      // nothing stored: zero output
+    if (blockIdx.x == 0 && !rag)
       for (int i = threadIdx.x; i < g.B * g.Hq * D; i += blockDim.x) out[i] = __float2bfloat16(0.f);
     return;
   }
+  // head hd = b H + hkv: its tokens, blocks and first flattened block; the
+  // head holding flattened block k
+  auto T_of = [&](int hd) { return rag ? s_T[hd / g.H] : T; };
+  auto nb_of = [&](int hd) { return rag ? (s_T[hd / g.H] + kBT - 1) / kBT : nb; };
+  auto start_of = [&](int hd) -> int64_t {
+    if (!rag) return (int64_t)hd * nb;
+    const int b = hd / g.H;
+    return s_pre[b] + (int64_t)(hd - b * g.H) * nb_of(hd);
+  };
+  auto head_at = [&](int64_t k, int* blk) -> int {
+    if (!rag) {
+      *blk = (int)(k % nb);
+      return (int)(k / nb);
+    }
+    int lo = 0, hi = g.B - 1;                        // last b with s_pre[b] <= k < s_pre[b + 1]
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_pre[mid] <= k) lo = mid; else hi = mid - 1;
+    }
+    while (s_pre[lo + 1] <= k) ++lo;                 // skip sequences holding no block
+    const int nbb = (s_T[lo] + kBT - 1) / kBT;
+    const int64_t r = k - s_pre[lo];
+    *blk = (int)(r % nbb);
+    return lo * g.H + (int)(r / nbb);
+  };
+  // first byte of head hd's token t in a plane (in a page of a paged cache)
+  auto run_ptr = [&](int plane, int hd, int t) -> const uint8_t* {
+    int pb = 0, hh = hd;
+    int64_t row = t;
+    if (paged) {
+      tok_loc(g, hd / g.H, t, &pb, &row);
+      hh = hd % g.H;
+    }
+    const Plane& pl = g.pl[plane];
+    return static_cast<const uint8_t*>(pl.p) + plane_index(pl, pb, hh, g.H, row, 0) * pl.elem;
+  };
   const int P = N < (int64_t)gridDim.x ? (int)N : (int)gridDim.x;
   if ((int)blockIdx.x >= P) return;
   const int64_t k0 = range_start(blockIdx.x, N, P), k1 = range_start(blockIdx.x + 1, N, P);
   const int nblk = (int)(k1 - k0);
-  const int tq = C::KIVI ? kivi_tq(T, g.R, 32) : T;  // coded tokens
+  const int tq = C::KIVI ? kivi_tq(T, g.R, 32) : T;  // coded tokens (uniform layout)
+  auto tq_of = [&](int hd) { return rag ? T_of(hd) : tq; };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < ns; ++i) {
@@ -147,7 +217,8 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   // ------------------------------------------------------------------ producer
   if (warp == kNW) {
     const int nst = (nblk + kSB - 1) / kSB;          // stages
-    int head = (int)(k0 / nb), blk = (int)(k0 % nb); // first block of the next stage
+    int blk;
+    int head = head_at(k0, &blk);                    // first block of the next stage
     int s = 0;
     for (; s < nst; ++s) {
       const int st = s % ns;
@@ -171,8 +242,10 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         int p_head = -1, p_end = -1;                 // end of the current run
 #pragma unroll
         for (int i = 0; i < kSB; ++i) {
-          if (i < nbs && bb * kBT < tq) {
-            if (!(hh == p_head && bb == p_end)) {    // a new run starts here
+          const int tqh = hh < BH ? tq_of(hh) : 0;
+          if (i < nbs && bb * kBT < tqh) {
+            // a new run starts here (a paged cache's runs stay in one page)
+            if (!(hh == p_head && bb == p_end) || (paged && bb % (kPageTok / kBT) == 0)) {
               if (cnt == myr) { r_head = hh; r_blk = bb; r_sub = i; }
               ++cnt;
             }
@@ -180,14 +253,18 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
             if (pass == 0) {
               // bytes of the block (the last coded block of a head may be
               // partial: whole 4-token groups are copied)
-              const int nt = (min(kBT, tq - bb * kBT) + 3) & ~3;
+              const int nt = (min(kBT, tqh - bb * kBT) + 3) & ~3;
               total += nt * (C::KCB + C::VCB) + (C::SYM ? 1 : 2) * nt * NG * 2;
               total += C::KIVI ? 2 * D * 2 : (C::SYM ? 1 : 2) * nt * NG * 2;
             }
             p_head = hh;
             p_end = bb + 1;
           }
-          if (i < nbs && ++bb == nb) { bb = 0; ++hh; }
+          if (i < nbs && ++bb == nb_of(hh)) {
+            bb = 0;
+            ++hh;
+            while (rag && hh < BH && nb_of(hh) == 0) ++hh;   // sequences holding nothing
+          }
         }
         if (pass == 0) {
           nrun = cnt;
@@ -198,29 +275,29 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         }
         if (lane < 30 && myr < nrun && (!C::SYM || myc < 4)) {
           const int t0 = r_blk * kBT;
-          const int n4 = (min(r_n * kBT, tq - t0) + 3) & ~3;
+          const int n4 = (min(r_n * kBT, tq_of(r_head) - t0) + 3) & ~3;
           const int tsub = r_sub * kBT;              // first token slot in the stage
           // plane rows of head h: plane_ptr(g, plane, 0, h, row) addresses (b, hkv) = h
           const uint8_t* src;
           unsigned char* dst;
           uint32_t bytes;
           if (myc == 0) {
-            src = plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, 0, r_head, t0);
+            src = run_ptr(KVQ_PLANE_K_CODES, r_head, t0);
             dst = sp + C::KC + tsub * C::KCB;
             bytes = n4 * C::KCB;
           } else if (myc == 1) {
-            src = plane_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, 0, r_head, t0);
+            src = run_ptr(KVQ_PLANE_V_CODES, r_head, t0);
             dst = sp + C::VC + tsub * C::VCB;
             bytes = n4 * C::VCB;
           } else if (myc == 2 || myc == 4) {
             const int pl = myc == 2 ? KVQ_PLANE_K_SCALE : KVQ_PLANE_K_ZERO;
-            src = reinterpret_cast<const uint8_t*>(
-                plane_ptr<__half>(g, pl, 0, r_head, C::KIVI ? r_blk : t0));
+            src = C::KIVI ? reinterpret_cast<const uint8_t*>(plane_ptr<__half>(g, pl, 0, r_head, r_blk))
+                          : run_ptr(pl, r_head, t0);
             dst = sp + (myc == 2 ? C::KS : C::KZ) + r_sub * C::KMETA;
             bytes = C::KIVI ? r_n * D * 2 : n4 * NG * 2;
           } else {
             const int pl = myc == 3 ? KVQ_PLANE_V_SCALE : KVQ_PLANE_V_ZERO;
-            src = reinterpret_cast<const uint8_t*>(plane_ptr<__half>(g, pl, 0, r_head, t0));
+            src = run_ptr(pl, r_head, t0);
             dst = sp + (myc == 3 ? C::VS : C::VZ) + r_sub * C::VMETA;
             bytes = n4 * NG * 2;
           }
@@ -654,10 +731,14 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   // The CTA's range crosses heads hfirst..hlast.  Every consumer warp runs
   // every segment (warps without blocks in it only join the merge), so the
   // named barriers below are reached by all of them.
-  const int hfirst = (int)(k0 / nb), hlast = (int)((k1 - 1) / nb);
+  int bdummy;
+  const int hfirst = head_at(k0, &bdummy), hlast = head_at(k1 - 1, &bdummy);
   for (int hd = hfirst; hd <= hlast; ++hd) {
-    const int64_t hs = (int64_t)hd * nb;
-    const int a = (int)(max(k0, hs) - k0), e = (int)(min(k1, hs + nb) - k0);
+    const int nbh = nb_of(hd);
+    if (nbh == 0) continue;                          // a sequence holding no token
+    const int64_t hs = start_of(hd);
+    const int a = (int)(max(k0, hs) - k0), e = (int)(min(k1, hs + nbh) - k0);
+    const int Th = T_of(hd), tqh = tq_of(hd);
     b = hd / g.H;
     hkv = hd % g.H;
     const int jst = a + ((warp - a) % kNW + kNW) % kNW;   // first block of this warp
@@ -673,11 +754,11 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         break;
       }
       const int t0 = (int)(k0 + j - hs) * kBT;
-      const int nv = min(kBT, T - t0);
+      const int nv = min(kBT, Th - t0);
       if (nv == kBT)
-        process(std::true_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tq);
+        process(std::true_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tqh);
       else
-        process(std::false_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tq);
+        process(std::false_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tqh);
       __syncwarp();
       if (lane == 0) mbar_arrive1(&empty[st]);
     }
@@ -729,7 +810,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
       mg->L[tc] = L;
     }
     consumer_sync();
-    const int c0 = cta_of(hs, N, P), c1 = cta_of(hs + nb - 1, N, P);
+    const int c0 = cta_of(hs, N, P), c1 = cta_of(hs + nbh - 1, N, P);
     const int nct = c1 - c0 + 1;
     if (nct > kMaxSplits) {                          // the host sizes the grid so this cannot happen
       if (tc == 0) atomicOr(err, 4);
@@ -795,9 +876,12 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
 }
 
 template <int D, int KB, int VB, int FMT>
-size_t stream_smem(int grp, int* ns) {
+size_t stream_smem(int grp, int B, bool rag, int* ns) {
   using C = SCfg<D, KB, VB, FMT>;
-  const size_t fixed = (size_t)kNW * grp * (D + 2) * 4 + sizeof(Merge);
+  // per-warp partial slots, merge scratch; ragged: each sequence's count and
+  // first block (rounded up so the mbarriers stay 8-byte aligned)
+  const size_t fixed = (size_t)kNW * grp * (D + 2) * 4 + sizeof(Merge) +
+                       (rag ? (size_t)((B + 2) & ~1) * 4 + (size_t)(B + 1) * 8 : 0);
   int n = (int)((kSmemMax - fixed) / (C::STAGE + 16));
   if (n > kMaxStages) n = kMaxStages;
   *ns = n;
@@ -809,7 +893,7 @@ cudaError_t launch_t(const Geom& g, const void* q, float scale, int* err, void* 
                      cudaStream_t s) {
   const int grp = g.Hq / g.H;
   int ns = 0;
-  const size_t sm = stream_smem<D, KB, VB, FMT>(grp, &ns);
+  const size_t sm = stream_smem<D, KB, VB, FMT>(grp, g.B, g.layout != KVQ_LAYOUT_UNIFORM, &ns);
   auto kern = decode_stream_kernel<D, KB, VB, FMT>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
@@ -838,13 +922,17 @@ int decode_stream_ctas(const Geom& g) {
   const int bh = g.B * g.H;
   int p = num_sms();
   if (p > 15 * bh) p = 15 * bh;
+  // ragged: the longest sequence's heads must not span more CTAs either
+  if (g.layout != KVQ_LAYOUT_UNIFORM && g.ragged_cta_cap > 0 && p > g.ragged_cta_cap)
+    p = g.ragged_cta_cap;
   return p < 1 ? 1 : p;
 }
 
 bool decode_stream_supported(const Geom& g) {
   const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC || g.fmt == KVQ_FMT_KIVI;
-  return fmt_ok && g.layout == KVQ_LAYOUT_UNIFORM && g.act == KVQ_BF16 && g.G == 32 &&
-         g.kb == g.vb && (g.kb == 2 || g.kb == 4) && (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
+  return fmt_ok && (g.layout == KVQ_LAYOUT_UNIFORM || g.fmt != KVQ_FMT_KIVI) &&
+         g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb && (g.kb == 2 || g.kb == 4) &&
+         (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
 }
 
 cudaError_t launch_decode_stream(const Geom& g, const void* q, float scale, int* err, void* out,

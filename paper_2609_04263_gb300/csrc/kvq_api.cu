@@ -548,6 +548,16 @@ static kvq_status attend_common(kvq_cache* cache, const void* q, int L, int n_q_
         return fail(KVQ_ERR_SHAPE, "sequence %d appended %d tokens, more than L = %d query rows",
                     b, cache->seq_n[b], L);
   if (!(scale > 0.f) || scale != scale) return fail(KVQ_ERR_ARG, "softmax_scale must be > 0");
+  if (cache->g.layout != KVQ_LAYOUT_UNIFORM) {
+    // a streaming decode over N blocks in P equal ranges gives a head of m
+    // blocks at most ceil(m P / N) + 1 CTAs: P <= 30 N / m keeps that <= 31
+    int64_t n = 0, m = 0;
+    for (int t : cache->seq_T) {
+      n += (int64_t)cache->g.H * ((t + 31) / 32);
+      m = std::max<int64_t>(m, (t + 31) / 32);
+    }
+    cache->g.ragged_cta_cap = m > 0 ? (int)std::max<int64_t>(1, std::min<int64_t>(1 << 20, 30 * n / m)) : 0;
+  }
   cudaError_t e = ensure_init(cache, (cudaStream_t)stream);
   if (e == cudaSuccess) e = launch_attend(cache->g, q, L, scale, out, decode, cache->T,
                                             (cudaStream_t)stream);

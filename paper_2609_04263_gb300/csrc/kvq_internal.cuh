@@ -51,14 +51,22 @@ struct Geom {
   Plane pl[KVQ_NUM_PLANES];
   // token layout (kvq_layout).  RAGGED / PAGED: seq_len[b] tokens of sequence
   // b, seq_new[b] of them appended by the last append; PAGED: token t of
-  // sequence b in pool page page_table[b max_pages + t / 64], and the planes
-  // hold the pool ([1][H][num_pages 64][cols]) instead of [B][H][Tmax][cols]
+  // sequence b in pool page page_table[b max_pages + t / kPageTok], and the
+  // planes hold the pool ([1][H][num_pages kPageTok][cols]) instead of
+  // [B][H][Tmax][cols]
   int32_t layout, max_pages;
+  // RAGGED / PAGED, host side: most streaming-decode CTAs for which no head
+  // spans more than kMaxSplits of them at the current lengths (set before
+  // each decode launch; 0 = no bound)
+  int32_t ragged_cta_cap;
   int32_t* seq_len;
   int32_t* seq_new;
   int32_t* page_table;
 };
 constexpr int kPageTok = KVQ_PAGE_TOKENS;
+constexpr int kPageShift = 8;
+static_assert(kPageTok == 1 << kPageShift && kPageTok % 64 == 0,
+              "pages hold whole 64-token tiles and decode chunks");
 
 __host__ __device__ inline int64_t plane_index(const Plane& pl, int b, int h, int H,
                                                int64_t row, int64_t col) {
@@ -268,12 +276,13 @@ __device__ __forceinline__ int seq_tokens(const Geom& g, int b) {
                                         : *reinterpret_cast<volatile int32_t*>(&g.seq_len[b]);
 }
 // Where token t of sequence b sits in a per-token plane: its batch index and
-// row (PAGED: the pool page's row).  Runs of tokens inside one 64-token page
+// row (PAGED: the pool page's row).  Runs of tokens inside one page
 // are contiguous rows in every layout.
 __device__ __forceinline__ void tok_loc(const Geom& g, int b, int t, int* pb, int64_t* row) {
   if (g.layout == KVQ_LAYOUT_PAGED) {
     *pb = 0;
-    *row = (int64_t)g.page_table[b * g.max_pages + (t >> 6)] * kPageTok + (t & (kPageTok - 1));
+    *row = (int64_t)g.page_table[b * g.max_pages + (t >> kPageShift)] * kPageTok +
+           (t & (kPageTok - 1));
   } else {
     *pb = b;
     *row = t;

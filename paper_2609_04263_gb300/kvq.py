@@ -17,7 +17,7 @@ KVQ_OK, KVQ_ERR_ARG, KVQ_ERR_SHAPE, KVQ_ERR_CAPACITY, KVQ_ERR_UNSUPPORTED, \
 KVQ_FMT_FLOAT, KVQ_FMT_AFFINE, KVQ_FMT_SYMMETRIC, KVQ_FMT_KIVI, KVQ_FMT_KVARN = range(5)
 KVQ_F32, KVQ_BF16 = 0, 1
 KVQ_LAYOUT_UNIFORM, KVQ_LAYOUT_RAGGED, KVQ_LAYOUT_PAGED = range(3)
-KVQ_PAGE_TOKENS = 64
+KVQ_PAGE_TOKENS = 256
 KVQ_MAX_SEQS = 512
 
 PLANES = ["k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "k_full",

@@ -242,25 +242,25 @@ def test_ragged_and_paged_layout_rules(kvq):
     d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_PAGED, num_pages=0)
     with pytest.raises(kvq.KvqError):                       # a pool needs pages
         kvq.kvq_cache_bytes(d)
-    d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_PAGED, num_pages=10)
+    d = _desc(kvq, **base, layout=kvq.KVQ_LAYOUT_PAGED, num_pages=5)
     n = kvq.kvq_cache_bytes(d)
     h = kvq.kvq_create_cache(d, fake, n)
     try:
-        assert kvq.kvq_free_pages(h) == 10
+        assert kvq.kvq_free_pages(h) == 5
         assert kvq.kvq_seq_pages(h, 0) == []
         assert kvq.kvq_seq_tokens(h, 2) == 0 and kvq.kvq_seq_tokens(h, 3) == -1
         v = kvq.kvq_cache_view(h)
-        assert v.dims[0][0] == 1 and v.dims[0][2] == 10 * 64       # codes: the pool
+        assert v.dims[0][0] == 1 and v.dims[0][2] == 5 * kvq.KVQ_PAGE_TOKENS    # the pool
         with pytest.raises(kvq.KvqError) as ei:                    # beyond max_tokens
             kvq.kvq_append_pack_ragged(h, P, P, 600, [600, 0, 0], 0)
         assert ei.value.status == kvq.KVQ_ERR_CAPACITY
         with pytest.raises(kvq.KvqError) as ei:                    # more pages than the pool
-            kvq.kvq_append_pack_ragged(h, P, P, 400, [400, 400, 0], 0)
+            kvq.kvq_append_pack_ragged(h, P, P, 500, [500, 500, 500], 0)
         assert ei.value.status == kvq.KVQ_ERR_CAPACITY
         with pytest.raises(kvq.KvqError) as ei:                    # a count above L
             kvq.kvq_append_pack_ragged(h, P, P, 4, [5, 0, 0], 0)
         assert ei.value.status == kvq.KVQ_ERR_ARG
-        assert kvq.kvq_free_pages(h) == 10                          # nothing was taken
+        assert kvq.kvq_free_pages(h) == 5                           # nothing was taken
     finally:
         kvq.kvq_destroy_cache(h)
     # a ragged cache of the same shape holds B x max_tokens rows and no pool

@@ -39,15 +39,18 @@ def _cache(spec, B, H, Hq, D, Tmax, layout, num_pages=0):
     return api.Cache(desc)
 
 
+PG = kvq.KVQ_PAGE_TOKENS
+
+
 def _seq_rows(gc, name, b, T):
     """Plane rows [H, T, cols] of sequence b's tokens (PAGED: through its pages)."""
     p = gc.planes()[name]
     if gc.desc.layout == kvq.KVQ_LAYOUT_PAGED:
         pages = gc.seq_pages(b)
-        assert len(pages) == (T + 63) // 64
+        assert len(pages) == (T + PG - 1) // PG
         if not pages:
             return p[0, :, :0]
-        rows = torch.cat([p[0, :, 64 * pg:64 * pg + 64] for pg in pages], dim=1)
+        rows = torch.cat([p[0, :, PG * pg:PG * pg + PG] for pg in pages], dim=1)
         return rows[:, :T]
     return p[b, :, :T]
 
@@ -126,7 +129,7 @@ class Batch:
 @pytest.mark.parametrize("layout", [kvq.KVQ_LAYOUT_RAGGED, kvq.KVQ_LAYOUT_PAGED])
 @pytest.mark.parametrize("fmt,B,H,Hq,D", [("affine4", 3, 2, 8, 64), ("sym2", 4, 2, 8, 128)])
 def test_ragged_batch_lifecycle(layout, fmt, B, H, Hq, D):
-    pages = 3 * B * 8 if layout == kvq.KVQ_LAYOUT_PAGED else 0
+    pages = 3 * B * 2 if layout == kvq.KVQ_LAYOUT_PAGED else 0
     bt = Batch(fmt, B, H, Hq, D, 512, layout, pages, seed=D + B)
     counts = [[100, 37, 0, 64][:B], [5, 64, 130, 1][:B], [0, 3, 200, 63][:B]]
     for n in counts:                          # ragged prefill chunks
@@ -140,7 +143,7 @@ def test_ragged_batch_lifecycle(layout, fmt, B, H, Hq, D):
     # sequence 1 finishes; its slot starts a new sequence while the others run on
     bt.release(1)
     if layout == kvq.KVQ_LAYOUT_PAGED:
-        held = sum((bt.oc[b].T + 63) // 64 for b in range(B))
+        held = sum((bt.oc[b].T + PG - 1) // PG for b in range(B))
         assert bt.gc.free_pages() == pages - held
     bt.check_decode()                         # the released sequence is empty
     n = [1] * B
@@ -155,17 +158,17 @@ def test_ragged_batch_lifecycle(layout, fmt, B, H, Hq, D):
 def test_paged_pool_exhaustion_and_reuse():
     """Appends that need more pages than the pool holds are refused whole;
     released pages serve the next sequence."""
-    bt = Batch("affine4", 2, 2, 4, 64, 1024, kvq.KVQ_LAYOUT_PAGED, num_pages=6, seed=3)
-    bt.append([130, 60])                      # 3 + 1 pages
-    assert bt.gc.free_pages() == 2
-    k = torch.zeros(2, 2, 200, 64, dtype=torch.bfloat16, device="cuda")
+    bt = Batch("affine4", 2, 2, 4, 64, 1024, kvq.KVQ_LAYOUT_PAGED, num_pages=4, seed=3)
+    bt.append([300, 60])                      # 2 + 1 pages of 256 tokens
+    assert bt.gc.free_pages() == 1
+    k = torch.zeros(2, 2, 600, 64, dtype=torch.bfloat16, device="cuda")
     with pytest.raises(kvq.KvqError) as ei:
-        bt.gc.append_ragged(k, k, [200, 0])   # would need 4 more pages
+        bt.gc.append_ragged(k, k, [600, 0])   # would need 2 more pages
     assert ei.value.status == kvq.KVQ_ERR_CAPACITY
-    assert bt.gc.free_pages() == 2 and bt.gc.seq_tokens(0) == 130
+    assert bt.gc.free_pages() == 1 and bt.gc.seq_tokens(0) == 300
     bt.release(0)
-    assert bt.gc.free_pages() == 5
-    L = bt.append([200, 10])                  # the released pages come back: 4 + 1
+    assert bt.gc.free_pages() == 3
+    L = bt.append([700, 10])                  # the released pages come back: 3 + 0
     bt.check_prefill(L)
     bt.check_planes()
     assert bt.gc.free_pages() == 0
@@ -201,3 +204,33 @@ def test_ragged_decode_step_positions():
         ref_o = O.attend(bt.oc[b], q[b:b + 1].float().cpu().numpy())
         check_attention(out[b:b + 1].float().cpu().numpy(), ref_o, "bf16", f"decode of sequence {b}")
     bt.check_planes()
+
+
+@pytest.mark.parametrize("layout", [kvq.KVQ_LAYOUT_RAGGED, kvq.KVQ_LAYOUT_PAGED])
+def test_streaming_decode_over_ragged_sequences(layout):
+    """Long ragged caches take the persistent streaming decode kernel (whose
+    work split follows each sequence's own block count, and whose copies stay
+    inside one page): sequences of very different lengths, one of them empty
+    and one holding a single token."""
+    B, H, Hq, D = 8, 4, 32, 64
+    lens = [4000, 10, 0, 3000, 4096, 1, 2500, 64]
+    pages = sum((t + PG - 1) // PG for t in lens) + 4
+    bt = Batch("sym2", B, H, Hq, D, 4160, layout, pages if layout == kvq.KVQ_LAYOUT_PAGED else 0,
+               seed=21)
+    for lo in range(0, max(lens), 1024):
+        bt.append([max(0, min(1024, t - lo)) for t in lens])
+    bt.check_decode()
+    bt.append([1, 1, 0, 1, 1, 1, 1, 1])       # one more token for all but the empty one
+    bt.check_decode()
+    bt.check_planes()
+
+
+def test_streaming_decode_one_long_sequence():
+    """One long sequence among single-token ones: the streaming decode takes
+    fewer CTAs so that the long sequence's head is not split across more of
+    them than its merge holds."""
+    bt = Batch("affine4", 4, 1, 4, 64, 8192, kvq.KVQ_LAYOUT_PAGED, num_pages=40, seed=31)
+    lens = [8000, 1, 1, 0]
+    for lo in range(0, 8000, 2048):
+        bt.append([max(0, min(2048, t - lo)) for t in lens])
+    bt.check_decode()
