@@ -527,18 +527,20 @@ def paged_decode_rates(run, peaks, flush):
     sequence at its own length: continuous batching) with the workload's head
     shape, batch and bit width, lengths spread evenly over [P/2, P] for a
     P-token prefill.  The workload's own format when a paged cache supports it
-    (affine, symmetric), otherwise an affine cache of the same bit width (KIVI
-    and KVarN caches are uniform only).  Against HBM: the coded tokens' bytes
-    of every sequence plus q and out."""
+    (affine, symmetric, KIVI), otherwise an affine cache of the same bit width
+    (KVarN caches are uniform only).  Against HBM: every sequence's coded and
+    full-precision tokens' bytes plus q and out."""
     from paper_2609_04263_gb300 import kvq
     wl, api = run.wl, run.api
     if wl.dtype != "bf16" or wl.head_dim not in (64, 128) or wl.key_bits not in (2, 4):
         return None
-    fmt = wl.fmt if wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC) else synth.FMT_AFFINE
+    own = wl.fmt in (synth.FMT_AFFINE, synth.FMT_SYMMETRIC, synth.FMT_KIVI)
+    fmt = wl.fmt if own else synth.FMT_AFFINE
     B, H, Hq, D, P = wl.batch, wl.n_kv_heads, wl.n_q_heads, wl.head_dim, wl.prefill
     lens = [P // 2 + (P - P // 2) * b // max(B - 1, 1) for b in range(B)]
     pages = sum((t + 256) // 256 for t in lens)
     desc = api.make_desc(fmt, wl.key_bits, wl.key_bits, 32, B, H, Hq, D, P + 64, torch.bfloat16,
+                         residual_tokens=wl.residual_tokens if own else 0,
                          layout=kvq.KVQ_LAYOUT_PAGED, num_pages=pages)
     cache = api.Cache(desc, device=run.dev)
     g = torch.Generator(device="cpu").manual_seed(3)
@@ -553,9 +555,13 @@ def paged_decode_rates(run, peaks, flush):
     q = torch.randn(B, Hq, 1, D, generator=g).to(torch.bfloat16).to(run.dev)
     out = torch.empty_like(q)
     ms = cold_graph_time_ms(lambda: cache.attend_decode(q, out=out), 10, flush)
-    per_tok = D * wl.key_bits // 8 * 2 + 2 * (D // 32) * (2 if fmt == synth.FMT_SYMMETRIC else 4)
-    nbytes = H * per_tok * sum(lens) + 2 * B * Hq * D * 2
-    return {"format": {synth.FMT_AFFINE: "affine", synth.FMT_SYMMETRIC: "symmetric"}[fmt],
+    if own:                                    # the workload's format: its own byte count
+        nbytes = H * sum(cache_read_bytes(wl, t) for t in lens) + 2 * B * Hq * D * 2
+    else:
+        per_tok = D * wl.key_bits // 8 * 2 + 2 * (D // 32) * 4
+        nbytes = H * per_tok * sum(lens) + 2 * B * Hq * D * 2
+    return {"format": {synth.FMT_AFFINE: "affine", synth.FMT_SYMMETRIC: "symmetric",
+                       synth.FMT_KIVI: "kivi"}[fmt],
             "bits": wl.key_bits, "sequences": B, "tokens_min": min(lens), "tokens_max": max(lens),
             "pages": pages, "mean_ms": round(ms, 5), "algorithmic_bytes": nbytes,
             "achieved": round(nbytes / ms / 1e6, 3), "unit": "GB/s",

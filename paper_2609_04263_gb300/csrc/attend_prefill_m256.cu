@@ -199,13 +199,13 @@ __device__ __forceinline__ void load_raw(const Geom& g, int b, int h, int t0, un
   // a tile is one 64-token page of a paged cache: tok_ptr finds its rows
   bulk_copy(raw + S::RKC, tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0), CB, bar);
   bulk_copy(raw + S::RVC, tok_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, h, t0), CB, bar);
-  // KIVI: two key blocks of D channels (uniform layout only)
-  const __half* ks = FMT == KVQ_FMT_KIVI ? plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t0 / 32)
+  // KIVI: two key blocks of D channels
+  const __half* ks = FMT == KVQ_FMT_KIVI ? blk_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t0 / 32)
                                          : tok_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, t0);
   bulk_copy(raw + S::RKS, ks, 4 * D, bar);
   if (FMT != KVQ_FMT_SYMMETRIC) {
     const __half* kz = FMT == KVQ_FMT_KIVI
-                           ? plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t0 / 32)
+                           ? blk_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t0 / 32)
                            : tok_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, t0);
     bulk_copy(raw + S::RKZ, kz, 4 * D, bar);
   }

@@ -207,9 +207,9 @@ __device__ void split_issue(const Geom& g, int b, int hkv, const SplitPlan& sp, 
   bulk_g2s(st + C::VC_OFF, tok_ptr<uint8_t>(g, KVQ_PLANE_V_CODES, b, hkv, c0), code_bytes,
            &bars[stage]);
   if (FMT == KVQ_FMT_KIVI) {
-    bulk_g2s(st + C::KS_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
+    bulk_g2s(st + C::KS_OFF, blk_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0 / 32), kmeta,
              &bars[stage]);
-    bulk_g2s(st + C::KZ_OFF, plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
+    bulk_g2s(st + C::KZ_OFF, blk_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, hkv, c0 / 32), kmeta,
              &bars[stage]);
   } else {
     bulk_g2s(st + C::KS_OFF, tok_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, hkv, c0), kmeta,

@@ -101,7 +101,7 @@ __host__ __device__ constexpr uint32_t pow2_h2(int e) {
   return ((uint32_t)(15 + e) << 10) | ((uint32_t)(15 + e) << 26);
 }
 
-template <int D, int KB, int VB, int FMT>
+template <int D, int KB, int VB, int FMT, bool RAG>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, int* err,
                      __nv_bfloat16* __restrict__ out, int ns) {
@@ -123,9 +123,10 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   int* s_T = reinterpret_cast<int*>(empty + ns);     // [B]
   int64_t* s_pre = reinterpret_cast<int64_t*>(s_T + ((g.B + 1) & ~1));   // [B + 1]
 
-  // (KIVI caches are uniform only)
-  const bool rag = !C::KIVI && g.layout != KVQ_LAYOUT_UNIFORM;
-  const bool paged = !C::KIVI && g.layout == KVQ_LAYOUT_PAGED;
+  // RAG: a ragged or paged cache (a separate instantiation, so the uniform
+  // kernel carries none of the per-sequence bookkeeping)
+  constexpr bool rag = RAG;
+  const bool paged = RAG && g.layout == KVQ_LAYOUT_PAGED;
   const int T = rag ? 0 : cache_tokens(g);
   const int BH = g.B * g.H;
   const int nb = (T + kBT - 1) / kBT;                // blocks per head (uniform layout)
@@ -198,12 +199,25 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
     const Plane& pl = g.pl[plane];
     return static_cast<const uint8_t*>(pl.p) + plane_index(pl, pb, hh, g.H, row, 0) * pl.elem;
   };
+  // first byte of head hd's 32-token block k in a per-block plane (KIVI keys)
+  auto blk_run_ptr = [&](int plane, int hd, int k) -> const uint8_t* {
+    int pb = 0, hh = hd;
+    int64_t row = k;
+    if (paged) {
+      blk_loc(g, hd / g.H, k, &pb, &row);
+      hh = hd % g.H;
+    }
+    const Plane& pl = g.pl[plane];
+    return static_cast<const uint8_t*>(pl.p) + plane_index(pl, pb, hh, g.H, row, 0) * pl.elem;
+  };
   const int P = N < (int64_t)gridDim.x ? (int)N : (int)gridDim.x;
   if ((int)blockIdx.x >= P) return;
   const int64_t k0 = range_start(blockIdx.x, N, P), k1 = range_start(blockIdx.x + 1, N, P);
   const int nblk = (int)(k1 - k0);
   const int tq = C::KIVI ? kivi_tq(T, g.R, 32) : T;  // coded tokens (uniform layout)
-  auto tq_of = [&](int hd) { return rag ? T_of(hd) : tq; };
+  auto tq_of = [&](int hd) {
+    return !rag ? tq : C::KIVI ? kivi_tq(T_of(hd), g.R, 32) : T_of(hd);
+  };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < ns; ++i) {
@@ -291,8 +305,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
             bytes = n4 * C::VCB;
           } else if (myc == 2 || myc == 4) {
             const int pl = myc == 2 ? KVQ_PLANE_K_SCALE : KVQ_PLANE_K_ZERO;
-            src = C::KIVI ? reinterpret_cast<const uint8_t*>(plane_ptr<__half>(g, pl, 0, r_head, r_blk))
-                          : run_ptr(pl, r_head, t0);
+            src = C::KIVI ? blk_run_ptr(pl, r_head, r_blk) : run_ptr(pl, r_head, t0);
             dst = sp + (myc == 2 ? C::KS : C::KZ) + r_sub * C::KMETA;
             bytes = C::KIVI ? r_n * D * 2 : n4 * NG * 2;
           } else {
@@ -894,7 +907,8 @@ cudaError_t launch_t(const Geom& g, const void* q, float scale, int* err, void* 
   const int grp = g.Hq / g.H;
   int ns = 0;
   const size_t sm = stream_smem<D, KB, VB, FMT>(grp, g.B, g.layout != KVQ_LAYOUT_UNIFORM, &ns);
-  auto kern = decode_stream_kernel<D, KB, VB, FMT>;
+  auto kern = g.layout == KVQ_LAYOUT_UNIFORM ? decode_stream_kernel<D, KB, VB, FMT, false>
+                                             : decode_stream_kernel<D, KB, VB, FMT, true>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   launch_pdl(kern, dim3(decode_stream_ctas(g)), dim3(kThreads), sm, s, g,

@@ -100,13 +100,14 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     fail(KVQ_ERR_ARG, "unknown layout %d", d->layout); *st = KVQ_ERR_ARG; return 0;
   }
   if (d->layout != KVQ_LAYOUT_UNIFORM) {
-    const bool ok = (d->fmt == KVQ_FMT_AFFINE || d->fmt == KVQ_FMT_SYMMETRIC) &&
+    const bool ok = (d->fmt == KVQ_FMT_AFFINE || d->fmt == KVQ_FMT_SYMMETRIC ||
+                     d->fmt == KVQ_FMT_KIVI) &&
                     d->dtype == KVQ_BF16 && G == 32 && d->key_bits == d->value_bits &&
                     (d->key_bits == 2 || d->key_bits == 4) && (D == 64 || D == 128) &&
                     d->q_heads / d->kv_heads <= 16;
     if (!ok) {
-      fail(KVQ_ERR_UNSUPPORTED, "ragged and paged layouts need a bf16 affine or symmetric cache "
-           "with group_size 32, key_bits == value_bits in {2, 4} and head_dim 64 or 128");
+      fail(KVQ_ERR_UNSUPPORTED, "ragged and paged layouts need a bf16 affine, symmetric or KIVI "
+           "cache with group_size 32, key_bits == value_bits in {2, 4} and head_dim 64 or 128");
       *st = KVQ_ERR_UNSUPPORTED; return 0;
     }
     if (d->batch > KVQ_MAX_SEQS) {
@@ -123,7 +124,6 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
   // whole chunks), so their rows are padded to a multiple of 64; a paged
   // cache's planes hold the page pool of all sequences (batch index 0)
   const int Tp = paged ? d->num_pages * kPageTok : (Tm + 63) / 64 * 64;
-  const int pb = paged ? 1 : B;               // batch extent of the cache planes
   const int act = d->dtype == KVQ_BF16 ? 2 : 4;
   memset(g, 0, sizeof *g);
   g->fmt = d->fmt; g->kb = d->key_bits; g->vb = d->value_bits; g->G = G;
@@ -196,7 +196,7 @@ size_t layout(const kvq_cache_desc* d, Geom* g, size_t off[KVQ_NUM_PLANES],
     Plane& p = g->pl[i];
     if (p.rows == 0) continue;
     off[i] = total;
-    total = align256(total + (size_t)pb * H * p.rows * p.cols * p.elem);
+    total = align256(total + (size_t)plane_batch(*g, i) * H * p.rows * p.cols * p.elem);
   }
   // decode workspace: [B][Hq][kMaxSplits][D + 2] fp32, indexed by q head
   off[KVQ_PLANE_WORKSPACE] = total;
@@ -387,7 +387,7 @@ kvq_status kvq_cache_view(const kvq_cache* cache, kvq_cache_planes* out) {
   const Geom& g = cache->g;
   for (int i = 0; i < KVQ_NUM_PLANES; ++i) {
     out->ptr[i] = g.pl[i].p;
-    out->dims[i][0] = g.pl[i].rows ? (g.layout == KVQ_LAYOUT_PAGED && i != KVQ_PLANE_WORKSPACE ? 1 : g.B) : 0;
+    out->dims[i][0] = g.pl[i].rows ? plane_batch(g, i) : 0;
     out->dims[i][1] = g.pl[i].rows ? (i == KVQ_PLANE_WORKSPACE ? g.Hq : g.H) : 0;
     out->dims[i][2] = g.pl[i].rows;
     out->dims[i][3] = g.pl[i].cols;

@@ -261,6 +261,27 @@ __device__ __forceinline__ void append_arrive(CacheState* st, int T0, int L, boo
   }
 }
 
+// Batch extent of plane `which`: a paged cache's per-token and per-block
+// planes hold the page pool (1); KIVI's full-precision ring stays per sequence.
+__host__ __device__ inline int plane_batch(const Geom& g, int which) {
+  const bool per_seq = which == KVQ_PLANE_K_FULL || which == KVQ_PLANE_V_FULL ||
+                       which == KVQ_PLANE_WORKSPACE;
+  return g.layout == KVQ_LAYOUT_PAGED && !per_seq ? 1 : g.B;
+}
+// Token count before this append, and tokens appended, for sequence b of an
+// append of L tokens: the uniform count T0u and L, or a ragged cache's
+// seq_len[b] and seq_new[b] (set for this append before its kernels run).
+__device__ __forceinline__ void append_span(const Geom& g, int b, int L, int T0u, int* T0,
+                                            int* n) {
+  if (g.layout == KVQ_LAYOUT_UNIFORM) {
+    *T0 = T0u;
+    *n = L;
+  } else {
+    *T0 = g.seq_len[b];
+    *n = g.seq_new[b];
+  }
+}
+
 // Tokens stored, as read by attention kernels.
 __device__ __forceinline__ int cache_tokens(const Geom& g) {
   return *reinterpret_cast<volatile int32_t*>(&g.state->tokens);
@@ -294,6 +315,26 @@ __device__ __forceinline__ T* tok_ptr(const Geom& g, int which, int b, int h, in
   int pb;
   int64_t row;
   tok_loc(g, b, t, &pb, &row);
+  return plane_ptr<T>(g, which, pb, h, row, col);
+}
+// Row of 32-token block k of sequence b in a per-block plane (KIVI's key
+// scales and zero points; a page holds kPageTok / 32 block rows).
+__device__ __forceinline__ void blk_loc(const Geom& g, int b, int k, int* pb, int64_t* row) {
+  constexpr int per = kPageTok / 32;
+  if (g.layout == KVQ_LAYOUT_PAGED) {
+    *pb = 0;
+    *row = (int64_t)g.page_table[b * g.max_pages + k / per] * per + k % per;
+  } else {
+    *pb = b;
+    *row = k;
+  }
+}
+template <typename T>
+__device__ __forceinline__ T* blk_ptr(const Geom& g, int which, int b, int h, int k,
+                                      int64_t col = 0) {
+  int pb;
+  int64_t row;
+  blk_loc(g, b, k, &pb, &row);
   return plane_ptr<T>(g, which, pb, h, row, col);
 }
 

@@ -119,53 +119,74 @@ __device__ __forceinline__ void pack_rows(const Geom& g, const TokSrc& src, int 
   }
 }
 
+// A ragged cache (layouts RAGGED and PAGED) appends per sequence: sequence b
+// codes its first seq_new[b] of the L new tokens at its own positions
+// seq_len[b] ..; the host has checked capacity and assigned the pages, and
+// the counts advance after the append's kernels.
 __global__ void pack_pertoken_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int kivi,
                                      int final_kernel, int lcpt, int llpg) {
   pdl_wait();
   pdl_trigger();
-  bool ok;
-  const int T0 = append_begin(g, L, &ok);
+  bool ok = true;
+  const bool rag = g.layout != KVQ_LAYOUT_UNIFORM;
+  const int T0u = rag ? 0 : append_begin(g, L, &ok);
   const int which = kivi ? 1 : blockIdx.z;
-  int t_begin = T0, t_end = T0 + L;
+  const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
+  int T0, n;
+  append_span(g, b, L, T0u, &T0, &n);
+  int t_begin = T0, t_end = T0 + n;
   if (kivi) {
     t_begin = kivi_tq(T0, g.R, g.G);
-    t_end = kivi_tq(T0 + L, g.R, g.G);
+    t_end = kivi_tq(T0 + n, g.R, g.G);
   }
   if (ok && t_end > t_begin) {
     TokSrc src = which ? sv : sk;
     src.T0 = T0;
-    const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
     pack_rows(g, src, b, h, t_begin, t_end - t_begin, which, sym, lcpt, llpg);
   }
-  if (final_kernel) append_arrive_spread(g.state, T0, L, ok);
+  if (final_kernel && !rag) append_arrive_spread(g.state, T0u, L, ok);
 }
 
-// Ragged append (layouts RAGGED and PAGED, affine or symmetric): sequence b
-// codes the first n.n[b] of its L new tokens at its own positions
-// seq_len[b] ..; the host has checked capacity and assigned the pages.
+// Ragged appends: this append's counts (first), and the sequences' counts
+// advanced by them (last).
 struct SeqCounts {
   int32_t n[KVQ_MAX_SEQS];
 };
 
-__global__ void pack_ragged_kernel(Geom g, int L, TokSrc sk, TokSrc sv, int sym, int lcpt,
-                                   int llpg, SeqCounts n) {
+__global__ void seq_counts_kernel(Geom g, SeqCounts n) {
   pdl_wait();
   pdl_trigger();
-  const int b = blockIdx.y / g.H, h = blockIdx.y - b * g.H;
-  const int nb = n.n[b];
-  if (nb <= 0) return;
-  TokSrc src = blockIdx.z ? sv : sk;
-  src.T0 = seq_tokens(g, b);
-  pack_rows(g, src, b, h, src.T0, nb, blockIdx.z, sym, lcpt, llpg);
+  for (int b = threadIdx.x; b < g.B; b += blockDim.x) g.seq_new[b] = n.n[b];
 }
 
-// After a ragged append: the sequences' counts.
-__global__ void seq_advance_kernel(Geom g, SeqCounts n) {
+__global__ void seq_advance_kernel(Geom g) {
   pdl_wait();
   pdl_trigger();
-  for (int b = threadIdx.x; b < g.B; b += blockDim.x) {
-    g.seq_len[b] += n.n[b];
-    g.seq_new[b] = n.n[b];
+  for (int b = threadIdx.x; b < g.B; b += blockDim.x) g.seq_len[b] += g.seq_new[b];
+}
+
+// KIVI's full-precision ring for a ragged cache: sequence b's new tokens that
+// stay outside its coded prefix, token t in slot t mod (R + G).
+__global__ void store_ring_ragged_kernel(Geom g, int L, const void* k, const void* v) {
+  pdl_wait();
+  pdl_trigger();
+  const int which = blockIdx.y;
+  const void* x = which ? v : k;
+  const int vec_per_tok = g.D * 2 / 16;                 // bf16
+  const int total = g.B * g.H * L * vec_per_tok;        // below 2^31 (checked by the host)
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    const int vi = i % vec_per_tok;
+    const int rest = i / vec_per_tok;
+    const int j = rest % L, row = rest / L;
+    const int h = row % g.H, b = row / g.H;
+    int T0, n;
+    append_span(g, b, L, 0, &T0, &n);
+    const int t = T0 + j;
+    if (j >= n || t < kivi_tq(T0 + n, g.R, g.G)) continue;
+    const int plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+    const uint4* src = reinterpret_cast<const uint4*>(x) + ((int64_t)row * L + j) * vec_per_tok;
+    uint4* dst = reinterpret_cast<uint4*>(plane_ptr<__nv_bfloat16>(g, plane, b, h, t % g.ring));
+    dst[vi] = src[vi];
   }
 }
 
@@ -241,10 +262,12 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
   pdl_wait();
   pdl_trigger();
   extern __shared__ float smem[];
-  bool ok;
-  const int T0 = append_begin(g, L, &ok);
+  bool ok = true;
+  const int T0u = g.layout == KVQ_LAYOUT_UNIFORM ? append_begin(g, L, &ok) : 0;
   const int G = g.G, D = g.D, bits = g.kb;
-  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + L, g.R, G);
+  int T0, n;
+  append_span(g, blockIdx.y / g.H, L, T0u, &T0, &n);
+  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + n, g.R, G);
   const int blk = q0 / G + blockIdx.x;
   if (!ok || blk >= q1 / G) return;
   src.T0 = T0;
@@ -297,8 +320,8 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
       for (int r = r0; r < r1; ++r)
         cs[r * D + d] = (uint8_t)affine_code(xs[r * D + d], mn, s, inv, bits);
     if (part == 0) {
-      *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
-      *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+      *blk_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
+      *blk_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
     }
   }
   __syncthreads();
@@ -323,7 +346,7 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
       };
       word = crumbs(u.x) | crumbs(u.y) << 8 | crumbs(u.z) << 16 | crumbs(u.w) << 24;
     }
-    reinterpret_cast<uint32_t*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
+    reinterpret_cast<uint32_t*>(tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
   }
 }
 
@@ -338,9 +361,11 @@ __global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, To
   pdl_wait();
   pdl_trigger();
   extern __shared__ float smem[];
-  bool ok;
-  const int T0 = append_begin(g, L, &ok);
-  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + L, g.R, G);
+  bool ok = true;
+  const int T0u = g.layout == KVQ_LAYOUT_UNIFORM ? append_begin(g, L, &ok) : 0;
+  int T0, n;
+  append_span(g, blockIdx.y / g.H, L, T0u, &T0, &n);
+  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + n, g.R, G);
   const int blk = q0 / G + blockIdx.x;
   if (!ok || blk >= q1 / G) return;
   src.T0 = T0;
@@ -396,8 +421,8 @@ __global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, To
 #pragma unroll
   for (int j = 0; j < TPP; ++j) cs[(r0 + j) * D + d] = (uint8_t)clamp_code(c[j], BITS);
   if (part == 0) {
-    *plane_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
-    *plane_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
+    *blk_ptr<__half>(g, KVQ_PLANE_K_SCALE, b, h, blk, d) = __float2half_rn(s);
+    *blk_ptr<__half>(g, KVQ_PLANE_K_ZERO, b, h, blk, d) = __float2half_rn(mn + 0.0f);
   }
   __syncthreads();
   for (int i = threadIdx.x; i < G * WPR; i += NT) {
@@ -418,7 +443,7 @@ __global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, To
       };
       word = crumbs(u.x) | crumbs(u.y) << 8 | crumbs(u.z) << 16 | crumbs(u.w) << 24;
     }
-    reinterpret_cast<uint32_t*>(plane_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
+    reinterpret_cast<uint32_t*>(tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
   }
 }
 
@@ -745,19 +770,57 @@ int grid_for(int64_t threads_needed, int block) {
   return (int)(n < 1 ? 1 : n);
 }
 
+// KIVI: code the key blocks and the value blocks this append completes
+// (before the ring takes the new tokens: the blocks read older tokens from it).
+cudaError_t launch_kivi_append(const Geom& g, int L, const void* k, const void* v,
+                               cudaStream_t s) {
+  TokSrc sk{k, 0, L, KVQ_PLANE_K_FULL, 0, g.ring}, sv{v, 0, L, KVQ_PLANE_V_FULL, 0, g.ring};
+  const int max_blocks = L / g.G + 1;     // most G-blocks an append of L completes
+  const size_t sm = (size_t)g.G * g.D * 5 + 2 * 256 * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(kivi_key_flush_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  const dim3 fgrid(max_blocks, g.B * g.H);
+  auto fk = kivi_key_flush_kernel;
+  if (g.G == 32) {
+    const int b = g.kb;
+    if (g.D == 64) fk = b == 2 ? kivi_key_flush32_kernel<64, 2> : b == 4 ? kivi_key_flush32_kernel<64, 4> : kivi_key_flush32_kernel<64, 8>;
+    if (g.D == 128) fk = b == 2 ? kivi_key_flush32_kernel<128, 2> : b == 4 ? kivi_key_flush32_kernel<128, 4> : kivi_key_flush32_kernel<128, 8>;
+    if (g.D == 256) fk = b == 2 ? kivi_key_flush32_kernel<256, 2> : b == 4 ? kivi_key_flush32_kernel<256, 4> : kivi_key_flush32_kernel<256, 8>;
+  }
+  if (fk != kivi_key_flush_kernel) {
+    e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+  }
+  launch_pdl(fk, fgrid, dim3(256), sm, s, g, L, sk);
+  launch_pdl(pack_pertoken_kernel, pertoken_grid(g, max_blocks * g.G, 1), dim3(256), 0, s, g,
+             L, sk, sv, 0, 1, 0, ilog2(g.D / 8), ilog2(g.G / 8));
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_append_ragged(const Geom& g, int L, const void* k, const void* v,
                                  const int* n, cudaStream_t s) {
-  TokSrc sk{k, 0, L, -1, 0, 1}, sv{v, 0, L, -1, 0, 1};
   SeqCounts c = {};
   for (int b = 0; b < g.B; ++b) c.n[b] = n[b];
-  const int sym = g.fmt == KVQ_FMT_SYMMETRIC;
-  launch_pdl(pack_ragged_kernel, pertoken_grid(g, L, 2), dim3(256), 0, s, g, L, sk, sv, sym,
-             ilog2(g.D / 8), ilog2(g.G / 8), c);
+  launch_pdl(seq_counts_kernel, dim3(1), dim3(256), 0, s, g, c);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  launch_pdl(seq_advance_kernel, dim3(1), dim3(256), 0, s, g, c);
+  if (g.fmt == KVQ_FMT_KIVI) {
+    e = launch_kivi_append(g, L, k, v, s);
+    if (e != cudaSuccess) return e;
+    launch_pdl(store_ring_ragged_kernel,
+               dim3(dim3(grid_for((int64_t)g.B * g.H * L * (g.D * 2 / 16), 256), 2)), dim3(256),
+               0, s, g, L, k, v);
+  } else {
+    TokSrc sk{k, 0, L, -1, 0, 1}, sv{v, 0, L, -1, 0, 1};
+    launch_pdl(pack_pertoken_kernel, pertoken_grid(g, L, 2), dim3(256), 0, s, g, L, sk, sv,
+               g.fmt == KVQ_FMT_SYMMETRIC ? 1 : 0, 0, 0, ilog2(g.D / 8), ilog2(g.G / 8));
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  launch_pdl(seq_advance_kernel, dim3(1), dim3(256), 0, s, g);
   return cudaGetLastError();
 }
 
@@ -794,27 +857,8 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       return cudaGetLastError();
     }
     case KVQ_FMT_KIVI: {
-      sk.ring_plane = KVQ_PLANE_K_FULL; sk.ring_rows = g.ring;
-      sv.ring_plane = KVQ_PLANE_V_FULL; sv.ring_rows = g.ring;
-      const size_t sm = (size_t)g.G * g.D * 5 + 2 * 256 * sizeof(float);
-      e = cudaFuncSetAttribute(kivi_key_flush_kernel,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+      e = launch_kivi_append(g, L, k, v, s);
       if (e != cudaSuccess) return e;
-      const dim3 fgrid(max_blocks, g.B * g.H);
-      auto fk = kivi_key_flush_kernel;
-      if (g.G == 32) {
-        const int b = g.kb;
-        if (g.D == 64) fk = b == 2 ? kivi_key_flush32_kernel<64, 2> : b == 4 ? kivi_key_flush32_kernel<64, 4> : kivi_key_flush32_kernel<64, 8>;
-        if (g.D == 128) fk = b == 2 ? kivi_key_flush32_kernel<128, 2> : b == 4 ? kivi_key_flush32_kernel<128, 4> : kivi_key_flush32_kernel<128, 8>;
-        if (g.D == 256) fk = b == 2 ? kivi_key_flush32_kernel<256, 2> : b == 4 ? kivi_key_flush32_kernel<256, 4> : kivi_key_flush32_kernel<256, 8>;
-      }
-      if (fk != kivi_key_flush_kernel) {
-        e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        if (e != cudaSuccess) return e;
-      }
-      launch_pdl(fk, fgrid, dim3(256), sm, s, g, L, sk);
-      launch_pdl(pack_pertoken_kernel, pertoken_grid(g, max_blocks * g.G, 1), dim3(256), 0, s, g,
-                 L, sk, sv, 0, 1, 0, ilog2(g.D / 8), ilog2(g.G / 8));
       launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
       return cudaGetLastError();
     }

@@ -33,6 +33,8 @@ FORMATS = {
                     residual_tokens=32),
     "kivi_k8": dict(fmt=O.FMT_KIVI, key_bits=8, value_bits=4, group_size=32,
                     residual_tokens=0),
+    "kivi4": dict(fmt=O.FMT_KIVI, key_bits=4, value_bits=4, group_size=32,
+                  residual_tokens=64),
     "kvarn": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=64,
                   sink_tokens=128, norm_iters=8),
     "kvarn_small": dict(fmt=O.FMT_KVARN, key_bits=4, value_bits=2, group_size=32,

@@ -234,7 +234,7 @@ def test_ragged_and_paged_layout_rules(kvq):
     fake = 1 << 32
     P = 1 << 33
     base = dict(batch=3, kv_heads=2, q_heads=8, head_dim=64, max_tokens=500)
-    for kw in (dict(fmt=kvq.KVQ_FMT_KIVI, residual_tokens=32), dict(dtype=kvq.KVQ_F32),
+    for kw in (dict(fmt=kvq.KVQ_FMT_KVARN, group_size=64, sink_tokens=16), dict(dtype=kvq.KVQ_F32),
                dict(key_bits=2), dict(group_size=64), dict(head_dim=256)):
         d = _desc(kvq, **{**base, **kw, "layout": kvq.KVQ_LAYOUT_RAGGED})
         with pytest.raises(kvq.KvqError):

@@ -18,11 +18,13 @@ import torch
 from oracle import kvq_oracle as O
 from paper_2609_04263_gb300 import kvq, synth
 from tests.gpu_common import require_gpu
-from tests.helpers import FORMATS, check_attention, check_projection, kv_pair, oracle_cache
+from tests.helpers import (FORMATS, check_attention, check_projection, kv_pair, live,
+                           oracle_cache, to_numpy_plane)
 
 pytestmark = pytest.mark.gpu
 
-PLANE_NAMES = ("k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero")
+PLANE_NAMES = ("k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "k_full",
+               "v_full")
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -35,7 +37,8 @@ def _cache(spec, B, H, Hq, D, Tmax, layout, num_pages=0):
     kw = dict(spec)
     fmt = kw.pop("fmt")
     desc = api.make_desc(fmt, kw["key_bits"], kw["value_bits"], kw["group_size"], B, H, Hq, D,
-                         Tmax, torch.bfloat16, layout=layout, num_pages=num_pages)
+                         Tmax, torch.bfloat16, residual_tokens=kw.get("residual_tokens", 0),
+                         layout=layout, num_pages=num_pages)
     return api.Cache(desc)
 
 
@@ -43,29 +46,37 @@ PG = kvq.KVQ_PAGE_TOKENS
 
 
 def _seq_rows(gc, name, b, T):
-    """Plane rows [H, T, cols] of sequence b's tokens (PAGED: through its pages)."""
+    """Sequence b's rows [1, H, rows, cols] of a plane (PAGED: gathered
+    through its pages; KIVI's key scales and zeros hold a row per 32-token
+    block, its full-precision ring stays per sequence)."""
     p = gc.planes()[name]
-    if gc.desc.layout == kvq.KVQ_LAYOUT_PAGED:
-        pages = gc.seq_pages(b)
-        assert len(pages) == (T + PG - 1) // PG
-        if not pages:
-            return p[0, :, :0]
-        rows = torch.cat([p[0, :, PG * pg:PG * pg + PG] for pg in pages], dim=1)
-        return rows[:, :T]
-    return p[b, :, :T]
+    if name.endswith("_full"):
+        return p[b:b + 1]
+    if gc.desc.layout != kvq.KVQ_LAYOUT_PAGED:
+        return p[b:b + 1]
+    per = PG // 32 if (gc.desc.fmt == kvq.KVQ_FMT_KIVI and name in ("k_scale", "k_zero")) else PG
+    pages = gc.seq_pages(b)
+    assert len(pages) == (T + PG - 1) // PG
+    if not pages:
+        return p[0:1, :, :0]
+    return torch.cat([p[0:1, :, per * pg:per * pg + per] for pg in pages], dim=2)
 
 
 def _compare_seq(gc, oc, b):
+    """Bit-exact comparison of sequence b's live rows with its oracle cache."""
     T = oc.T
     assert gc.seq_tokens(b) == T
     for name in PLANE_NAMES:
         if name not in oc.planes or oc.planes[name].size == 0:
             continue
-        got = _seq_rows(gc, name, b, T).contiguous().cpu().numpy()
-        ref = oc.planes[name][0, :, :T]
+        got = live(name, to_numpy_plane(_seq_rows(gc, name, b, T).contiguous()), oc)
+        ref = live(name, oc.planes[name], oc)
         assert got.shape == ref.shape, (name, got.shape, ref.shape)
-        assert np.array_equal(got.view(np.uint8), ref.view(np.uint8)), \
-            f"sequence {b} plane {name} differs"
+        if got.dtype == np.float32:         # full-precision rows (bf16 read as fp32)
+            same = np.array_equal(got, ref.astype(np.float32))
+        else:
+            same = np.array_equal(got.view(np.uint8), ref.view(np.uint8))
+        assert same, f"sequence {b} plane {name} differs"
 
 
 class Batch:
@@ -127,7 +138,8 @@ class Batch:
 
 
 @pytest.mark.parametrize("layout", [kvq.KVQ_LAYOUT_RAGGED, kvq.KVQ_LAYOUT_PAGED])
-@pytest.mark.parametrize("fmt,B,H,Hq,D", [("affine4", 3, 2, 8, 64), ("sym2", 4, 2, 8, 128)])
+@pytest.mark.parametrize("fmt,B,H,Hq,D", [("affine4", 3, 2, 8, 64), ("sym2", 4, 2, 8, 128),
+                                          ("kivi2", 3, 2, 8, 128), ("kivi4", 3, 2, 4, 64)])
 def test_ragged_batch_lifecycle(layout, fmt, B, H, Hq, D):
     pages = 3 * B * 2 if layout == kvq.KVQ_LAYOUT_PAGED else 0
     bt = Batch(fmt, B, H, Hq, D, 512, layout, pages, seed=D + B)
@@ -207,7 +219,8 @@ def test_ragged_decode_step_positions():
 
 
 @pytest.mark.parametrize("layout", [kvq.KVQ_LAYOUT_RAGGED, kvq.KVQ_LAYOUT_PAGED])
-def test_streaming_decode_over_ragged_sequences(layout):
+@pytest.mark.parametrize("fmt", ["sym2", "kivi2"])
+def test_streaming_decode_over_ragged_sequences(layout, fmt):
     """Long ragged caches take the persistent streaming decode kernel (whose
     work split follows each sequence's own block count, and whose copies stay
     inside one page): sequences of very different lengths, one of them empty
@@ -215,7 +228,7 @@ def test_streaming_decode_over_ragged_sequences(layout):
     B, H, Hq, D = 8, 4, 32, 64
     lens = [4000, 10, 0, 3000, 4096, 1, 2500, 64]
     pages = sum((t + PG - 1) // PG for t in lens) + 4
-    bt = Batch("sym2", B, H, Hq, D, 4160, layout, pages if layout == kvq.KVQ_LAYOUT_PAGED else 0,
+    bt = Batch(fmt, B, H, Hq, D, 4160, layout, pages if layout == kvq.KVQ_LAYOUT_PAGED else 0,
                seed=21)
     for lo in range(0, max(lens), 1024):
         bt.append([max(0, min(1024, t - lo)) for t in lens])
