@@ -106,9 +106,10 @@ typedef struct {
  *            tokens taken from one pool of num_pages pages by the library's
  *            allocator as the sequence grows, and returned by
  *            kvq_seq_release; a sequence holds ceil(T_b / 256) pages.
- * RAGGED and PAGED caches are built for bf16 AFFINE and SYMMETRIC caches with
- * group_size 32, key_bits == value_bits in {2, 4}, head_dim 64 or 128, at most
- * 16 query heads per kv head and at most KVQ_MAX_SEQS sequences. */
+ * RAGGED and PAGED caches are built for bf16 AFFINE, SYMMETRIC and KIVI caches
+ * with group_size 32, key_bits == value_bits in {2, 4}, head_dim 64 or 128, at
+ * most 16 query heads per kv head and at most KVQ_MAX_SEQS sequences (KIVI's
+ * residual ring stays per sequence; its coded blocks go to pages). */
 typedef enum { KVQ_LAYOUT_UNIFORM = 0, KVQ_LAYOUT_RAGGED = 1, KVQ_LAYOUT_PAGED = 2 } kvq_layout;
 #define KVQ_PAGE_TOKENS 256
 #define KVQ_MAX_SEQS 512
