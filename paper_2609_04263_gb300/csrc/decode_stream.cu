@@ -254,9 +254,11 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         const int myr = pass * 5 + lane / 6, myc = lane % 6;
         int hh = h_st, bb = b_st, cnt = 0, r_head = 0, r_blk = 0, r_n = 0, r_sub = 0;
         int p_head = -1, p_end = -1;                 // end of the current run
+        // the current head's blocks and coded tokens, refreshed when the walk
+        // moves to the next head (ragged caches divide to find them)
+        int nbh = hh < BH ? nb_of(hh) : 0, tqh = hh < BH ? tq_of(hh) : 0;
 #pragma unroll
         for (int i = 0; i < kSB; ++i) {
-          const int tqh = hh < BH ? tq_of(hh) : 0;
           if (i < nbs && bb * kBT < tqh) {
             // a new run starts here (a paged cache's runs stay in one page)
             if (!(hh == p_head && bb == p_end) || (paged && bb % (kPageTok / kBT) == 0)) {
@@ -274,10 +276,12 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
             p_head = hh;
             p_end = bb + 1;
           }
-          if (i < nbs && ++bb == nb_of(hh)) {
+          if (i < nbs && ++bb == nbh) {
             bb = 0;
             ++hh;
             while (rag && hh < BH && nb_of(hh) == 0) ++hh;   // sequences holding nothing
+            nbh = hh < BH ? nb_of(hh) : 0;
+            tqh = hh < BH ? tq_of(hh) : 0;
           }
         }
         if (pass == 0) {
@@ -944,8 +948,7 @@ int decode_stream_ctas(const Geom& g) {
 
 bool decode_stream_supported(const Geom& g) {
   const bool fmt_ok = g.fmt == KVQ_FMT_AFFINE || g.fmt == KVQ_FMT_SYMMETRIC || g.fmt == KVQ_FMT_KIVI;
-  return fmt_ok && (g.layout == KVQ_LAYOUT_UNIFORM || g.fmt != KVQ_FMT_KIVI) &&
-         g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb && (g.kb == 2 || g.kb == 4) &&
+  return fmt_ok && g.act == KVQ_BF16 && g.G == 32 && g.kb == g.vb && (g.kb == 2 || g.kb == 4) &&
          (g.D == 64 || g.D == 128) && g.Hq / g.H <= 8;
 }
 
