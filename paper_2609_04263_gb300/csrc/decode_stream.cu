@@ -42,6 +42,11 @@ namespace {
 using namespace dattn;
 using namespace stream;
 
+// blocks per ring stage (copied together): 16 (half the producer's per-stage
+// bookkeeping of 8-block stages; 77.9 -> 73.4 us on the 8B-shaped KIVI cache),
+// where KVarN's larger blocks keep stream_common's 8
+constexpr int kSBD = 16;
+
 template <int D, int KB, int VB, int FMT>
 struct SCfg {
   static constexpr int NG = D / 32;                    // groups of 32 channels
@@ -53,14 +58,14 @@ struct SCfg {
   // per block: K metadata (KIVI: one row of D per block; else per token), V metadata
   static constexpr int KMETA = KIVI ? D * 2 : kBT * NG * 2;
   static constexpr int VMETA = kBT * NG * 2;
-  // a stage holds kSB consecutive blocks, each plane contiguous over them
+  // a stage holds kSBD consecutive blocks, each plane contiguous over them
   static constexpr int KC = 0;
-  static constexpr int VC = KC + kSB * kBT * KCB;
-  static constexpr int KS = VC + kSB * kBT * VCB;
-  static constexpr int KZ = KS + kSB * KMETA;
-  static constexpr int VS = KZ + (SYM ? 0 : kSB * KMETA);
-  static constexpr int VZ = VS + kSB * VMETA;
-  static constexpr int STAGE = (VZ + (SYM ? 0 : kSB * VMETA) + 127) / 128 * 128;
+  static constexpr int VC = KC + kSBD * kBT * KCB;
+  static constexpr int KS = VC + kSBD * kBT * VCB;
+  static constexpr int KZ = KS + kSBD * KMETA;
+  static constexpr int VS = KZ + (SYM ? 0 : kSBD * KMETA);
+  static constexpr int VZ = VS + kSBD * VMETA;
+  static constexpr int STAGE = (VZ + (SYM ? 0 : kSBD * VMETA) + 127) / 128 * 128;
 };
 
 // Two tokens' fp16 metadata of group gq packed as (token a, token b), from
@@ -222,7 +227,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
   if (threadIdx.x == 0) {
     for (int i = 0; i < ns; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kSB);                     // one arrival per block
+      mbar_init(&empty[i], kSBD);                     // one arrival per block
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -230,7 +235,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
 
   // ------------------------------------------------------------------ producer
   if (warp == kNW) {
-    const int nst = (nblk + kSB - 1) / kSB;          // stages
+    const int nst = (nblk + kSBD - 1) / kSBD;          // stages
     int blk;
     int head = head_at(k0, &blk);                    // first block of the next stage
     int s = 0;
@@ -245,7 +250,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
       // split the stage's blocks into runs of one head's coded blocks; in
       // pass p, lane 6 r + c issues copy c of run 5 p + r (every lane walks
       // the same blocks, so the bookkeeping stays in registers)
-      const int nbs = min(kSB, nblk - s * kSB);
+      const int nbs = min(kSBD, nblk - s * kSBD);
       const int h_st = head, b_st = blk;             // the stage's first block
       unsigned char* sp = smem + (size_t)st * C::STAGE;
       int nrun = 0;
@@ -258,7 +263,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         // moves to the next head (ragged caches divide to find them)
         int nbh = hh < BH ? nb_of(hh) : 0, tqh = hh < BH ? tq_of(hh) : 0;
 #pragma unroll
-        for (int i = 0; i < kSB; ++i) {
+        for (int i = 0; i < kSBD; ++i) {
           if (i < nbs && bb * kBT < tqh) {
             // a new run starts here (a paged cache's runs stay in one page)
             if (!(hh == p_head && bb == p_end) || (paged && bb % (kPageTok / kBT) == 0)) {
@@ -762,7 +767,7 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
     const bool mine = jst < e;
     if (mine) load_q();
     for (int j = jst; j < e && !bad; j += kNW) {
-      const int sj = j / kSB, st = sj % ns;
+      const int sj = j / kSBD, st = sj % ns;
       bool ok = true;
       if (lane == 0) ok = mbar_wait(&full[st], (sj / ns) & 1);
       if (!__shfl_sync(0xffffffffu, ok, 0)) {
@@ -773,9 +778,9 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
       const int t0 = (int)(k0 + j - hs) * kBT;
       const int nv = min(kBT, Th - t0);
       if (nv == kBT)
-        process(std::true_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tqh);
+        process(std::true_type(), smem + (size_t)st * C::STAGE, j % kSBD, t0, nv, t0 < tqh);
       else
-        process(std::false_type(), smem + (size_t)st * C::STAGE, j % kSB, t0, nv, t0 < tqh);
+        process(std::false_type(), smem + (size_t)st * C::STAGE, j % kSBD, t0, nv, t0 < tqh);
       __syncwarp();
       if (lane == 0) mbar_arrive1(&empty[st]);
     }
