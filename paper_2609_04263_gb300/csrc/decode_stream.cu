@@ -238,6 +238,42 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
     const int nst = (nblk + kSBD - 1) / kSBD;          // stages
     int blk;
     int head = head_at(k0, &blk);                    // first block of the next stage
+    // the head's blocks and coded tokens (ragged caches divide to find them)
+    int cur_nb = nb_of(head), cur_tq = tq_of(head);
+    // bytes of one whole coded block
+    constexpr uint32_t kBlockBytes = kBT * (C::KCB + C::VCB) + (C::SYM ? 1 : 2) * kBT * NG * 2 +
+                                     (C::KIVI ? 2 * D * 2 : (C::SYM ? 1 : 2) * kBT * NG * 2);
+    // copy c (codes of K, V; metadata planes) of a run of r_n blocks of head
+    // r_head from its block r_blk into the stage's block slots from r_sub
+    auto issue = [&](unsigned char* sp, int st, int myc, int r_head, int r_blk, int r_n,
+                     int r_sub) {
+      const int t0 = r_blk * kBT;
+      const int n4 = (min(r_n * kBT, tq_of(r_head) - t0) + 3) & ~3;
+      const int tsub = r_sub * kBT;                  // first token slot in the stage
+      const uint8_t* src;
+      unsigned char* dst;
+      uint32_t bytes;
+      if (myc == 0) {
+        src = run_ptr(KVQ_PLANE_K_CODES, r_head, t0);
+        dst = sp + C::KC + tsub * C::KCB;
+        bytes = n4 * C::KCB;
+      } else if (myc == 1) {
+        src = run_ptr(KVQ_PLANE_V_CODES, r_head, t0);
+        dst = sp + C::VC + tsub * C::VCB;
+        bytes = n4 * C::VCB;
+      } else if (myc == 2 || myc == 4) {
+        const int pl = myc == 2 ? KVQ_PLANE_K_SCALE : KVQ_PLANE_K_ZERO;
+        src = C::KIVI ? blk_run_ptr(pl, r_head, r_blk) : run_ptr(pl, r_head, t0);
+        dst = sp + (myc == 2 ? C::KS : C::KZ) + r_sub * C::KMETA;
+        bytes = C::KIVI ? r_n * D * 2 : n4 * NG * 2;
+      } else {
+        const int pl = myc == 3 ? KVQ_PLANE_V_SCALE : KVQ_PLANE_V_ZERO;
+        src = run_ptr(pl, r_head, t0);
+        dst = sp + (myc == 3 ? C::VS : C::VZ) + r_sub * C::VMETA;
+        bytes = n4 * NG * 2;
+      }
+      bulk_g2s(dst, src, bytes, &full[st]);
+    };
     int s = 0;
     for (; s < nst; ++s) {
       const int st = s % ns;
@@ -247,21 +283,43 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
         if (lane == 0) atomicOr(err, 1);
         break;
       }
+      const int nbs = min(kSBD, nblk - s * kSBD);
+      unsigned char* sp = smem + (size_t)st * C::STAGE;
+      if (blk + nbs <= cur_nb && (blk + nbs) * kBT <= cur_tq) {
+        // the common case: the stage's blocks are whole coded blocks of one
+        // head, one run (a paged cache: one run per page it touches, at most 3)
+        if (lane == 0) mbar_expect_tx(&full[st], nbs * kBlockBytes);
+        __syncwarp();
+        constexpr int PB = kPageTok / kBT;               // blocks per page
+        const int nsub = paged ? (blk % PB + nbs + PB - 1) / PB : 1;
+        const int sub = lane / 6, myc = lane % 6;
+        if (sub < nsub && myc < (C::SYM ? 4 : 6)) {
+          const int b0 = sub == 0 ? blk : (blk / PB + sub) * PB;
+          const int b1 = paged ? min(blk + nbs, (blk / PB + sub + 1) * PB) : blk + nbs;
+          issue(sp, st, myc, head, b0, b1 - b0, b0 - blk);
+        }
+        blk += nbs;
+        if (blk == cur_nb) {
+          blk = 0;
+          ++head;
+          while (rag && head < BH && nb_of(head) == 0) ++head;   // sequences holding nothing
+          cur_nb = head < BH ? nb_of(head) : 0;
+          cur_tq = head < BH ? tq_of(head) : 0;
+        }
+        continue;
+      }
       // split the stage's blocks into runs of one head's coded blocks; in
       // pass p, lane 6 r + c issues copy c of run 5 p + r (every lane walks
       // the same blocks, so the bookkeeping stays in registers)
-      const int nbs = min(kSBD, nblk - s * kSBD);
       const int h_st = head, b_st = blk;             // the stage's first block
-      unsigned char* sp = smem + (size_t)st * C::STAGE;
+      const int nb_st = cur_nb, tq_st = cur_tq;      // and its head's counts
       int nrun = 0;
       uint32_t total = 0;
       for (int pass = 0; pass == 0 || pass * 5 < nrun; ++pass) {
         const int myr = pass * 5 + lane / 6, myc = lane % 6;
         int hh = h_st, bb = b_st, cnt = 0, r_head = 0, r_blk = 0, r_n = 0, r_sub = 0;
         int p_head = -1, p_end = -1;                 // end of the current run
-        // the current head's blocks and coded tokens, refreshed when the walk
-        // moves to the next head (ragged caches divide to find them)
-        int nbh = hh < BH ? nb_of(hh) : 0, tqh = hh < BH ? tq_of(hh) : 0;
+        int nbh = nb_st, tqh = tq_st;                // head hh's blocks and coded tokens
 #pragma unroll
         for (int i = 0; i < kSBD; ++i) {
           if (i < nbs && bb * kBT < tqh) {
@@ -293,38 +351,13 @@ decode_stream_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale, i
           nrun = cnt;
           head = hh;                                 // first block of the next stage
           blk = bb;
+          cur_nb = nbh;
+          cur_tq = tqh;
           if (lane == 0) mbar_expect_tx(&full[st], total);   // 0: nothing to copy
           __syncwarp();
         }
-        if (lane < 30 && myr < nrun && (!C::SYM || myc < 4)) {
-          const int t0 = r_blk * kBT;
-          const int n4 = (min(r_n * kBT, tq_of(r_head) - t0) + 3) & ~3;
-          const int tsub = r_sub * kBT;              // first token slot in the stage
-          // plane rows of head h: plane_ptr(g, plane, 0, h, row) addresses (b, hkv) = h
-          const uint8_t* src;
-          unsigned char* dst;
-          uint32_t bytes;
-          if (myc == 0) {
-            src = run_ptr(KVQ_PLANE_K_CODES, r_head, t0);
-            dst = sp + C::KC + tsub * C::KCB;
-            bytes = n4 * C::KCB;
-          } else if (myc == 1) {
-            src = run_ptr(KVQ_PLANE_V_CODES, r_head, t0);
-            dst = sp + C::VC + tsub * C::VCB;
-            bytes = n4 * C::VCB;
-          } else if (myc == 2 || myc == 4) {
-            const int pl = myc == 2 ? KVQ_PLANE_K_SCALE : KVQ_PLANE_K_ZERO;
-            src = C::KIVI ? blk_run_ptr(pl, r_head, r_blk) : run_ptr(pl, r_head, t0);
-            dst = sp + (myc == 2 ? C::KS : C::KZ) + r_sub * C::KMETA;
-            bytes = C::KIVI ? r_n * D * 2 : n4 * NG * 2;
-          } else {
-            const int pl = myc == 3 ? KVQ_PLANE_V_SCALE : KVQ_PLANE_V_ZERO;
-            src = run_ptr(pl, r_head, t0);
-            dst = sp + (myc == 3 ? C::VS : C::VZ) + r_sub * C::VMETA;
-            bytes = n4 * NG * 2;
-          }
-          bulk_g2s(dst, src, bytes, &full[st]);
-        }
+        if (lane < 30 && myr < nrun && (!C::SYM || myc < 4))
+          issue(sp, st, myc, r_head, r_blk, r_n, r_sub);
       }
     }
     // keep the CTA alive until the last copies have landed (the consumers
