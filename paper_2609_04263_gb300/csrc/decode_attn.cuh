@@ -96,6 +96,10 @@ __device__ __forceinline__ uint64_t ld_tagged(const uint64_t* p) {
   asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
   return w;
 }
+// two adjacent tagged words (16-byte aligned) in one access
+__device__ __forceinline__ void ld_tagged2(const uint64_t* p, uint64_t& a, uint64_t& b) {
+  asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p) : "memory");
+}
 __device__ __forceinline__ float tagged_value(uint64_t w) { return __uint_as_float((uint32_t)w); }
 __device__ __forceinline__ bool tag_is(uint64_t w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
 
@@ -225,16 +229,22 @@ __device__ void split_issue(const Geom& g, int b, int hkv, const SplitPlan& sp, 
              &bars[stage]);
 }
 
-// Initialise the stage barriers and issue the first STAGES chunks of a split.
-// Every thread of the CTA calls it.
+// Initialise the stage barriers and issue the first STAGES chunks of a split,
+// lane c of warp 0 the copies of chunk c (the chunks' copies are issued
+// together rather than one chunk after another).  Every thread of the CTA
+// calls it.
 template <int D, int BITS, int FMT, int STAGES>
 __device__ void split_prologue(const Geom& g, int b, int hkv, const SplitPlan& sp,
                                unsigned char* smem, uint64_t* bars) {
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < STAGES; ++i) mbar_init(&bars[i], 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    for (int c = 0; c < min(STAGES, sp.nchunks); ++c)
-      split_issue<D, BITS, FMT, STAGES>(g, b, hkv, sp, c, smem, bars);
+  static_assert(STAGES <= 32, "one lane per stage");
+  if (threadIdx.x < 32) {
+    if (threadIdx.x == 0) {
+      for (int i = 0; i < STAGES; ++i) mbar_init(&bars[i], 1);
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    if ((int)threadIdx.x < min(STAGES, sp.nchunks))
+      split_issue<D, BITS, FMT, STAGES>(g, b, hkv, sp, threadIdx.x, smem, bars);
   }
   __syncthreads();
 }
@@ -254,29 +264,35 @@ __device__ void merge_tagged(const Geom& g, __nv_bfloat16* __restrict__ out, int
     float M = -INFINITY, L = 0.f, a0 = 0.f, a1 = 0.f;
     for (int s0 = 0; s0 < S; s0 += SB) {
       float ms[SB], ls[SB], v0[SB], v1[SB];
+      // every word of the block is loaded before any is checked (the loads
+      // are in flight together: one L2 round trip per poll)
+      uint64_t wv[SB][4];
       for (long it = 0;; ++it) {
-        bool ok = true;
 #pragma unroll
         for (int k = 0; k < SB; ++k) {
-          const int sp = s0 + k;
-          ms[k] = -INFINITY;
-          ls[k] = v0[k] = v1[k] = 0.f;
-          if (sp < S) {
-            const uint64_t* ws = w + sp * (D + kWsStride);
-            const uint64_t wm = ld_tagged(ws), wl = ld_tagged(ws + 1);
-            const uint64_t w0 = ld_tagged(ws + 2 + d), w1 = ld_tagged(ws + 3 + d);
-            ok = ok && tag_is(wm, tag) && tag_is(wl, tag) && tag_is(w0, tag) && tag_is(w1, tag);
-            ms[k] = tagged_value(wm);
-            ls[k] = tagged_value(wl);
-            v0[k] = tagged_value(w0);
-            v1[k] = tagged_value(w1);
-          }
+          const uint64_t* ws = w + min(s0 + k, S - 1) * (D + kWsStride);
+          ld_tagged2(ws, wv[k][0], wv[k][1]);        // rows of D + 2 words, d even:
+          ld_tagged2(ws + 2 + d, wv[k][2], wv[k][3]); // both pairs 16-byte aligned
         }
+        bool ok = true;
+#pragma unroll
+        for (int k = 0; k < SB; ++k)
+          if (s0 + k < S)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) ok = ok && tag_is(wv[k][c], tag);
         if (ok) break;
         if (it > kPollLimit) {
           atomicOr(err, 2);
           break;
         }
+      }
+#pragma unroll
+      for (int k = 0; k < SB; ++k) {
+        const bool live = s0 + k < S;
+        ms[k] = live ? tagged_value(wv[k][0]) : -INFINITY;
+        ls[k] = live ? tagged_value(wv[k][1]) : 0.f;
+        v0[k] = live ? tagged_value(wv[k][2]) : 0.f;
+        v1[k] = live ? tagged_value(wv[k][3]) : 0.f;
       }
       float Mb = M;
 #pragma unroll

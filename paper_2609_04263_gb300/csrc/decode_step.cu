@@ -345,6 +345,7 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
   __shared__ uint64_t ubar[kMaxSlots];
   __shared__ uint64_t abar[AST];
   __shared__ uint64_t bbar;
+  __shared__ uint64_t xbar;
   __shared__ __align__(16) float ush[kWarpsF][128];
   const Geom& g = a.g;
   CacheState* st = g.state;
@@ -357,6 +358,7 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
   if (threadIdx.x == 0) {
     for (int i = 0; i < a.nslot; ++i) dattn::mbar_init(&ubar[i], 1);
     dattn::mbar_init(&bbar, 1);
+    dattn::mbar_init(&xbar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
@@ -396,6 +398,16 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
   pdl_trigger();
   pdl_wait();
 
+  // x (the step's input, written by the preceding kernel) to shared memory:
+  // one bulk copy per row, in flight with the token-count read below
+  unsigned char* xs = sm + a.xs_off;
+  const int M = g.B;
+  const bool x_bulk = (reinterpret_cast<uintptr_t>(a.x) & 15) == 0;
+  if (x_bulk && threadIdx.x == 0) {
+    dattn::mbar_expect_tx(&xbar, (uint32_t)(M * 2 * a.d_in));
+    for (int m = 0; m < M; ++m)
+      dattn::bulk_g2s(xs + m * a.xstride, a.x + (int64_t)m * a.d_in, 2 * a.d_in, &xbar);
+  }
   // tokens before this step and the launch epoch: read once (thread 0) and
   // shared, so that both reads are complete before this CTA arrives on the
   // counter below
@@ -411,9 +423,7 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
   const uint32_t tag = 0xFFC00000u | ((epoch + 1) & 0x003FFFFFu);   // a NaN no arithmetic makes
   const bool room = T0 >= 0 && T0 + 1 <= g.Tmax;
   const int T = T0 + 1;
-  const int M = g.B;
   unsigned char* asmem = sm + a.att_off;
-  unsigned char* xs = sm + a.xs_off;
   uint64_t* part = reinterpret_cast<uint64_t*>(g.pl[KVQ_PLANE_WORKSPACE].p) + a.part_off;
   const bool attend_here = room && (int)blockIdx.x < items3;
   int early = 0;                           // attention chunks issued ahead of the split
@@ -423,10 +433,13 @@ decode_step_kernel(const __grid_constant__ StepArgs a) {
     dattn::split_prologue<D, BITS, FMT, AST>(g, rest / g.H, rest % g.H, sp, asmem, abar);
     early = min(AST, sp.nchunks);
   }
-  for (int i = threadIdx.x * 8; i < M * a.d_in; i += blockDim.x * 8) {
-    const int m = i / a.d_in, k = i - m * a.d_in;
-    *reinterpret_cast<uint4*>(xs + m * a.xstride + 2 * k) =
-        __ldg(reinterpret_cast<const uint4*>(a.x + i));
+  if (x_bulk) {
+    if (threadIdx.x == 0 && !dattn::mbar_wait(&xbar, 0)) atomicOr(a.err, 1);
+  } else {                                 // x not 16-byte aligned: element loads
+    for (int i = threadIdx.x; i < M * a.d_in; i += blockDim.x) {
+      const int m = i / a.d_in, k = i - m * a.d_in;
+      *reinterpret_cast<__nv_bfloat16*>(xs + m * a.xstride + 2 * k) = a.x[i];
+    }
   }
   __syncthreads();
   // Every CTA has read the token count and the epoch once it arrives here;
