@@ -289,7 +289,8 @@ __global__ void combine_kernel(Geom g, int splits, int extra, void* out) {
 // refolded when the token block changes (a lane's channels lie in one group);
 // sinks and staged tokens are rotated forward in registers.  The values
 // accumulate in the rotated basis; the split's output is rotated back before
-// its (m, l, o) partial goes to the workspace, which combine_kernel merges.
+// its (m, l, o) partial goes to the workspace, and the last split CTA of a
+// (sequence, kv head) to finish merges the partials into the output.
 // ---------------------------------------------------------------------------
 template <int D>
 __device__ __forceinline__ void fwht_contig(float (&x)[D / 32], int lane, float inv_sqrt_d) {
@@ -323,7 +324,7 @@ __device__ __forceinline__ uint32_t lane_codes(const uint8_t* row, int lane, int
 template <int D, int GM>
 __global__ void __launch_bounds__(256)
 attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float scale,
-                           float inv_sqrt_d, int full_only) {
+                           float inv_sqrt_d, int full_only, void* out) {
   pdl_wait();
   pdl_trigger();
   constexpr int NS = D / 32;
@@ -483,10 +484,47 @@ attend_kvarn_decode_kernel(Geom g, const __nv_bfloat16* __restrict__ q, float sc
 #pragma unroll
     for (int i = 0; i < NS; ++i) wsr[2 + NS * lane + i] = x[i];
   }
+  // ---- the last split CTA of this (sequence, kv head) merges the splits
+  // and, with full_only, the coded tokens' partial (slot kMaxSplits - 1,
+  // written by the streaming kernel that ran before this one) ----
+  __shared__ int last_cta;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    last_cta = atomicAdd(&g.counters[b * g.H + hkv], 1u) == (unsigned)g.splits - 1;
+  }
+  __syncthreads();
+  if (!last_cta) return;
+  __threadfence();
+  const int n = g.splits + (full_only ? 1 : 0);
+  for (int h = warp; h < grp; h += 8) {
+    const float* w = ws_row(g, b, hkv * grp + h);
+    auto row = [&](int i) { return w + (int64_t)(i < g.splits ? i : kMaxSplits - 1) * (D + kWsStride); };
+    float M = -INFINITY;
+    for (int i = lane; i < n; i += 32) M = fmaxf(M, __ldcg(row(i)));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float L = 0.f, acc[NS];
+#pragma unroll
+    for (int i = 0; i < NS; ++i) acc[i] = 0.f;
+    for (int i = 0; i < n; ++i) {
+      const float mi = __ldcg(row(i));
+      if (mi == -INFINITY) continue;
+      const float f = expf(mi - M);
+      L += f * __ldcg(row(i) + 1);
+#pragma unroll
+      for (int k = 0; k < NS; ++k) acc[k] += f * __ldcg(row(i) + 2 + lane + 32 * k);
+    }
+#pragma unroll
+    for (int k = 0; k < NS; ++k)
+      st_act(out, ((int64_t)b * g.Hq + hkv * grp + h) * D + lane + 32 * k, acc[k] / L, g.act);
+  }
+  if (threadIdx.x == 0) g.counters[b * g.H + hkv] = 0;   // ready for the next call
 }
 
 template <int D>
-cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, int full_only, cudaStream_t s) {
+cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, int full_only, void* out,
+                           cudaStream_t s) {
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)D));
   dim3 grid(g.splits, g.H, g.B);
@@ -495,7 +533,7 @@ cudaError_t launch_kvarn_d(const Geom& g, const void* q, float scale, int full_o
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     launch_pdl(kern, dim3(grid), dim3(256), sm, s, g, reinterpret_cast<const __nv_bfloat16*>(q),
-               scale, inv_sqrt_d, full_only);
+               scale, inv_sqrt_d, full_only, out);
     return cudaGetLastError();
   };
   if (grp <= 2) return run(attend_kvarn_decode_kernel<D, 2>, 2);
@@ -555,13 +593,10 @@ cudaError_t launch_attend(const Geom& g, const void* q, int L, float scale, void
       cudaError_t e = launch_decode_stream_kvarn(g, q, scale, err, s);
       if (e != cudaSuccess) return e;
     }
-    cudaError_t e = g.D == 64 ? launch_kvarn_d<64>(g, q, scale, streamed, s)
-                  : g.D == 128 ? launch_kvarn_d<128>(g, q, scale, streamed, s)
-                               : launch_kvarn_d<256>(g, q, scale, streamed, s);
-    if (e != cudaSuccess) return e;
-    launch_pdl(combine_kernel, dim3(dim3(g.Hq, g.B)), dim3(64), 0, s, g, g.splits,
-               streamed ? kMaxSplits - 1 : -1, out);
-    return cudaGetLastError();
+    // the split kernel's last CTA per (sequence, kv head) merges everything
+    return g.D == 64 ? launch_kvarn_d<64>(g, q, scale, streamed, out, s)
+         : g.D == 128 ? launch_kvarn_d<128>(g, q, scale, streamed, out, s)
+                      : launch_kvarn_d<256>(g, q, scale, streamed, out, s);
   }
   const int grp = g.Hq / g.H;
   const float inv_sqrt_d = (float)(1.0 / sqrt((double)g.D));

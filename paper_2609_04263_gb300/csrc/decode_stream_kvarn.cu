@@ -21,8 +21,8 @@
 //     c_v,j when the block's contribution is added.
 // The sinks and the staged tokens (full precision, original basis) are left
 // to attend_kvarn_decode_kernel; this kernel leaves each head's result as one
-// more split partial (m, l, o rotated back) in workspace slot kFinalSlot, and
-// combine_kernel merges it with the other partials.
+// more split partial (m, l, o rotated back) in workspace slot kFinalSlot,
+// which that kernel (launched next) merges with its own partials.
 #include "decode_attn.cuh"
 #include "stream_common.cuh"
 
