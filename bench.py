@@ -883,7 +883,12 @@ def main():
     run.prefill(timer)
     mean_ms = timer.mean_ms()
     run.xs.copy_(run.x_dec[0])
-    reps = 10
+    # each decode graph replay appends one token per layer: two untimed
+    # replays and `reps` timed ones must fit the cache's decode room
+    reps = min(10, wl.decode - 2)
+    if reps < 1:
+        raise SystemExit("bench.py: the per-kernel timing needs --decode-steps >= 3 "
+                         "(or --timed-only)")
     n_dec = wl.layers * wl.decode
     work = {
         "project": ("tensor", proj_flops(wl, wl.batch * wl.prefill), wl.layers),
