@@ -674,9 +674,19 @@ kvq_status kvq_project_lora_nf4(const void* x, int B, int L, int d_in, const voi
     }
   }
   void* out[3] = {q, k, v};
-  cudaError_t e = launch_project_nf4(x, B, L, d_in, w_codes, w_absmax, a, bm, r, alpha_over_r,
-                                     n_q_heads, n_kv_heads, head_dim, pos0, pos_dev, rope_base,
-                                     out, (cudaStream_t)stream, pos_stride);
+  cudaError_t e;
+  if (B * L > 16 && project_tc_nf4_supported(n_q_heads, n_kv_heads, head_dim, d_in)) {
+    // prefill rows: tcgen05, the base dequantised in the kernel's operand path
+    int* err = device_error_word();
+    if (!err) return cuda_fail(cudaErrorInvalidDevice, "kvq_project_lora_nf4");
+    e = launch_project_tc_nf4(x, B, L, d_in, w_codes, w_absmax, a, bm, r, alpha_over_r,
+                              n_q_heads, n_kv_heads, head_dim, pos0, pos_dev, rope_base, out, err,
+                              (cudaStream_t)stream, pos_stride);
+  } else {
+    e = launch_project_nf4(x, B, L, d_in, w_codes, w_absmax, a, bm, r, alpha_over_r, n_q_heads,
+                           n_kv_heads, head_dim, pos0, pos_dev, rope_base, out,
+                           (cudaStream_t)stream, pos_stride);
+  }
   if (e != cudaSuccess) return cuda_fail(e, "kvq_project_lora_nf4 launch");
   return KVQ_OK;
 }

@@ -160,6 +160,15 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
                               cudaStream_t s, const Geom* append_to = nullptr, int pos_stride = 0);
 int project_tc_tile(int Hq, int Hkv, int D, int d_in);
+// The same kernel over an NF4 base (codes [N][d_in/2], fp32 absmax [N][d_in/64],
+// dequantised in the kernel's operand path).
+bool project_tc_nf4_supported(int Hq, int Hkv, int D, int d_in);
+cudaError_t launch_project_tc_nf4(const void* x, int B, int L, int d_in, const void* codes,
+                                  const void* absmax, const void* const a[3],
+                                  const void* const bm[3], const int r[3], float alpha_over_r,
+                                  int Hq, int Hkv, int D, int pos0, const int* pos_dev,
+                                  float rope_base, void* const out[3], int* err, cudaStream_t s,
+                                  int pos_stride = 0);
 
 // Projection over an NF4 base (project_nf4.cu): codes [N][d_in/2], fp32 absmax
 // [N][d_in/64]; bf16 activations.

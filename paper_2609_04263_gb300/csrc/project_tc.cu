@@ -35,8 +35,16 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;              // bf16 elements per 128-byte swizzle row
 constexpr int kStages = 3;
-constexpr int kThreads = 128;
+constexpr int kThreads = 128;      // + 256 dequantising threads over an NF4 base
+constexpr int kDqWarps = 8;
 using namespace tc;
+
+// The 16 NF4 levels, code 0 .. 15, as QLoRA publishes the data type.
+__constant__ float c_nf4_lv[16] = {
+    -1.0f, -0.6961928009986877f, -0.5250730514526367f, -0.39491748809814453f,
+    -0.28444138169288635f, -0.18477343022823334f, -0.09105003625154495f, 0.0f,
+    0.07958029955625534f, 0.16093020141124725f, 0.24611230194568634f, 0.33791524171829224f,
+    0.44070982933044434f, 0.5626170039176941f, 0.7229568362236023f, 1.0f};
 
 struct TcArgs {
   void* out[3];
@@ -51,6 +59,8 @@ struct TcArgs {
   int k_blocks;
   int* err;
   int pack;                     // 1: code k and v into the cache g instead of storing them
+  const uint8_t* nf4_codes;     // NF4 base: codes [N][d_in / 2] (two inputs a byte, low first)
+  const float* nf4_absmax;      //           and one absmax per 64 inputs of a row [N][d_in / 64]
   Geom g;
   float theta_hi[128], theta_lo[128];
 };
@@ -129,21 +139,28 @@ struct Smem {
   static constexpr int TOTAL = BP_OFF + BN * BK * 2 + 1024;   // + alignment slack
 };
 
-template <int BN>
-__global__ void __launch_bounds__(kThreads, 1)
+// NF4: W arrives as 4-bit NormalFloat codes; warps 4-11 (256 threads: one
+// per tile row at BN = 256, two at BN = 128) turn each 64-input K slice into
+// the bf16 tile the TMA would have landed (level x absmax in fp32, rounded
+// once), 128-byte swizzled, and signal it on w_full; the x and A_p slices
+// still come by TMA.
+template <int BN, bool NF4>
+__global__ void __launch_bounds__(NF4 ? kThreads + 32 * kDqWarps : kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
                   const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_a1,
                   const __grid_constant__ CUtensorMap tm_a2, const __grid_constant__ CUtensorMap tm_b0,
                   const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_b2,
                   const TcArgs args) {
+  static_assert(!NF4 || BN == 128 || BN == 256, "256 dequantising threads cover the tile's rows");
   pdl_wait();
   pdl_trigger();
   using S = Smem<BN>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ uint64_t full_bar[kStages], empty_bar[kStages];
+  __shared__ uint64_t full_bar[kStages], empty_bar[kStages], w_full[kStages];
   __shared__ uint64_t u_bar, bp_bar, acc_bar;
+  __shared__ float nf4_lv[16];
   __shared__ uint32_t tmem_base;
   __shared__ int fail;
 
@@ -160,6 +177,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&full_bar[i], 1);
       mbar_init(&empty_bar[i], 1);
+      mbar_init(&w_full[i], kDqWarps);     // NF4: one arrival per dequantising warp
     }
     mbar_init(&u_bar, 1);
     mbar_init(&bp_bar, 1);
@@ -167,6 +185,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (NF4 && threadIdx.x < 16) nf4_lv[threadIdx.x] = c_nf4_lv[threadIdx.x];
   if (warp == 1) {   // TMEM: 512 columns (main BN + LoRA <= 64)
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;"
                  ::"r"(smem_u32(&tmem_base)));
@@ -192,9 +211,9 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
         break;
       }
       unsigned char* st = smem + s * S::STAGE_B;
-      mbar_expect_tx(&full_bar[s], S::A_B + S::B_B + (r > 0 ? rp * BK * 2 : 0));
+      mbar_expect_tx(&full_bar[s], S::A_B + (NF4 ? 0 : S::B_B) + (r > 0 ? rp * BK * 2 : 0));
       tma_load_2d(st, &tm_x, kb * BK, m0, &full_bar[s]);
-      tma_load_2d(st + S::A_B, &tm_w, kb * BK, n0, &full_bar[s]);
+      if (!NF4) tma_load_2d(st + S::A_B, &tm_w, kb * BK, n0, &full_bar[s]);
       if (r > 0) tma_load_2d(st + S::A_B + S::B_B, tm_a, kb * BK, 0, &full_bar[s]);
     }
   } else if (threadIdx.x == 32) {
@@ -204,7 +223,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     bool ok = true;
     for (int kb = 0; kb < KB; ++kb) {
       const int s = kb % kStages;
-      if (!mbar_wait(&full_bar[s], (kb / kStages) & 1)) {
+      if (!mbar_wait(&full_bar[s], (kb / kStages) & 1) ||
+          (NF4 && !mbar_wait(&w_full[s], (kb / kStages) & 1))) {
         ok = false;
         break;
       }
@@ -220,13 +240,96 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     }
     if (!ok) atomicOr(&fail, 1);
     umma_commit(&u_bar);                   // all main-loop MMAs done
+  } else if (NF4 && warp >= 4) {
+    // ---------- NF4 dequantisation: TPR threads per tile row ----------
+    constexpr int TPR = 32 * kDqWarps / BN;               // 1 (BN = 256) or 2 (BN = 128)
+    constexpr int NQ = 2 / TPR;                           // 16-byte code words per thread and slice
+    const int dt = threadIdx.x - kThreads;                // 0 .. 255
+    const int n = dt / TPR, h = dt % TPR;                 // row, part of the slice
+    const int nkb = args.k_blocks;
+    const uint8_t* crow = args.nf4_codes + (int64_t)(n0 + n) * (nkb * 32) + h * 16;
+    const float* arow = args.nf4_absmax + (int64_t)(n0 + n) * nkb;
+    // codes and absmax of this and the next two K slices in registers
+    // (rotated each slice, so no array is indexed at run time)
+    uint4 cq[3][NQ];
+    float am[3];
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+#pragma unroll
+      for (int q = 0; q < NQ; ++q) cq[i][q] = make_uint4(0, 0, 0, 0);
+      am[i] = 0.f;
+    }
+    auto fetch = [&](int kb, uint4 (&x)[NQ], float& xa) {
+      if (kb < KB) {
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) x[q] = __ldg(reinterpret_cast<const uint4*>(crow + kb * 32 + 16 * q));
+        xa = __ldg(arow + kb);
+      }
+    };
+    fetch(0, cq[0], am[0]);
+    fetch(1, cq[1], am[1]);
+    const int rsw = (n >> 3) * 1024 + (n & 7) * 128;      // the row in the swizzled tile
+    for (int kb = 0; kb < KB; ++kb) {
+      const int s = kb % kStages;
+      fetch(kb + 2, cq[2], am[2]);
+      if (kb >= kStages) {                                // lane 0 waits for the slot, then the warp
+        bool ok = true;
+        if (lane == 0) ok = mbar_wait(&empty_bar[s], ((kb / kStages) - 1) & 1);
+        if (!__shfl_sync(0xffffffffu, ok, 0)) {
+          if (lane == 0) atomicOr(&fail, 1);
+          break;
+        }
+      }
+      unsigned char* wt = smem + s * S::STAGE_B + S::A_B;
+      uint32_t w8[4 * NQ];
+#pragma unroll
+      for (int q = 0; q < NQ; ++q) {
+        w8[4 * q] = cq[0][q].x; w8[4 * q + 1] = cq[0][q].y;
+        w8[4 * q + 2] = cq[0][q].z; w8[4 * q + 3] = cq[0][q].w;
+      }
+      const float a = am[0];
+#pragma unroll
+      for (int q = 0; q < NQ; ++q) {
+        cq[0][q] = cq[1][q];
+        cq[1][q] = cq[2][q];
+      }
+      am[0] = am[1];
+      am[1] = am[2];
+      uint64_t a2;
+      asm("mov.b64 %0, {%1, %1};" : "=l"(a2) : "f"(a));
+#pragma unroll
+      for (int j = 0; j < 4 * NQ; ++j) {                  // chunk c: inputs 8c .. 8c + 7
+        const int c = 4 * NQ * h + j;
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {                     // byte i of word j: inputs 8c + 2i, + 1
+          // the two levels times absmax as one packed fp32 multiply (each
+          // product rounded as a scalar one would be), then one bf16 pair
+          const char* lvb = reinterpret_cast<const char*>(nf4_lv);
+          const uint32_t w = w8[j];
+          const float l0 = *reinterpret_cast<const float*>(
+              lvb + ((i == 0 ? w << 2 : w >> (8 * i - 2)) & 0x3Cu));
+          const float l1 = *reinterpret_cast<const float*>(lvb + ((w >> (8 * i + 2)) & 0x3Cu));
+          uint64_t p2, l2;
+          asm("mov.b64 %0, {%1, %2};" : "=l"(l2) : "f"(l0), "f"(l1));
+          asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(p2) : "l"(l2), "l"(a2));
+          float q0, q1;
+          asm("mov.b64 {%0, %1}, %2;" : "=f"(q0), "=f"(q1) : "l"(p2));
+          o[i] = pack_bf16(q0, q1);
+        }
+        *reinterpret_cast<uint4*>(wt + rsw + ((c ^ (n & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // for the MMA's reads
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&w_full[s]);
+    }
   }
   // ---------------- (alpha/r) x A^T -> bf16 operand in shared memory ----------
   const bool u_ok = __syncthreads_and(mbar_wait(&u_bar, 0)) != 0;   // uniform
   tc_fence_after();
   const int row = warp * 32 + lane;            // TMEM lane = tile row
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  if (r > 0 && u_ok) {
+  if (r > 0 && u_ok && warp < 4) {
     unsigned char* us = smem + S::U_OFF;
     for (int c0 = 0; c0 < rp; c0 += 16) {
       float v[16];
@@ -270,7 +373,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
   tc_fence_after();
   const int m = m0 + row;
   const bool active = m < args.M;                     // rows past M: load, do not store
-  if (good) {
+  if (good && warp < 4) {
     const int D = args.D, half = D / 2;
     const int mm = active ? m : 0;
     const int b = mm / args.L, l = mm % args.L;
@@ -398,14 +501,14 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
   return res == CUDA_SUCCESS;
 }
 
-template <int BN>
+template <int BN, bool NF4 = false>
 cudaError_t launch_bn(const CUtensorMap maps[8], const TcArgs& a, cudaStream_t s) {
   const int smem = Smem<BN>::TOTAL;
-  auto kern = project_tc_kernel<BN>;
+  auto kern = project_tc_kernel<BN, NF4>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_off[3] / BN, (a.M + BM - 1) / BM);
-  launch_pdl(kern, dim3(grid), dim3(kThreads), smem, s, maps[0], maps[1], maps[2], maps[3], maps[4], maps[5],
+  launch_pdl(kern, dim3(grid), dim3(NF4 ? kThreads + 32 * kDqWarps : kThreads), smem, s, maps[0], maps[1], maps[2], maps[3], maps[4], maps[5],
                                     maps[6], maps[7], a);
   return cudaGetLastError();
 }
@@ -424,14 +527,19 @@ int project_tc_tile(int Hq, int Hkv, int D, int d_in) {
   return 0;
 }
 
-cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void* w,
-                              const void* const a[3], const void* const bm[3], const int r[3],
-                              float alpha_over_r, int Hq, int Hkv, int D, int pos0,
-                              const int* pos_dev, float rope_base, void* const out[3], int* err,
-                              cudaStream_t s, const Geom* append_to, int pos_stride) {
+// NF4 base (codes, absmax) when `w` is null.
+static cudaError_t launch_tc(const void* x, int B, int L, int d_in, const void* w,
+                             const uint8_t* nf4_codes, const float* nf4_absmax,
+                             const void* const a[3], const void* const bm[3], const int r[3],
+                             float alpha_over_r, int Hq, int Hkv, int D, int pos0,
+                             const int* pos_dev, float rope_base, void* const out[3], int* err,
+                             cudaStream_t s, const Geom* append_to, int pos_stride) {
+  const bool nf4 = w == nullptr;
   const int bn = project_tc_tile(Hq, Hkv, D, d_in);
   if (!bn) return cudaErrorNotSupported;
   TcArgs t;
+  t.nf4_codes = nf4_codes;
+  t.nf4_absmax = nf4_absmax;
   t.pack = append_to != nullptr;
   if (append_to) t.g = *append_to;
   else memset(&t.g, 0, sizeof t.g);
@@ -447,8 +555,9 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
   t.rope = rope_base > 0.f; t.k_blocks = d_in / 64; t.err = err;
   rope_theta_table(rope_base, D, t.theta_hi, t.theta_lo);
   CUtensorMap maps[8];
-  bool ok = make_map(&maps[0], x, M, d_in, BM) &&
-            make_map(&maps[1], w, (uint64_t)t.n_off[3], d_in, bn);
+  bool ok = make_map(&maps[0], x, M, d_in, BM);
+  if (nf4) maps[1] = maps[0];                       // unused: any valid map
+  else ok = ok && make_map(&maps[1], w, (uint64_t)t.n_off[3], d_in, bn);
   const int dout[3] = {Hq * D, Hkv * D, Hkv * D};
   for (int p = 0; p < 3 && ok; ++p) {
     if (r[p] > 0) {
@@ -460,7 +569,33 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
     }
   }
   if (!ok) return cudaErrorInvalidValue;
+  if (nf4) return bn == 256 ? launch_bn<256, true>(maps, t, s) : launch_bn<128, true>(maps, t, s);
   return bn == 256 ? launch_bn<256>(maps, t, s) : launch_bn<128>(maps, t, s);
+}
+
+cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void* w,
+                              const void* const a[3], const void* const bm[3], const int r[3],
+                              float alpha_over_r, int Hq, int Hkv, int D, int pos0,
+                              const int* pos_dev, float rope_base, void* const out[3], int* err,
+                              cudaStream_t s, const Geom* append_to, int pos_stride) {
+  if (!w) return cudaErrorInvalidValue;
+  return launch_tc(x, B, L, d_in, w, nullptr, nullptr, a, bm, r, alpha_over_r, Hq, Hkv, D, pos0,
+                   pos_dev, rope_base, out, err, s, append_to, pos_stride);
+}
+
+bool project_tc_nf4_supported(int Hq, int Hkv, int D, int d_in) {
+  return project_tc_tile(Hq, Hkv, D, d_in) != 0;
+}
+
+cudaError_t launch_project_tc_nf4(const void* x, int B, int L, int d_in, const void* codes,
+                                  const void* absmax, const void* const a[3],
+                                  const void* const bm[3], const int r[3], float alpha_over_r,
+                                  int Hq, int Hkv, int D, int pos0, const int* pos_dev,
+                                  float rope_base, void* const out[3], int* err, cudaStream_t s,
+                                  int pos_stride) {
+  return launch_tc(x, B, L, d_in, nullptr, static_cast<const uint8_t*>(codes),
+                   static_cast<const float*>(absmax), a, bm, r, alpha_over_r, Hq, Hkv, D, pos0,
+                   pos_dev, rope_base, out, err, s, nullptr, pos_stride);
 }
 
 }  // namespace kvq
