@@ -301,15 +301,17 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
       for (int j = 0; j < 4 * NQ; ++j) {                  // chunk c: inputs 8c .. 8c + 7
         const int c = 4 * NQ * h + j;
         uint32_t o[4];
+        // byte offsets into the level table (4 x code) of the word's low and
+        // high nibbles, four at a time
+        const uint32_t lo4 = (w8[j] << 2) & 0x3C3C3C3Cu, hi4 = (w8[j] >> 2) & 0x3C3C3C3Cu;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {                     // byte i of word j: inputs 8c + 2i, + 1
           // the two levels times absmax as one packed fp32 multiply (each
           // product rounded as a scalar one would be), then one bf16 pair
           const char* lvb = reinterpret_cast<const char*>(nf4_lv);
-          const uint32_t w = w8[j];
-          const float l0 = *reinterpret_cast<const float*>(
-              lvb + ((i == 0 ? w << 2 : w >> (8 * i - 2)) & 0x3Cu));
-          const float l1 = *reinterpret_cast<const float*>(lvb + ((w >> (8 * i + 2)) & 0x3Cu));
+          const uint32_t sel = 0x4440u | (uint32_t)i;     // byte i into byte 0, zeros above
+          const float l0 = *reinterpret_cast<const float*>(lvb + __byte_perm(lo4, 0u, sel));
+          const float l1 = *reinterpret_cast<const float*>(lvb + __byte_perm(hi4, 0u, sel));
           uint64_t p2, l2;
           asm("mov.b64 %0, {%1, %2};" : "=l"(l2) : "f"(l0), "f"(l1));
           asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(p2) : "l"(l2), "l"(a2));
