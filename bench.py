@@ -574,12 +574,14 @@ def paged_decode_rates(run, peaks, flush):
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
 
 
-def ste_backward_rates(run, flush, max_len=2048):
+def ste_backward_rates(run, peaks, flush, max_len=2048):
     """The straight-through backward of one layer (kvq_attend_backward, then
     kvq_lora_backward with d_x) for one sequence of min(prefill, 2048) tokens
-    of the workload's shape and cache format: the adapter-training step.  Its
-    products run on fp32 SIMT GEMMs, so the rates are against the fp32 FMA
-    rate.  None for KVarN caches (no backward)."""
+    of the workload's shape and cache format: the adapter-training step.  The
+    attention products run on fp32 SIMT GEMMs (rated against the fp32 FMA
+    rate); with bf16 activations the adapters' dominant product, d_x = g W,
+    runs on the tensor cores (rated against the sustained bf16 peak).  None for
+    KVarN caches (no backward)."""
     from paper_2609_04263_gb300 import kvq
     wl, api = run.wl, run.api
     if wl.fmt == synth.FMT_KVARN:
@@ -601,7 +603,7 @@ def ste_backward_rates(run, flush, max_len=2048):
         torch.empty(1, Hkv, L, D, **f32)
     ws_bytes = kvq.kvq_attend_backward_workspace(cache.handle, L, Hq) * Hkv
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
-    lws_bytes = kvq.kvq_lora_backward_workspace(1, L, Hq, Hkv, D, r, r, r)
+    lws_bytes = kvq.kvq_lora_backward_workspace(1, L, d_in, Hq, Hkv, D, r, r, r)
     lws = torch.empty(lws_bytes, dtype=torch.uint8, device=dev)
     grads = [torch.empty(lora[p][i].shape, **f32) for p in "qkv" for i in (0, 1)]
     dx = torch.empty(1, L, d_in, **f32)
@@ -627,15 +629,20 @@ def ste_backward_rates(run, flush, max_len=2048):
     lora_flops = (2 * L * d_in * 3 * r + 2 * 2 * L * r * n_out + 2 * L * r * 3 * d_in
                   + 2 * L * n_out * d_in + 2 * L * 3 * r * d_in)
     rate = lambda f, ms: round(f / ms / 1e9, 3)
+    fma = {"bound": "alu", "value": round(FP32_FMA_TFLOPS, 2), "unit": "TFLOP/s",
+           "what": "fp32 FMA: 152 SMs x 128 lanes x 2 flops x 2070 MHz"}
+    tensor = dt == torch.bfloat16 and d_in % 128 == 0 and n_out % 64 == 0
+    lpeak = ({"bound": "tensor", "value": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s",
+              "what": "measured sustained bf16 (d_x = g W as bf16 high + low parts of g: "
+                      "twice the algorithmic MMA work)"} if tensor else fma)
     return {"tokens": L, "sequences": 1,
             "attention": {"mean_ms": round(att_ms, 4), "flops": att_flops,
                           "achieved": rate(att_flops, att_ms), "unit": "TFLOP/s",
-                          "frac": round(att_flops / att_ms / 1e9 / FP32_FMA_TFLOPS, 4)},
+                          "frac": round(att_flops / att_ms / 1e9 / fma["value"], 4), "peak": fma},
             "adapters": {"mean_ms": round(lora_ms, 4), "flops": lora_flops,
                          "achieved": rate(lora_flops, lora_ms), "unit": "TFLOP/s",
-                         "frac": round(lora_flops / lora_ms / 1e9 / FP32_FMA_TFLOPS, 4)},
-            "peak": {"bound": "alu", "value": round(FP32_FMA_TFLOPS, 2), "unit": "TFLOP/s",
-                     "what": "fp32 FMA: 152 SMs x 128 lanes x 2 flops x 2070 MHz"},
+                         "frac": round(lora_flops / lora_ms / 1e9 / lpeak["value"], 4),
+                         "peak": lpeak},
             "l2": "flushed before each timed launch"}
 
 
@@ -923,7 +930,7 @@ def main():
                         "l2": "flushed before each replay of all layers' calls",
                         "traffic": measured_traffic(wl.name, "decode_attention")}
     nf4 = nf4_projection_rates(run, peaks, flush) if wl.dtype == "bf16" else None
-    ste = ste_backward_rates(run, flush)
+    ste = ste_backward_rates(run, peaks, flush)
     paged = paged_decode_rates(run, peaks, flush)
     share = {k: mean_ms[k] * work[k][2] for k in work}
     dominant = max(share, key=share.get)

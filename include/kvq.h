@@ -393,10 +393,15 @@ kvq_status kvq_attend_backward(kvq_cache* cache, const void* q, const void* d_ou
  *   d_x [B][L][d_in] = g W + sum_p (alpha/r) (g_p B_p) A_p   (needs w_qkv).
  * x, w_qkv and the factors are in `dtype`, laid out as for kvq_project_lora;
  * a projection with r_p = 0 has no factors and its gradients are not written.
- * workspace: at least kvq_lora_backward_workspace() bytes.
+ * With bf16 activations, d_in a multiple of 128 and (Hq + 2 Hkv) D a multiple of
+ * 64, g W runs on the tensor cores: g is split in the workspace into bf16 high and
+ * low parts (about 16 significant bits) against W^T, which the call also writes
+ * into the workspace.
+ * workspace: at least kvq_lora_backward_workspace() bytes (a function of the
+ * shape alone; 16-byte aligned).
  */
-size_t kvq_lora_backward_workspace(int B, int L, int n_q_heads, int n_kv_heads, int head_dim,
-                                   int r_q, int r_k, int r_v);
+size_t kvq_lora_backward_workspace(int B, int L, int d_in, int n_q_heads, int n_kv_heads,
+                                   int head_dim, int r_q, int r_k, int r_v);
 kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* w_qkv,
                              const void* a_q, const void* b_q, int r_q,
                              const void* a_k, const void* b_k, int r_k,

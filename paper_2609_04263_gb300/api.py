@@ -247,7 +247,7 @@ def lora_backward(x, w_qkv, lora, alpha_over_r, n_q_heads, n_kv_heads, head_dim,
     D = head_dim
     r = [0 if lora.get(p) is None else lora[p][0].shape[0] for p in "qkv"]
     if workspace is None:
-        nb = kvq.kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, D, *r)
+        nb = kvq.kvq_lora_backward_workspace(B, L, d_in, n_q_heads, n_kv_heads, D, *r)
         workspace = torch.empty(nb, dtype=torch.uint8, device=x.device)
     f32 = dict(dtype=torch.float32, device=x.device)
     grads, args = {}, []

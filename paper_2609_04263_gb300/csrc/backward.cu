@@ -358,6 +358,45 @@ __global__ void lora_gather_kernel(GatherArgs a) {
   }
 }
 
+// Rows of G [rows][n] fp32, in place, as [rows][2n] bf16: the high parts
+// (g rounded to bf16) then the bf16 of the remainders, so that the two halves
+// carry about 16 significant bits of g for a bf16 tensor-core product.  One
+// CTA per row at a time: the row goes through shared memory first.
+__global__ void __launch_bounds__(256) bwd_split_rows_kernel(float* G, int rows, int n) {
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ float rowbuf[];
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    float* g = G + (int64_t)r * n;
+    for (int j = threadIdx.x; j < n; j += blockDim.x) rowbuf[j] = g[j];
+    __syncthreads();
+    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(g);
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+      const float v = rowbuf[j];
+      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+      o[j] = hi;
+      o[n + j] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    }
+    __syncthreads();
+  }
+}
+
+// Wt [d][n] = W [n][d] (bf16), 32 x 32 tiles through shared memory.
+__global__ void __launch_bounds__(256) bwd_transpose_kernel(const __nv_bfloat16* __restrict__ W,
+                                                            __nv_bfloat16* __restrict__ Wt, int n,
+                                                            int d) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ __nv_bfloat16 tile[32][33];
+  const int n0 = blockIdx.y * 32, d0 = blockIdx.x * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 8 rows per pass
+  for (int i = ty; i < 32; i += 8)
+    if (n0 + i < n && d0 + tx < d) tile[i][tx] = W[(int64_t)(n0 + i) * d + d0 + tx];
+  __syncthreads();
+  for (int i = ty; i < 32; i += 8)
+    if (d0 + i < d && n0 + tx < n) Wt[(int64_t)(d0 + i) * n + n0 + tx] = tile[tx][i];
+}
+
 int grid_for(int64_t n, int threads) {
   const int64_t blocks = (n + threads - 1) / threads;
   return (int)std::min<int64_t>(blocks, (int64_t)num_sms() * 16);
@@ -444,11 +483,18 @@ cudaError_t launch_attend_backward(const Geom& g, int T, const void* q, const vo
   return e;
 }
 
-size_t lora_backward_bytes(int B, int L, int Hq, int Hkv, int D, const int r[3]) {
+size_t lora_backward_bytes(int B, int L, int d_in, int Hq, int Hkv, int D, const int r[3]) {
   const size_t BL = (size_t)B * L;
   size_t n = a256(BL * (Hq + 2 * Hkv) * D * sizeof(float));
   for (int p = 0; p < 3; ++p) n += 2 * a256(BL * r[p] * sizeof(float));
+  n += a256((size_t)d_in * (Hq + 2 * Hkv) * D * 2);   // W^T in bf16 for the d_x product
   return n;
+}
+
+// d_x on tcgen05 needs bf16 activations and whole 64-element K slices and
+// 128-column output tiles.
+static bool dx_on_tc(int act, int d_in, int ntot) {
+  return act == KVQ_BF16 && d_in % 128 == 0 && ntot % 64 == 0;
 }
 
 cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const void* w,
@@ -473,6 +519,7 @@ cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const vo
     V[p] = reinterpret_cast<float*>(wp);
     wp += a256((size_t)BL * r[p] * sizeof(float));
   }
+  __nv_bfloat16* Wt = reinterpret_cast<__nv_bfloat16*>(wp);   // [d_in][ntot]
   GatherArgs ga;
   ga.dq = dq; ga.dk = dk; ga.dv = dv; ga.G = G;
   ga.B = B; ga.L = L; ga.Hq = Hq; ga.Hkv = Hkv; ga.D = D; ga.kv_rows = kv_rows; ga.pos0 = pos0;
@@ -482,12 +529,17 @@ cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const vo
   cudaError_t e = cudaGetLastError();
   for (int p = 0; p < 3 && e == cudaSuccess; ++p) {
     if (r[p] == 0) continue;
-    // U_p = x A_p^T  [BL][r]
+    // U_p = x A_p^T  [BL][r] and V_p = g_p B_p  [BL][r]: narrow outputs over
+    // long K, split over K (accumulated atomically into zeroed outputs)
     GemmArgs gu = gemm_args(x, d_in, 0, a[p], d_in, 0, U[p], r[p], 0, BL, r[p], d_in, 1, 1.f);
-    e = gemm_act_ab<true, true>(gu, act, s);
-    // V_p = g_p B_p  [BL][r]
+    gu.splits = choose_splits(BL, r[p], d_in, 1);
+    if (gu.splits > 1) e = cudaMemsetAsync(U[p], 0, (size_t)BL * r[p] * sizeof(float), s);
+    if (e == cudaSuccess) e = gemm_act_ab<true, true>(gu, act, s);
     GemmArgs gv = gemm_args(G + off[p], ntot, 0, bm[p], r[p], 0, V[p], r[p], 0, BL, r[p],
                             nout[p], 1, 1.f);
+    gv.splits = choose_splits(BL, r[p], nout[p], 1);
+    if (e == cudaSuccess && gv.splits > 1)
+      e = cudaMemsetAsync(V[p], 0, (size_t)BL * r[p] * sizeof(float), s);
     if (e == cudaSuccess) e = gemm_act_b<true, false>(gv, act, s);
     // dB_p = (alpha/r) g_p^T U_p  [n_p][r], split over the BL rows
     GemmArgs gb = gemm_args(G + off[p], ntot, 0, U[p], r[p], 0, db[p], r[p], 0, nout[p], r[p],
@@ -506,8 +558,28 @@ cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const vo
   }
   if (dx && e == cudaSuccess) {
     // dx = g W + sum_p (alpha/r) V_p A_p
-    GemmArgs gx = gemm_args(G, ntot, 0, w, d_in, 0, dx, d_in, 0, BL, d_in, ntot, 1, 1.f);
-    e = gemm_act_b<true, false>(gx, act, s);
+    if (dx_on_tc(act, d_in, ntot)) {
+      // g W on tcgen05: g split into bf16 high and low parts in place (G is
+      // not read again), [g_hi | g_lo] times [W^T | W^T] along K
+      int* err = device_error_word();
+      if (!err) return cudaErrorInvalidDevice;
+      launch_pdl(bwd_transpose_kernel, dim3((d_in + 31) / 32, (ntot + 31) / 32), dim3(256), 0, s,
+                 reinterpret_cast<const __nv_bfloat16*>(w), Wt, ntot, d_in);
+      e = cudaGetLastError();
+      const size_t sm = (size_t)ntot * sizeof(float);
+      if (e == cudaSuccess && sm > 48 * 1024)
+        e = cudaFuncSetAttribute(bwd_split_rows_kernel,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+      if (e == cudaSuccess) {
+        launch_pdl(bwd_split_rows_kernel, dim3(std::min(BL, num_sms() * 8)), dim3(256), sm, s, G,
+                   BL, ntot);
+        e = cudaGetLastError();
+      }
+      if (e == cudaSuccess) e = launch_gemm_tc_bf16(G, BL, 2 * ntot, Wt, d_in, ntot, dx, err, s);
+    } else {
+      GemmArgs gx = gemm_args(G, ntot, 0, w, d_in, 0, dx, d_in, 0, BL, d_in, ntot, 1, 1.f);
+      e = gemm_act_b<true, false>(gx, act, s);
+    }
     for (int p = 0; p < 3 && e == cudaSuccess; ++p) {
       if (r[p] == 0) continue;
       GemmArgs gl = gemm_args(V[p], r[p], 0, a[p], d_in, 0, dx, d_in, 0, BL, d_in, r[p], 1,

@@ -858,13 +858,13 @@ kvq_status kvq_attend_backward(kvq_cache* cache, const void* q, const void* d_ou
   return KVQ_OK;
 }
 
-size_t kvq_lora_backward_workspace(int B, int L, int n_q_heads, int n_kv_heads, int head_dim,
-                                   int r_q, int r_k, int r_v) {
-  if (B <= 0 || L <= 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0 || r_q < 0 ||
-      r_k < 0 || r_v < 0)
+size_t kvq_lora_backward_workspace(int B, int L, int d_in, int n_q_heads, int n_kv_heads,
+                                   int head_dim, int r_q, int r_k, int r_v) {
+  if (B <= 0 || L <= 0 || d_in <= 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0 ||
+      r_q < 0 || r_k < 0 || r_v < 0)
     return 0;
   const int r[3] = {r_q, r_k, r_v};
-  return lora_backward_bytes(B, L, n_q_heads, n_kv_heads, head_dim, r);
+  return lora_backward_bytes(B, L, d_in, n_q_heads, n_kv_heads, head_dim, r);
 }
 
 kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* w_qkv,
@@ -897,7 +897,7 @@ kvq_status kvq_lora_backward(const void* x, int B, int L, int d_in, const void* 
     if (r[p] > 0 && (!a[p] || !bm[p] || !da[p] || !db[p]))
       return fail(KVQ_ERR_ARG, "rank %d but a NULL factor or gradient", r[p]);
   }
-  const size_t need = lora_backward_bytes(B, L, n_q_heads, n_kv_heads, head_dim, r);
+  const size_t need = lora_backward_bytes(B, L, d_in, n_q_heads, n_kv_heads, head_dim, r);
   if (workspace_bytes < need)
     return fail(KVQ_ERR_CAPACITY, "workspace of %zu bytes < %zu", workspace_bytes, need);
   if (misaligned(workspace)) return fail(KVQ_ERR_ARG, "workspace must be 16-byte aligned");

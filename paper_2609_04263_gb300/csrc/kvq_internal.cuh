@@ -160,6 +160,10 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
                               const int* pos_dev, float rope_base, void* const out[3], int* err,
                               cudaStream_t s, const Geom* append_to = nullptr, int pos_stride = 0);
 int project_tc_tile(int Hq, int Hkv, int D, int d_in);
+// The same kernel as a plain product: C [M][N] fp32 = A [M][K] B^T, A and Bt
+// bf16 K-major, Bt's rows of Kb elements repeated along K (K a multiple of Kb).
+cudaError_t launch_gemm_tc_bf16(const void* a, int M, int K, const void* bt, int N, int Kb,
+                                float* c, int* err, cudaStream_t s);
 // The same kernel over an NF4 base (codes [N][d_in/2], fp32 absmax [N][d_in/64],
 // dequantised in the kernel's operand path).
 bool project_tc_nf4_supported(int Hq, int Hkv, int D, int d_in);
@@ -188,7 +192,7 @@ size_t attend_backward_pair_bytes(const Geom& g, int T, int L);
 cudaError_t launch_attend_backward(const Geom& g, int T, const void* q, const void* d_out,
                                    int L, float scale, float* dq, float* dk, float* dv,
                                    void* ws, size_t ws_bytes, cudaStream_t s);
-size_t lora_backward_bytes(int B, int L, int Hq, int Hkv, int D, const int r[3]);
+size_t lora_backward_bytes(int B, int L, int d_in, int Hq, int Hkv, int D, const int r[3]);
 cudaError_t launch_lora_backward(const void* x, int B, int L, int d_in, const void* w,
                                  const void* const a[3], const void* const bm[3],
                                  const int r[3], float alpha_over_r, int Hq, int Hkv, int D,

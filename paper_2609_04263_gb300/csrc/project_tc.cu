@@ -61,6 +61,8 @@ struct TcArgs {
   int pack;                     // 1: code k and v into the cache g instead of storing them
   const uint8_t* nf4_codes;     // NF4 base: codes [N][d_in / 2] (two inputs a byte, low first)
   const float* nf4_absmax;      //           and one absmax per 64 inputs of a row [N][d_in / 64]
+  float* plain_out;             // plain product: fp32 [M][N] row-major, no RoPE, no adapters
+  int kb_wrap;                  // > 0: K slice kb of W is slice kb % kb_wrap (W repeated along K)
   Geom g;
   float theta_hi[128], theta_lo[128];
 };
@@ -213,7 +215,9 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
       unsigned char* st = smem + s * S::STAGE_B;
       mbar_expect_tx(&full_bar[s], S::A_B + (NF4 ? 0 : S::B_B) + (r > 0 ? rp * BK * 2 : 0));
       tma_load_2d(st, &tm_x, kb * BK, m0, &full_bar[s]);
-      if (!NF4) tma_load_2d(st + S::A_B, &tm_w, kb * BK, n0, &full_bar[s]);
+      if (!NF4)
+        tma_load_2d(st + S::A_B, &tm_w, (args.kb_wrap ? kb % args.kb_wrap : kb) * BK, n0,
+                    &full_bar[s]);
       if (r > 0) tma_load_2d(st + S::A_B + S::B_B, tm_a, kb * BK, 0, &full_bar[s]);
     }
   } else if (threadIdx.x == 32) {
@@ -384,7 +388,18 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constan
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(args.out[proj]);
     const bool rope = args.rope && proj < 2;
     const int pos = args.pos0 + pos_of(args.pos_dev, args.pos_stride, b) + l;
-    if (args.pack && proj > 0) {
+    if (args.plain_out) {
+      // plain product: the accumulator row as fp32
+      const int N = args.n_off[3];
+      for (int c = 0; c < BN; c += 16) {
+        float v[16];
+        tmem_ld16(tmem + lane_base + c, v);
+        if (!active) continue;
+        float4* d = reinterpret_cast<float4*>(args.plain_out + (int64_t)m * N + n0 + c);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+    } else if (args.pack && proj > 0) {
       // append: k (after RoPE) and v rounded to bf16, then coded per token
       // in groups of 32 channels straight into the cache planes
       const Geom& gg = args.g;
@@ -542,6 +557,8 @@ static cudaError_t launch_tc(const void* x, int B, int L, int d_in, const void* 
   TcArgs t;
   t.nf4_codes = nf4_codes;
   t.nf4_absmax = nf4_absmax;
+  t.plain_out = nullptr;
+  t.kb_wrap = 0;
   t.pack = append_to != nullptr;
   if (append_to) t.g = *append_to;
   else memset(&t.g, 0, sizeof t.g);
@@ -583,6 +600,26 @@ cudaError_t launch_project_tc(const void* x, int B, int L, int d_in, const void*
   if (!w) return cudaErrorInvalidValue;
   return launch_tc(x, B, L, d_in, w, nullptr, nullptr, a, bm, r, alpha_over_r, Hq, Hkv, D, pos0,
                    pos_dev, rope_base, out, err, s, append_to, pos_stride);
+}
+
+// C [M][N] fp32 = A [M][K] B^T on tcgen05, A bf16 K-major, B's rows bf16 of Kb
+// elements repeated along K (K a multiple of Kb: B(k) = Bt[:, k mod Kb]).
+cudaError_t launch_gemm_tc_bf16(const void* a, int M, int K, const void* bt, int N, int Kb,
+                                float* c, int* err, cudaStream_t s) {
+  if (M <= 0 || N <= 0 || K <= 0 || K % 64 || Kb % 64 || K % Kb) return cudaErrorInvalidValue;
+  const int bn = N % 256 == 0 ? 256 : N % 128 == 0 ? 128 : 0;
+  if (!bn) return cudaErrorNotSupported;
+  TcArgs t;
+  memset(&t, 0, sizeof t);
+  t.B = 1; t.L = M; t.M = M; t.D = 64; t.Hq = N / 64; t.Hkv = 1;
+  t.n_off[0] = 0; t.n_off[1] = N; t.n_off[2] = N; t.n_off[3] = N;
+  t.k_blocks = K / 64; t.kb_wrap = Kb / 64 == K / 64 ? 0 : Kb / 64; t.err = err;
+  t.plain_out = c;
+  CUtensorMap maps[8];
+  if (!make_map(&maps[0], a, M, K, BM) || !make_map(&maps[1], bt, N, Kb, bn))
+    return cudaErrorInvalidValue;
+  for (int i = 2; i < 8; ++i) maps[i] = maps[0];   // unused: no adapters
+  return bn == 256 ? launch_bn<256>(maps, t, s) : launch_bn<128>(maps, t, s);
 }
 
 bool project_tc_nf4_supported(int Hq, int Hkv, int D, int d_in) {

@@ -96,7 +96,7 @@ _SIGS = {
                                     c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
                                     c_void_p]),
     "kvq_lora_backward_workspace": (c_size_t, [c_int, c_int, c_int, c_int, c_int, c_int, c_int,
-                                               c_int]),
+                                               c_int, c_int]),
     "kvq_lora_backward": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p,
                                   c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int,
                                   c_void_p, c_void_p, c_int, c_float, c_int, c_int, c_int,
@@ -259,9 +259,10 @@ def kvq_attend_backward(handle, q, d_out, L, n_q_heads, softmax_scale, d_q, d_k,
                                      c_void_p(stream or 0)))
 
 
-def kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, head_dim, r_q, r_k, r_v) -> int:
-    return lib().kvq_lora_backward_workspace(B, L, n_q_heads, n_kv_heads, head_dim, r_q, r_k,
-                                             r_v)
+def kvq_lora_backward_workspace(B, L, d_in, n_q_heads, n_kv_heads, head_dim, r_q, r_k,
+                                r_v) -> int:
+    return lib().kvq_lora_backward_workspace(B, L, d_in, n_q_heads, n_kv_heads, head_dim, r_q,
+                                             r_k, r_v)
 
 
 def kvq_lora_backward(x, B, L, d_in, w_qkv, a_q, b_q, r_q, a_k, b_k, r_k, a_v, b_v, r_v,

@@ -212,8 +212,10 @@ def test_backward_host_rules(kvq):
 
     def a256(n):
         return (n + 255) // 256 * 256
-    want = a256(B * L * (Hq + 2 * Hkv) * D * 4) + sum(2 * a256(B * L * x * 4) for x in r)
-    assert kvq.kvq_lora_backward_workspace(B, L, Hq, Hkv, D, *r) == want
+    d_in = 256
+    want = (a256(B * L * (Hq + 2 * Hkv) * D * 4) + sum(2 * a256(B * L * x * 4) for x in r)
+            + a256(d_in * (Hq + 2 * Hkv) * D * 2))
+    assert kvq.kvq_lora_backward_workspace(B, L, d_in, Hq, Hkv, D, *r) == want
     with pytest.raises(kvq.KvqError) as ei:
         kvq.kvq_lora_backward(P, B, L, 256, P, P, P, 16, None, None, 0, P, P, 8, 2.0, Hq, Hkv, D,
                               0, 1e4, kvq.KVQ_BF16, P, P, P, L, P, P, None, None, P, P, None,

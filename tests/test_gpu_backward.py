@@ -124,6 +124,8 @@ LORA_CASES = [
     ("bf16", 2, 70, 256, 8, 2, 64, (16, 16, 16), 0, 3, 10000.0),
     ("bf16", 1, 40, 512, 4, 4, 128, (8, 0, 24), 25, 100, 500000.0),   # d_k rows beyond L
     ("f32", 3, 17, 128, 2, 1, 64, (8, 8, 8), 0, 0, 0.0),              # no RoPE
+    ("bf16", 2, 300, 1024, 8, 2, 128, (16, 16, 16), 0, 0, 500000.0),  # d_x on tensor cores: ragged row tile, 4 column tiles
+    ("bf16", 1, 33, 192, 4, 2, 64, (8, 8, 8), 0, 0, 10000.0),        # d_in not a multiple of 128: the SIMT d_x
 ]
 
 
