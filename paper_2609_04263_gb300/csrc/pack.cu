@@ -354,26 +354,17 @@ __global__ void __launch_bounds__(256) kivi_key_flush_kernel(Geom g, int L, TokS
 // compile time (the KIVI configuration): 256 threads, 256 / D of them per
 // channel over 32 D / 256 tokens each; codes go to shared memory as bytes and
 // leave as whole packed words.  Same arithmetic as kivi_key_flush_kernel.
+// One 32-token key block `blk` of the (b, h) row, by the CTA's 256 threads
+// (src.T0 set: tokens below it come from the residual ring).
 template <int D, int BITS>
-__global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, TokSrc src) {
+__device__ __forceinline__ void kivi_key_flush32_block(const Geom& g, const TokSrc& src, int b,
+                                                       int h, int blk, float* smem) {
   constexpr int G = 32, NT = 256, CPT = D / 8, PARTS = NT / D, TPP = G / PARTS;
   constexpr int CPW = 32 / BITS, WPR = D / CPW;
-  pdl_wait();
-  pdl_trigger();
-  extern __shared__ float smem[];
-  bool ok = true;
-  const int T0u = g.layout == KVQ_LAYOUT_UNIFORM ? append_begin(g, L, &ok) : 0;
-  int T0, n;
-  append_span(g, blockIdx.y / g.H, L, T0u, &T0, &n);
-  const int q0 = kivi_tq(T0, g.R, G), q1 = kivi_tq(T0 + n, g.R, G);
-  const int blk = q0 / G + blockIdx.x;
-  if (!ok || blk >= q1 / G) return;
-  src.T0 = T0;
   float* xs = smem;                                      // [G][D]
   uint8_t* cs = reinterpret_cast<uint8_t*>(xs + G * D);  // [G][D]
   float* pmn = reinterpret_cast<float*>(cs + G * D);     // [PARTS][D]
   float* pmx = pmn + PARTS * D;
-  const int h = blockIdx.y % g.H, b = blockIdx.y / g.H;
   const int t0 = blk * G;
 #pragma unroll
   for (int k = 0; k < G * CPT / NT; ++k) {
@@ -445,6 +436,63 @@ __global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, To
     }
     reinterpret_cast<uint32_t*>(tok_ptr<uint8_t>(g, KVQ_PLANE_K_CODES, b, h, t0 + r))[w] = word;
   }
+}
+
+template <int D, int BITS>
+__global__ void __launch_bounds__(256) kivi_key_flush32_kernel(Geom g, int L, TokSrc src) {
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ float smem[];
+  bool ok = true;
+  const int T0u = g.layout == KVQ_LAYOUT_UNIFORM ? append_begin(g, L, &ok) : 0;
+  int T0, n;
+  append_span(g, blockIdx.y / g.H, L, T0u, &T0, &n);
+  const int q0 = kivi_tq(T0, g.R, 32), q1 = kivi_tq(T0 + n, g.R, 32);
+  const int blk = q0 / 32 + blockIdx.x;
+  if (!ok || blk >= q1 / 32) return;
+  src.T0 = T0;
+  kivi_key_flush32_block<D, BITS>(g, src, blockIdx.y / g.H, blockIdx.y % g.H, blk, smem);
+}
+
+// One decode token (L = 1) of a uniform KIVI cache with 32-token blocks, in
+// one launch instead of three: one CTA per (b, h) codes the key block and
+// the value tokens that this token completes (read from the residual ring,
+// with the code of kivi_key_flush32_kernel and pack_pertoken_kernel), then
+// stores the new key and value in the ring (as store_full_kernel does), and
+// the last CTA advances the token count.  The block's ring slots and the new
+// token's slot differ (the ring holds R + 32 tokens).
+template <int D, int BITS>
+__global__ void __launch_bounds__(256) kivi_decode_append_kernel(Geom g, const void* k,
+                                                                 const void* v, int lcpt,
+                                                                 int llpg) {
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ float smem[];
+  bool ok = true;
+  const int T0 = append_begin(g, 1, &ok);
+  // grid (1, B H): pack_rows spreads a row's chunks over blockIdx.x
+  const int b = blockIdx.y / g.H, h = blockIdx.y % g.H;
+  const int q0 = kivi_tq(T0, g.R, 32), q1 = kivi_tq(T0 + 1, g.R, 32);
+  if (ok && q1 > q0) {
+    const TokSrc sk{k, T0, 1, KVQ_PLANE_K_FULL, 0, g.ring};
+    kivi_key_flush32_block<D, BITS>(g, sk, b, h, q0 / 32, smem);
+    const TokSrc sv{v, T0, 1, KVQ_PLANE_V_FULL, 0, g.ring};
+    pack_rows(g, sv, b, h, q0, q1 - q0, 1, 0, lcpt, llpg);
+  }
+  if (ok && T0 >= q1) {                      // the new token stays in full precision
+    constexpr int V16 = D * 2 / 16;          // 16-byte pieces of a bf16 row
+    if ((int)threadIdx.x < 2 * V16) {
+      const int which = threadIdx.x / V16, vi = threadIdx.x % V16;
+      const int plane = which ? KVQ_PLANE_V_FULL : KVQ_PLANE_K_FULL;
+      const uint4* src = reinterpret_cast<const uint4*>(which ? v : k) +
+                         ((int64_t)b * g.H + h) * V16;
+      const Plane& pl = g.pl[plane];
+      uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<char*>(pl.p) +
+                                            plane_index(pl, b, h, g.H, T0 % g.ring, 0) * 2);
+      dst[vi] = src[vi];
+    }
+  }
+  append_arrive_spread(g.state, T0, 1, ok);
 }
 
 // ---------------------------------------------------------------------------
@@ -857,6 +905,19 @@ cudaError_t launch_append(const Geom& g, int L, const void* k, const void* v, cu
       return cudaGetLastError();
     }
     case KVQ_FMT_KIVI: {
+      if (L == 1 && g.G == 32 && g.act == KVQ_BF16 && g.kb == g.vb &&
+          (g.D == 64 || g.D == 128 || g.D == 256) && (g.kb == 2 || g.kb == 4 || g.kb == 8)) {
+        // a decode token: one launch
+        auto kern = kivi_decode_append_kernel<128, 2>;
+        if (g.D == 64) kern = g.kb == 2 ? kivi_decode_append_kernel<64, 2> : g.kb == 4 ? kivi_decode_append_kernel<64, 4> : kivi_decode_append_kernel<64, 8>;
+        if (g.D == 128) kern = g.kb == 2 ? kivi_decode_append_kernel<128, 2> : g.kb == 4 ? kivi_decode_append_kernel<128, 4> : kivi_decode_append_kernel<128, 8>;
+        if (g.D == 256) kern = g.kb == 2 ? kivi_decode_append_kernel<256, 2> : g.kb == 4 ? kivi_decode_append_kernel<256, 4> : kivi_decode_append_kernel<256, 8>;
+        const size_t sm = (size_t)32 * g.D * 5 + 2 * 256 * sizeof(float);
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        if (e != cudaSuccess) return e;
+        launch_pdl(kern, dim3(1, g.B * g.H), dim3(256), sm, s, g, k, v, ilog2(g.D / 8), ilog2(32 / 8));
+        return cudaGetLastError();
+      }
       e = launch_kivi_append(g, L, k, v, s);
       if (e != cudaSuccess) return e;
       launch_pdl(store_full_kernel, dim3(dim3(grid_for(full_threads, 256), 2)), dim3(256), 0, s, g, L, k, v);
