@@ -988,6 +988,12 @@ def main():
         run.x_dec_host.numel() * run.x_dec_host.element_size()
     d2h = o_host.numel() * o_host.element_size() + od_host.numel() * od_host.element_size()
     copy_stream = torch.cuda.Stream()
+    # untimed passes first, as for the device-timed steps: the first copies
+    # between these pinned buffers and the device run far slower (106 ms
+    # instead of 43 ms for the 1 GB prefill input on the 8B-shaped job)
+    for _ in range(min(args.warmup, 2)):
+        run.job_e2e(run.x_pre_host, run.x_dec_host, o_host, od_host, copy_stream)
+    torch.cuda.synchronize()
     for s in range(args.steps):
         l2_flush(flush)
         torch.cuda.synchronize()
