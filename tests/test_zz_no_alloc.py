@@ -12,8 +12,8 @@ whose partials do not fit the scratch.
 The caches below reach every kernel that writes or reads the partials: the
 persistent streaming decode (a long affine cache), the split kernel with its
 in-kernel merge (short caches), the KVarN tensor-core kernel with its sink
-kernel and combine (a long KVarN cache), and the fp32 generic kernel with its
-combine.  Calls on different caches are interleaved so that rows another path
+kernel, whose last CTA merges (a long KVarN cache), and the fp32 generic kernel
+with its combine.  Calls on different caches are interleaved so that rows another path
 left in the scratch are there when the next one runs.
 
 Collected last so that a failure here cannot hide the other GPU tests.
@@ -78,7 +78,7 @@ def test_matches_existing_entry_point_on_consecutive_calls():
         "split kernel (symmetric 2-bit, D 128)": _filled(FORMATS["sym2"], 1, 4, 8, 128, 40,
                                                          "bf16", 3),
         # 2 x 2 heads, up to 60 CTAs: 4 x coded / 32 >= 16 x 60 needs 7680 coded tokens
-        "KVarN tensor-core kernel + sinks + combine": _filled(FORMATS["kvarn_small"], 2, 2, 8,
+        "KVarN tensor-core kernel + sinks with the merge": _filled(FORMATS["kvarn_small"], 2, 2, 8,
                                                               64, 7800, "bf16", 4),
         "generic fp32 kernel + combine": _filled(FORMATS["affine4"], 2, 2, 4, 64, 300, "f32", 5),
     }
